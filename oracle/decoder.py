@@ -1,0 +1,338 @@
+"""Plain float64 CPU oracle of the Llama-family decoder forward.
+
+TEST INFRASTRUCTURE ONLY (see the package docstring): the product path never
+imports this module, and this module imports nothing from the product.
+
+What it computes follows the Axon paper (arxiv 2608.19889):
+
+* the pre-norm residual block -- `h <- NN.rmsnorm@ln x; a <- attention h ...;
+  return x + a` (Sec. "The Axon Language", Syntax paragraph);
+* the core built-ins `NN.embedding`, `NN.linear` (weights `[out, in]`, default
+  `bias=true` that Llama checkpoints leave out except on q/k/v), `NN.rmsnorm`
+  (Sec. "Built-In Libraries", core built-ins listing; running example of the
+  compiler stages for the `bias=true` default);
+* `Attention.attention` with grouped-query heads, causal masks and the
+  `1.0 / sqrt HD` scale (Sec. "Built-In Libraries", the tensor/math listing
+  `scale_heads` and the attention-and-masking paragraph);
+* `Positions.position_ids ... past_length=past_len` and the `Cache`
+  built-ins, dynamic and static overlays with one interface (Sec.
+  "Built-In Libraries", positions and cache management);
+* `Act.swiglu` between `NN.linear@up` and `NN.linear@down` (appendix,
+  function application and composition listing);
+* the model skeleton -- embedding, a `for` loop over layers that threads the
+  cache, final norm and a tied or untied LM head (appendix GPT-2 causal_lm
+  listing);
+* greedy generation, counting generated tokens (Sec. "Results", Measures).
+
+The paper prints no formulas for these operations. Each place where it is
+silent takes the reading listed in READINGS below.
+
+Precision: every input (weights that are exact bf16 values, ids) is widened
+to float64 and every product, sum and transcendental is float64. Nothing is
+rounded back to bf16: the oracle is the exact-arithmetic target the GPU path
+is compared against.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass
+
+import numpy as np
+
+READINGS = [
+    "RMSNorm: y = x / sqrt(mean(x^2) + eps) * g; the gain multiplies the "
+    "normalised vector (not 1+g); eps sits inside the square root.",
+    "RoPE: rotate-half pairing (j, j + d/2), inv_freq_j = theta^(-2j/d), "
+    "angle = position * inv_freq_j, no frequency scaling.",
+    "Positions: the i-th new token of sequence b has position past_b + i, "
+    "past_b = tokens already in the cache.",
+    "GQA: query head h reads KV head floor(h / (H/G)) (contiguous groups).",
+    "Attention scale 1/sqrt(d), causal mask keeps keys with position <= "
+    "query position, softmax with max subtraction.",
+    "Biases: q, k, v only (when attention_bias); never on o, gate, up, down.",
+    "SwiGLU: silu(h Wg^T) * (h Wu^T), silu(z) = z / (1 + exp(-z)).",
+    "LM head: logits = rmsnorm(x) Whead^T with Whead = embedding when tied.",
+    "Greedy next token: argmax of the logits, lowest index on ties.",
+    "KV cache: keys stored after RoPE; the paged overlay maps position p of "
+    "sequence b to block_table[b][p // block_size], offset p % block_size.",
+]
+
+
+@dataclass(frozen=True)
+class DecoderConfig:
+    """HF config.json equivalents read through `Config.dim @@key` (appendix
+    GPT-2 causal_lm listing reads n_embd, n_layer, n_head, vocab_size the same
+    way)."""
+
+    L: int  # num_hidden_layers
+    D: int  # hidden_size
+    H: int  # num_attention_heads
+    G: int  # num_key_value_heads
+    d: int  # head_dim
+    F: int  # intermediate_size
+    V: int  # vocab_size
+    tie: bool  # tie_word_embeddings
+    bias: bool  # attention_bias (q, k, v)
+    theta: float  # rope_theta
+    eps: float  # rms_norm_eps
+
+    @staticmethod
+    def from_dict(c: dict) -> "DecoderConfig":
+        return DecoderConfig(L=int(c["L"]), D=int(c["D"]), H=int(c["H"]), G=int(c["G"]),
+                             d=int(c["d"]), F=int(c["F"]), V=int(c["V"]), tie=bool(c["tie"]),
+                             bias=bool(c["bias"]), theta=float(c["theta"]), eps=float(c["eps"]))
+
+
+# ---------------------------------------------------------------------------
+# Elementary operations
+# ---------------------------------------------------------------------------
+
+def rmsnorm(x, g, eps):
+    """NN.rmsnorm (Sec. Built-In Libraries, core built-ins listing; the
+    pre-norm block of Sec. The Axon Language): scale each vector along the
+    last axis to unit root-mean-square, then multiply by the gain g."""
+    x = np.asarray(x, dtype=np.float64)
+    ms = np.mean(x * x, axis=-1, keepdims=True)
+    return x / np.sqrt(ms + eps) * np.asarray(g, dtype=np.float64)
+
+
+def linear(x, W, b=None):
+    """NN.linear (Sec. Built-In Libraries; compiler running example): y = x W^T
+    (+ b), W stored `[out, in]` as in HF checkpoints."""
+    y = np.asarray(x, dtype=np.float64) @ np.asarray(W, dtype=np.float64).T
+    if b is not None:
+        y = y + np.asarray(b, dtype=np.float64)
+    return y
+
+
+def rope_inv_freq(d, theta):
+    """Positions (Sec. Built-In Libraries, positions and cache management):
+    rotary inverse frequencies theta^(-2j/d), j = 0 .. d/2-1."""
+    j = np.arange(d // 2, dtype=np.float64)
+    return np.power(float(theta), -2.0 * j / d)
+
+
+def rope(x, pos, theta):
+    """Rotary embedding applied by `rope_apply` (Table 6 call counts) with the
+    rotate-half pairing: for j < d/2,
+        out_j       = x_j cos(p f_j) - x_{j+d/2} sin(p f_j)
+        out_{j+d/2} = x_{j+d/2} cos(p f_j) + x_j sin(p f_j).
+    x: [..., d]; pos broadcasts against x[..., 0]."""
+    x = np.asarray(x, dtype=np.float64)
+    d = x.shape[-1]
+    f = rope_inv_freq(d, theta)
+    ang = np.asarray(pos, dtype=np.float64)[..., None] * f
+    c, s = np.cos(ang), np.sin(ang)
+    x1, x2 = x[..., : d // 2], x[..., d // 2:]
+    return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
+
+
+def silu(z):
+    """Activations.silu (Sec. Built-In Libraries, activations): z / (1 + e^-z)."""
+    z = np.asarray(z, dtype=np.float64)
+    with np.errstate(over="ignore"):
+        return z / (1.0 + np.exp(-z))
+
+
+def swiglu(gate, up):
+    """Act.swiglu between NN.linear@up and NN.linear@down (appendix, function
+    application listing): silu(gate) * up."""
+    return silu(gate) * np.asarray(up, dtype=np.float64)
+
+
+def softmax(s, axis=-1):
+    """Tensor.softmax (Sec. Built-In Libraries, tensor and math primitives),
+    with the row maximum subtracted first; -inf entries get weight 0."""
+    s = np.asarray(s, dtype=np.float64)
+    m = np.max(s, axis=axis, keepdims=True)
+    e = np.exp(s - m)
+    return e / np.sum(e, axis=axis, keepdims=True)
+
+
+def attention_one_query(q, K, V, H, G):
+    """Grouped-query scaled dot-product attention for one query position
+    (Sec. Built-In Libraries, attention and masking; scale from `scale_heads`).
+    q: [H, d]; K, V: [T, G, d] holding exactly the visible keys.
+    Returns o: [H, d]."""
+    q = np.asarray(q, dtype=np.float64)
+    d = q.shape[-1]
+    o = np.empty_like(q)
+    per = H // G
+    for h in range(H):
+        g = h // per
+        s = (K[:, g, :] @ q[h]) / math.sqrt(d)
+        o[h] = softmax(s) @ V[:, g, :]
+    return o
+
+
+def causal_attention(q, K, V, q_pos, H, G):
+    """Masking.causal_mask + Attention.attention for S queries of one sequence
+    (Sec. Built-In Libraries, attention and masking).
+    q: [S, H, d] at positions q_pos [S]; K, V: [T, G, d] at positions 0..T-1.
+    Key t is visible to query i iff t <= q_pos[i]. Returns o: [S, H, d]."""
+    q = np.asarray(q, dtype=np.float64)
+    S, _, d = q.shape
+    T = K.shape[0]
+    keep = np.arange(T)[None, :] <= np.asarray(q_pos)[:, None]  # [S, T]
+    o = np.empty_like(q)
+    per = H // G
+    for h in range(H):
+        g = h // per
+        s = (q[:, h, :] @ K[:, g, :].T) / math.sqrt(d)  # [S, T]
+        s = np.where(keep, s, -np.inf)
+        o[:, h, :] = softmax(s, axis=-1) @ V[:, g, :]
+    return o
+
+
+def argmax_lowest(logits):
+    """Greedy selection in `generate()` (Sec. Results, Measures): the index of
+    the largest logit, the lowest such index on ties (np.argmax's rule)."""
+    return np.argmax(np.asarray(logits), axis=-1).astype(np.int64)
+
+
+# ---------------------------------------------------------------------------
+# KV caches (Sec. Built-In Libraries: dynamic vs static `Cache` overlays with
+# one interface; the paged manager is vLLM's PagedAttention, Sec. Related Work)
+# ---------------------------------------------------------------------------
+
+class ContiguousKV:
+    """Static-overlay cache: per layer K, V of shape [B, Tmax, G, d], float64."""
+
+    def __init__(self, L, B, Tmax, G, d):
+        self.K = [np.zeros((B, Tmax, G, d)) for _ in range(L)]
+        self.V = [np.zeros((B, Tmax, G, d)) for _ in range(L)]
+
+    def write(self, l, b, pos, k, v):
+        """Cache.update: store k, v [S, G, d] at positions pos [S]."""
+        self.K[l][b, pos] = k
+        self.V[l][b, pos] = v
+
+    def read(self, l, b, T):
+        """Cache.read: keys and values at positions 0 .. T-1."""
+        return self.K[l][b, :T], self.V[l][b, :T]
+
+
+def slot_of(block_table, b, p, block_size):
+    """Paged slot of position p of sequence b: (block, offset) with
+    block = block_table[b][p // block_size] and offset = p % block_size."""
+    return int(block_table[b][p // block_size]), int(p % block_size)
+
+
+class PagedKV:
+    """Paged cache: per layer a pool [num_blocks, block_size, G, d] and an
+    integer block table [B, max_blocks] naming the pool block of each
+    sequence's logical block."""
+
+    def __init__(self, L, num_blocks, block_size, G, d, block_table):
+        self.bs = int(block_size)
+        self.bt = np.asarray(block_table, dtype=np.int64)
+        self.K = [np.zeros((num_blocks, block_size, G, d)) for _ in range(L)]
+        self.V = [np.zeros((num_blocks, block_size, G, d)) for _ in range(L)]
+
+    def write(self, l, b, pos, k, v):
+        for i, p in enumerate(np.asarray(pos).tolist()):
+            blk, off = slot_of(self.bt, b, p, self.bs)
+            self.K[l][blk, off] = k[i]
+            self.V[l][blk, off] = v[i]
+
+    def read(self, l, b, T):
+        pos = np.arange(T)
+        blk = self.bt[b][pos // self.bs]
+        off = pos % self.bs
+        return self.K[l][blk, off], self.V[l][blk, off]
+
+
+# ---------------------------------------------------------------------------
+# The decoder
+# ---------------------------------------------------------------------------
+
+class Oracle:
+    """Decoder forward over HF-named weights (appendix GPT-2 causal_lm listing
+    for the skeleton; Llama naming `model.layers.{i}.self_attn.q_proj.weight`
+    as in the `_param(...)` lookups of the Python-overhead appendix).
+
+    weights: name -> array (float32 holding exact bf16 values, or float64).
+    keep_f64: convert every matrix to float64 once (faster, 8 bytes/param);
+    otherwise each matmul widens its matrix on the fly.
+    """
+
+    def __init__(self, cfg: DecoderConfig, weights: dict, keep_f64: bool = True):
+        self.cfg = cfg
+        conv = (lambda a: np.asarray(a, dtype=np.float64)) if keep_f64 else (lambda a: np.asarray(a))
+        self.W = {k: conv(v) for k, v in weights.items()}
+
+    def _w(self, name):
+        return self.W[name]
+
+    def new_contiguous_cache(self, B, Tmax):
+        c = self.cfg
+        return ContiguousKV(c.L, B, Tmax, c.G, c.d)
+
+    def new_paged_cache(self, num_blocks, block_size, block_table):
+        c = self.cfg
+        return PagedKV(c.L, num_blocks, block_size, c.G, c.d, block_table)
+
+    def forward(self, ids, cache, past_lens, last_hidden_only=False):
+        """One pass over new tokens ids [B, S] whose sequence b already holds
+        past_lens[b] cached tokens. Writes their K, V into the cache
+        (Cache.update / Cache.append) and returns logits [B, S, V]."""
+        c = self.cfg
+        ids = np.asarray(ids, dtype=np.int64)
+        B, S = ids.shape
+        past = np.asarray(past_lens, dtype=np.int64).reshape(B)
+        pos = past[:, None] + np.arange(S)[None, :]  # Positions.position_ids
+
+        x = self._w("model.embed_tokens.weight")[ids].astype(np.float64)  # NN.embedding
+        for l in range(c.L):
+            p = f"model.layers.{l}."
+            h = rmsnorm(x, self._w(p + "input_layernorm.weight"), c.eps)
+            bq = self._w(p + "self_attn.q_proj.bias") if c.bias else None
+            bk = self._w(p + "self_attn.k_proj.bias") if c.bias else None
+            bv = self._w(p + "self_attn.v_proj.bias") if c.bias else None
+            q = linear(h, self._w(p + "self_attn.q_proj.weight"), bq).reshape(B, S, c.H, c.d)
+            k = linear(h, self._w(p + "self_attn.k_proj.weight"), bk).reshape(B, S, c.G, c.d)
+            v = linear(h, self._w(p + "self_attn.v_proj.weight"), bv).reshape(B, S, c.G, c.d)
+            q = rope(q, pos[:, :, None], c.theta)
+            k = rope(k, pos[:, :, None], c.theta)
+            o = np.empty((B, S, c.H, c.d))
+            for b in range(B):
+                cache.write(l, b, pos[b], k[b], v[b])
+                Kb, Vb = cache.read(l, b, int(pos[b, -1]) + 1)
+                o[b] = causal_attention(q[b], Kb, Vb, pos[b], c.H, c.G)
+            x = x + linear(o.reshape(B, S, c.H * c.d), self._w(p + "self_attn.o_proj.weight"))
+            h2 = rmsnorm(x, self._w(p + "post_attention_layernorm.weight"), c.eps)
+            u = swiglu(linear(h2, self._w(p + "mlp.gate_proj.weight")),
+                       linear(h2, self._w(p + "mlp.up_proj.weight")))
+            x = x + linear(u, self._w(p + "mlp.down_proj.weight"))
+        if last_hidden_only:
+            x = x[:, -1:, :]
+        head = self._w("model.embed_tokens.weight") if c.tie else self._w("lm_head.weight")
+        return linear(rmsnorm(x, self._w("model.norm.weight"), c.eps), head)
+
+    def prefill(self, ids, cache, last_only=False):
+        """Prompt pass from an empty cache; logits for every position, or for
+        the last one only."""
+        B = np.asarray(ids).shape[0]
+        return self.forward(ids, cache, np.zeros(B, dtype=np.int64), last_hidden_only=last_only)
+
+    def decode_step(self, tokens, cache, context_lens):
+        """One KV-cached decode step: token b enters at position
+        context_lens[b]. Returns logits [B, V]."""
+        tokens = np.asarray(tokens, dtype=np.int64).reshape(-1, 1)
+        return self.forward(tokens, cache, context_lens)[:, 0, :]
+
+    def generate(self, prompt, n_new, cache, forced=None):
+        """Greedy generation: prefill, then n_new - 1 decode steps feeding
+        back the argmax (or, teacher-forced, the given tokens forced[:, t]).
+        Returns (tokens [B, n_new], logits [B, n_new, V])."""
+        prompt = np.asarray(prompt, dtype=np.int64)
+        B, S = prompt.shape
+        logits = [self.prefill(prompt, cache, last_only=True)[:, -1, :]]
+        toks = [argmax_lowest(logits[-1])]
+        lens = np.full(B, S, dtype=np.int64)
+        for t in range(1, n_new):
+            feed = toks[-1] if forced is None else np.asarray(forced)[:, t - 1]
+            logits.append(self.decode_step(feed, cache, lens))
+            toks.append(argmax_lowest(logits[-1]))
+            lens = lens + 1
+        return np.stack(toks, axis=1), np.stack(logits, axis=1)

@@ -1,0 +1,186 @@
+"""Model-level pins for the oracle: a pure-Python loop restatement on tiny
+shapes, the L=0 closed form, causality, KV-cached decode versus full
+recompute, paged versus contiguous caches and batch independence."""
+import math
+
+import numpy as np
+import pytest
+
+import synth_inputs as si
+from oracle import decoder as od
+
+
+def tiny_model(L=2, D=8, H=4, G=2, d=4, F=12, V=16, tie=False, bias=True, theta=100.0, eps=1e-5, seed=0):
+    m = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=bias, theta=theta, eps=eps)
+    w = si.weights_as_f32_numpy(si.make_weights(m, seed=seed))
+    # Large-ish weights so that every term matters at tiny widths.
+    w = {k: (v if k.endswith("layernorm.weight") or k == "model.norm.weight" else v * 20.0)
+         for k, v in w.items()}
+    return od.DecoderConfig.from_dict(m), w
+
+
+# ----------------------------------------------------- brute-force restatement
+def _bf_forward(cfg, W, ids):
+    """Element-by-element restatement with Python loops and the math module:
+    full recompute of every position from scratch, no cache, no numpy
+    vectorisation."""
+    L, D, H, G, d, F, V = cfg.L, cfg.D, cfg.H, cfg.G, cfg.d, cfg.F, cfg.V
+    S = len(ids)
+
+    def rms(vec, g):
+        ms = sum(t * t for t in vec) / len(vec)
+        r = 1.0 / math.sqrt(ms + cfg.eps)
+        return [vec[i] * r * float(g[i]) for i in range(len(vec))]
+
+    def lin(vec, Wm, b=None):
+        out = []
+        for o in range(Wm.shape[0]):
+            acc = 0.0
+            for k in range(Wm.shape[1]):
+                acc += vec[k] * float(Wm[o, k])
+            if b is not None:
+                acc += float(b[o])
+            out.append(acc)
+        return out
+
+    def rot(vec, p):
+        half = d // 2
+        out = [0.0] * d
+        for j in range(half):
+            ang = p * cfg.theta ** (-2.0 * j / d)
+            out[j] = vec[j] * math.cos(ang) - vec[j + half] * math.sin(ang)
+            out[j + half] = vec[j + half] * math.cos(ang) + vec[j] * math.sin(ang)
+        return out
+
+    xs = [[float(W["model.embed_tokens.weight"][t, i]) for i in range(D)] for t in ids]
+    for l in range(L):
+        p = f"model.layers.{l}."
+        qs, ks, vs = [], [], []
+        for s in range(S):
+            h = rms(xs[s], W[p + "input_layernorm.weight"])
+            q = lin(h, W[p + "self_attn.q_proj.weight"], W.get(p + "self_attn.q_proj.bias"))
+            k = lin(h, W[p + "self_attn.k_proj.weight"], W.get(p + "self_attn.k_proj.bias"))
+            v = lin(h, W[p + "self_attn.v_proj.weight"], W.get(p + "self_attn.v_proj.bias"))
+            qs.append([rot(q[hh * d:(hh + 1) * d], s) for hh in range(H)])
+            ks.append([rot(k[g * d:(g + 1) * d], s) for g in range(G)])
+            vs.append([v[g * d:(g + 1) * d] for g in range(G)])
+        new_x = []
+        for s in range(S):
+            o = []
+            for hh in range(H):
+                g = hh * G // H
+                sc = [sum(qs[s][hh][j] * ks[t][g][j] for j in range(d)) / math.sqrt(d) for t in range(s + 1)]
+                mx = max(sc)
+                e = [math.exp(c - mx) for c in sc]
+                z = sum(e)
+                for j in range(d):
+                    o.append(sum(e[t] / z * vs[t][g][j] for t in range(s + 1)))
+            a = lin(o, W[p + "self_attn.o_proj.weight"])
+            x1 = [xs[s][i] + a[i] for i in range(D)]
+            h2 = rms(x1, W[p + "post_attention_layernorm.weight"])
+            gt = lin(h2, W[p + "mlp.gate_proj.weight"])
+            up = lin(h2, W[p + "mlp.up_proj.weight"])
+            u = [gt[i] / (1.0 + math.exp(-gt[i])) * up[i] for i in range(F)]
+            dn = lin(u, W[p + "mlp.down_proj.weight"])
+            new_x.append([x1[i] + dn[i] for i in range(D)])
+        xs = new_x
+    head = W["model.embed_tokens.weight"] if cfg.tie else W["lm_head.weight"]
+    return [lin(rms(x, W["model.norm.weight"]), head) for x in xs]
+
+
+@pytest.mark.parametrize("tie,bias,H,G", [(False, True, 4, 2), (True, False, 2, 2), (False, False, 4, 1)])
+def test_oracle_matches_bruteforce_loops(tie, bias, H, G):
+    cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8)
+    ids = [3, 15, 0, 7, 7]
+    ref = np.array(_bf_forward(cfg, W, ids))
+    o = od.Oracle(cfg, W)
+    got = o.prefill(np.array([ids]), o.new_contiguous_cache(1, 8))[0]
+    assert np.allclose(got, ref, rtol=1e-12, atol=1e-12)
+
+
+# ------------------------------------------------------------- special cases
+def test_zero_layers_is_norm_then_head():
+    cfg, W = tiny_model(L=0)
+    ids = np.array([[1, 4, 9]])
+    o = od.Oracle(cfg, W)
+    got = o.prefill(ids, o.new_contiguous_cache(1, 4))
+    E = W["model.embed_tokens.weight"].astype(np.float64)
+    x = E[ids[0]]
+    r = 1.0 / np.sqrt(np.mean(x * x, -1, keepdims=True) + cfg.eps)
+    want = (x * r * W["model.norm.weight"]) @ W["lm_head.weight"].astype(np.float64).T
+    assert np.allclose(got[0], want, rtol=1e-13, atol=1e-13)
+    # Tied head reads the embedding matrix.
+    cfg_t, W_t = tiny_model(L=0, tie=True)
+    ot = od.Oracle(cfg_t, W_t)
+    got_t = ot.prefill(ids, ot.new_contiguous_cache(1, 4))
+    Et = W_t["model.embed_tokens.weight"].astype(np.float64)
+    xt = Et[ids[0]]
+    rt = 1.0 / np.sqrt(np.mean(xt * xt, -1, keepdims=True) + cfg_t.eps)
+    assert np.allclose(got_t[0], (xt * rt * W_t["model.norm.weight"]) @ Et.T, rtol=1e-13, atol=1e-13)
+
+
+# ---------------------------------------------------------------- invariants
+def test_appending_tokens_leaves_earlier_logits_unchanged():
+    cfg, W = tiny_model()
+    o = od.Oracle(cfg, W)
+    ids = np.array([[5, 1, 2, 11, 3, 8]])
+    full = o.prefill(ids, o.new_contiguous_cache(1, 8))
+    for k in (1, 3, 5):
+        part = o.prefill(ids[:, :k], o.new_contiguous_cache(1, 8))
+        assert np.allclose(part, full[:, :k], rtol=1e-12, atol=1e-12)
+
+
+def test_incremental_decode_equals_full_recompute():
+    cfg, W = tiny_model()
+    o = od.Oracle(cfg, W)
+    ids = np.array([[5, 1, 2, 11, 3, 8, 0, 14], [2, 2, 9, 4, 1, 1, 7, 6]])
+    full = o.prefill(ids, o.new_contiguous_cache(2, 8))
+    cache = o.new_contiguous_cache(2, 8)
+    o.prefill(ids[:, :3], cache)
+    for t in range(3, 8):
+        step = o.decode_step(ids[:, t], cache, np.array([t, t]))
+        assert np.allclose(step, full[:, t], rtol=1e-12, atol=1e-12)
+
+
+def test_paged_cache_is_bit_identical_to_contiguous():
+    cfg, W = tiny_model()
+    o = od.Oracle(cfg, W)
+    B, S, bs = 2, 7, 2
+    ids = np.array([[5, 1, 2, 11, 3, 8, 0], [2, 2, 9, 4, 1, 1, 7]])
+    bt = si.make_block_table([S + 3, S + 3], bs, 6, 12, seed=3)
+    c_cont = o.new_contiguous_cache(B, 12)
+    c_page = o.new_paged_cache(12, bs, bt)
+    a = o.prefill(ids, c_cont)
+    b = o.prefill(ids, c_page)
+    assert np.array_equal(a, b)
+    lens = np.array([S, S])
+    for t in range(3):
+        tok = od.argmax_lowest(a[:, -1] if t == 0 else sa)
+        sa = o.decode_step(tok, c_cont, lens)
+        sb = o.decode_step(tok, c_page, lens)
+        assert np.array_equal(sa, sb)
+        lens = lens + 1
+    # Cache contents sit at the slots the block table names.
+    for b_ in range(B):
+        for p in range(S + 3):
+            blk, off = od.slot_of(bt, b_, p, bs)
+            assert np.array_equal(c_page.K[1][blk, off], c_cont.K[1][b_, p])
+
+
+def test_batch_rows_are_independent():
+    cfg, W = tiny_model()
+    o = od.Oracle(cfg, W)
+    ids = np.array([[5, 1, 2, 11], [2, 2, 9, 4], [0, 13, 13, 1]])
+    both = o.prefill(ids, o.new_contiguous_cache(3, 4))
+    for b in range(3):
+        one = o.prefill(ids[b:b + 1], o.new_contiguous_cache(1, 4))
+        assert np.allclose(one[0], both[b], rtol=1e-13, atol=1e-13)
+
+
+def test_generate_teacher_forced_matches_free_running_when_forced_on_own_tokens():
+    cfg, W = tiny_model()
+    o = od.Oracle(cfg, W)
+    ids = np.array([[5, 1, 2]])
+    toks, logits = o.generate(ids, 4, o.new_contiguous_cache(1, 8))
+    toks2, logits2 = o.generate(ids, 4, o.new_contiguous_cache(1, 8), forced=toks)
+    assert np.array_equal(toks, toks2) and np.allclose(logits, logits2, rtol=1e-14, atol=1e-14)
