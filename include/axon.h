@@ -1,0 +1,192 @@
+/*
+ * axon.h -- C ABI of the GB300 (sm_103a) Llama-family decoder forward.
+ *
+ * The operation behind these calls is the forward pass that the Axon paper
+ * (arxiv 2608.19889) compiles to its backends: a model definition plus a
+ * safetensors checkpoint go in (Fig. 1; Sec. "The Axon Compiler", Phase 3:
+ * backends implement `forward` and `generate` with static-cache scaffolding),
+ * logits and greedy next tokens come out (Sec. "Results", Measures). The
+ * per-layer math is the pre-norm block of Sec. "The Axon Language" (RMSNorm,
+ * grouped-query causal attention with rotary positions and a KV cache,
+ * residual add, SwiGLU MLP) built from the library of Sec. "Built-In
+ * Libraries"; the model skeleton follows the appendix causal_lm listing
+ * (embedding, layer loop threading the cache, final norm, tied or untied
+ * LM head).
+ *
+ * Conventions for every call
+ *   - Return value: AXON_OK (0) or one AXON_ERR_* code. Nothing aborts or
+ *     throws across the ABI. axon_status_string() names a code.
+ *   - Pointers named d_* are DEVICE pointers (CUDA global memory of the
+ *     device current when the model was created). The caller owns them.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL =
+ *     the legacy default stream). Argument errors are reported
+ *     synchronously; device-side range checks (token ids, block-table
+ *     entries, positions) set a device error word that
+ *     axon_check_device() reads, and the offending access is skipped.
+ *   - Token ids, context lengths and block tables are int32.
+ *   - Floating point: weights bf16 (or fp32 widened in AXON_FP32_DEBUG),
+ *     fp32 accumulation everywhere, fp32 residual stream and logits.
+ */
+#ifndef AXON_H
+#define AXON_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+enum {
+  AXON_OK = 0,
+  AXON_ERR_INVALID_ARG = 1,    /* null pointer, bad enum, B or S out of range */
+  AXON_ERR_SHAPE_MISMATCH = 2, /* a weight's shape disagrees with the config */
+  AXON_ERR_MISSING_WEIGHT = 3, /* a required weight name is absent */
+  AXON_ERR_UNSUPPORTED = 4,    /* config outside what the kernels implement */
+  AXON_ERR_OOM = 5,            /* device allocation failed */
+  AXON_ERR_CUDA = 6,           /* a CUDA runtime call failed */
+  AXON_ERR_TIMEOUT = 7,        /* a bounded device wait expired */
+  AXON_ERR_DEVICE_CHECK = 8    /* a device-side range check fired */
+};
+
+/* KV cache layouts (Sec. Built-In Libraries: a static, preallocated cache
+ * overlay; vLLM's PagedAttention manager, Sec. Related Work). */
+enum { AXON_KV_CONTIGUOUS = 0, AXON_KV_PAGED = 1 };
+
+/* Arithmetic mode: bf16 weights/activations with fp32 accumulation, or an
+ * all-fp32 debug mode (Sec. Results: bf16 primary, fp32 fallback). */
+enum { AXON_BF16 = 0, AXON_FP32_DEBUG = 1 };
+
+/* Element types of weight tensors handed to axon_model_create. */
+enum { AXON_DTYPE_BF16 = 0, AXON_DTYPE_F32 = 1 };
+
+/* Which positions of a prefill get logits written. */
+enum { AXON_LOGITS_LAST = 0, AXON_LOGITS_ALL = 1 };
+
+/* Model configuration: HF config.json equivalents (the appendix causal_lm
+ * listing reads hidden size, layer and head counts and vocabulary size
+ * through `Config.dim @@key`), plus capacity and layout fields. */
+typedef struct axon_config {
+  int32_t num_hidden_layers;   /* L */
+  int32_t hidden_size;         /* D, multiple of 64 */
+  int32_t num_attention_heads; /* H, multiple of num_key_value_heads */
+  int32_t num_key_value_heads; /* G */
+  int32_t head_dim;            /* d: 64 or 128 */
+  int32_t intermediate_size;   /* F, multiple of 64 */
+  int32_t vocab_size;          /* V */
+  int32_t tie_word_embeddings; /* 1: LM head = embedding matrix */
+  int32_t attention_bias;      /* 1: q, k, v projections carry biases */
+  float rope_theta;            /* rotary base */
+  float rms_norm_eps;          /* RMSNorm epsilon */
+  int32_t max_batch;           /* sequences (contiguous cache slots) */
+  int32_t max_context;         /* tokens per sequence, multiple of 16 */
+  int32_t max_prefill_tokens;  /* largest B*S per axon_prefill; 0 = max_batch*max_context */
+  int32_t kv_layout;           /* AXON_KV_CONTIGUOUS or AXON_KV_PAGED */
+  int32_t kv_block_size;       /* tokens per block: must be 16 */
+  int32_t kv_num_blocks;       /* paged pool size in blocks (ignored if contiguous) */
+  int32_t precision;           /* AXON_BF16 or AXON_FP32_DEBUG */
+} axon_config;
+
+/* One named checkpoint tensor, HF Llama naming and [out, in] matrices, as a
+ * safetensors file stores them (Fig. 1; weights looked up by flat dotted
+ * path, appendix "Python Overhead"):
+ *   model.embed_tokens.weight                       [V, D]
+ *   model.layers.{i}.input_layernorm.weight         [D]
+ *   model.layers.{i}.self_attn.{q,k,v}_proj.weight  [H*d | G*d | G*d, D]
+ *   model.layers.{i}.self_attn.{q,k,v}_proj.bias    (if attention_bias)
+ *   model.layers.{i}.self_attn.o_proj.weight        [D, H*d]
+ *   model.layers.{i}.post_attention_layernorm.weight[D]
+ *   model.layers.{i}.mlp.{gate,up}_proj.weight      [F, D]
+ *   model.layers.{i}.mlp.down_proj.weight           [D, F]
+ *   model.norm.weight                               [D]
+ *   lm_head.weight                                  [V, D] (absent if tied)
+ * `data` may be a host or a device pointer (unified addressing); it is
+ * only read during axon_model_create. Row-major, contiguous. */
+typedef struct axon_tensor {
+  const char* name;
+  const void* data;
+  int32_t dtype; /* AXON_DTYPE_BF16 or AXON_DTYPE_F32 */
+  int32_t ndim;  /* 1 or 2 */
+  int64_t shape[4];
+} axon_tensor;
+
+typedef struct axon_model axon_model;
+
+/* Build a model: validate the config against the named weights (symbolic
+ * dimensions, Sec. The Axon Language, Types), allocate and repack weights
+ * into the kernels' layout (fused QKV, interleaved gate/up), allocate the KV
+ * cache and workspace. The weight table is copied; the caller may free it
+ * on return. Work is done on `stream` and synchronised before returning.
+ * *out receives the model, or NULL on error. */
+int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_t n_weights,
+                      void* stream, axon_model** out);
+
+/* Prompt pass (Positions.position_ids with past_length 0; Cache.update of
+ * every prompt token; Sec. Built-In Libraries).
+ *   d_ids          [B, S] token ids.
+ *   B              1 .. max_batch; sequence b uses contiguous slot b, or the
+ *                  blocks named by row b of d_block_table.
+ *   S              1 .. max_context, B*S <= max_prefill_tokens.
+ *   d_block_table  paged layout: [B, ceil(max_context/16)] pool block ids,
+ *                  row b for sequence b (entries past the prompt unused);
+ *                  must be NULL for the contiguous layout.
+ *   logits_mode    AXON_LOGITS_LAST: d_logits is [B, V], the last position;
+ *                  AXON_LOGITS_ALL: d_logits is [B, S, V].
+ *   d_logits       fp32 output, or NULL to skip storing logits.
+ *   d_next         [B] greedy next token (argmax of the last position's
+ *                  logits, lowest index on ties), or NULL.
+ * Previous contents of the used cache slots are overwritten. */
+int axon_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S,
+                 const int32_t* d_block_table, int32_t logits_mode, float* d_logits,
+                 int32_t* d_next, void* stream);
+
+/* One KV-cached greedy decode step for B sequences (generate loop, Sec.
+ * Results; Cache.append in the appendix causal_lm listing).
+ *   d_tokens        [B] the newest token of each sequence.
+ *   d_context_lens  [B] IN/OUT: tokens already cached for sequence b; the
+ *                   new token takes position context_lens[b]. The step adds
+ *                   1 to every entry (in stream order, after all reads), so
+ *                   consecutive steps can be replayed without host work.
+ *   d_block_table   paged layout: [B, ceil(max_context/16)], else NULL.
+ *   d_logits        [B, V] fp32 output, or NULL.
+ *   d_next          [B] greedy next token; may alias d_tokens.
+ * The step's launches are recorded once per (B, pointer set) into a CUDA
+ * graph and replayed afterwards (set AXON_NO_GRAPH=1 to launch directly). */
+int axon_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,
+                     const int32_t* d_block_table, float* d_logits, int32_t* d_next, void* stream);
+
+/* Forget cached sequences: zero the KV cache and clear the device error
+ * word. Synchronous. */
+int axon_reset(axon_model* m);
+
+/* Synchronise `stream` and read the device error word. Returns AXON_OK,
+ * AXON_ERR_DEVICE_CHECK (a range check fired) or AXON_ERR_TIMEOUT (a
+ * bounded wait expired). *bits (optional) receives the raw word; the word
+ * is cleared. */
+int axon_check_device(axon_model* m, void* stream, int32_t* bits);
+
+/* Read-only view of the KV pools for inspection (tests check cache
+ * placement through it). Layout of either pool: [L][num_blocks][G][16][d],
+ * element type bf16 (fp32 in AXON_FP32_DEBUG). In the contiguous layout,
+ * sequence b's logical block j is pool block b*blocks_per_seq + j. */
+typedef struct axon_kv_view {
+  void* k_pool;
+  void* v_pool;
+  int64_t num_blocks;
+  int32_t blocks_per_seq;
+  int32_t block_size;
+  int32_t elem_bytes;
+} axon_kv_view;
+int axon_kv_view_get(const axon_model* m, axon_kv_view* out);
+
+/* Release everything the model owns. NULL is a no-op. */
+void axon_free(axon_model* m);
+
+/* Static string naming a status code. */
+const char* axon_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AXON_H */

@@ -1,0 +1,835 @@
+// C ABI of the decoder forward: model creation (config validation, weight
+// repack, KV cache and workspace), prefill and decode launch plans, and the
+// per-(B, pointer set) CUDA-graph cache of the decode step.
+//
+// The launch plans are the layer loop of the paper's causal_lm listing
+// (`for@h i <- [0..NUM_LAYERS) carry (x, work_kv)`), with every block of the
+// pre-norm layer turned into one fused kernel:
+//   QKV projection (+norm scale, bias, RoPE, KV store) -> attention ->
+//   O projection (+residual, next norm's operand) -> gate/up (+SwiGLU) ->
+//   down projection (+residual, next norm's operand),
+// then final norm + LM head (+argmax) and the greedy-token finaliser.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "../../include/axon.h"
+#include "kernels.h"
+
+namespace {
+
+struct LayerW {
+  void* wqkv = nullptr;
+  float* bqkv = nullptr;
+  void* wo = nullptr;
+  void* wgu = nullptr;
+  void* wd = nullptr;
+  float* g1 = nullptr;
+  float* g2 = nullptr;
+  GemmMaps m_qkv{}, m_o{}, m_gu{}, m_d{};
+};
+
+using GraphKey = std::tuple<int, const void*, const void*, const void*, const void*, const void*>;
+
+bool env_flag(const char* name) {
+  const char* v = getenv(name);
+  return v && v[0] && v[0] != '0';
+}
+
+}  // namespace
+
+struct axon_model {
+  axon_config cfg{};
+  int L = 0, D = 0, H = 0, G = 0, d = 0, F = 0, V = 0, Nqkv = 0;
+  bool fp32 = false;
+  size_t esz = 2;
+  int device = 0;
+  int num_sms = 148;
+  // weights
+  std::vector<void*> allocs;
+  void* embed = nullptr;
+  void* head = nullptr;
+  float* gf = nullptr;
+  std::vector<LayerW> layers;
+  GemmMaps m_head{};
+  // KV cache
+  void* kpool = nullptr;
+  void* vpool = nullptr;
+  long long num_blocks = 0;
+  int blocks_per_seq = 0;
+  size_t layer_kv_elems = 0;
+  float2* rope = nullptr;
+  // workspace
+  int Mcap = 0;
+  int Pmax = 0;
+  float* x = nullptr;
+  void* a = nullptr;
+  float* ss = nullptr;
+  void* q = nullptr;
+  void* o = nullptr;
+  void* u = nullptr;
+  unsigned long long* keys = nullptr;
+  float* rinv = nullptr;   // [Mcap] per-row inverse RMS from decode producers
+  int* ticket = nullptr;   // last-CTA counter of the residual producers
+  float* attn_part = nullptr;
+  int* attn_cnt = nullptr;
+  int max_splits = 1;
+  int* err = nullptr;
+  CUtensorMap t_a{}, t_o{}, t_u{};
+  // decode graphs
+  cudaStream_t cap_stream = nullptr;
+  std::map<GraphKey, cudaGraphExec_t> graphs;
+  bool use_graphs = true;
+  bool use_pdl = true;
+};
+
+namespace {
+
+#define CK(call)                                                                    \
+  do {                                                                              \
+    cudaError_t e_ = (call);                                                        \
+    if (e_ != cudaSuccess) {                                                        \
+      if (env_flag("AXON_DEBUG"))                                                   \
+        fprintf(stderr, "axon: %s failed: %s (%s:%d)\n", #call, cudaGetErrorString(e_), __FILE__, __LINE__); \
+      return AXON_ERR_CUDA;                                                         \
+    }                                                                               \
+  } while (0)
+
+int dev_alloc(axon_model* m, void** p, size_t bytes) {
+  if (bytes == 0) bytes = 16;
+  if (cudaMalloc(p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    *p = nullptr;
+    return AXON_ERR_OOM;
+  }
+  m->allocs.push_back(*p);
+  return AXON_OK;
+}
+
+// dst[p][:] = src[rowmap[p]][:] with dtype conversion (bf16/f32 -> bf16/f32).
+__global__ void gather_rows_kernel(void* dst, int dst_f32, const void* src, int src_f32, const int* rowmap, int rows,
+                                   int cols) {
+  const int p = blockIdx.x;
+  if (p >= rows) return;
+  const long long sr = rowmap ? rowmap[p] : p;
+  for (int c = threadIdx.x; c < cols; c += blockDim.x) {
+    const float v = src_f32 ? static_cast<const float*>(src)[sr * cols + c]
+                            : __bfloat162float(static_cast<const bf16*>(src)[sr * cols + c]);
+    if (dst_f32)
+      static_cast<float*>(dst)[static_cast<long long>(p) * cols + c] = v;
+    else
+      static_cast<bf16*>(dst)[static_cast<long long>(p) * cols + c] = __float2bfloat16_rn(v);
+  }
+}
+
+struct Builder {
+  axon_model* m;
+  const axon_tensor* w;
+  int n;
+  cudaStream_t st;
+  void* staging = nullptr;
+  size_t staging_bytes = 0;
+  int* d_rowmap = nullptr;
+  size_t rowmap_cap = 0;
+
+  const axon_tensor* find(const std::string& name) const {
+    for (int i = 0; i < n; ++i)
+      if (w[i].name && name == w[i].name) return &w[i];
+    return nullptr;
+  }
+  int check(const axon_tensor* t, int64_t d0, int64_t d1) const {
+    if (!t) return AXON_ERR_MISSING_WEIGHT;
+    if (!t->data || (t->dtype != AXON_DTYPE_BF16 && t->dtype != AXON_DTYPE_F32)) return AXON_ERR_INVALID_ARG;
+    if (d1 < 0) {
+      if (t->ndim != 1 || t->shape[0] != d0) return AXON_ERR_SHAPE_MISMATCH;
+    } else {
+      if (t->ndim != 2 || t->shape[0] != d0 || t->shape[1] != d1) return AXON_ERR_SHAPE_MISMATCH;
+    }
+    return AXON_OK;
+  }
+  // Copy a checkpoint tensor (host or device) into device staging.
+  int stage(const axon_tensor* t, size_t elems) {
+    const size_t bytes = elems * (t->dtype == AXON_DTYPE_F32 ? 4 : 2);
+    if (bytes > staging_bytes) {
+      if (staging) cudaFree(staging);
+      staging = nullptr;
+      if (cudaMalloc(&staging, bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return AXON_ERR_OOM;
+      }
+      staging_bytes = bytes;
+    }
+    CK(cudaMemcpyAsync(staging, t->data, bytes, cudaMemcpyDefault, st));
+    return AXON_OK;
+  }
+  int gather(void* dst, bool dst_f32, const axon_tensor* t, const std::vector<int>* rowmap, int rows, int cols) {
+    int rc = stage(t, static_cast<size_t>(t->ndim == 2 ? t->shape[0] : 1) * cols);
+    if (rc) return rc;
+    const int* dm = nullptr;
+    if (rowmap) {
+      if (rowmap->size() > rowmap_cap) {
+        if (d_rowmap) cudaFree(d_rowmap);
+        if (cudaMalloc(&d_rowmap, rowmap->size() * sizeof(int)) != cudaSuccess) {
+          cudaGetLastError();
+          return AXON_ERR_OOM;
+        }
+        rowmap_cap = rowmap->size();
+      }
+      CK(cudaMemcpyAsync(d_rowmap, rowmap->data(), rowmap->size() * sizeof(int), cudaMemcpyHostToDevice, st));
+      dm = d_rowmap;
+    }
+    gather_rows_kernel<<<rows, 256, 0, st>>>(dst, dst_f32 ? 1 : 0, staging, t->dtype == AXON_DTYPE_F32 ? 1 : 0, dm,
+                                             rows, cols);
+    CK(cudaGetLastError());
+    // staging and rowmap are reused by the next call
+    CK(cudaStreamSynchronize(st));
+    return AXON_OK;
+  }
+  ~Builder() {
+    if (staging) cudaFree(staging);
+    if (d_rowmap) cudaFree(d_rowmap);
+  }
+};
+
+int validate_config(const axon_config* c) {
+  if (c->num_hidden_layers < 0 || c->hidden_size <= 0 || c->num_attention_heads <= 0 ||
+      c->num_key_value_heads <= 0 || c->intermediate_size <= 0 || c->vocab_size <= 0 || c->max_batch <= 0 ||
+      c->max_context <= 0)
+    return AXON_ERR_INVALID_ARG;
+  if (c->kv_layout != AXON_KV_CONTIGUOUS && c->kv_layout != AXON_KV_PAGED) return AXON_ERR_INVALID_ARG;
+  if (c->precision != AXON_BF16 && c->precision != AXON_FP32_DEBUG) return AXON_ERR_INVALID_ARG;
+  if (c->kv_block_size != 16) return AXON_ERR_UNSUPPORTED;
+  if (c->kv_layout == AXON_KV_PAGED && c->kv_num_blocks <= 0) return AXON_ERR_INVALID_ARG;
+  if (c->num_attention_heads % c->num_key_value_heads) return AXON_ERR_UNSUPPORTED;
+  if (c->num_attention_heads / c->num_key_value_heads > 16) return AXON_ERR_UNSUPPORTED;
+  if (c->head_dim != 64 && c->head_dim != 128) return AXON_ERR_UNSUPPORTED;
+  if (c->hidden_size % 64 || c->intermediate_size % 64 || (c->num_attention_heads * c->head_dim) % 64)
+    return AXON_ERR_UNSUPPORTED;
+  if (c->max_context % 16) return AXON_ERR_UNSUPPORTED;
+  if (c->max_batch > 64 && c->max_prefill_tokens == 0) return AXON_ERR_UNSUPPORTED;
+  return AXON_OK;
+}
+
+// Packed row p of one head (QKV): chunk c = p / 16 holds natural dims
+// c*8 + i (slots 0..7) and c*8 + i + d/2 (slots 8..15).
+int qkv_natural(int p, int d) {
+  const int c = p >> 4, i = p & 15;
+  return i < 8 ? c * 8 + i : c * 8 + (i - 8) + d / 2;
+}
+
+void kv_layout_args(const axon_model* m, int layer, const int* block_table, EpiArgs& e) {
+  e.k_cache = static_cast<char*>(m->kpool) + static_cast<size_t>(layer) * m->layer_kv_elems * m->esz;
+  e.v_cache = static_cast<char*>(m->vpool) + static_cast<size_t>(layer) * m->layer_kv_elems * m->esz;
+  e.block_table = block_table;
+  e.bt_stride = m->blocks_per_seq;
+  e.blocks_per_seq = m->blocks_per_seq;
+  e.num_blocks = static_cast<int>(m->num_blocks);
+}
+
+EpiArgs base_epi(const axon_model* m) {
+  EpiArgs e;
+  memset(&e, 0, sizeof(e));
+  e.max_pos = m->cfg.max_context;
+  e.inv_D = 1.0f / static_cast<float>(m->D);
+  e.eps = m->cfg.rms_norm_eps;
+  e.H = m->H;
+  e.G = m->G;
+  e.d = m->d;
+  e.rope = m->rope;
+  e.err = m->err;
+  return e;
+}
+
+AttnArgs base_attn(const axon_model* m, int layer, const int* block_table) {
+  AttnArgs a;
+  memset(&a, 0, sizeof(a));
+  a.q = m->q;
+  a.o = m->o;
+  a.k = static_cast<char*>(m->kpool) + static_cast<size_t>(layer) * m->layer_kv_elems * m->esz;
+  a.v = static_cast<char*>(m->vpool) + static_cast<size_t>(layer) * m->layer_kv_elems * m->esz;
+  a.block_table = block_table;
+  a.bt_stride = m->blocks_per_seq;
+  a.blocks_per_seq = m->blocks_per_seq;
+  a.num_blocks = static_cast<int>(m->num_blocks);
+  a.H = m->H;
+  a.G = m->G;
+  a.d = m->d;
+  a.scale_log2 = static_cast<float>(1.0 / std::sqrt(static_cast<double>(m->d)) * 1.4426950408889634);
+  a.err = m->err;
+  return a;
+}
+
+// Which form the next norm's scale is available in after a producer: the
+// reduced per-row inverse RMS (`rinv` buffer) or `parts` partial sums of
+// squares per row in `ss`.
+struct NormState {
+  bool rinv = false;
+  int parts = 1;
+};
+
+void set_norm(const axon_model* m, const NormState& ns, EpiArgs& e, int row_offset = 0, int row_stride = 1) {
+  if (ns.rinv) {
+    e.rinv = m->rinv + row_offset;
+    e.rinv_stride = row_stride;
+  } else {
+    e.ss = m->ss + static_cast<size_t>(row_offset) * m->Pmax;
+    e.ss_stride = row_stride * m->Pmax;
+    e.ss_parts = ns.parts;
+  }
+}
+
+// One projection: picks the kernel for the mode and row count.
+struct Proj {
+  const axon_model* m;
+  LaunchCtx lc;
+  cudaError_t rc = cudaSuccess;
+  // act: activation rows (row stride act_stride elements), M rows. Returns
+  // the norm state a RESID producer leaves behind.
+  NormState run(int kind, const void* W, const GemmMaps* maps, int N, int K, const void* act, long long act_stride,
+                int M, EpiArgs& ep) {
+    ep.M = M;
+    ep.N = N;
+    NormState ns;
+    const bool gemv = M <= 64 || (!m->fp32 && maps == nullptr);
+    if (gemv && kind == EPI_RESID) {
+      ep.rinv_out = m->rinv;
+      ep.ticket = m->ticket;
+      ns.rinv = true;
+    }
+    if (gemv) {
+      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep);
+      ns.parts = N / 16;
+    } else if (m->fp32) {
+      rc = launch_gemm_simt(lc, kind, static_cast<const float*>(act), act_stride, static_cast<const float*>(W), M, N,
+                            K, ep);
+      ns.parts = N / 16;
+    } else {
+      rc = launch_gemm_tc(lc, kind, *maps, M, N, K, ep);
+      ns.parts = (N + 255) / 256;
+    }
+    return ns;
+  }
+};
+
+int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32_t* bt, int logits_mode, float* logits,
+                    int32_t* next, cudaStream_t st) {
+  const int M = B * S;
+  LaunchCtx lc{st, m->use_pdl, m->num_sms};
+  Proj pj{m, lc};
+  const int D = m->D, Hd = m->H * m->d;
+  CK(launch_embed(lc, m->fp32, m->embed, m->V, D, ids, M, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
+                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err));
+  NormState ns;
+  ns.rinv = true;
+  for (int l = 0; l < m->L; ++l) {
+    const LayerW& w = m->layers[l];
+    EpiArgs e = base_epi(m);
+    e.S = S;
+    set_norm(m, ns, e);
+    e.bias = w.bqkv;
+    e.q_out = m->q;
+    kv_layout_args(m, l, bt, e);
+    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, M, e);
+    CK(pj.rc);
+
+    AttnArgs at = base_attn(m, l, bt);
+    at.S = S;
+    CK(launch_attn_prefill(lc, m->fp32, at, B));
+
+    EpiArgs r = base_epi(m);
+    r.S = S;
+    r.x = m->x;
+    r.a_out = m->a;
+    r.gain = w.g2;
+    r.ss_out = m->ss;
+    r.ss_out_stride = m->Pmax;
+    ns = pj.run(EPI_RESID, w.wo, &w.m_o, D, Hd, m->o, Hd, M, r);
+    CK(pj.rc);
+
+    EpiArgs g = base_epi(m);
+    g.S = S;
+    set_norm(m, ns, g);
+    g.u_out = m->u;
+    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, M, g);
+    CK(pj.rc);
+
+    EpiArgs dn = base_epi(m);
+    dn.S = S;
+    dn.x = m->x;
+    dn.a_out = m->a;
+    dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
+    dn.ss_out = m->ss;
+    dn.ss_out_stride = m->Pmax;
+    ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, M, dn);
+    CK(pj.rc);
+  }
+  EpiArgs h = base_epi(m);
+  h.S = S;
+  h.keys = m->keys;
+  h.logits = logits;
+  h.logits_stride = m->V;
+  if (logits_mode == AXON_LOGITS_ALL) {
+    set_norm(m, ns, h);
+    pj.run(EPI_LOGITS, m->head, &m->m_head, m->V, D, m->a, D, M, h);
+    CK(pj.rc);
+    CK(launch_finalize(lc, m->keys, M, S, S - 1, B, next, nullptr));
+  } else {
+    // Last position of each sequence: rows S-1, 2S-1, ... as a B-row GEMV.
+    const size_t off = static_cast<size_t>(S - 1) * D * m->esz;
+    set_norm(m, ns, h, S - 1, S);
+    h.M = B;
+    h.N = m->V;
+    CK(launch_gemv(lc, EPI_LOGITS, m->fp32, m->head, m->V, D, static_cast<char*>(m->a) + off,
+                   static_cast<long long>(S) * D, B, h));
+    CK(launch_finalize(lc, m->keys, B, 1, 0, B, next, nullptr));
+  }
+  return AXON_OK;
+}
+
+int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt, float* logits,
+                   int32_t* next, cudaStream_t st) {
+  LaunchCtx lc{st, m->use_pdl, m->num_sms};
+  Proj pj{m, lc};
+  const int D = m->D, Hd = m->H * m->d;
+  CK(launch_embed(lc, m->fp32, m->embed, m->V, D, tokens, B, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
+                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err));
+  NormState ns;
+  ns.rinv = true;
+  const int splits = m->fp32 ? 1 : attn_decode_splits(B, m->G, m->blocks_per_seq, m->num_sms);
+  for (int l = 0; l < m->L; ++l) {
+    const LayerW& w = m->layers[l];
+    EpiArgs e = base_epi(m);
+    e.S = 1;
+    e.ctx = ctx;
+    set_norm(m, ns, e);
+    e.bias = w.bqkv;
+    e.q_out = m->q;
+    kv_layout_args(m, l, bt, e);
+    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e);
+    CK(pj.rc);
+
+    AttnArgs at = base_attn(m, l, bt);
+    at.ctx = ctx;
+    at.S = 1;
+    at.splits = splits;
+    at.part = m->attn_part;
+    at.counter = m->attn_cnt;
+    CK(launch_attn_decode(lc, m->fp32, at, B));
+
+    EpiArgs r = base_epi(m);
+    r.S = 1;
+    r.ctx = ctx;
+    r.x = m->x;
+    r.a_out = m->a;
+    r.gain = w.g2;
+    r.ss_out = m->ss;
+    r.ss_out_stride = m->Pmax;
+    ns = pj.run(EPI_RESID, w.wo, nullptr, D, Hd, m->o, Hd, B, r);
+    CK(pj.rc);
+
+    EpiArgs g = base_epi(m);
+    g.S = 1;
+    g.ctx = ctx;
+    set_norm(m, ns, g);
+    g.u_out = m->u;
+    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g);
+    CK(pj.rc);
+
+    EpiArgs dn = base_epi(m);
+    dn.S = 1;
+    dn.ctx = ctx;
+    dn.x = m->x;
+    dn.a_out = m->a;
+    dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
+    dn.ss_out = m->ss;
+    dn.ss_out_stride = m->Pmax;
+    ns = pj.run(EPI_RESID, w.wd, nullptr, D, m->F, m->u, m->F, B, dn);
+    CK(pj.rc);
+  }
+  EpiArgs h = base_epi(m);
+  h.S = 1;
+  h.ctx = ctx;
+  set_norm(m, ns, h);
+  h.keys = m->keys;
+  h.logits = logits;
+  h.logits_stride = m->V;
+  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h);
+  CK(pj.rc);
+  CK(launch_finalize(lc, m->keys, B, 1, 0, B, next, ctx));
+  return AXON_OK;
+}
+
+void free_model(axon_model* m) {
+  if (!m) return;
+  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+  m->graphs.clear();
+  if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
+  for (void* p : m->allocs) cudaFree(p);
+  delete m;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* axon_status_string(int status) {
+  switch (status) {
+    case AXON_OK: return "ok";
+    case AXON_ERR_INVALID_ARG: return "invalid argument";
+    case AXON_ERR_SHAPE_MISMATCH: return "weight shape does not match the config";
+    case AXON_ERR_MISSING_WEIGHT: return "required weight missing";
+    case AXON_ERR_UNSUPPORTED: return "configuration not supported by the kernels";
+    case AXON_ERR_OOM: return "device out of memory";
+    case AXON_ERR_CUDA: return "CUDA runtime error";
+    case AXON_ERR_TIMEOUT: return "bounded device wait expired";
+    case AXON_ERR_DEVICE_CHECK: return "device-side range check failed";
+    default: return "unknown status";
+  }
+}
+
+int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_t n_weights, void* stream,
+                      axon_model** out) {
+  if (!out) return AXON_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg || (!weights && n_weights > 0) || n_weights < 0) return AXON_ERR_INVALID_ARG;
+  int rc = validate_config(cfg);
+  if (rc) return rc;
+  axon_model* m = new axon_model();
+  m->cfg = *cfg;
+  if (m->cfg.max_prefill_tokens <= 0) m->cfg.max_prefill_tokens = cfg->max_batch * cfg->max_context;
+  m->L = cfg->num_hidden_layers;
+  m->D = cfg->hidden_size;
+  m->H = cfg->num_attention_heads;
+  m->G = cfg->num_key_value_heads;
+  m->d = cfg->head_dim;
+  m->F = cfg->intermediate_size;
+  m->V = cfg->vocab_size;
+  m->Nqkv = (m->H + 2 * m->G) * m->d;
+  m->fp32 = cfg->precision == AXON_FP32_DEBUG;
+  m->esz = m->fp32 ? 4 : 2;
+  m->use_graphs = !env_flag("AXON_NO_GRAPH");
+  m->use_pdl = !env_flag("AXON_NO_PDL");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  auto fail = [&](int code) {
+    cudaStreamSynchronize(st);
+    free_model(m);
+    return code;
+  };
+  if (cudaGetDevice(&m->device) != cudaSuccess) return fail(AXON_ERR_CUDA);
+  cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
+  int major = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, m->device);
+  if (major < 10) return fail(AXON_ERR_UNSUPPORTED);
+  if (prepare_attn_kernels() != cudaSuccess || prepare_gemm_kernels() != cudaSuccess) return fail(AXON_ERR_CUDA);
+
+  Builder bl{m, weights, n_weights, st};
+  const int D = m->D, Hd = m->H * m->d, Gd = m->G * m->d, F = m->F, V = m->V;
+  // ---- validate every name and shape before allocating
+  if ((rc = bl.check(bl.find("model.embed_tokens.weight"), V, D))) return fail(rc);
+  if ((rc = bl.check(bl.find("model.norm.weight"), D, -1))) return fail(rc);
+  if (!cfg->tie_word_embeddings && (rc = bl.check(bl.find("lm_head.weight"), V, D))) return fail(rc);
+  for (int l = 0; l < m->L; ++l) {
+    const std::string p = "model.layers." + std::to_string(l) + ".";
+    if ((rc = bl.check(bl.find(p + "input_layernorm.weight"), D, -1))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "post_attention_layernorm.weight"), D, -1))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "self_attn.q_proj.weight"), Hd, D))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "self_attn.k_proj.weight"), Gd, D))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "self_attn.v_proj.weight"), Gd, D))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "self_attn.o_proj.weight"), D, Hd))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "mlp.gate_proj.weight"), F, D))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "mlp.up_proj.weight"), F, D))) return fail(rc);
+    if ((rc = bl.check(bl.find(p + "mlp.down_proj.weight"), D, F))) return fail(rc);
+    if (cfg->attention_bias) {
+      if ((rc = bl.check(bl.find(p + "self_attn.q_proj.bias"), Hd, -1))) return fail(rc);
+      if ((rc = bl.check(bl.find(p + "self_attn.k_proj.bias"), Gd, -1))) return fail(rc);
+      if ((rc = bl.check(bl.find(p + "self_attn.v_proj.bias"), Gd, -1))) return fail(rc);
+    }
+  }
+
+  // ---- weights
+  const bool f32 = m->fp32;
+  const size_t es = m->esz;
+  if ((rc = dev_alloc(m, &m->embed, static_cast<size_t>(V) * D * es))) return fail(rc);
+  if ((rc = bl.gather(m->embed, f32, bl.find("model.embed_tokens.weight"), nullptr, V, D))) return fail(rc);
+  if (cfg->tie_word_embeddings) {
+    m->head = m->embed;
+  } else {
+    if ((rc = dev_alloc(m, &m->head, static_cast<size_t>(V) * D * es))) return fail(rc);
+    if ((rc = bl.gather(m->head, f32, bl.find("lm_head.weight"), nullptr, V, D))) return fail(rc);
+  }
+  void* gfp = nullptr;
+  if ((rc = dev_alloc(m, &gfp, D * 4))) return fail(rc);
+  m->gf = static_cast<float*>(gfp);
+  if ((rc = bl.gather(m->gf, true, bl.find("model.norm.weight"), nullptr, 1, D))) return fail(rc);
+
+  std::vector<int> qmap(Hd), kmap(Gd), gmap(F), umap(F);
+  for (int h = 0; h < m->H; ++h)
+    for (int p = 0; p < m->d; ++p) qmap[h * m->d + p] = h * m->d + qkv_natural(p, m->d);
+  for (int h = 0; h < m->G; ++h)
+    for (int p = 0; p < m->d; ++p) kmap[h * m->d + p] = h * m->d + qkv_natural(p, m->d);
+  m->layers.resize(m->L);
+  for (int l = 0; l < m->L; ++l) {
+    LayerW& w = m->layers[l];
+    const std::string p = "model.layers." + std::to_string(l) + ".";
+    if ((rc = dev_alloc(m, &w.wqkv, static_cast<size_t>(m->Nqkv) * D * es))) return fail(rc);
+    char* q0 = static_cast<char*>(w.wqkv);
+    if ((rc = bl.gather(q0, f32, bl.find(p + "self_attn.q_proj.weight"), &qmap, Hd, D))) return fail(rc);
+    if ((rc = bl.gather(q0 + static_cast<size_t>(Hd) * D * es, f32, bl.find(p + "self_attn.k_proj.weight"), &kmap,
+                        Gd, D)))
+      return fail(rc);
+    if ((rc = bl.gather(q0 + static_cast<size_t>(Hd + Gd) * D * es, f32, bl.find(p + "self_attn.v_proj.weight"),
+                        &kmap, Gd, D)))
+      return fail(rc);
+    if (cfg->attention_bias) {
+      void* bp = nullptr;
+      if ((rc = dev_alloc(m, &bp, static_cast<size_t>(m->Nqkv) * 4))) return fail(rc);
+      w.bqkv = static_cast<float*>(bp);
+      // A bias vector is a [n, 1] matrix for the gather.
+      axon_tensor tq = *bl.find(p + "self_attn.q_proj.bias"), tk = *bl.find(p + "self_attn.k_proj.bias"),
+                  tv = *bl.find(p + "self_attn.v_proj.bias");
+      tq.ndim = tk.ndim = tv.ndim = 2;
+      tq.shape[1] = tk.shape[1] = tv.shape[1] = 1;
+      if ((rc = bl.gather(w.bqkv, true, &tq, &qmap, Hd, 1))) return fail(rc);
+      if ((rc = bl.gather(w.bqkv + Hd, true, &tk, &kmap, Gd, 1))) return fail(rc);
+      if ((rc = bl.gather(w.bqkv + Hd + Gd, true, &tv, &kmap, Gd, 1))) return fail(rc);
+    }
+    if ((rc = dev_alloc(m, &w.wo, static_cast<size_t>(D) * Hd * es))) return fail(rc);
+    if ((rc = bl.gather(w.wo, f32, bl.find(p + "self_attn.o_proj.weight"), nullptr, D, Hd))) return fail(rc);
+    // gate/up interleave: packed row r: chunk r/16, slots 0..7 gate, 8..15 up.
+    if ((rc = dev_alloc(m, &w.wgu, static_cast<size_t>(2 * F) * D * es))) return fail(rc);
+    {
+      // Build the interleaved matrix in two gathers over a [2F] row map whose
+      // entries index a virtual [gate; up] stack: stage gate and up into one
+      // contiguous buffer first.
+      const axon_tensor* tg = bl.find(p + "mlp.gate_proj.weight");
+      const axon_tensor* tu = bl.find(p + "mlp.up_proj.weight");
+      void* tmp = nullptr;
+      const size_t half = static_cast<size_t>(F) * D * es;
+      if (cudaMalloc(&tmp, 2 * half) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(AXON_ERR_OOM);
+      }
+      int r1 = bl.gather(tmp, f32, tg, nullptr, F, D);
+      if (!r1) r1 = bl.gather(static_cast<char*>(tmp) + half, f32, tu, nullptr, F, D);
+      if (!r1) {
+        std::vector<int> imap(2 * F);
+        for (int r = 0; r < 2 * F; ++r) {
+          const int c = r >> 4, i = r & 15;
+          imap[r] = i < 8 ? c * 8 + i : F + c * 8 + (i - 8);
+        }
+        axon_tensor stack{};
+        stack.name = "gate_up";
+        stack.data = tmp;
+        stack.dtype = f32 ? AXON_DTYPE_F32 : AXON_DTYPE_BF16;
+        stack.ndim = 2;
+        stack.shape[0] = 2 * F;
+        stack.shape[1] = D;
+        r1 = bl.gather(w.wgu, f32, &stack, &imap, 2 * F, D);
+      }
+      cudaFree(tmp);
+      if (r1) return fail(r1);
+    }
+    if ((rc = dev_alloc(m, &w.wd, static_cast<size_t>(D) * F * es))) return fail(rc);
+    if ((rc = bl.gather(w.wd, f32, bl.find(p + "mlp.down_proj.weight"), nullptr, D, F))) return fail(rc);
+    void* g1 = nullptr;
+    void* g2 = nullptr;
+    if ((rc = dev_alloc(m, &g1, D * 4))) return fail(rc);
+    if ((rc = dev_alloc(m, &g2, D * 4))) return fail(rc);
+    w.g1 = static_cast<float*>(g1);
+    w.g2 = static_cast<float*>(g2);
+    if ((rc = bl.gather(w.g1, true, bl.find(p + "input_layernorm.weight"), nullptr, 1, D))) return fail(rc);
+    if ((rc = bl.gather(w.g2, true, bl.find(p + "post_attention_layernorm.weight"), nullptr, 1, D)))
+      return fail(rc);
+  }
+
+  // ---- KV cache: pools [L][num_blocks][G][16][d]
+  m->blocks_per_seq = cfg->max_context / 16;
+  m->num_blocks = cfg->kv_layout == AXON_KV_PAGED ? cfg->kv_num_blocks
+                                                  : static_cast<long long>(cfg->max_batch) * m->blocks_per_seq;
+  m->layer_kv_elems = static_cast<size_t>(m->num_blocks) * m->G * 16 * m->d;
+  const size_t kv_bytes = m->layer_kv_elems * m->L * es;
+  if ((rc = dev_alloc(m, &m->kpool, kv_bytes))) return fail(rc);
+  if ((rc = dev_alloc(m, &m->vpool, kv_bytes))) return fail(rc);
+  if (cudaMemsetAsync(m->kpool, 0, kv_bytes, st) != cudaSuccess ||
+      cudaMemsetAsync(m->vpool, 0, kv_bytes, st) != cudaSuccess)
+    return fail(AXON_ERR_CUDA);
+
+  // ---- RoPE table in double precision: (cos, sin)(p * theta^(-2j/d))
+  {
+    const int half = m->d / 2;
+    std::vector<float2> tab(static_cast<size_t>(cfg->max_context) * half);
+    for (int pos = 0; pos < cfg->max_context; ++pos)
+      for (int j = 0; j < half; ++j) {
+        const double f = std::pow(static_cast<double>(cfg->rope_theta), -2.0 * j / m->d);
+        const double ang = pos * f;
+        tab[static_cast<size_t>(pos) * half + j] = make_float2(static_cast<float>(std::cos(ang)),
+                                                               static_cast<float>(std::sin(ang)));
+      }
+    void* rp = nullptr;
+    if ((rc = dev_alloc(m, &rp, tab.size() * sizeof(float2)))) return fail(rc);
+    m->rope = static_cast<float2*>(rp);
+    if (cudaMemcpy(m->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(AXON_ERR_CUDA);
+  }
+
+  // ---- workspace
+  int Mcap = m->cfg.max_prefill_tokens;
+  if (Mcap < cfg->max_batch) Mcap = cfg->max_batch;
+  Mcap = (Mcap + 127) / 128 * 128;
+  m->Mcap = Mcap;
+  m->Pmax = D / 16;
+  void* p = nullptr;
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * D * 4))) return fail(rc);
+  m->x = static_cast<float*>(p);
+  if ((rc = dev_alloc(m, &m->a, static_cast<size_t>(Mcap) * D * es))) return fail(rc);
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * m->Pmax * 4))) return fail(rc);
+  m->ss = static_cast<float*>(p);
+  if ((rc = dev_alloc(m, &m->q, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
+  if ((rc = dev_alloc(m, &m->o, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
+  if ((rc = dev_alloc(m, &m->u, static_cast<size_t>(Mcap) * F * es))) return fail(rc);
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * 8))) return fail(rc);
+  m->keys = static_cast<unsigned long long*>(p);
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * 4))) return fail(rc);
+  m->rinv = static_cast<float*>(p);
+  if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
+  m->ticket = static_cast<int*>(p);
+  m->max_splits = 64;
+  const int dec_b = cfg->max_batch < 64 ? cfg->max_batch : 64;
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(dec_b) * m->G * m->max_splits * 16 * (m->d + 2) * 4))) return fail(rc);
+  m->attn_part = static_cast<float*>(p);
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(dec_b) * m->G * 4))) return fail(rc);
+  m->attn_cnt = static_cast<int*>(p);
+  if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
+  m->err = static_cast<int*>(p);
+  if (cudaMemsetAsync(m->keys, 0, static_cast<size_t>(Mcap) * 8, st) != cudaSuccess ||
+      cudaMemsetAsync(m->attn_cnt, 0, static_cast<size_t>(dec_b) * m->G * 4, st) != cudaSuccess ||
+      cudaMemsetAsync(m->err, 0, 16, st) != cudaSuccess || cudaMemsetAsync(m->ticket, 0, 16, st) != cudaSuccess ||
+      cudaMemsetAsync(m->x, 0, static_cast<size_t>(Mcap) * D * 4, st) != cudaSuccess ||
+      cudaMemsetAsync(m->a, 0, static_cast<size_t>(Mcap) * D * es, st) != cudaSuccess ||
+      cudaMemsetAsync(m->o, 0, static_cast<size_t>(Mcap) * Hd * es, st) != cudaSuccess ||
+      cudaMemsetAsync(m->u, 0, static_cast<size_t>(Mcap) * F * es, st) != cudaSuccess)
+    return fail(AXON_ERR_CUDA);
+
+  // ---- TMA descriptors (bf16 tensor-core path)
+  if (!f32) {
+    bool ok = make_tma_2d_bf16(&m->t_a, m->a, Mcap, D, 128) && make_tma_2d_bf16(&m->t_o, m->o, Mcap, Hd, 128) &&
+              make_tma_2d_bf16(&m->t_u, m->u, Mcap, F, 128);
+    for (int l = 0; l < m->L && ok; ++l) {
+      LayerW& w = m->layers[l];
+      w.m_qkv.a = m->t_a;
+      ok = ok && make_tma_2d_bf16(&w.m_qkv.w, w.wqkv, m->Nqkv, D, 256);
+      w.m_o.a = m->t_o;
+      ok = ok && make_tma_2d_bf16(&w.m_o.w, w.wo, D, Hd, 256);
+      w.m_gu.a = m->t_a;
+      ok = ok && make_tma_2d_bf16(&w.m_gu.w, w.wgu, 2 * F, D, 256);
+      w.m_d.a = m->t_u;
+      ok = ok && make_tma_2d_bf16(&w.m_d.w, w.wd, D, F, 256);
+    }
+    m->m_head.a = m->t_a;
+    ok = ok && make_tma_2d_bf16(&m->m_head.w, m->head, V, D, 256);
+    if (!ok) return fail(AXON_ERR_CUDA);
+  }
+  if (cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking) != cudaSuccess) return fail(AXON_ERR_CUDA);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return fail(AXON_ERR_CUDA);
+  *out = m;
+  return AXON_OK;
+}
+
+int axon_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S, const int32_t* d_block_table,
+                 int32_t logits_mode, float* d_logits, int32_t* d_next, void* stream) {
+  if (!m || !d_ids) return AXON_ERR_INVALID_ARG;
+  if (B < 1 || B > m->cfg.max_batch || S < 1 || S > m->cfg.max_context) return AXON_ERR_INVALID_ARG;
+  if (static_cast<long long>(B) * S > m->cfg.max_prefill_tokens) return AXON_ERR_INVALID_ARG;
+  if (logits_mode != AXON_LOGITS_LAST && logits_mode != AXON_LOGITS_ALL) return AXON_ERR_INVALID_ARG;
+  if (B > 64 && logits_mode == AXON_LOGITS_LAST) return AXON_ERR_UNSUPPORTED;
+  const bool paged = m->cfg.kv_layout == AXON_KV_PAGED;
+  if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
+  return enqueue_prefill(m, d_ids, B, S, d_block_table, logits_mode, d_logits, d_next,
+                         static_cast<cudaStream_t>(stream));
+}
+
+int axon_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,
+                     const int32_t* d_block_table, float* d_logits, int32_t* d_next, void* stream) {
+  if (!m || !d_tokens || !d_context_lens || !d_next) return AXON_ERR_INVALID_ARG;
+  if (B < 1 || B > m->cfg.max_batch || B > 64) return AXON_ERR_INVALID_ARG;
+  const bool paged = m->cfg.kv_layout == AXON_KV_PAGED;
+  if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (!m->use_graphs) return enqueue_decode(m, d_tokens, B, d_context_lens, d_block_table, d_logits, d_next, st);
+  const GraphKey key{B, d_tokens, d_context_lens, d_block_table, d_logits, d_next};
+  auto it = m->graphs.find(key);
+  if (it == m->graphs.end()) {
+    if (m->graphs.size() >= 64) {
+      for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+      m->graphs.clear();
+    }
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(m->cap_stream, cudaStreamCaptureModeThreadLocal));
+    const int rc = enqueue_decode(m, d_tokens, B, d_context_lens, d_block_table, d_logits, d_next, m->cap_stream);
+    const cudaError_t ec = cudaStreamEndCapture(m->cap_stream, &g);
+    if (rc != AXON_OK || ec != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      cudaGetLastError();
+      return rc != AXON_OK ? rc : AXON_ERR_CUDA;
+    }
+    cudaGraphExec_t ex = nullptr;
+    const cudaError_t ei = cudaGraphInstantiate(&ex, g, 0);
+    cudaGraphDestroy(g);
+    if (ei != cudaSuccess) {
+      cudaGetLastError();
+      return AXON_ERR_CUDA;
+    }
+    it = m->graphs.emplace(key, ex).first;
+  }
+  CK(cudaGraphLaunch(it->second, st));
+  return AXON_OK;
+}
+
+int axon_reset(axon_model* m) {
+  if (!m) return AXON_ERR_INVALID_ARG;
+  CK(cudaDeviceSynchronize());
+  const size_t kv_bytes = m->layer_kv_elems * m->L * m->esz;
+  CK(cudaMemset(m->kpool, 0, kv_bytes));
+  CK(cudaMemset(m->vpool, 0, kv_bytes));
+  CK(cudaMemset(m->err, 0, 16));
+  CK(cudaDeviceSynchronize());
+  return AXON_OK;
+}
+
+int axon_check_device(axon_model* m, void* stream, int32_t* bits) {
+  if (!m) return AXON_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  int word = 0;
+  CK(cudaMemcpy(&word, m->err, sizeof(int), cudaMemcpyDeviceToHost));
+  CK(cudaMemset(m->err, 0, sizeof(int)));
+  if (bits) *bits = word;
+  if (word & DEVERR_TIMEOUT) return AXON_ERR_TIMEOUT;
+  if (word) return AXON_ERR_DEVICE_CHECK;
+  return AXON_OK;
+}
+
+int axon_kv_view_get(const axon_model* m, axon_kv_view* out) {
+  if (!m || !out) return AXON_ERR_INVALID_ARG;
+  out->k_pool = m->kpool;
+  out->v_pool = m->vpool;
+  out->num_blocks = m->num_blocks;
+  out->blocks_per_seq = m->blocks_per_seq;
+  out->block_size = 16;
+  out->elem_bytes = static_cast<int32_t>(m->esz);
+  return AXON_OK;
+}
+
+void axon_free(axon_model* m) {
+  if (!m) return;
+  cudaDeviceSynchronize();
+  free_model(m);
+}
+
+}  // extern "C"

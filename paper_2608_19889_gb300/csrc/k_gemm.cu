@@ -1,0 +1,261 @@
+// Prefill projections on the 5th-generation tensor cores: a persistent,
+// warp-specialised tcgen05 GEMM, out[m][n] = A[m] . W[n] (A = bf16
+// activations [M][K], W = bf16 weights [N][K], fp32 accumulation in TMEM),
+// followed by the fused epilogues of epilogue.cuh.
+//
+//   warp 0      : TMA producer -- one lane streams 128x64 A and 256x64 W
+//                 tiles (128-byte swizzle) into a 4-stage shared-memory ring,
+//                 completion tracked by mbarrier transaction bytes;
+//   warp 1      : MMA issuer -- allocates 512 TMEM columns (two 128x256 fp32
+//                 accumulators), one lane issues tcgen05.mma kind::f16
+//                 (M=128, N=256, K=16) and frees ring slots / publishes
+//                 finished accumulators with tcgen05.commit;
+//   warps 2..5  : epilogue -- each reads its 32 TMEM lanes (rows) 16 columns
+//                 at a time with tcgen05.ld and applies the fused epilogue,
+//                 overlapping the next tile's main loop (double-buffered
+//                 accumulators).
+// Tiles are visited in groups of 8 M-blocks per N sweep so the A and W
+// working sets of the concurrently running CTAs stay L2-resident.
+// Every mbarrier wait is bounded (DEVERR_TIMEOUT instead of a hang).
+#include "kernels.h"
+
+#include <cudaTypedefs.h>
+
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4, GROUP_M = 8;
+constexpr int A_BYTES = BM * BK * 2;  // 16 KB
+constexpr int B_BYTES = BN * BK * 2;  // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
+constexpr int NUM_THREADS = 192;
+constexpr uint32_t TMEM_COLS = 2 * BN;
+
+AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
+  const int per_group = GROUP_M * num_n;
+  const int g = t / per_group;
+  const int first_m = g * GROUP_M;
+  const int gm = min(GROUP_M, num_m - first_m);
+  const int local = t - g * per_group;
+  nb = local / gm;
+  mb = first_m + (local - nb * gm);
+}
+
+template <int KIND>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
+                   int K, EpiArgs ep) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const uint32_t sA = base, sB = base + STAGES * A_BYTES;
+  const uint32_t bars = base + STAGES * STAGE_BYTES;
+  const uint32_t tmem_slot = bars + 8 * (2 * STAGES + 4);
+  const uint32_t* tmem_slot_ptr =
+      reinterpret_cast<const uint32_t*>(smem_raw + (tmem_slot - raw));
+  auto full_bar = [&](int s) { return bars + 8 * s; };
+  auto empty_bar = [&](int s) { return bars + 8 * (STAGES + s); };
+  auto accf_bar = [&](int i) { return bars + 8 * (2 * STAGES + i); };
+  auto acce_bar = [&](int i) { return bars + 8 * (2 * STAGES + 2 + i); };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(accf_bar(i), 1);
+      mbar_init(acce_bar(i), 128);
+    }
+    fence_mbar_init();
+    fence_proxy_async();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot_ptr;
+
+  grid_dep_wait();
+  const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN;
+  const int tiles = num_m * num_n, KB = K / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        int mb, nb;
+        tile_coords(t, num_m, num_n, mb, nb);
+        for (int kb = 0; kb < KB; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          if (!mbar_wait(empty_bar(s), ph ^ 1, ep.err)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full_bar(s), STAGE_BYTES);
+          tma_load_2d(sA + s * A_BYTES, &tmA, full_bar(s), kb * BK, mb * BM);
+          tma_load_2d(sB + s * B_BYTES, &tmB, full_bar(s), kb * BK, nb * BN);
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      int it = 0, lt = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++lt) {
+        const int buf = lt & 1;
+        const uint32_t aph = (lt >> 1) & 1;
+        if (!mbar_wait(acce_bar(buf), aph ^ 1, ep.err)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + buf * BN;
+        for (int kb = 0; kb < KB; ++kb, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1;
+          if (!mbar_wait(full_bar(s), ph, ep.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = smem_desc_sw128(sA + s * A_BYTES);
+          const uint64_t bd = smem_desc_sw128(sB + s * B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K inside the swizzle atom
+            tc_mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
+          tc_commit(empty_bar(s));
+        }
+        if (ok) tc_commit(accf_bar(buf));
+      }
+    }
+    __syncwarp();
+  } else {
+    const int q4 = warp & 3;  // TMEM lane quarter this warp may read
+    const int row = q4 * 32 + lane;
+    int lt = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
+      int mb, nb;
+      tile_coords(t, num_m, num_n, mb, nb);
+      const int buf = lt & 1;
+      const uint32_t aph = (lt >> 1) & 1;
+      const bool got = mbar_wait(accf_bar(buf), aph, ep.err);
+      __syncwarp();
+      if (!got) break;
+      tc_fence_after();
+      const int m = mb * BM + row;
+      const bool mval = m < M;
+      float rinv = 1.f;
+      if (KIND != EPI_RESID && mval) rinv = row_rinv(ep, m);
+      float ssum = 0.f;
+      unsigned long long best = 0ull;
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(q4 * 32) << 16) + buf * BN;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 16) {
+        uint32_t v[16];
+        tmem_ld16(taddr + c, v);
+        tmem_wait_ld();
+        const int n0 = nb * BN + c;
+        if (mval && n0 < N) {
+          float f[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(v[i]);
+          if (KIND == EPI_QKV) {
+            epi_qkv16<bf16>(ep, m, n0, f, rinv);
+          } else if (KIND == EPI_RESID) {
+            ssum += epi_resid16<bf16>(ep, m, n0, f);
+          } else if (KIND == EPI_SWIGLU) {
+            epi_swiglu16<bf16>(ep, m, n0, f, rinv);
+          } else {
+            const unsigned long long k = epi_logits16(ep, m, n0, f, rinv);
+            best = k > best ? k : best;
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(acce_bar(buf));
+      if (KIND == EPI_RESID && mval) ep.ss_out[static_cast<long long>(m) * ep.ss_out_stride + nb] = ssum;
+      if (KIND == EPI_LOGITS && mval) argmax_commit(ep.keys + m, best);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+template <int KIND>
+cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep) {
+  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+  const int grid = tiles < lc.num_sms ? tiles : lc.num_sms;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.stream = lc.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = lc.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND>, maps.a, maps.w, M, N, K, ep);
+}
+
+}  // namespace
+
+bool make_tma_2d_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn || (reinterpret_cast<uintptr_t>(base) & 15) || ((cols * 2) & 15)) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+cudaError_t prepare_gemm_kernels() {
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_LOGITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  return e;
+}
+
+cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K,
+                           const EpiArgs& ep) {
+  if (M < 1 || N < 1 || K < BK || (K % BK)) return cudaErrorInvalidValue;
+  switch (kind) {
+    case EPI_QKV: return launch_kind<EPI_QKV>(lc, maps, M, N, K, ep);
+    case EPI_RESID: return launch_kind<EPI_RESID>(lc, maps, M, N, K, ep);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU>(lc, maps, M, N, K, ep);
+    default: return launch_kind<EPI_LOGITS>(lc, maps, M, N, K, ep);
+  }
+}

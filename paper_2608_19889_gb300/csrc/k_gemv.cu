@@ -1,0 +1,346 @@
+// Decode-side kernels: the weight-streaming projection (skinny GEMV on
+// tensor cores), the embedding gather and the greedy-token finaliser.
+//
+// Projection layout: one CTA owns 16 consecutive weight rows and all B <= 64
+// tokens; its KW warps split K into 64-wide chunks. Each lane streams 2 rows
+// x 32 bytes per chunk with 16-byte L1-bypassing loads (4 lanes cover 128
+// contiguous bytes of a row), so the whole matrix is read exactly once at
+// full 128-byte-line efficiency. Products run on mma.sync m16n8k16 with the
+// weights as the 16-row A operand and tokens as the 8-wide N operand: the
+// dot product is order-free in k, so each lane feeds its contiguous 16
+// elements into the fragment slots in a fixed permutation that the token
+// operand mirrors. Partial sums meet in shared memory in a fixed warp order
+// (deterministic), then one thread per token runs the fused epilogue.
+#include "kernels.h"
+
+namespace {
+
+constexpr int GEMV_KW = 8;  // warps per CTA along K
+
+// Inverse RMS of each token for the consuming epilogue: either read back
+// (producer already reduced it) or summed from the producer's partials by
+// one warp.
+AXON_DEV void load_rinv(const EpiArgs& ep, int B, float* rinv_s, int lane) {
+  if (ep.rinv) {
+    for (int b = lane; b < B; b += 32) rinv_s[b] = ep.rinv[static_cast<long long>(b) * ep.rinv_stride];
+    return;
+  }
+  for (int b = 0; b < B; ++b) {
+    const float* p = ep.ss + static_cast<long long>(b) * ep.ss_stride;
+    float s = 0.f;
+    for (int i = lane; i < ep.ss_parts; i += 32) s += p[i];
+    s = warp_sum(s);
+    if (lane == 0) rinv_s[b] = 1.0f / sqrtf(s * ep.inv_D + ep.eps);
+  }
+}
+
+// Residual producers: the last CTA to finish reduces every token's partial
+// sums of squares (fixed order, deterministic) into rinv_out and re-arms the
+// ticket. No CTA waits on another.
+AXON_DEV void finish_rinv(const EpiArgs& ep, int B, int nparts) {
+  __shared__ int is_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) is_last = (atomicAdd(ep.ticket, 1) == static_cast<int>(gridDim.x) - 1);
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int b = warp; b < B; b += nw) {
+    const float* p = ep.ss_out + static_cast<long long>(b) * ep.ss_out_stride;
+    float s = 0.f;
+    for (int i = lane; i < nparts; i += 32) s += __ldcg(p + i);
+    s = warp_sum(s);
+    if (lane == 0) ep.rinv_out[b] = 1.0f / sqrtf(s * ep.inv_D + ep.eps);
+  }
+  if (threadIdx.x == 0) *ep.ticket = 0;
+}
+
+template <int NT, int KIND>
+__global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __restrict__ W, int N, int K,
+                                                               const bf16* __restrict__ act, long long act_stride,
+                                                               int B, EpiArgs ep) {
+  constexpr int TOK = NT * 8;
+  __shared__ float red[GEMV_KW][16][TOK + 1];
+  __shared__ float rinv_s[TOK];
+
+  // Let the next kernel in the stream start launching now: it only reads our
+  // outputs after its own griddepcontrol.wait.
+  grid_dep_launch();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = lane >> 2, q = lane & 3;
+  const int n0 = blockIdx.x * 16;
+  const int row0 = min(n0 + r, N - 1), row1 = min(n0 + r + 8, N - 1);
+  const bf16* w0 = W + static_cast<long long>(row0) * K + 16 * q;
+  const bf16* w1 = W + static_cast<long long>(row1) * K + 16 * q;
+  const int nchunks = K >> 6;
+
+  float acc[NT][4];
+#pragma unroll
+  for (int t = 0; t < NT; ++t) acc[t][0] = acc[t][1] = acc[t][2] = acc[t][3] = 0.f;
+
+  const bf16* arow[NT];
+  bool aval[NT];
+#pragma unroll
+  for (int t = 0; t < NT; ++t) {
+    const int tok = t * 8 + r;
+    aval[t] = tok < B;
+    arow[t] = act + static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q;
+  }
+
+  auto chunk = [&](int c, const uint4& wa0, const uint4& wa1, const uint4& wb0, const uint4& wb1) {
+    const uint32_t A0[8] = {wa0.x, wa0.y, wa0.z, wa0.w, wa1.x, wa1.y, wa1.z, wa1.w};
+    const uint32_t A1[8] = {wb0.x, wb0.y, wb0.z, wb0.w, wb1.x, wb1.y, wb1.z, wb1.w};
+#pragma unroll
+    for (int t = 0; t < NT; ++t) {
+      uint4 x0 = make_uint4(0, 0, 0, 0), x1 = make_uint4(0, 0, 0, 0);
+      if (aval[t]) {
+        x0 = ld16(arow[t] + c * 64);
+        x1 = ld16(arow[t] + c * 64 + 8);
+      }
+      const uint32_t Bv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t a[4] = {A0[2 * j], A1[2 * j], A0[2 * j + 1], A1[2 * j + 1]};
+        const uint32_t bb[2] = {Bv[2 * j], Bv[2 * j + 1]};
+        mma_bf16_16816(acc[t], a, bb);
+      }
+    }
+  };
+
+  // Weights do not depend on earlier kernels: the first iteration's weight
+  // loads are in flight before waiting for the activations.
+  int c = warp;
+  const uint4 z = make_uint4(0, 0, 0, 0);
+  uint4 a0 = z, a1 = z, b0 = z, b1 = z, a2 = z, a3 = z, b2 = z, b3 = z;
+  if (c < nchunks) {
+    a0 = ld_stream16(w0 + c * 64);
+    a1 = ld_stream16(w0 + c * 64 + 8);
+    b0 = ld_stream16(w1 + c * 64);
+    b1 = ld_stream16(w1 + c * 64 + 8);
+  }
+  if (c + GEMV_KW < nchunks) {
+    const int c2 = c + GEMV_KW;
+    a2 = ld_stream16(w0 + c2 * 64);
+    a3 = ld_stream16(w0 + c2 * 64 + 8);
+    b2 = ld_stream16(w1 + c2 * 64);
+    b3 = ld_stream16(w1 + c2 * 64 + 8);
+  }
+  grid_dep_wait();
+  if (c < nchunks) chunk(c, a0, a1, b0, b1);
+  if (c + GEMV_KW < nchunks) chunk(c + GEMV_KW, a2, a3, b2, b3);
+  for (c += 2 * GEMV_KW; c + GEMV_KW < nchunks; c += 2 * GEMV_KW) {
+    const int c2 = c + GEMV_KW;
+    a0 = ld_stream16(w0 + c * 64);
+    a1 = ld_stream16(w0 + c * 64 + 8);
+    b0 = ld_stream16(w1 + c * 64);
+    b1 = ld_stream16(w1 + c * 64 + 8);
+    a2 = ld_stream16(w0 + c2 * 64);
+    a3 = ld_stream16(w0 + c2 * 64 + 8);
+    b2 = ld_stream16(w1 + c2 * 64);
+    b3 = ld_stream16(w1 + c2 * 64 + 8);
+    chunk(c, a0, a1, b0, b1);
+    chunk(c2, a2, a3, b2, b3);
+  }
+  if (c < nchunks) {
+    a0 = ld_stream16(w0 + c * 64);
+    a1 = ld_stream16(w0 + c * 64 + 8);
+    b0 = ld_stream16(w1 + c * 64);
+    b1 = ld_stream16(w1 + c * 64 + 8);
+    chunk(c, a0, a1, b0, b1);
+  }
+
+  if (KIND != EPI_RESID && warp == GEMV_KW - 1) load_rinv(ep, B, rinv_s, lane);
+#pragma unroll
+  for (int t = 0; t < NT; ++t) {
+    red[warp][r][t * 8 + 2 * q] = acc[t][0];
+    red[warp][r][t * 8 + 2 * q + 1] = acc[t][1];
+    red[warp][r + 8][t * 8 + 2 * q] = acc[t][2];
+    red[warp][r + 8][t * 8 + 2 * q + 1] = acc[t][3];
+  }
+  __syncthreads();
+
+  const int b = threadIdx.x;
+  if (b < B) {
+    float v[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float s = 0.f;
+#pragma unroll
+      for (int w = 0; w < GEMV_KW; ++w) s += red[w][i][b];
+      v[i] = s;
+    }
+    if (KIND == EPI_QKV) {
+      epi_qkv16<bf16>(ep, b, n0, v, rinv_s[b]);
+    } else if (KIND == EPI_RESID) {
+      const float s = epi_resid16<bf16>(ep, b, n0, v);
+      ep.ss_out[static_cast<long long>(b) * ep.ss_out_stride + blockIdx.x] = s;
+    } else if (KIND == EPI_SWIGLU) {
+      epi_swiglu16<bf16>(ep, b, n0, v, rinv_s[b]);
+    } else {
+      const unsigned long long k = epi_logits16(ep, b, n0, v, rinv_s[b]);
+      argmax_commit(ep.keys + b, k);
+    }
+  }
+  if (KIND == EPI_RESID && ep.rinv_out) finish_rinv(ep, B, gridDim.x);
+}
+
+// fp32 debug projection: same CTA shape, CUDA-core FMAs on fp32 weights.
+template <int KIND>
+__global__ void __launch_bounds__(GEMV_KW * 32) gemv_f32_kernel(const float* __restrict__ W, int N, int K,
+                                                               const float* __restrict__ act, long long act_stride,
+                                                               int B, EpiArgs ep) {
+  __shared__ float red[GEMV_KW][16][65];
+  __shared__ float rinv_s[64];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n0 = blockIdx.x * 16;
+  grid_dep_launch();
+  grid_dep_wait();
+  if (KIND != EPI_RESID && warp == GEMV_KW - 1) load_rinv(ep, B, rinv_s, lane);
+  // Warp w: rows n0 + 2w, n0 + 2w + 1; lanes stride over K.
+  for (int rr = 0; rr < 2; ++rr) {
+    const int i = warp * 2 + rr;
+    const int row = min(n0 + i, N - 1);
+    const float* w = W + static_cast<long long>(row) * K;
+    for (int b = 0; b < B; ++b) {
+      const float* a = act + static_cast<long long>(b) * act_stride;
+      float s = 0.f;
+      for (int k = lane; k < K; k += 32) s = fmaf(w[k], a[k], s);
+      s = warp_sum(s);
+      if (lane == 0) red[0][i][b] = s;
+    }
+  }
+  __syncthreads();
+  const int b = threadIdx.x;
+  if (b < B) {
+    float v[16];
+    for (int i = 0; i < 16; ++i) v[i] = red[0][i][b];
+    if (KIND == EPI_QKV) {
+      epi_qkv16<float>(ep, b, n0, v, rinv_s[b]);
+    } else if (KIND == EPI_RESID) {
+      const float s = epi_resid16<float>(ep, b, n0, v);
+      ep.ss_out[static_cast<long long>(b) * ep.ss_out_stride + blockIdx.x] = s;
+    } else if (KIND == EPI_SWIGLU) {
+      epi_swiglu16<float>(ep, b, n0, v, rinv_s[b]);
+    } else {
+      const unsigned long long k = epi_logits16(ep, b, n0, v, rinv_s[b]);
+      argmax_commit(ep.keys + b, k);
+    }
+  }
+  if (KIND == EPI_RESID && ep.rinv_out) finish_rinv(ep, B, gridDim.x);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) embed_kernel(const T* __restrict__ E, int V, int D, const int* __restrict__ ids,
+                                                    float* __restrict__ x, T* __restrict__ a,
+                                                    const float* __restrict__ g, float* __restrict__ ss, int ss_stride,
+                                                    float* __restrict__ rinv, float eps, int* err) {
+  __shared__ float red[4];
+  grid_dep_launch();
+  grid_dep_wait();
+  const int m = blockIdx.x;
+  int id = ids[m];
+  if (id < 0 || id >= V) {
+    if (threadIdx.x == 0) set_err(err, DEVERR_TOKEN);
+    id = 0;
+  }
+  const T* e = E + static_cast<long long>(id) * D;
+  float* xr = x + static_cast<long long>(m) * D;
+  T* ar = a + static_cast<long long>(m) * D;
+  float s = 0.f;
+  for (int k = threadIdx.x; k < D; k += blockDim.x) {
+    const float v = to_f(e[k]);
+    xr[k] = v;
+    ar[k] = from_f<T>(v * g[k]);
+    s += v * v;
+  }
+  s = warp_sum(s);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const float tot = red[0] + red[1] + red[2] + red[3];
+    ss[static_cast<long long>(m) * ss_stride] = tot;
+    if (rinv) rinv[m] = 1.0f / sqrtf(tot / static_cast<float>(D) + eps);
+  }
+}
+
+// One CTA: read the B greedy tokens, then clear every key row used.
+__global__ void __launch_bounds__(1024) finalize_kernel(unsigned long long* keys, int n_keys, int key_stride,
+                                                        int key_offset, int B, int* next, int* ctx) {
+  grid_dep_launch();
+  grid_dep_wait();
+  const int i = threadIdx.x;
+  if (i < B) {
+    const unsigned long long k = keys[static_cast<long long>(i) * key_stride + key_offset];
+    if (next) next[i] = static_cast<int>(0xffffffffu - static_cast<uint32_t>(k & 0xffffffffull));
+    if (ctx) ctx[i] += 1;
+  }
+  __syncthreads();
+  for (int j = i; j < n_keys; j += blockDim.x) keys[j] = 0ull;
+}
+
+template <typename K, typename... Args>
+cudaError_t launch_k(const LaunchCtx& lc, K kernel, dim3 grid, dim3 block, size_t smem, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = lc.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = lc.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+template <int NT>
+cudaError_t gemv_nt(const LaunchCtx& lc, int kind, const void* W, int N, int K, const void* act, long long st, int B,
+                    const EpiArgs& ep) {
+  const dim3 grid((N + 15) / 16), block(GEMV_KW * 32);
+  const bf16* w = static_cast<const bf16*>(W);
+  const bf16* a = static_cast<const bf16*>(act);
+  switch (kind) {
+    case EPI_QKV: return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV>, grid, block, 0, w, N, K, a, st, B, ep);
+    case EPI_RESID: return launch_k(lc, gemv_mma_kernel<NT, EPI_RESID>, grid, block, 0, w, N, K, a, st, B, ep);
+    case EPI_SWIGLU: return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU>, grid, block, 0, w, N, K, a, st, B, ep);
+    default: return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS>, grid, block, 0, w, N, K, a, st, B, ep);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
+                        long long act_stride, int B, const EpiArgs& ep) {
+  if (B < 1 || B > 64 || (K & 63) || N < 1) return cudaErrorInvalidValue;
+  if (fp32) {
+    const dim3 grid((N + 15) / 16), block(GEMV_KW * 32);
+    const float* w = static_cast<const float*>(W);
+    const float* a = static_cast<const float*>(act);
+    switch (kind) {
+      case EPI_QKV: return launch_k(lc, gemv_f32_kernel<EPI_QKV>, grid, block, 0, w, N, K, a, act_stride, B, ep);
+      case EPI_RESID: return launch_k(lc, gemv_f32_kernel<EPI_RESID>, grid, block, 0, w, N, K, a, act_stride, B, ep);
+      case EPI_SWIGLU: return launch_k(lc, gemv_f32_kernel<EPI_SWIGLU>, grid, block, 0, w, N, K, a, act_stride, B, ep);
+      default: return launch_k(lc, gemv_f32_kernel<EPI_LOGITS>, grid, block, 0, w, N, K, a, act_stride, B, ep);
+    }
+  }
+  if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep);
+  if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep);
+  if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep);
+  return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep);
+}
+
+cudaError_t launch_embed(const LaunchCtx& lc, bool fp32, const void* E, int V, int D, const int* ids, int M, float* x,
+                         void* a, const float* g, float* ss, int ss_stride, float* rinv, float eps, int* err) {
+  if (fp32)
+    return launch_k(lc, embed_kernel<float>, dim3(M), dim3(128), 0, static_cast<const float*>(E), V, D, ids, x,
+                    static_cast<float*>(a), g, ss, ss_stride, rinv, eps, err);
+  return launch_k(lc, embed_kernel<bf16>, dim3(M), dim3(128), 0, static_cast<const bf16*>(E), V, D, ids, x,
+                  static_cast<bf16*>(a), g, ss, ss_stride, rinv, eps, err);
+}
+
+cudaError_t launch_finalize(const LaunchCtx& lc, unsigned long long* keys, int n_keys, int key_stride, int key_offset,
+                            int B, int* next, int* ctx) {
+  if (B > 1024) return cudaErrorInvalidValue;
+  return launch_k(lc, finalize_kernel, dim3(1), dim3(1024), 0, keys, n_keys, key_stride, key_offset, B, next, ctx);
+}

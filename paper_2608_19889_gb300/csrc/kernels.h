@@ -1,0 +1,72 @@
+// Host-side launchers of the CUDA kernels (one translation unit each).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda.h>
+#include <stdint.h>
+
+#include "epilogue.cuh"
+
+// Launch options shared by every launcher: stream and whether to request
+// programmatic dependent launch (overlap with the previous kernel's tail).
+struct LaunchCtx {
+  cudaStream_t stream;
+  bool pdl;
+  int num_sms;
+};
+
+// ---- decode projections (k_gemv.cu): out[b][n] = act[b] . W[n], B <= 64
+// tokens, 16 weight rows per CTA, fused epilogue `kind`.
+cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
+                        long long act_stride, int B, const EpiArgs& ep);
+
+// ---- embedding gather producing x, a = x * g and the row sum of squares.
+// rinv (optional): 1 / sqrt(mean(x^2) + eps) per row.
+cudaError_t launch_embed(const LaunchCtx& lc, bool fp32, const void* E, int V, int D, const int* ids, int M, float* x,
+                         void* a, const float* g, float* ss, int ss_stride, float* rinv, float eps, int* err);
+
+// ---- greedy token from argmax keys; clears the keys; optionally advances
+// context lengths.
+cudaError_t launch_finalize(const LaunchCtx& lc, unsigned long long* keys, int n_keys, int key_stride,
+                            int key_offset, int B, int* next, int* ctx);
+
+// ---- attention (k_attn.cu)
+struct AttnArgs {
+  const void* q;  // [rows][H*d]
+  const void* k;  // layer pool [num_blocks][G][16][d]
+  const void* v;
+  void* o;        // [rows][H*d]
+  const int* ctx;  // decode: [B] tokens cached before the step
+  const int* block_table;
+  int bt_stride;
+  int blocks_per_seq;
+  int num_blocks;
+  int H, G, d;
+  int S;        // prefill prompt length
+  int splits;   // decode split-KV factor
+  float scale_log2;
+  float* part;  // decode partials
+  int* counter;  // decode [B][G] tickets
+  int* err;
+};
+cudaError_t launch_attn_decode(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B);
+cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B);
+int attn_decode_splits(int B, int G, int max_blocks, int num_sms);
+// Set kernel attributes (dynamic shared memory limits) once, before any
+// launch or graph capture.
+cudaError_t prepare_attn_kernels();
+cudaError_t prepare_gemm_kernels();
+
+// ---- prefill projections (k_gemm.cu): tcgen05 + TMA persistent GEMM,
+// out[m][n] = A[m] . W[n], M x N x K with K % 64 == 0.
+struct GemmMaps {
+  CUtensorMap a;  // activations [rows][K] bf16, box 64 x 128
+  CUtensorMap w;  // weights [N][K] bf16, box 64 x 256
+};
+bool make_tma_2d_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep);
+
+// ---- fp32 debug projections (k_simt.cu): plain tiled CUDA-core GEMM with
+// the same epilogues, any M.
+cudaError_t launch_gemm_simt(const LaunchCtx& lc, int kind, const float* A, long long a_stride, const float* W, int M,
+                             int N, int K, const EpiArgs& ep);

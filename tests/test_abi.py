@@ -1,0 +1,69 @@
+"""CPU-side checks of the C ABI: the library loads without a GPU and exports
+every function include/axon.h declares; the binding's structs match the
+header's field order."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "axon.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:int|void|const char\*)\s+(axon_\w+)\s*\(", src, flags=re.M)))
+
+
+@pytest.fixture(scope="module")
+def built():
+    from paper_2608_19889_gb300 import build
+    build.build()
+    import paper_2608_19889_gb300 as ax
+    return ax
+
+
+def test_header_declares_the_boundary():
+    fns = declared_functions()
+    for f in ("axon_model_create", "axon_prefill", "axon_decode_step", "axon_free"):
+        assert f in fns
+
+
+def test_library_exports_every_declared_symbol(built):
+    lib = built.lib()
+    for f in declared_functions():
+        assert hasattr(lib, f), f"missing export {f}"
+    assert sorted(built.EXPORTED) == declared_functions()
+
+
+def test_status_strings_without_gpu(built):
+    assert built.axon_status_string(0) == "ok"
+    assert "argument" in built.axon_status_string(built.AXON_ERR_INVALID_ARG)
+    assert built.axon_status_string(12345) == "unknown status"
+
+
+def test_null_arguments_are_rejected_without_touching_the_device(built):
+    lib = built.lib()
+    out = ctypes.c_void_p()
+    assert lib.axon_model_create(None, None, 0, None, ctypes.byref(out)) == built.AXON_ERR_INVALID_ARG
+    assert lib.axon_prefill(None, None, 1, 1, None, 0, None, None, None) == built.AXON_ERR_INVALID_ARG
+    assert lib.axon_decode_step(None, None, 1, None, None, None, None, None) == built.AXON_ERR_INVALID_ARG
+    lib.axon_free(None)
+
+
+def test_config_struct_layout_matches_header():
+    import paper_2608_19889_gb300 as ax
+    src = open(os.path.join(ROOT, "include", "axon.h")).read()
+    body = src[src.index("typedef struct axon_config {"):src.index("} axon_config;")]
+    names = re.findall(r"(\w+);", re.sub(r"/\*.*?\*/", "", body, flags=re.S))
+    # fields declared several per line: expand "int32_t a, b, c;"
+    fields = []
+    for decl in re.sub(r"/\*.*?\*/", "", body, flags=re.S).split(";")[:-1]:
+        decl = decl.replace("typedef struct axon_config {", "")
+        parts = decl.split()
+        if not parts:
+            continue
+        fields += [p.strip(",") for p in " ".join(parts[1:]).split(",")]
+    assert [f[0] for f in ax.axon_config._fields_] == [f.strip() for f in fields]
+    assert names

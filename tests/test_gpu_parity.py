@@ -1,0 +1,249 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle on
+the same seeded weights and ids. Tiny shapes span several 16-row / 128-row
+tiles with ragged tails; the 135M and 0.5B workloads run at full width."""
+import numpy as np
+import pytest
+
+import synth_inputs as si
+from helpers import FP32_REL_TOL, LOGIT_TOL, TOP1_MIN, create, gpu_weights, oracle_for, parity
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+# Two layers, two KV heads x 2 query heads each, head_dim 64, a vocabulary
+# that is not a multiple of 16, biases on q/k/v.
+TINY = dict(L=2, D=128, H=4, G=2, d=64, F=192, V=1000, tie=False, bias=True, theta=1e4, eps=1e-5)
+TINY128 = dict(L=2, D=256, H=6, G=2, d=128, F=320, V=777, tie=True, bias=False, theta=5e5, eps=1e-6)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_19889_gb300 import build
+    build.build()
+
+
+class _DevBuf:
+    """Wraps a raw device pointer for torch.as_tensor (CUDA array interface)."""
+
+    def __init__(self, ptr, nbytes):
+        self.__cuda_array_interface__ = {"shape": (nbytes,), "typestr": "|u1", "data": (int(ptr), False),
+                                         "version": 3}
+
+
+def device_bytes(ptr, nbytes):
+    return torch.as_tensor(_DevBuf(ptr, nbytes), device="cuda").clone()
+
+
+def _ax():
+    import paper_2608_19889_gb300 as ax
+    return ax
+
+
+def run_prefill(m, ids_np, mode, V, block_table=None):
+    ax = _ax()
+    B, S = ids_np.shape
+    ids = torch.from_numpy(ids_np.astype(np.int32)).cuda()
+    logits = torch.full((B, S, V) if mode == ax.AXON_LOGITS_ALL else (B, V), float("nan"), device="cuda")
+    nxt = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    ax.axon_prefill(m, ids, block_table=block_table, logits_mode=mode, logits=logits, next_tokens=nxt)
+    torch.cuda.synchronize()
+    return logits.cpu().numpy(), nxt.cpu().numpy()
+
+
+def decode_steps(m, first_tokens, ctx0, n_steps, V, block_table=None):
+    """n_steps greedy steps; returns logits [B, n, V] and tokens fed [B, n]."""
+    ax = _ax()
+    B = len(first_tokens)
+    tok = torch.from_numpy(np.asarray(first_tokens, dtype=np.int32)).cuda()
+    ctx = torch.from_numpy(np.asarray(ctx0, dtype=np.int32)).cuda()
+    fed, outs = [], []
+    for _ in range(n_steps):
+        fed.append(tok.cpu().numpy().copy())
+        logits = torch.full((B, V), float("nan"), device="cuda")
+        nxt = torch.empty(B, dtype=torch.int32, device="cuda")
+        ax.axon_decode_step(m, tok, ctx, block_table=block_table, logits=logits, next_tokens=nxt)
+        torch.cuda.synchronize()
+        lg = logits.cpu().numpy()
+        assert np.array_equal(nxt.cpu().numpy(), lg.argmax(-1)), "next token != argmax of the step's logits"
+        outs.append(lg)
+        tok = nxt
+    assert np.array_equal(ctx.cpu().numpy(), np.asarray(ctx0) + n_steps)
+    return np.stack(outs, 1), np.stack(fed, 1)
+
+
+def check(gpu, ref, tol=LOGIT_TOL, what="", top1=False):
+    """max |delta logit| <= tol and no top-1 mismatch outside a near tie;
+    with top1=True also >= 99% top-1 agreement among the positions whose
+    oracle top-2 gap is outside the bf16 noise band (2 max |delta|): random
+    init leaves many positions with gaps inside it, where either token is a
+    correct greedy choice at this precision."""
+    maxd, agree, hard = parity(gpu, ref)
+    srt = np.sort(np.asarray(ref), axis=-1)
+    near = float(np.mean((srt[..., -1] - srt[..., -2]) <= 2 * maxd))
+    print(f"{what}: max|dlogit| {maxd:.3e}  top1 {agree:.4f}  hard mismatches {hard}  "
+          f"near-tie positions {near:.3f}")
+    assert np.isfinite(gpu).all(), f"{what}: non-finite logits"
+    assert maxd <= tol, f"{what}: max|dlogit| {maxd} > {tol}"
+    assert hard == 0, f"{what}: {hard} top-1 mismatches beyond near ties"
+    if top1:
+        g = np.asarray(gpu).argmax(-1)
+        r = np.asarray(ref).argmax(-1)
+        clear = (srt[..., -1] - srt[..., -2]) > 2 * maxd
+        if clear.sum():
+            assert float(np.mean(g[clear] == r[clear])) >= TOP1_MIN
+
+
+def oracle_decode(o, cache, fed, ctx0):
+    lens = np.asarray(ctx0, dtype=np.int64).copy()
+    outs = []
+    for t in range(fed.shape[1]):
+        outs.append(o.decode_step(fed[:, t], cache, lens))
+        lens += 1
+    return np.stack(outs, 1)
+
+
+@pytest.mark.parametrize("shape,B,S", [(TINY, 2, 20), (TINY, 3, 45), (TINY128, 2, 33)])
+def test_tiny_prefill_all_positions_and_decode_gemv_path(shape, B, S):
+    """B*S <= 64: projections on the decode GEMV, attention on the prefill
+    kernel; every position's logits, then 6 cached decode steps."""
+    ax = _ax()
+    w = gpu_weights(shape)
+    m = create(shape, w, max_batch=4, max_context=128)
+    try:
+        ids = si.make_ids(B, S, shape["V"])
+        lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_ALL, shape["V"])
+        o = oracle_for(shape, w)
+        cache = o.new_contiguous_cache(B, 128)
+        ref = o.prefill(ids, cache)
+        check(lg, ref, what="prefill all")
+        assert np.array_equal(nxt, lg[:, -1].argmax(-1))
+        dl, fed = decode_steps(m, nxt, [S] * B, 6, shape["V"])
+        check(dl, oracle_decode(o, cache, fed, [S] * B), what="decode")
+        assert ax.axon_check_device(m)[0] == 0
+    finally:
+        ax.axon_free(m)
+
+
+@pytest.mark.parametrize("shape,B,S", [(TINY, 2, 100), (TINY128, 1, 300)])
+def test_tiny_prefill_tensor_core_path(shape, B, S):
+    """B*S > 64: projections on the tcgen05 GEMM (ragged 128-row tail)."""
+    ax = _ax()
+    w = gpu_weights(shape)
+    m = create(shape, w, max_batch=2, max_context=320)
+    try:
+        ids = si.make_ids(B, S, shape["V"], seed=5)
+        lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_ALL, shape["V"])
+        o = oracle_for(shape, w)
+        cache = o.new_contiguous_cache(B, 320)
+        ref = o.prefill(ids, cache)
+        check(lg, ref, what="prefill all (tcgen05)")
+        lg2, nxt2 = run_prefill(m, ids, ax.AXON_LOGITS_LAST, shape["V"])
+        check(lg2, ref[:, -1], what="prefill last")
+        assert np.array_equal(nxt2, lg2.argmax(-1))
+        dl, fed = decode_steps(m, nxt2, [S] * B, 4, shape["V"])
+        check(dl, oracle_decode(o, cache, fed, [S] * B), what="decode after tcgen05 prefill")
+        assert ax.axon_check_device(m)[0] == 0
+    finally:
+        ax.axon_free(m)
+
+
+def test_paged_cache_shuffled_blocks_and_placement():
+    ax = _ax()
+    shape = TINY
+    B, S, n_new, max_ctx = 3, 37, 5, 64
+    num_blocks = 40
+    w = gpu_weights(shape)
+    bt_np = si.make_block_table([max_ctx] * B, 16, max_ctx // 16, num_blocks, seed=si.SEED_BLOCKS)
+    m = create(shape, w, max_batch=B, max_context=max_ctx, layout="paged", num_blocks=num_blocks)
+    try:
+        bt = torch.from_numpy(bt_np).cuda()
+        ids = si.make_ids(B, S, shape["V"], seed=7)
+        lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_LAST, shape["V"], block_table=bt)
+        o = oracle_for(shape, w)
+        cache = o.new_paged_cache(num_blocks, 16, bt_np)
+        ref = o.prefill(ids, cache, last_only=True)[:, -1]
+        check(lg, ref, what="paged prefill")
+        dl, fed = decode_steps(m, nxt, [S] * B, n_new, shape["V"], block_table=bt)
+        check(dl, oracle_decode(o, cache, fed, [S] * B), what="paged decode")
+        # Cache placement: every written slot holds the oracle's K/V (bf16),
+        # every other slot of the pool is still zero.
+        v = ax.axon_kv_view_get(m)
+        G, d, L = shape["G"], shape["d"], shape["L"]
+        n_el = L * num_blocks * G * 16 * d
+        assert v.num_blocks == num_blocks and v.elem_bytes == 2
+        kp = device_bytes(v.k_pool, n_el * 2).view(torch.bfloat16).float()
+        kp = kp.view(L, num_blocks, G, 16, d).cpu().numpy()
+        written = np.zeros((num_blocks, 16), dtype=bool)
+        T = S + n_new
+        for b in range(B):
+            for p in range(T):
+                blk, off = bt_np[b][p // 16], p % 16
+                written[blk, off] = True
+                for l in range(L):
+                    ref_k = cache.K[l][blk, off]  # [G, d]
+                    assert np.max(np.abs(kp[l, blk, :, off, :] - ref_k)) <= 2e-2 * (1 + np.abs(ref_k).max())
+        assert np.all(kp.transpose(0, 1, 3, 2, 4)[:, ~written] == 0.0)
+    finally:
+        ax.axon_free(m)
+
+
+def test_fp32_debug_mode_relative_error():
+    ax = _ax()
+    shape = TINY
+    B, S = 2, 70  # > 64 rows: tiled CUDA-core GEMM; decode: fp32 GEMV
+    w = gpu_weights(shape)
+    m = create(shape, w, max_batch=B, max_context=128, fp32=True)
+    try:
+        ids = si.make_ids(B, S, shape["V"], seed=9)
+        lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_ALL, shape["V"])
+        o = oracle_for(shape, w)
+        cache = o.new_contiguous_cache(B, 128)
+        ref = o.prefill(ids, cache)
+        rel = np.max(np.abs(lg - ref)) / np.max(np.abs(ref))
+        print("fp32 prefill rel", rel)
+        assert rel <= FP32_REL_TOL
+        dl, fed = decode_steps(m, nxt, [S] * B, 4, shape["V"])
+        refd = oracle_decode(o, cache, fed, [S] * B)
+        reld = np.max(np.abs(dl - refd)) / np.max(np.abs(refd))
+        print("fp32 decode rel", reld)
+        assert reld <= FP32_REL_TOL
+    finally:
+        ax.axon_free(m)
+
+
+def _workload(name, n_check_steps=None):
+    ax = _ax()
+    wl = si.WORKLOADS[name]
+    shape = si.MODEL_SHAPES[wl["model"]]
+    B, S, n_new = wl["B"], wl["S"], wl["n_new"]
+    steps = n_new - 1 if n_check_steps is None else n_check_steps
+    w = gpu_weights(shape)
+    max_ctx = (S + n_new + 15) // 16 * 16
+    m = create(shape, w, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S)
+    try:
+        ids = si.make_ids(B, S, shape["V"])
+        lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_LAST, shape["V"])
+        dl, fed = decode_steps(m, nxt, [S] * B, steps, shape["V"])
+        o = oracle_for(shape, w)
+        cache = o.new_contiguous_cache(B, max_ctx)
+        ref = o.prefill(ids, cache, last_only=True)[:, -1]
+        refd = oracle_decode(o, cache, fed, [S] * B)
+        check(lg, ref, what=f"{name} prefill")
+        check(dl, refd, what=f"{name} decode")
+        # greedy agreement over every generated token (teacher-forced)
+        check(np.concatenate([lg[:, None], dl], 1), np.concatenate([ref[:, None], refd], 1),
+              what=f"{name} all tokens", top1=B * (steps + 1) >= 100)
+        assert ax.axon_check_device(m)[0] == 0
+    finally:
+        ax.axon_free(m)
+
+
+def test_workload_135m():
+    _workload("135m_b1_s16_n16")
+
+
+@pytest.mark.slow
+def test_workload_0_5b():
+    _workload("0.5b_b1_s512_n128")
