@@ -77,6 +77,7 @@ struct axon_model {
   void* u = nullptr;
   unsigned long long* keys = nullptr;
   float* rinv = nullptr;   // [Mcap] per-row inverse RMS from decode producers
+  SplitKWork splitk{};     // decode projections' cross-CTA split-K workspace
   int* ticket = nullptr;   // last-CTA counter of the residual producers
   float* attn_part = nullptr;
   int* attn_cnt = nullptr;
@@ -304,7 +305,7 @@ struct Proj {
       ns.rinv = true;
     }
     if (gemv) {
-      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep);
+      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk);
       ns.parts = N / 16;
     } else if (m->fp32) {
       rc = launch_gemm_simt(lc, kind, static_cast<const float*>(act), act_stride, static_cast<const float*>(W), M, N,
@@ -387,7 +388,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     h.M = B;
     h.N = m->V;
     CK(launch_gemv(lc, EPI_LOGITS, m->fp32, m->head, m->V, D, static_cast<char*>(m->a) + off,
-                   static_cast<long long>(S) * D, B, h));
+                   static_cast<long long>(S) * D, B, h, m->splitk));
     CK(launch_finalize(lc, m->keys, B, 1, 0, B, next, nullptr));
   }
   return AXON_OK;
@@ -700,6 +701,14 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->rinv = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
   m->ticket = static_cast<int*>(p);
+  m->splitk.max_tiles = 1024;
+  m->splitk.max_ctas = 2048;
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->splitk.max_ctas) * 16 * 64 * 4))) return fail(rc);
+  m->splitk.part = static_cast<float*>(p);
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->splitk.max_tiles) * 4))) return fail(rc);
+  m->splitk.ticket = static_cast<int*>(p);
+  if (cudaMemsetAsync(m->splitk.ticket, 0, static_cast<size_t>(m->splitk.max_tiles) * 4, st) != cudaSuccess)
+    return fail(AXON_ERR_CUDA);
   m->max_splits = 64;
   const int dec_b = cfg->max_batch < 64 ? cfg->max_batch : 64;
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(dec_b) * m->G * m->max_splits * 16 * (m->d + 2) * 4))) return fail(rc);

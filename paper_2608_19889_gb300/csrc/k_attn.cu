@@ -25,6 +25,7 @@
 namespace {
 
 constexpr float NEG_INF = -INFINITY;
+constexpr int DEC_WARPS = 8;  // warps per decode CTA (one key block each per round)
 
 template <int HD>
 AXON_DEV uint32_t swz(uint32_t base, int tok, int ch) {
@@ -148,7 +149,7 @@ AXON_DEV int block_of(const AttnArgs& p, int b, int j, bool& ok) {
 
 // --------------------------------------------------------------- decode
 template <int HD>
-__global__ void __launch_bounds__(128) attn_decode_kernel(AttnArgs p) {
+__global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p) {
   extern __shared__ __align__(128) uint8_t sm[];
   constexpr int TILE = 16 * HD * 2;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, r = lane >> 2, q = lane & 3;
@@ -166,7 +167,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(AttnArgs p) {
   if (T < 1) T = 1;
   const int nblk = (T + 15) >> 4;
   // At least one block per warp; splits beyond the ones needed exit at once.
-  const int per = max((nblk + p.splits - 1) / p.splits, 4);
+  const int per = max((nblk + p.splits - 1) / p.splits, DEC_WARPS);
   const int n_used = (nblk + per - 1) / per;
   if (s >= n_used) return;
   const int jb = s * per, je = min(jb + per, nblk);
@@ -177,7 +178,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(AttnArgs p) {
 
   WarpState<HD> st;
   st.init();
-  const uint32_t wbase = smem_u32(sm) + warp * 4 * TILE;  // [stage][K | V]
+  const uint32_t wbase = smem_u32(sm) + warp * 4 * TILE;  // per warp: [stage][K | V]
   const bf16* kp = static_cast<const bf16*>(p.k);
   const bf16* vp = static_cast<const bf16*>(p.v);
   auto issue = [&](int j, int stg) {
@@ -190,8 +191,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(AttnArgs p) {
   };
   int j = jb + warp, stg = 0;
   if (j < je) issue(j, 0);
-  for (; j < je; j += 4) {
-    const int jn = j + 4;
+  for (; j < je; j += DEC_WARPS) {
+    const int jn = j + DEC_WARPS;
     if (jn < je) {
       issue(jn, stg ^ 1);
       cp_async_wait<1>();
@@ -210,10 +211,10 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(AttnArgs p) {
   st.l1 += __shfl_xor_sync(0xffffffffu, st.l1, 2);
   __syncthreads();
 
-  // Merge the 4 warps' states in shared memory.
-  float* wm = reinterpret_cast<float*>(sm);  // [4][16]
-  float* wl = wm + 64;                       // [4][16]
-  float* wo = wl + 64;                       // [4][16][HD]
+  // Merge the warps' states in shared memory.
+  float* wm = reinterpret_cast<float*>(sm);  // [DEC_WARPS][16]
+  float* wl = wm + DEC_WARPS * 16;           // [DEC_WARPS][16]
+  float* wo = wl + DEC_WARPS * 16;           // [DEC_WARPS][16][HD]
   if (q == 0) {
     wm[warp * 16 + r] = st.m0;
     wm[warp * 16 + r + 8] = st.m1;
@@ -237,11 +238,11 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(AttnArgs p) {
     const int i = idx / HD, dd = idx - i * HD;
     float M = NEG_INF;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w * 16 + i]);
+    for (int w = 0; w < DEC_WARPS; ++w) M = fmaxf(M, wm[w * 16 + i]);
     float O = 0.f, L = 0.f;
     if (M != NEG_INF) {
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
+      for (int w = 0; w < DEC_WARPS; ++w) {
         const float f = exp2f(wm[w * 16 + i] - M);
         O += wo[(w * 16 + i) * HD + dd] * f;
         L += wl[w * 16 + i] * f;
@@ -294,11 +295,20 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(AttnArgs p) {
   __syncthreads();
   for (int idx = threadIdx.x; idx < HPG * HD; idx += blockDim.x) {
     const int i = idx / HD, dd = idx - i * HD;
-    float O = 0.f;
-#pragma unroll 8
-    for (int t = 0; t < n_used; ++t) O += cw[i][t] * __ldcg(part + (static_cast<long long>(t) * 16 + i) * rowlen + dd);
+    const float* pc = part + static_cast<long long>(i) * rowlen + dd;
+    float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
+    int t = 0;
+    for (; t + 4 <= n_used; t += 4) {
+      const float v0 = __ldcg(pc + (t + 0) * 16 * rowlen), v1 = __ldcg(pc + (t + 1) * 16 * rowlen);
+      const float v2 = __ldcg(pc + (t + 2) * 16 * rowlen), v3 = __ldcg(pc + (t + 3) * 16 * rowlen);
+      O0 += cw[i][t] * v0;
+      O1 += cw[i][t + 1] * v1;
+      O2 += cw[i][t + 2] * v2;
+      O3 += cw[i][t + 3] * v3;
+    }
+    for (; t < n_used; ++t) O0 += cw[i][t] * __ldcg(pc + t * 16 * rowlen);
     bf16* og = static_cast<bf16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
-    *og = __float2bfloat16_rn(O * cinv[i]);
+    *og = __float2bfloat16_rn(((O0 + O1) + (O2 + O3)) * cinv[i]);
   }
   if (threadIdx.x == 0) p.counter[b * p.G + g] = 0;
 }
@@ -461,14 +471,14 @@ cudaError_t launch_k(const LaunchCtx& lc, K kernel, dim3 grid, dim3 block, size_
 }
 
 template <int HD>
-constexpr size_t decode_smem() { return 4 * 4 * 16 * HD * 2; }  // 4 warps x 2 stages x (K, V)
+constexpr size_t decode_smem() { return DEC_WARPS * 4 * 16 * HD * 2; }  // warps x 2 stages x (K, V)
 template <int HD>
 constexpr size_t prefill_smem() { return 2 * 4 * 2 * 16 * HD * 2; }  // 2 stages x 4 blocks x (K, V)
 
 template <int HD>
 cudaError_t decode_hd(const LaunchCtx& lc, const AttnArgs& a, int B) {
   const size_t smem = decode_smem<HD>();
-  return launch_k(lc, attn_decode_kernel<HD>, dim3(a.splits, a.G, B), dim3(128), smem, a);
+  return launch_k(lc, attn_decode_kernel<HD>, dim3(a.splits, a.G, B), dim3(DEC_WARPS * 32), smem, a);
 }
 
 template <int HD>

@@ -59,7 +59,7 @@ AXON_DEV void finish_rinv(const EpiArgs& ep, int B, int nparts) {
 template <int NT, int KIND>
 __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __restrict__ W, int N, int K,
                                                                const bf16* __restrict__ act, long long act_stride,
-                                                               int B, EpiArgs ep) {
+                                                               int B, EpiArgs ep, SplitK sk) {
   constexpr int TOK = NT * 8;
   __shared__ float red[GEMV_KW][16][TOK + 1];
   __shared__ float rinv_s[TOK];
@@ -71,9 +71,12 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __re
   const int r = lane >> 2, q = lane & 3;
   const int n0 = blockIdx.x * 16;
   const int row0 = min(n0 + r, N - 1), row1 = min(n0 + r + 8, N - 1);
-  const bf16* w0 = W + static_cast<long long>(row0) * K + 16 * q;
-  const bf16* w1 = W + static_cast<long long>(row1) * K + 16 * q;
-  const int nchunks = K >> 6;
+  // K-split blockIdx.y covers chunks [c_begin, c_end) of 64 columns.
+  const int per = (K >> 6) / sk.count;
+  const int c_begin = blockIdx.y * per;
+  const int nchunks = (blockIdx.y == sk.count - 1) ? (K >> 6) - c_begin : per;
+  const bf16* w0 = W + static_cast<long long>(row0) * K + 16 * q + c_begin * 64;
+  const bf16* w1 = W + static_cast<long long>(row1) * K + 16 * q + c_begin * 64;
 
   float acc[NT][4];
 #pragma unroll
@@ -85,7 +88,7 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __re
   for (int t = 0; t < NT; ++t) {
     const int tok = t * 8 + r;
     aval[t] = tok < B;
-    arow[t] = act + static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q;
+    arow[t] = act + static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q + c_begin * 64;
   }
 
   auto chunk = [&](int c, const uint4& wa0, const uint4& wa1, const uint4& wb0, const uint4& wb1) {
@@ -161,8 +164,8 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __re
   __syncthreads();
 
   const int b = threadIdx.x;
+  float v[16];
   if (b < B) {
-    float v[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       float s = 0.f;
@@ -170,6 +173,34 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __re
       for (int w = 0; w < GEMV_KW; ++w) s += red[w][i][b];
       v[i] = s;
     }
+  }
+  if (sk.count > 1) {
+    // Cross-CTA split-K: publish this split's partial tile; the last split to
+    // arrive sums all of them in split order (deterministic) and runs the
+    // epilogue. No CTA waits on another.
+    __shared__ int last_split;
+    float* pt = sk.part + (static_cast<long long>(blockIdx.x) * sk.count) * 16 * 64;
+    if (b < B) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) pt[(blockIdx.y * 16 + i) * 64 + b] = v[i];
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) last_split = (atomicAdd(sk.ticket + blockIdx.x, 1) == sk.count - 1);
+    __syncthreads();
+    if (!last_split) return;
+    __threadfence();
+    if (b < B) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      for (int y = 0; y < sk.count; ++y) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] += __ldcg(pt + (y * 16 + i) * 64 + b);
+      }
+    }
+    if (threadIdx.x == 0) sk.ticket[blockIdx.x] = 0;
+  }
+  if (b < B) {
     if (KIND == EPI_QKV) {
       epi_qkv16<bf16>(ep, b, n0, v, rinv_s[b]);
     } else if (KIND == EPI_RESID) {
@@ -231,11 +262,11 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_f32_kernel(const float* __r
 }
 
 template <typename T>
-__global__ void __launch_bounds__(128) embed_kernel(const T* __restrict__ E, int V, int D, const int* __restrict__ ids,
+__global__ void __launch_bounds__(256) embed_kernel(const T* __restrict__ E, int V, int D, const int* __restrict__ ids,
                                                     float* __restrict__ x, T* __restrict__ a,
                                                     const float* __restrict__ g, float* __restrict__ ss, int ss_stride,
                                                     float* __restrict__ rinv, float eps, int* err) {
-  __shared__ float red[4];
+  __shared__ float red[8];
   grid_dep_launch();
   grid_dep_wait();
   const int m = blockIdx.x;
@@ -248,17 +279,26 @@ __global__ void __launch_bounds__(128) embed_kernel(const T* __restrict__ E, int
   float* xr = x + static_cast<long long>(m) * D;
   T* ar = a + static_cast<long long>(m) * D;
   float s = 0.f;
-  for (int k = threadIdx.x; k < D; k += blockDim.x) {
-    const float v = to_f(e[k]);
-    xr[k] = v;
-    ar[k] = from_f<T>(v * g[k]);
-    s += v * v;
+  // 8 consecutive elements per thread and step (D is a multiple of 64).
+  for (int k = threadIdx.x * 8; k < D; k += blockDim.x * 8) {
+    float v[8], ag[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = to_f(e[k + i]);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      ag[i] = v[i] * g[k + i];
+      s += v[i] * v[i];
+    }
+    reinterpret_cast<float4*>(xr + k)[0] = make_float4(v[0], v[1], v[2], v[3]);
+    reinterpret_cast<float4*>(xr + k)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    store8<T>(ar + k, ag);
   }
   s = warp_sum(s);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
   __syncthreads();
   if (threadIdx.x == 0) {
-    const float tot = red[0] + red[1] + red[2] + red[3];
+    float tot = 0.f;
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) tot += red[w];
     ss[static_cast<long long>(m) * ss_stride] = tot;
     if (rinv) rinv[m] = 1.0f / sqrtf(tot / static_cast<float>(D) + eps);
   }
@@ -296,22 +336,38 @@ cudaError_t launch_k(const LaunchCtx& lc, K kernel, dim3 grid, dim3 block, size_
 
 template <int NT>
 cudaError_t gemv_nt(const LaunchCtx& lc, int kind, const void* W, int N, int K, const void* act, long long st, int B,
-                    const EpiArgs& ep) {
-  const dim3 grid((N + 15) / 16), block(GEMV_KW * 32);
+                    const EpiArgs& ep, SplitK sk) {
+  const dim3 grid((N + 15) / 16, sk.count), block(GEMV_KW * 32);
   const bf16* w = static_cast<const bf16*>(W);
   const bf16* a = static_cast<const bf16*>(act);
   switch (kind) {
-    case EPI_QKV: return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV>, grid, block, 0, w, N, K, a, st, B, ep);
-    case EPI_RESID: return launch_k(lc, gemv_mma_kernel<NT, EPI_RESID>, grid, block, 0, w, N, K, a, st, B, ep);
-    case EPI_SWIGLU: return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU>, grid, block, 0, w, N, K, a, st, B, ep);
-    default: return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS>, grid, block, 0, w, N, K, a, st, B, ep);
+    case EPI_QKV: return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV>, grid, block, 0, w, N, K, a, st, B, ep, sk);
+    case EPI_RESID: return launch_k(lc, gemv_mma_kernel<NT, EPI_RESID>, grid, block, 0, w, N, K, a, st, B, ep, sk);
+    case EPI_SWIGLU: return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU>, grid, block, 0, w, N, K, a, st, B, ep, sk);
+    default: return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS>, grid, block, 0, w, N, K, a, st, B, ep, sk);
   }
+}
+
+// K-split count: enough CTAs for ~4 per SM, each warp keeping >= 2 chunks,
+// bounded by the partial-tile workspace.
+SplitK choose_split(const LaunchCtx& lc, int N, int K, const SplitKWork& wk) {
+  SplitK sk{1, wk.part, wk.ticket};
+  if (!wk.part || !wk.ticket) return sk;
+  const int tiles = (N + 15) / 16;
+  const int target = 4 * lc.num_sms;
+  if (tiles >= target || tiles > wk.max_tiles) return sk;
+  int ks = (target + tiles - 1) / tiles;
+  const int max_by_k = (K >> 6) / (2 * GEMV_KW);
+  if (ks > max_by_k) ks = max_by_k;
+  while (ks > 1 && static_cast<long long>(tiles) * ks > wk.max_ctas) --ks;
+  sk.count = ks < 1 ? 1 : ks;
+  return sk;
 }
 
 }  // namespace
 
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
-                        long long act_stride, int B, const EpiArgs& ep) {
+                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk) {
   if (B < 1 || B > 64 || (K & 63) || N < 1) return cudaErrorInvalidValue;
   if (fp32) {
     const dim3 grid((N + 15) / 16), block(GEMV_KW * 32);
@@ -324,18 +380,19 @@ cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W,
       default: return launch_k(lc, gemv_f32_kernel<EPI_LOGITS>, grid, block, 0, w, N, K, a, act_stride, B, ep);
     }
   }
-  if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep);
-  if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep);
-  if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep);
-  return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep);
+  const SplitK sk = choose_split(lc, N, K, wk);
+  if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
+  if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
+  if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
+  return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
 }
 
 cudaError_t launch_embed(const LaunchCtx& lc, bool fp32, const void* E, int V, int D, const int* ids, int M, float* x,
                          void* a, const float* g, float* ss, int ss_stride, float* rinv, float eps, int* err) {
   if (fp32)
-    return launch_k(lc, embed_kernel<float>, dim3(M), dim3(128), 0, static_cast<const float*>(E), V, D, ids, x,
+    return launch_k(lc, embed_kernel<float>, dim3(M), dim3(256), 0, static_cast<const float*>(E), V, D, ids, x,
                     static_cast<float*>(a), g, ss, ss_stride, rinv, eps, err);
-  return launch_k(lc, embed_kernel<bf16>, dim3(M), dim3(128), 0, static_cast<const bf16*>(E), V, D, ids, x,
+  return launch_k(lc, embed_kernel<bf16>, dim3(M), dim3(256), 0, static_cast<const bf16*>(E), V, D, ids, x,
                   static_cast<bf16*>(a), g, ss, ss_stride, rinv, eps, err);
 }
 

@@ -16,9 +16,22 @@ struct LaunchCtx {
 };
 
 // ---- decode projections (k_gemv.cu): out[b][n] = act[b] . W[n], B <= 64
-// tokens, 16 weight rows per CTA, fused epilogue `kind`.
+// tokens, 16 weight rows per CTA, fused epilogue `kind`. Projections with
+// few row tiles split K over CTAs; the partial tiles go to `part` and the
+// per-tile tickets (zeroed, re-armed by the kernel) pick the CTA that sums.
+struct SplitKWork {
+  float* part;     // [max_ctas][16][64]
+  int* ticket;     // [max_tiles]
+  int max_tiles;
+  int max_ctas;
+};
+struct SplitK {
+  int count;
+  float* part;
+  int* ticket;
+};
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
-                        long long act_stride, int B, const EpiArgs& ep);
+                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk);
 
 // ---- embedding gather producing x, a = x * g and the row sum of squares.
 // rinv (optional): 1 / sqrt(mean(x^2) + eps) per row.
