@@ -291,6 +291,37 @@ def main():
     # embed + 5 per layer + LM head + finaliser, for the prefill and each decode step
     launches_per_step = (5 * m["L"] + 3) * (1 + n_new)
 
+    # ---- per-kernel timing (CUDA events around each launch, no graph) of one
+    # prefill and of decode steps at the start, middle and end of the run.
+    with torch.cuda.stream(st):
+        prof_pre = ax.axon_profile_prefill(model, ids, next_tokens=tok, stream=st)
+        prof_dec = {}
+        for T in (S, S + n_new // 2, S + n_new - 1):
+            ctx.fill_(T)
+            for e in ax.axon_profile_decode_step(model, tok, ctx, next_tokens=tok, stream=st):
+                a = prof_dec.setdefault(e["name"], dict(launches=0, total_ms=0.0, bytes=0.0, flops=0.0))
+                for k in ("launches", "total_ms", "bytes", "flops"):
+                    a[k] += e[k]
+    torch.cuda.synchronize()
+    # whole-run weight of each kernel kind: prefill once + n_new decode steps
+    kinds = []
+    for e in prof_pre:
+        kinds.append((e["total_ms"], e["name"], e["launches"], e["total_ms"], e["bytes"], e["flops"]))
+    for name, e in prof_dec.items():
+        kinds.append((e["total_ms"] / 3 * n_new, name, e["launches"], e["total_ms"], e["bytes"], e["flops"]))
+    kinds.sort(reverse=True)
+    _, top_name, top_n, top_ms, top_bytes, top_flops = kinds[0]
+    per_launch_ms = top_ms / top_n
+    if top_name.startswith("prefill") and top_flops > 0 and top_bytes / top_flops < 0.05:
+        ach = top_flops / top_n / (per_launch_ms / 1e3) / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": tf_burst, "unit": "TFLOP/s", "frac": ach / tf_burst}
+    else:
+        ach = top_bytes / top_n / (per_launch_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm}
+    roof.update({"kernel": top_name, "launch_ms": per_launch_ms, "per_launch_units": (top_bytes if roof["bound"] == "hbm" else top_flops) / top_n,
+                 "peak_kind": peak_kind, "traffic": None})
+    kernel_table = {k[1]: {"share_of_run": k[0] / sum(x[0] for x in kinds), "launch_ms": k[3] / k[2]} for k in kinds}
+
     out = {
         "metric": METRIC,
         "value": world * B * n_new / (ms / 1e3),
@@ -311,11 +342,14 @@ def main():
         "decode_tok_s": world * B * n_new / (dec_ms / 1e3),
         "prefill_ms": pre_ms,
         "decode_ms": dec_ms,
-        "roofline": {"bound": "hbm", "kernel": "decode step (fused GEMV/attention chain, CUDA graph)",
-                     "achieved": dec_gbs, "peak": hbm, "unit": "GB/s", "frac": dec_gbs / hbm,
-                     "peak_kind": peak_kind, "traffic": None},
-        "roofline_prefill": {"bound": "tensor", "achieved": pre_tflops, "peak": tf_burst, "unit": "TFLOP/s",
-                             "frac": pre_tflops / tf_burst, "peak_kind": peak_kind},
+        "roofline": roof,
+        "roofline_decode_step": {"bound": "hbm", "achieved": dec_gbs, "peak": hbm, "unit": "GB/s",
+                                 "frac": dec_gbs / hbm, "peak_kind": peak_kind,
+                                 "what": "all decode bytes (weights + KV + logits) / timed decode phase"},
+        "roofline_prefill_phase": {"bound": "tensor", "achieved": pre_tflops, "peak": tf_burst, "unit": "TFLOP/s",
+                                   "frac": pre_tflops / tf_burst, "peak_kind": peak_kind,
+                                   "what": "prefill FLOPs / timed prefill phase"},
+        "kernels": kernel_table,
         "e2e": {"value": world * e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": B * S * 4,
                 "d2h_bytes_per_step": B * n_new * 4},
         "gpu_launches": args.steps * launches_per_step,

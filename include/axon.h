@@ -179,6 +179,34 @@ typedef struct axon_kv_view {
 } axon_kv_view;
 int axon_kv_view_get(const axon_model* m, axon_kv_view* out);
 
+/* Per-kernel timing of one pass (tracing hook; the paper profiles its
+ * generate loop's GPU kernels, appendix "Python Overhead", Table 5).
+ * The pass runs exactly as axon_prefill / axon_decode_step would (same
+ * kernels, same side effects on the cache and, for decode, on
+ * d_context_lens), but launched one kernel at a time with a CUDA event pair
+ * around each launch and no CUDA graph or programmatic overlap, then
+ * synchronised. Entries aggregate launches of one kind:
+ *   name       kernel kind ("decode_gateup", "prefill_qkv", ...)
+ *   launches   number of launches in the pass
+ *   total_ms   summed event time of those launches
+ *   bytes      algorithmic HBM bytes of those launches (weights once, KV
+ *              cache reads/writes, activations in/out)
+ *   flops      algorithmic floating-point operations
+ * `out` receives at most max_out entries (16 suffice); *n_out their count.
+ * Prefill logits are not stored (LAST mode, next tokens only). */
+typedef struct axon_kernel_time {
+  char name[32];
+  int32_t launches;
+  float total_ms;
+  double bytes;
+  double flops;
+} axon_kernel_time;
+int axon_profile_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,
+                             const int32_t* d_block_table, int32_t* d_next, void* stream, axon_kernel_time* out,
+                             int32_t max_out, int32_t* n_out);
+int axon_profile_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S, const int32_t* d_block_table,
+                         int32_t* d_next, void* stream, axon_kernel_time* out, int32_t max_out, int32_t* n_out);
+
 /* Release everything the model owns. NULL is a no-op. */
 void axon_free(axon_model* m);
 

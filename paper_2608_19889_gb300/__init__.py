@@ -30,7 +30,8 @@ AXON_DTYPE_BF16, AXON_DTYPE_F32 = 0, 1
 AXON_LOGITS_LAST, AXON_LOGITS_ALL = 0, 1
 
 EXPORTED = ["axon_model_create", "axon_prefill", "axon_decode_step", "axon_reset", "axon_check_device",
-            "axon_kv_view_get", "axon_free", "axon_status_string"]
+            "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill", "axon_free",
+            "axon_status_string"]
 
 
 class axon_config(ctypes.Structure):
@@ -50,6 +51,11 @@ class axon_tensor(ctypes.Structure):
 class axon_kv_view(ctypes.Structure):
     _fields_ = [("k_pool", ctypes.c_void_p), ("v_pool", ctypes.c_void_p), ("num_blocks", ctypes.c_int64),
                 ("blocks_per_seq", ctypes.c_int32), ("block_size", ctypes.c_int32), ("elem_bytes", ctypes.c_int32)]
+
+
+class axon_kernel_time(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int32), ("total_ms", ctypes.c_float),
+                ("bytes", ctypes.c_double), ("flops", ctypes.c_double)]
 
 
 class AxonError(RuntimeError):
@@ -76,12 +82,15 @@ def lib() -> ctypes.CDLL:
         L.axon_reset.argtypes = [vp]
         L.axon_check_device.argtypes = [vp, vp, p_i32]
         L.axon_kv_view_get.argtypes = [vp, ctypes.POINTER(axon_kv_view)]
+        L.axon_profile_decode_step.argtypes = [vp, vp, i32, vp, vp, vp, vp, ctypes.POINTER(axon_kernel_time), i32,
+                                               p_i32]
+        L.axon_profile_prefill.argtypes = [vp, vp, i32, i32, vp, vp, vp, ctypes.POINTER(axon_kernel_time), i32, p_i32]
         L.axon_free.argtypes = [vp]
         L.axon_free.restype = None
         L.axon_status_string.argtypes = [ctypes.c_int]
         L.axon_status_string.restype = ctypes.c_char_p
         for n in ("axon_model_create", "axon_prefill", "axon_decode_step", "axon_reset", "axon_check_device",
-                  "axon_kv_view_get"):
+                  "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill"):
             getattr(L, n).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -168,6 +177,32 @@ def axon_kv_view_get(m) -> axon_kv_view:
     v = axon_kv_view()
     _check("axon_kv_view_get", lib().axon_kv_view_get(m, ctypes.byref(v)))
     return v
+
+
+def _profile_result(arr, n):
+    return [dict(name=arr[i].name.decode(), launches=arr[i].launches, total_ms=arr[i].total_ms,
+                 bytes=arr[i].bytes, flops=arr[i].flops) for i in range(n.value)]
+
+
+def axon_profile_decode_step(m, tokens, context_lens, block_table=None, next_tokens=None, stream=None):
+    """Per-kernel-kind timing of one decode step (runs the step)."""
+    arr = (axon_kernel_time * 16)()
+    n = ctypes.c_int32(0)
+    B = tokens.shape[0]
+    _check("axon_profile_decode_step", lib().axon_profile_decode_step(
+        m, _ptr(tokens), B, _ptr(context_lens), _ptr(block_table), _ptr(next_tokens), _stream(stream), arr, 16,
+        ctypes.byref(n)))
+    return _profile_result(arr, n)
+
+
+def axon_profile_prefill(m, ids, block_table=None, next_tokens=None, stream=None):
+    """Per-kernel-kind timing of one prefill (LAST-position logits not stored)."""
+    arr = (axon_kernel_time * 16)()
+    n = ctypes.c_int32(0)
+    B, S = ids.shape
+    _check("axon_profile_prefill", lib().axon_profile_prefill(
+        m, _ptr(ids), B, S, _ptr(block_table), _ptr(next_tokens), _stream(stream), arr, 16, ctypes.byref(n)))
+    return _profile_result(arr, n)
 
 
 def axon_free(m):

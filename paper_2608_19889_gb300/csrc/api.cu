@@ -286,6 +286,43 @@ void set_norm(const axon_model* m, const NormState& ns, EpiArgs& e, int row_offs
   }
 }
 
+// Optional per-launch timing (axon_profile_*): an event pair around every
+// kernel, with the launch's algorithmic bytes and FLOPs.
+struct Prof {
+  struct Entry {
+    std::string name;
+    cudaEvent_t a, b;
+    double bytes, flops;
+  };
+  cudaStream_t st;
+  std::vector<Entry> entries;
+  void begin(const char* name) {
+    Entry e{name, nullptr, nullptr, 0, 0};
+    cudaEventCreate(&e.a);
+    cudaEventCreate(&e.b);
+    cudaEventRecord(e.a, st);
+    entries.push_back(e);
+  }
+  void end(double bytes, double flops) {
+    Entry& e = entries.back();
+    cudaEventRecord(e.b, st);
+    e.bytes = bytes;
+    e.flops = flops;
+  }
+  ~Prof() {
+    for (auto& e : entries) {
+      cudaEventDestroy(e.a);
+      cudaEventDestroy(e.b);
+    }
+  }
+};
+inline void pbeg(Prof* p, const char* n) {
+  if (p) p->begin(n);
+}
+inline void pend(Prof* p, double bytes, double flops) {
+  if (p) p->end(bytes, flops);
+}
+
 // One projection: picks the kernel for the mode and row count.
 struct Proj {
   const axon_model* m;
@@ -320,13 +357,19 @@ struct Proj {
 };
 
 int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32_t* bt, int logits_mode, float* logits,
-                    int32_t* next, cudaStream_t st) {
+                    int32_t* next, cudaStream_t st, Prof* pf = nullptr) {
   const int M = B * S;
-  LaunchCtx lc{st, m->use_pdl, m->num_sms};
+  LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms};
+  const double es = static_cast<double>(m->esz);
+  const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * m->H * m->d * es,
+               wgu = 2.0 * m->F * m->D * es, wdn = static_cast<double>(m->D) * m->F * es,
+               whd = static_cast<double>(m->V) * m->D * es;
   Proj pj{m, lc};
   const int D = m->D, Hd = m->H * m->d;
+  pbeg(pf, "embed");
   CK(launch_embed(lc, m->fp32, m->embed, m->V, D, ids, M, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
                   m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err));
+  pend(pf, static_cast<double>(M) * D * (es + 4 + es), 0);
   NormState ns;
   ns.rinv = true;
   for (int l = 0; l < m->L; ++l) {
@@ -337,12 +380,17 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     e.bias = w.bqkv;
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
+    pbeg(pf, "prefill_qkv");
     pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, M, e);
     CK(pj.rc);
+    pend(pf, wq + M * (D + m->Nqkv) * es, 2.0 * M * m->Nqkv * D);
 
     AttnArgs at = base_attn(m, l, bt);
     at.S = S;
+    pbeg(pf, "prefill_attention");
     CK(launch_attn_prefill(lc, m->fp32, at, B));
+    pend(pf, static_cast<double>(M) * (m->H + 2 * m->G) * m->d * es + static_cast<double>(M) * Hd * es,
+         4.0 * B * m->H * m->d * (static_cast<double>(S) * (S + 1) / 2));
 
     EpiArgs r = base_epi(m);
     r.S = S;
@@ -351,15 +399,19 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     r.gain = w.g2;
     r.ss_out = m->ss;
     r.ss_out_stride = m->Pmax;
+    pbeg(pf, "prefill_o");
     ns = pj.run(EPI_RESID, w.wo, &w.m_o, D, Hd, m->o, Hd, M, r);
     CK(pj.rc);
+    pend(pf, wo + M * (Hd * es + D * (8 + es)), 2.0 * M * D * Hd);
 
     EpiArgs g = base_epi(m);
     g.S = S;
     set_norm(m, ns, g);
     g.u_out = m->u;
+    pbeg(pf, "prefill_gateup");
     pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, M, g);
     CK(pj.rc);
+    pend(pf, wgu + M * (D + m->F) * es, 2.0 * M * 2 * m->F * D);
 
     EpiArgs dn = base_epi(m);
     dn.S = S;
@@ -368,8 +420,10 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
+    pbeg(pf, "prefill_down");
     ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, M, dn);
     CK(pj.rc);
+    pend(pf, wdn + M * (m->F * es + D * (8 + es)), 2.0 * M * D * m->F);
   }
   EpiArgs h = base_epi(m);
   h.S = S;
@@ -378,29 +432,43 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
   h.logits_stride = m->V;
   if (logits_mode == AXON_LOGITS_ALL) {
     set_norm(m, ns, h);
+    pbeg(pf, "prefill_lm_head");
     pj.run(EPI_LOGITS, m->head, &m->m_head, m->V, D, m->a, D, M, h);
     CK(pj.rc);
+    pend(pf, whd + M * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * M * m->V * D);
+    pbeg(pf, "finalize");
     CK(launch_finalize(lc, m->keys, M, S, S - 1, B, next, nullptr));
+    pend(pf, 8.0 * M, 0);
   } else {
     // Last position of each sequence: rows S-1, 2S-1, ... as a B-row GEMV.
     const size_t off = static_cast<size_t>(S - 1) * D * m->esz;
     set_norm(m, ns, h, S - 1, S);
     h.M = B;
     h.N = m->V;
+    pbeg(pf, "prefill_lm_head");
     CK(launch_gemv(lc, EPI_LOGITS, m->fp32, m->head, m->V, D, static_cast<char*>(m->a) + off,
                    static_cast<long long>(S) * D, B, h, m->splitk));
+    pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
+    pbeg(pf, "finalize");
     CK(launch_finalize(lc, m->keys, B, 1, 0, B, next, nullptr));
+    pend(pf, 8.0 * B, 0);
   }
   return AXON_OK;
 }
 
 int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt, float* logits,
-                   int32_t* next, cudaStream_t st) {
-  LaunchCtx lc{st, m->use_pdl, m->num_sms};
+                   int32_t* next, cudaStream_t st, Prof* pf = nullptr, double kv_tokens = 0) {
+  LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms};
   Proj pj{m, lc};
   const int D = m->D, Hd = m->H * m->d;
+  const double es = static_cast<double>(m->esz);
+  const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * Hd * es,
+               wgu = 2.0 * m->F * m->D * es, wdn = static_cast<double>(m->D) * m->F * es,
+               whd = static_cast<double>(m->V) * m->D * es;
+  pbeg(pf, "embed");
   CK(launch_embed(lc, m->fp32, m->embed, m->V, D, tokens, B, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
                   m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err));
+  pend(pf, static_cast<double>(B) * D * (es + 4 + es), 0);
   NormState ns;
   ns.rinv = true;
   const int splits = m->fp32 ? 1 : attn_decode_splits(B, m->G, m->blocks_per_seq, m->num_sms);
@@ -413,8 +481,10 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     e.bias = w.bqkv;
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
+    pbeg(pf, "decode_qkv");
     pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e);
     CK(pj.rc);
+    pend(pf, wq + B * (D + m->Nqkv) * es, 2.0 * B * m->Nqkv * D);
 
     AttnArgs at = base_attn(m, l, bt);
     at.ctx = ctx;
@@ -422,7 +492,9 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     at.splits = splits;
     at.part = m->attn_part;
     at.counter = m->attn_cnt;
+    pbeg(pf, "decode_attention");
     CK(launch_attn_decode(lc, m->fp32, at, B));
+    pend(pf, kv_tokens * 2.0 * m->G * m->d * es + 2.0 * B * Hd * es, 4.0 * kv_tokens * m->H * m->d);
 
     EpiArgs r = base_epi(m);
     r.S = 1;
@@ -432,16 +504,20 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     r.gain = w.g2;
     r.ss_out = m->ss;
     r.ss_out_stride = m->Pmax;
+    pbeg(pf, "decode_o");
     ns = pj.run(EPI_RESID, w.wo, nullptr, D, Hd, m->o, Hd, B, r);
     CK(pj.rc);
+    pend(pf, wo + B * (Hd * es + D * (8 + es)), 2.0 * B * D * Hd);
 
     EpiArgs g = base_epi(m);
     g.S = 1;
     g.ctx = ctx;
     set_norm(m, ns, g);
     g.u_out = m->u;
+    pbeg(pf, "decode_gateup");
     pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g);
     CK(pj.rc);
+    pend(pf, wgu + B * (D + m->F) * es, 2.0 * B * 2 * m->F * D);
 
     EpiArgs dn = base_epi(m);
     dn.S = 1;
@@ -451,8 +527,10 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
+    pbeg(pf, "decode_down");
     ns = pj.run(EPI_RESID, w.wd, nullptr, D, m->F, m->u, m->F, B, dn);
     CK(pj.rc);
+    pend(pf, wdn + B * (m->F * es + D * (8 + es)), 2.0 * B * D * m->F);
   }
   EpiArgs h = base_epi(m);
   h.S = 1;
@@ -461,9 +539,13 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   h.keys = m->keys;
   h.logits = logits;
   h.logits_stride = m->V;
+  pbeg(pf, "decode_lm_head");
   pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h);
   CK(pj.rc);
+  pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
+  pbeg(pf, "finalize");
   CK(launch_finalize(lc, m->keys, B, 1, 0, B, next, ctx));
+  pend(pf, 16.0 * B, 0);
   return AXON_OK;
 }
 
@@ -799,6 +881,70 @@ int axon_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t*
   }
   CK(cudaGraphLaunch(it->second, st));
   return AXON_OK;
+}
+
+namespace {
+int collect_profile(Prof& pf, axon_kernel_time* out, int32_t max_out, int32_t* n_out) {
+  CK(cudaStreamSynchronize(pf.st));
+  std::vector<axon_kernel_time> agg;
+  for (auto& e : pf.entries) {
+    float ms = 0.f;
+    CK(cudaEventElapsedTime(&ms, e.a, e.b));
+    axon_kernel_time* slot = nullptr;
+    for (auto& a : agg)
+      if (e.name == a.name) slot = &a;
+    if (!slot) {
+      axon_kernel_time t;
+      memset(&t, 0, sizeof(t));
+      snprintf(t.name, sizeof(t.name), "%s", e.name.c_str());
+      agg.push_back(t);
+      slot = &agg.back();
+    }
+    slot->launches += 1;
+    slot->total_ms += ms;
+    slot->bytes += e.bytes;
+    slot->flops += e.flops;
+  }
+  const int n = static_cast<int>(agg.size()) < max_out ? static_cast<int>(agg.size()) : max_out;
+  for (int i = 0; i < n; ++i) out[i] = agg[i];
+  if (n_out) *n_out = n;
+  return AXON_OK;
+}
+}  // namespace
+
+int axon_profile_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,
+                             const int32_t* d_block_table, int32_t* d_next, void* stream, axon_kernel_time* out,
+                             int32_t max_out, int32_t* n_out) {
+  if (!m || !d_tokens || !d_context_lens || !d_next || !out || max_out < 1) return AXON_ERR_INVALID_ARG;
+  if (B < 1 || B > m->cfg.max_batch || B > 64) return AXON_ERR_INVALID_ARG;
+  const bool paged = m->cfg.kv_layout == AXON_KV_PAGED;
+  if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  std::vector<int32_t> h(B);
+  CK(cudaMemcpyAsync(h.data(), d_context_lens, B * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  CK(cudaStreamSynchronize(st));
+  double kv_tokens = 0;
+  for (int b = 0; b < B; ++b) kv_tokens += h[b] + 1;
+  Prof pf;
+  pf.st = st;
+  const int rc = enqueue_decode(m, d_tokens, B, d_context_lens, d_block_table, nullptr, d_next, st, &pf, kv_tokens);
+  if (rc) return rc;
+  return collect_profile(pf, out, max_out, n_out);
+}
+
+int axon_profile_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S, const int32_t* d_block_table,
+                         int32_t* d_next, void* stream, axon_kernel_time* out, int32_t max_out, int32_t* n_out) {
+  if (!m || !d_ids || !out || max_out < 1) return AXON_ERR_INVALID_ARG;
+  if (B < 1 || B > m->cfg.max_batch || S < 1 || S > m->cfg.max_context) return AXON_ERR_INVALID_ARG;
+  if (static_cast<long long>(B) * S > m->cfg.max_prefill_tokens || B > 64) return AXON_ERR_INVALID_ARG;
+  const bool paged = m->cfg.kv_layout == AXON_KV_PAGED;
+  if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Prof pf;
+  pf.st = st;
+  const int rc = enqueue_prefill(m, d_ids, B, S, d_block_table, AXON_LOGITS_LAST, nullptr, d_next, st, &pf);
+  if (rc) return rc;
+  return collect_profile(pf, out, max_out, n_out);
 }
 
 int axon_reset(axon_model* m) {
