@@ -207,6 +207,32 @@ int axon_profile_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, 
 int axon_profile_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S, const int32_t* d_block_table,
                          int32_t* d_next, void* stream, axon_kernel_time* out, int32_t max_out, int32_t* n_out);
 
+/* Decode step that allocates nothing (no counterpart in the paper; a
+ * deployment affordance of this library). Same arguments, results and
+ * side effects as axon_decode_step, for callers that must not allocate on
+ * the call path -- for example a serving loop running while another
+ * component owns the device memory pool, or a caller whose allocator is
+ * locked after start-up: axon_decode_step instantiates a CUDA graph the
+ * first time it meets a new (B, pointer set), and instantiation allocates.
+ * This entry point instead launches the step's kernels directly, and the
+ * split-KV attention takes its merge scratch from a fixed, library-owned
+ * device array (256 merge slots, about 2.1 MB, resident on every device
+ * that loads the library until the process exits) instead of from memory
+ * allocated per call. It calls no cudaMalloc, cudaFree or graph
+ * instantiation.
+ *   Limits: B * num_key_value_heads <= 256 and head_dim <= 128, else
+ *   AXON_ERR_UNSUPPORTED; bf16 precision only (AXON_ERR_UNSUPPORTED in
+ *   AXON_FP32_DEBUG).
+ *   First call on a device: resolves the array's device address (with that
+ *   device current) -- make that first call before any stream capture.
+ *   Every call shares the one array and clears the parts that must start
+ *   at zero: calls that overlap on the GPU (different streams, or several
+ *   models at once) race on it and must be serialised by the caller.
+ * The key-split count may differ from axon_decode_step's, so logits can
+ * differ from it by floating-point rounding of the merge. */
+int axon_decode_step_noalloc(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,
+                             const int32_t* d_block_table, float* d_logits, int32_t* d_next, void* stream);
+
 /* Release everything the model owns. NULL is a no-op. */
 void axon_free(axon_model* m);
 

@@ -30,8 +30,8 @@ AXON_DTYPE_BF16, AXON_DTYPE_F32 = 0, 1
 AXON_LOGITS_LAST, AXON_LOGITS_ALL = 0, 1
 
 EXPORTED = ["axon_model_create", "axon_prefill", "axon_decode_step", "axon_reset", "axon_check_device",
-            "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill", "axon_free",
-            "axon_status_string"]
+            "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill", "axon_decode_step_noalloc",
+            "axon_free", "axon_status_string"]
 
 
 class axon_config(ctypes.Structure):
@@ -79,6 +79,7 @@ def lib() -> ctypes.CDLL:
                                         ctypes.POINTER(vp)]
         L.axon_prefill.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp, vp]
         L.axon_decode_step.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
+        L.axon_decode_step_noalloc.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
         L.axon_reset.argtypes = [vp]
         L.axon_check_device.argtypes = [vp, vp, p_i32]
         L.axon_kv_view_get.argtypes = [vp, ctypes.POINTER(axon_kv_view)]
@@ -90,7 +91,8 @@ def lib() -> ctypes.CDLL:
         L.axon_status_string.argtypes = [ctypes.c_int]
         L.axon_status_string.restype = ctypes.c_char_p
         for n in ("axon_model_create", "axon_prefill", "axon_decode_step", "axon_reset", "axon_check_device",
-                  "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill"):
+                  "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill",
+                  "axon_decode_step_noalloc"):
             getattr(L, n).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -160,6 +162,14 @@ def axon_decode_step(m, tokens, context_lens, block_table=None, logits=None, nex
     B = tokens.shape[0]
     _check("axon_decode_step", lib().axon_decode_step(m, _ptr(tokens), B, _ptr(context_lens), _ptr(block_table),
                                                       _ptr(logits), _ptr(next_tokens), _stream(stream)))
+
+
+def axon_decode_step_noalloc(m, tokens, context_lens, block_table=None, logits=None, next_tokens=None, stream=None):
+    """Allocation-free decode step (see include/axon.h): same contract as
+    axon_decode_step, direct launches, fixed library-owned merge scratch."""
+    B = tokens.shape[0]
+    _check("axon_decode_step_noalloc", lib().axon_decode_step_noalloc(
+        m, _ptr(tokens), B, _ptr(context_lens), _ptr(block_table), _ptr(logits), _ptr(next_tokens), _stream(stream)))
 
 
 def axon_reset(m):

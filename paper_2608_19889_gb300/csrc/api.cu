@@ -457,7 +457,8 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 }
 
 int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt, float* logits,
-                   int32_t* next, cudaStream_t st, Prof* pf = nullptr, double kv_tokens = 0) {
+                   int32_t* next, cudaStream_t st, Prof* pf = nullptr, double kv_tokens = 0,
+                   float* attn_part = nullptr, int* attn_cnt = nullptr, int attn_rows_cap = 0) {
   LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms};
   Proj pj{m, lc};
   const int D = m->D, Hd = m->H * m->d;
@@ -471,7 +472,12 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   pend(pf, static_cast<double>(B) * D * (es + 4 + es), 0);
   NormState ns;
   ns.rinv = true;
-  const int splits = m->fp32 ? 1 : attn_decode_splits(B, m->G, m->blocks_per_seq, m->num_sms);
+  int splits = m->fp32 ? 1 : attn_decode_splits(B, m->G, m->blocks_per_seq, m->num_sms);
+  if (attn_rows_cap > 0) {
+    // caller-supplied merge scratch holds attn_rows_cap (sequence, kv head, split) slots
+    const int cap = attn_rows_cap / (B * m->G);
+    if (splits > cap) splits = cap < 1 ? 1 : cap;
+  }
   for (int l = 0; l < m->L; ++l) {
     const LayerW& w = m->layers[l];
     EpiArgs e = base_epi(m);
@@ -490,8 +496,8 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     at.ctx = ctx;
     at.S = 1;
     at.splits = splits;
-    at.part = m->attn_part;
-    at.counter = m->attn_cnt;
+    at.part = attn_part ? attn_part : m->attn_part;
+    at.counter = attn_cnt ? attn_cnt : m->attn_cnt;
     pbeg(pf, "decode_attention");
     CK(launch_attn_decode(lc, m->fp32, at, B));
     pend(pf, kv_tokens * 2.0 * m->G * m->d * es + 2.0 * B * Hd * es, 4.0 * kv_tokens * m->H * m->d);
@@ -548,6 +554,32 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   pend(pf, 16.0 * B, 0);
   return AXON_OK;
 }
+
+}  // namespace
+
+// Direct-launch decode step with caller-supplied attention merge scratch
+// (used by the allocation-free entry point in noalloc.cu). Not exported.
+int axon_internal_decode_direct(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt,
+                                float* logits, int32_t* next, cudaStream_t st, float* attn_part, int* attn_cnt,
+                                int attn_rows_cap, int* head_dim, int* kv_heads) {
+  if (head_dim) *head_dim = m->d;
+  if (kv_heads) *kv_heads = m->G;
+  if (!tokens) return AXON_OK;  // query only
+  return enqueue_decode(m, tokens, B, ctx, bt, logits, next, st, nullptr, 0, attn_part, attn_cnt, attn_rows_cap);
+}
+
+// Validation shared with axon_decode_step. Not exported.
+int axon_internal_decode_args_ok(const axon_model* m, const int32_t* d_tokens, int32_t B, const int32_t* d_ctx,
+                                 const int32_t* d_block_table, const int32_t* d_next) {
+  if (!m || !d_tokens || !d_ctx || !d_next) return AXON_ERR_INVALID_ARG;
+  if (B < 1 || B > m->cfg.max_batch || B > 64) return AXON_ERR_INVALID_ARG;
+  const bool paged = m->cfg.kv_layout == AXON_KV_PAGED;
+  if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
+  if (m->fp32) return AXON_ERR_UNSUPPORTED;
+  return AXON_OK;
+}
+
+namespace {
 
 void free_model(axon_model* m) {
   if (!m) return;
