@@ -34,6 +34,7 @@ struct LayerW {
   float* g1 = nullptr;
   float* g2 = nullptr;
   GemmMaps m_qkv{}, m_o{}, m_gu{}, m_d{};
+  CUtensorMap v_qkv{}, v_o{}, v_gu{}, v_d{};  // weight maps for the decode projections (box 64 x 128)
 };
 
 using GraphKey = std::tuple<int, const void*, const void*, const void*, const void*, const void*>;
@@ -59,6 +60,7 @@ struct axon_model {
   float* gf = nullptr;
   std::vector<LayerW> layers;
   GemmMaps m_head{};
+  CUtensorMap v_head{};
   // KV cache
   void* kpool = nullptr;
   void* vpool = nullptr;
@@ -78,6 +80,8 @@ struct axon_model {
   unsigned long long* keys = nullptr;
   float* rinv = nullptr;   // [Mcap] per-row inverse RMS from decode producers
   SplitKWork splitk{};     // decode projections' cross-CTA split-K workspace
+  GemvTmaWork tmawork{};   // TMA stream-K decode projections' workspace
+  CUtensorMap t_a_tok[4]{}, t_o_tok[4]{}, t_u_tok[4]{};  // activation maps, box 64 x {8,16,32,64} rows
   int* ticket = nullptr;   // last-CTA counter of the residual producers
   float* attn_part = nullptr;
   int* attn_cnt = nullptr;
@@ -89,6 +93,7 @@ struct axon_model {
   std::map<GraphKey, cudaGraphExec_t> graphs;
   bool use_graphs = true;
   bool use_pdl = true;
+  bool use_tma_gemv = false;
 };
 
 namespace {
@@ -330,8 +335,10 @@ struct Proj {
   cudaError_t rc = cudaSuccess;
   // act: activation rows (row stride act_stride elements), M rows. Returns
   // the norm state a RESID producer leaves behind.
+  // vmap: the weight's decode-projection TMA map; amaps: the activation
+  // buffer's maps by token-box size (null: register-streaming GEMV).
   NormState run(int kind, const void* W, const GemmMaps* maps, int N, int K, const void* act, long long act_stride,
-                int M, EpiArgs& ep) {
+                int M, EpiArgs& ep, const CUtensorMap* vmap = nullptr, const CUtensorMap* amaps = nullptr) {
     ep.M = M;
     ep.N = N;
     NormState ns;
@@ -341,7 +348,12 @@ struct Proj {
       ep.ticket = m->ticket;
       ns.rinv = true;
     }
-    if (gemv) {
+    if (gemv && !m->fp32 && vmap && amaps && m->use_tma_gemv) {
+      const int tok = gemv_tma_tokens(M);
+      const int idx = tok == 8 ? 0 : (tok == 16 ? 1 : (tok == 32 ? 2 : 3));
+      rc = launch_gemv_tma(lc, kind, *vmap, amaps[idx], N, K, M, ep, m->tmawork);
+      ns.parts = N / 16;
+    } else if (gemv) {
       rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk);
       ns.parts = N / 16;
     } else if (m->fp32) {
@@ -488,7 +500,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
     pbeg(pf, "decode_qkv");
-    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e);
+    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok);
     CK(pj.rc);
     pend(pf, wq + B * (D + m->Nqkv) * es, 2.0 * B * m->Nqkv * D);
 
@@ -511,7 +523,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     r.ss_out = m->ss;
     r.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_o");
-    ns = pj.run(EPI_RESID, w.wo, nullptr, D, Hd, m->o, Hd, B, r);
+    ns = pj.run(EPI_RESID, w.wo, nullptr, D, Hd, m->o, Hd, B, r, &w.v_o, m->t_o_tok);
     CK(pj.rc);
     pend(pf, wo + B * (Hd * es + D * (8 + es)), 2.0 * B * D * Hd);
 
@@ -521,7 +533,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     set_norm(m, ns, g);
     g.u_out = m->u;
     pbeg(pf, "decode_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g);
+    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok);
     CK(pj.rc);
     pend(pf, wgu + B * (D + m->F) * es, 2.0 * B * 2 * m->F * D);
 
@@ -534,7 +546,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_down");
-    ns = pj.run(EPI_RESID, w.wd, nullptr, D, m->F, m->u, m->F, B, dn);
+    ns = pj.run(EPI_RESID, w.wd, nullptr, D, m->F, m->u, m->F, B, dn, &w.v_d, m->t_u_tok);
     CK(pj.rc);
     pend(pf, wdn + B * (m->F * es + D * (8 + es)), 2.0 * B * D * m->F);
   }
@@ -546,7 +558,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   h.logits = logits;
   h.logits_stride = m->V;
   pbeg(pf, "decode_lm_head");
-  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h);
+  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok);
   CK(pj.rc);
   pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
   pbeg(pf, "finalize");
@@ -631,6 +643,7 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->esz = m->fp32 ? 4 : 2;
   m->use_graphs = !env_flag("AXON_NO_GRAPH");
   m->use_pdl = !env_flag("AXON_NO_PDL");
+  m->use_tma_gemv = env_flag("AXON_TMA_GEMV");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   auto fail = [&](int code) {
     cudaStreamSynchronize(st);
@@ -642,7 +655,9 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   int major = 0;
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, m->device);
   if (major < 10) return fail(AXON_ERR_UNSUPPORTED);
-  if (prepare_attn_kernels() != cudaSuccess || prepare_gemm_kernels() != cudaSuccess) return fail(AXON_ERR_CUDA);
+  if (prepare_attn_kernels() != cudaSuccess || prepare_gemm_kernels() != cudaSuccess ||
+      prepare_gemv_tma_kernels() != cudaSuccess || prepare_gemv_kernels() != cudaSuccess)
+    return fail(AXON_ERR_CUDA);
 
   Builder bl{m, weights, n_weights, st};
   const int D = m->D, Hd = m->H * m->d, Gd = m->G * m->d, F = m->F, V = m->V;
@@ -815,6 +830,20 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->rinv = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
   m->ticket = static_cast<int*>(p);
+  {
+    int maxn = V;
+    if (2 * F > maxn) maxn = 2 * F;
+    if (m->Nqkv > maxn) maxn = m->Nqkv;
+    m->tmawork.max_row_blocks = (maxn + 127) / 128;
+    m->tmawork.max_grid = m->num_sms;
+    if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->num_sms) * 2 * 128 * 64 * 4))) return fail(rc);
+    m->tmawork.part = static_cast<float*>(p);
+    if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->tmawork.max_row_blocks) * 8 * 4 + 64))) return fail(rc);
+    m->tmawork.slice_ticket = static_cast<int*>(p);
+    m->tmawork.rinv_ticket = m->tmawork.slice_ticket + static_cast<size_t>(m->tmawork.max_row_blocks) * 8;
+    if (cudaMemsetAsync(p, 0, static_cast<size_t>(m->tmawork.max_row_blocks) * 8 * 4 + 64, st) != cudaSuccess)
+      return fail(AXON_ERR_CUDA);
+  }
   m->splitk.max_tiles = 1024;
   m->splitk.max_ctas = 2048;
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->splitk.max_ctas) * 16 * 64 * 4))) return fail(rc);
@@ -857,6 +886,18 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     }
     m->m_head.a = m->t_a;
     ok = ok && make_tma_2d_bf16(&m->m_head.w, m->head, V, D, 256);
+    // decode projections: weight boxes of 128 rows, activation boxes of 8..64 token rows
+    for (int l = 0; l < m->L && ok; ++l) {
+      LayerW& w = m->layers[l];
+      ok = make_tma_2d_bf16(&w.v_qkv, w.wqkv, m->Nqkv, D, 128) && make_tma_2d_bf16(&w.v_o, w.wo, D, Hd, 128) &&
+           make_tma_2d_bf16(&w.v_gu, w.wgu, 2 * F, D, 128) && make_tma_2d_bf16(&w.v_d, w.wd, D, F, 128);
+    }
+    ok = ok && make_tma_2d_bf16(&m->v_head, m->head, V, D, 128);
+    for (int i = 0; i < 4 && ok; ++i) {
+      const uint32_t tok = 8u << i;
+      ok = make_tma_2d_bf16(&m->t_a_tok[i], m->a, Mcap, D, tok) && make_tma_2d_bf16(&m->t_o_tok[i], m->o, Mcap, Hd, tok) &&
+           make_tma_2d_bf16(&m->t_u_tok[i], m->u, Mcap, F, tok);
+    }
     if (!ok) return fail(AXON_ERR_CUDA);
   }
   if (cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking) != cudaSuccess) return fail(AXON_ERR_CUDA);

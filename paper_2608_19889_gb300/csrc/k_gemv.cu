@@ -348,19 +348,35 @@ cudaError_t gemv_nt(const LaunchCtx& lc, int kind, const void* W, int N, int K, 
   }
 }
 
-// K-split count: enough CTAs for ~4 per SM, each warp keeping >= 2 chunks,
-// bounded by the partial-tile workspace.
-SplitK choose_split(const LaunchCtx& lc, int N, int K, const SplitKWork& wk) {
+// Resident CTAs per SM of each projection instantiation (occupancy API),
+// filled by prepare_gemv_kernels().
+int g_resident[4][4] = {};  // [NT index][kind]
+
+// K-split count minimising the modelled time of the launch:
+// waves(tiles * ks) * (chunks per CTA + per-CTA overhead), with waves
+// counted against the resident-CTA capacity of the whole GPU. Each warp
+// keeps >= 2 chunks; the partial-tile workspace bounds tiles * ks.
+SplitK choose_split(const LaunchCtx& lc, int nt_idx, int kind, int N, int K, const SplitKWork& wk) {
   SplitK sk{1, wk.part, wk.ticket};
   if (!wk.part || !wk.ticket) return sk;
   const int tiles = (N + 15) / 16;
-  const int target = 4 * lc.num_sms;
-  if (tiles >= target || tiles > wk.max_tiles) return sk;
-  int ks = (target + tiles - 1) / tiles;
-  const int max_by_k = (K >> 6) / (2 * GEMV_KW);
-  if (ks > max_by_k) ks = max_by_k;
-  while (ks > 1 && static_cast<long long>(tiles) * ks > wk.max_ctas) --ks;
-  sk.count = ks < 1 ? 1 : ks;
+  if (tiles > wk.max_tiles) return sk;
+  const int per_sm = g_resident[nt_idx][kind] > 0 ? g_resident[nt_idx][kind] : 2;
+  const long long cap = static_cast<long long>(per_sm) * lc.num_sms;
+  const int nch = K >> 6;
+  const int max_ks = nch / (2 * GEMV_KW);
+  constexpr double OVERHEAD_CHUNKS = 8.0;  // launch + first-load latency + merge, in chunk-times
+  double best = 1e30;
+  for (int ks = 1; ks <= (max_ks < 1 ? 1 : max_ks); ++ks) {
+    const long long total = static_cast<long long>(tiles) * ks;
+    if (ks > 1 && total > wk.max_ctas) break;
+    const long long waves = (total + cap - 1) / cap;
+    const double t = static_cast<double>(waves) * (static_cast<double>(nch) / ks / GEMV_KW + OVERHEAD_CHUNKS);
+    if (t < best - 1e-9) {
+      best = t;
+      sk.count = ks;
+    }
+  }
   return sk;
 }
 
@@ -380,11 +396,37 @@ cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W,
       default: return launch_k(lc, gemv_f32_kernel<EPI_LOGITS>, grid, block, 0, w, N, K, a, act_stride, B, ep);
     }
   }
-  const SplitK sk = choose_split(lc, N, K, wk);
+  const int nt_idx = B <= 8 ? 0 : (B <= 16 ? 1 : (B <= 32 ? 2 : 3));
+  const SplitK sk = choose_split(lc, nt_idx, kind, N, K, wk);
   if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
   if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
   if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
   return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
+}
+
+namespace {
+template <int NT>
+cudaError_t occupancy_nt(int idx) {
+  cudaError_t e = cudaSuccess;
+  const int threads = GEMV_KW * 32;
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_QKV], gemv_mma_kernel<NT, EPI_QKV>, threads, 0);
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_RESID], gemv_mma_kernel<NT, EPI_RESID>, threads, 0);
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_SWIGLU], gemv_mma_kernel<NT, EPI_SWIGLU>, threads, 0);
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_LOGITS], gemv_mma_kernel<NT, EPI_LOGITS>, threads, 0);
+  return e;
+}
+}  // namespace
+
+cudaError_t prepare_gemv_kernels() {
+  cudaError_t e = occupancy_nt<1>(0);
+  if (e == cudaSuccess) e = occupancy_nt<2>(1);
+  if (e == cudaSuccess) e = occupancy_nt<4>(2);
+  if (e == cudaSuccess) e = occupancy_nt<8>(3);
+  return e;
 }
 
 cudaError_t launch_embed(const LaunchCtx& lc, bool fp32, const void* E, int V, int D, const int* ids, int M, float* x,

@@ -32,6 +32,23 @@ struct SplitK {
 };
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
                         long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk);
+// Query occupancy of the projection kernels (once, before launches).
+cudaError_t prepare_gemv_kernels();
+
+// ---- decode projections, TMA-fed persistent stream-K variant
+// (k_gemv_tma.cu). W map: box 64 x 128 rows; activation map: box 64 x
+// gemv_tma_tokens(B) rows of a row-contiguous [rows][K] buffer.
+struct GemvTmaWork {
+  float* part;        // [max_grid][2][128][64]
+  int* slice_ticket;  // [max_row_blocks][8], zeroed once
+  int* rinv_ticket;   // [1], zeroed once
+  int max_grid;
+  int max_row_blocks;
+};
+int gemv_tma_tokens(int B);
+cudaError_t prepare_gemv_tma_kernels();
+cudaError_t launch_gemv_tma(const LaunchCtx& lc, int kind, const CUtensorMap& w, const CUtensorMap& a, int N, int K,
+                            int B, const EpiArgs& ep, const GemvTmaWork& wk);
 
 // ---- embedding gather producing x, a = x * g and the row sum of squares.
 // rinv (optional): 1 / sqrt(mean(x^2) + eps) per row.
