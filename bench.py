@@ -168,6 +168,159 @@ def run_reference(args, rank, world):
     }), flush=True)
 
 
+class GenerateRun:
+    """Contiguous-cache workload: one step = prefill B x S + n_new decode steps."""
+
+    def __init__(self, ax, torch, model, m, wl, st):
+        self.ax, self.torch, self.model, self.m, self.st = ax, torch, model, m, st
+        self.B, self.S, self.n_new = wl["B"], wl["S"], wl["n_new"]
+        B = self.B
+        self.ids = torch.from_numpy(si.make_ids(B, self.S, m["V"])).cuda()
+        self.tok = torch.empty(B, dtype=torch.int32, device="cuda")
+        self.ctx = torch.empty(B, dtype=torch.int32, device="cuda")
+        self.logits = torch.empty(B, m["V"], device="cuda")
+        self.bt = None
+        self.kind = "contiguous"
+
+    def step(self, ev=None):
+        ax, st = self.ax, self.st
+        if ev:
+            ev[0].record(st)
+        ax.axon_prefill(self.model, self.ids, logits_mode=ax.AXON_LOGITS_LAST, logits=self.logits,
+                        next_tokens=self.tok, stream=st)
+        if ev:
+            ev[1].record(st)
+        self.ctx.fill_(self.S)  # positions restart at the prompt length (torch fill on the same stream)
+        for _ in range(self.n_new):
+            ax.axon_decode_step(self.model, self.tok, self.ctx, logits=self.logits, next_tokens=self.tok, stream=st)
+        if ev:
+            ev[2].record(st)
+
+    def e2e_step(self, ids_h, out_h, hist, ids_d):
+        ax, st = self.ax, self.st
+        ids_d.copy_(ids_h, non_blocking=True)
+        ax.axon_prefill(self.model, ids_d, logits_mode=ax.AXON_LOGITS_LAST, logits=None, next_tokens=self.tok,
+                        stream=st)
+        self.ctx.fill_(self.S)
+        for t in range(self.n_new):
+            ax.axon_decode_step(self.model, self.tok, self.ctx, logits=None, next_tokens=self.tok, stream=st)
+            hist[t].copy_(self.tok)
+        out_h.copy_(hist, non_blocking=True)
+
+    def host_inputs(self):
+        return self.torch.from_numpy(si.make_ids(self.B, self.S, self.m["V"])).pin_memory(), self.ids
+
+    def decode_positions(self):
+        return [[self.S + i] * self.B for i in range(self.n_new)]
+
+    def generated_per_step(self):
+        return self.B * self.n_new
+
+    def launches_per_step(self):
+        # embed + 5 per layer + LM head + finaliser, for the prefill and each decode step
+        return (5 * self.m["L"] + 3) * (1 + self.n_new)
+
+    def profile_positions(self):
+        return [[self.S] * self.B, [self.S + self.n_new // 2] * self.B, [self.S + self.n_new - 1] * self.B]
+
+
+class PagedDecodeRun:
+    """Paged-cache workload: sequences with context lengths drawn from [lo, hi]
+    are prefilled one by one into a shuffled block pool (set-up, timed
+    separately); one step = n_new decode steps of the whole batch."""
+
+    def __init__(self, ax, torch, model, m, wl, st, lens, bt_np):
+        self.ax, self.torch, self.model, self.m, self.st = ax, torch, model, m, st
+        self.B, self.n_new = wl["B"], wl["n_new"]
+        self.lens = torch.from_numpy(lens.astype(np.int32)).cuda()
+        self.lens_np = lens
+        self.bt = torch.from_numpy(bt_np).cuda()
+        self.tok = torch.empty(self.B, dtype=torch.int32, device="cuda")
+        self.first_tok = torch.empty(self.B, dtype=torch.int32, device="cuda")
+        self.ctx = torch.empty(self.B, dtype=torch.int32, device="cuda")
+        self.logits = torch.empty(self.B, m["V"], device="cuda")
+        self.kind = "paged"
+        # varlen prefill: one call per sequence on its block-table row
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        nxt = torch.empty(1, dtype=torch.int32, device="cuda")
+        with torch.cuda.stream(st):
+            ev[0].record(st)
+            for b in range(self.B):
+                ids = torch.from_numpy(si.make_ids(1, int(lens[b]), m["V"], seed=100 + b)).cuda()
+                ax.axon_prefill(model, ids, block_table=self.bt[b:b + 1], next_tokens=nxt, stream=st)
+                self.first_tok[b:b + 1].copy_(nxt)
+            ev[1].record(st)
+        torch.cuda.synchronize()
+        self.prefill_ms = ev[0].elapsed_time(ev[1])
+        self.prefill_tokens = int(lens.sum())
+
+    def step(self, ev=None):
+        ax, st = self.ax, self.st
+        self.ctx.copy_(self.lens)
+        self.tok.copy_(self.first_tok)
+        if ev:
+            ev[0].record(st)
+            ev[1].record(st)
+        for _ in range(self.n_new):
+            ax.axon_decode_step(self.model, self.tok, self.ctx, block_table=self.bt, logits=self.logits,
+                                next_tokens=self.tok, stream=st)
+        if ev:
+            ev[2].record(st)
+
+    def e2e_step(self, tok_h, out_h, hist, tok_d):
+        ax, st = self.ax, self.st
+        tok_d.copy_(tok_h, non_blocking=True)
+        self.ctx.copy_(self.lens)
+        for t in range(self.n_new):
+            ax.axon_decode_step(self.model, tok_d, self.ctx, block_table=self.bt, logits=None, next_tokens=tok_d,
+                                stream=st)
+            hist[t].copy_(tok_d)
+        out_h.copy_(hist, non_blocking=True)
+
+    def host_inputs(self):
+        return self.first_tok.cpu().pin_memory(), self.tok
+
+    def decode_positions(self):
+        return [list(self.lens_np + i) for i in range(self.n_new)]
+
+    def generated_per_step(self):
+        return self.B * self.n_new
+
+    def launches_per_step(self):
+        return (5 * self.m["L"] + 3) * self.n_new
+
+    def profile_positions(self):
+        return [list(self.lens_np), list(self.lens_np + self.n_new // 2), list(self.lens_np + self.n_new - 1)]
+
+
+def build_model(ax, torch, wl, m, st, layers=None, vocab=None):
+    m = dict(m)
+    if layers is not None:
+        m["L"] = layers
+    if vocab is not None:
+        m["V"] = vocab
+    w = si.make_weights(m, device="cuda")
+    lens = bt_np = None
+    if wl["layout"] == "paged":
+        B, (lo, hi) = wl["B"], wl["ctx"]
+        lens = si.make_context_lens(B, lo, hi)
+        max_ctx = (hi + wl["n_new"] + 15) // 16 * 16
+        caps = lens + wl["n_new"]
+        num_blocks = int(sum(-(-int(c) // 16) for c in caps)) + 64
+        bt_np = si.make_block_table(caps, 16, max_ctx // 16, num_blocks)
+        cfg = ax.make_config(m, max_batch=B, max_context=max_ctx, kv_layout=ax.AXON_KV_PAGED,
+                             kv_num_blocks=num_blocks, max_prefill_tokens=hi)
+    else:
+        B, S = wl["B"], wl["S"]
+        max_ctx = (S + wl["n_new"] + 15) // 16 * 16
+        cfg = ax.make_config(m, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S)
+    with torch.cuda.stream(st):
+        model = ax.axon_model_create(cfg, w, stream=st)
+    del w
+    torch.cuda.empty_cache()
+    return model, m, lens, bt_np
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -176,6 +329,12 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(si.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--case", action="store_true",
+                    help="profiling case: build the workload's model, run one prefill and --case-steps decode "
+                         "steps, print nothing but a status line (for ncu)")
+    ap.add_argument("--case-layers", type=int, default=None)
+    ap.add_argument("--case-vocab", type=int, default=None)
+    ap.add_argument("--case-steps", type=int, default=2)
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -196,40 +355,35 @@ def main():
         dist.init_process_group("nccl")
 
     wl = si.WORKLOADS[args.workload]
-    m = si.MODEL_SHAPES[wl["model"]]
-    if wl["layout"] != "contiguous":
-        raise SystemExit("paged workloads are benchmarked by a later revision")
-    B, S, n_new = wl["B"], wl["S"], wl["n_new"]
-    max_ctx = (S + n_new + 15) // 16 * 16
-    w = si.make_weights(m, device="cuda")
-    cfg = ax.make_config(m, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S)
     st = torch.cuda.Stream()
-    with torch.cuda.stream(st):
-        model = ax.axon_model_create(cfg, w, stream=st)
-    del w
-    torch.cuda.empty_cache()
+    model, m, lens, bt_np = build_model(ax, torch, wl, si.MODEL_SHAPES[wl["model"]], st,
+                                        layers=args.case_layers if args.case else None,
+                                        vocab=args.case_vocab if args.case else None)
+    if wl["layout"] == "paged":
+        run = PagedDecodeRun(ax, torch, model, m, wl, st, lens, bt_np)
+    else:
+        run = GenerateRun(ax, torch, model, m, wl, st)
+    B, n_new = run.B, run.n_new
 
-    ids = torch.from_numpy(si.make_ids(B, S, m["V"])).cuda()
-    tok = torch.empty(B, dtype=torch.int32, device="cuda")
-    ctx = torch.empty(B, dtype=torch.int32, device="cuda")
-    logits = torch.empty(B, m["V"], device="cuda")
+    if args.case:
+        with torch.cuda.stream(st):
+            if run.kind == "contiguous":
+                ax.axon_prefill(model, run.ids, next_tokens=run.tok, stream=st)
+                run.ctx.fill_(run.S)
+            else:
+                run.ctx.copy_(run.lens)
+                run.tok.copy_(run.first_tok)
+            for _ in range(args.case_steps):
+                ax.axon_decode_step(model, run.tok, run.ctx, block_table=run.bt, next_tokens=run.tok, stream=st)
+        torch.cuda.synchronize()
+        print("case ok", ax.axon_check_device(model, stream=st), flush=True)
+        ax.axon_free(model)
+        return
+
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-
-    def one_step(events=None):
-        if events:
-            events[0].record(st)
-        ax.axon_prefill(model, ids, logits_mode=ax.AXON_LOGITS_LAST, logits=logits, next_tokens=tok, stream=st)
-        if events:
-            events[1].record(st)
-        ctx.fill_(S)  # positions restart at the prompt length (torch fill on the same stream)
-        for _ in range(n_new):
-            ax.axon_decode_step(model, tok, ctx, logits=logits, next_tokens=tok, stream=st)
-        if events:
-            events[2].record(st)
-
     with torch.cuda.stream(st):
         for _ in range(args.warmup):
-            one_step()
+            run.step()
     torch.cuda.synchronize()
     rc, bits = ax.axon_check_device(model, stream=st)
     if rc != 0:
@@ -242,7 +396,7 @@ def main():
     t0 = time.perf_counter()
     with torch.cuda.stream(st):
         for k in range(args.steps):
-            one_step(ev[k])
+            run.step(ev[k])
     torch.cuda.synchronize()
     wall = time.perf_counter() - t0
     if dist:
@@ -257,54 +411,46 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
 
-    # ---- end to end through the public API with host buffers: pinned ids in,
-    # generated tokens out, copies inside the timed region.
-    ids_h = torch.from_numpy(si.make_ids(B, S, m["V"])).pin_memory()
+    # ---- end to end through the public API with host buffers: inputs copied in
+    # from pinned memory, generated tokens copied out, inside the timed region.
+    in_h, in_d_like = run.host_inputs()
+    in_d = torch.empty_like(in_d_like)
     out_h = torch.empty(n_new, B, dtype=torch.int32).pin_memory()
     hist = torch.empty(n_new, B, dtype=torch.int32, device="cuda")
-    ids_d = torch.empty_like(ids)
     e2e_ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
     e2e_ms = []
     with torch.cuda.stream(st):
+        run.e2e_step(in_h, out_h, hist, in_d)  # untimed: records this pointer set's decode graph
+        torch.cuda.synchronize()
         for k in range(args.steps):
             e2e_ev[0].record(st)
-            ids_d.copy_(ids_h, non_blocking=True)
-            ax.axon_prefill(model, ids_d, logits_mode=ax.AXON_LOGITS_LAST, logits=None, next_tokens=tok, stream=st)
-            ctx.fill_(S)
-            for t in range(n_new):
-                ax.axon_decode_step(model, tok, ctx, logits=None, next_tokens=tok, stream=st)
-                hist[t].copy_(tok)
-            out_h.copy_(hist, non_blocking=True)
+            run.e2e_step(in_h, out_h, hist, in_d)
             e2e_ev[1].record(st)
             e2e_ev[1].synchronize()
             e2e_ms.append(e2e_ev[0].elapsed_time(e2e_ev[1]))
-    e2e_val = B * n_new / (float(np.mean(e2e_ms)) / 1e3)
+    e2e_val = run.generated_per_step() / (float(np.mean(e2e_ms)) / 1e3)
 
     hbm, tf_burst, tf_sus, peak_kind = read_peaks()
-    T_list = [S + i for i in range(n_new)]
-    dec_bytes = sum(decode_bytes_per_step(m, B, [T] * B) for T in T_list)
+    dec_bytes = sum(decode_bytes_per_step(m, B, T) for T in run.decode_positions())
     dec_ms = float(np.mean(t_dec))
     dec_gbs = dec_bytes / (dec_ms / 1e3) / 1e9
-    pre_flops = prefill_flops(m, B, S)
-    pre_ms = float(np.mean(t_pre))
-    pre_tflops = pre_flops / (pre_ms / 1e3) / 1e12
-    # embed + 5 per layer + LM head + finaliser, for the prefill and each decode step
-    launches_per_step = (5 * m["L"] + 3) * (1 + n_new)
 
-    # ---- per-kernel timing (CUDA events around each launch, no graph) of one
-    # prefill and of decode steps at the start, middle and end of the run.
+    # ---- per-kernel timing (CUDA events around each launch, no graph) of
+    # decode steps at the start, middle and end of the run (and one prefill).
+    prof_pre = []
+    prof_dec = {}
     with torch.cuda.stream(st):
-        prof_pre = ax.axon_profile_prefill(model, ids, next_tokens=tok, stream=st)
-        prof_dec = {}
-        for T in (S, S + n_new // 2, S + n_new - 1):
-            ctx.fill_(T)
-            for e in ax.axon_profile_decode_step(model, tok, ctx, next_tokens=tok, stream=st):
+        if run.kind == "contiguous":
+            prof_pre = ax.axon_profile_prefill(model, run.ids, next_tokens=run.tok, stream=st)
+        for pos in run.profile_positions():
+            run.ctx.copy_(torch.tensor(pos, dtype=torch.int32))
+            for e in ax.axon_profile_decode_step(model, run.tok, run.ctx, block_table=run.bt, next_tokens=run.tok,
+                                                 stream=st):
                 a = prof_dec.setdefault(e["name"], dict(launches=0, total_ms=0.0, bytes=0.0, flops=0.0))
                 for k in ("launches", "total_ms", "bytes", "flops"):
                     a[k] += e[k]
     torch.cuda.synchronize()
-    # whole-run weight of each kernel kind: prefill once + n_new decode steps
-    kinds = []
+    kinds = []  # (weight over the run, name, launches, ms, bytes, flops)
     for e in prof_pre:
         kinds.append((e["total_ms"], e["name"], e["launches"], e["total_ms"], e["bytes"], e["flops"]))
     for name, e in prof_dec.items():
@@ -318,13 +464,18 @@ def main():
     else:
         ach = top_bytes / top_n / (per_launch_ms / 1e3) / 1e9
         roof = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm}
-    roof.update({"kernel": top_name, "launch_ms": per_launch_ms, "per_launch_units": (top_bytes if roof["bound"] == "hbm" else top_flops) / top_n,
+    roof.update({"kernel": top_name, "launch_ms": per_launch_ms,
+                 "per_launch_units": (top_bytes if roof["bound"] == "hbm" else top_flops) / top_n,
                  "peak_kind": peak_kind, "traffic": None})
-    kernel_table = {k[1]: {"share_of_run": k[0] / sum(x[0] for x in kinds), "launch_ms": k[3] / k[2]} for k in kinds}
+    total_w = sum(x[0] for x in kinds)
+    kernel_table = {k[1]: {"share_of_run": k[0] / total_w, "launch_ms": k[3] / k[2]} for k in kinds}
 
+    config = {"workload": args.workload, "B": B, "n_new": n_new, "layers": m["L"], "hidden": m["D"],
+              "vocab": m["V"], "kv": run.kind,
+              "l2": "inputs larger than L2 (weights " + f"{2 * sum(model_bytes(m)) / 1e9:.2f} GB > 129 MB)"}
     out = {
         "metric": METRIC,
-        "value": world * B * n_new / (ms / 1e3),
+        "value": world * run.generated_per_step() / (ms / 1e3),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
@@ -335,28 +486,36 @@ def main():
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded random-init weights N(0,0.02), uniform random ids)",
-        "config": {"workload": args.workload, "B": B, "S": S, "n_new": n_new, "layers": m["L"],
-                   "hidden": m["D"], "vocab": m["V"], "kv": "contiguous",
-                   "l2": "inputs larger than L2 (weights " + f"{2 * sum(model_bytes(m)) / 1e9:.2f} GB > 129 MB)"},
-        "prefill_tok_s": world * B * S / (pre_ms / 1e3),
+        "config": config,
         "decode_tok_s": world * B * n_new / (dec_ms / 1e3),
-        "prefill_ms": pre_ms,
         "decode_ms": dec_ms,
         "roofline": roof,
         "roofline_decode_step": {"bound": "hbm", "achieved": dec_gbs, "peak": hbm, "unit": "GB/s",
                                  "frac": dec_gbs / hbm, "peak_kind": peak_kind,
                                  "what": "all decode bytes (weights + KV + logits) / timed decode phase"},
-        "roofline_prefill_phase": {"bound": "tensor", "achieved": pre_tflops, "peak": tf_burst, "unit": "TFLOP/s",
-                                   "frac": pre_tflops / tf_burst, "peak_kind": peak_kind,
-                                   "what": "prefill FLOPs / timed prefill phase"},
         "kernels": kernel_table,
-        "e2e": {"value": world * e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": B * S * 4,
-                "d2h_bytes_per_step": B * n_new * 4},
-        "gpu_launches": args.steps * launches_per_step,
+        "e2e": {"value": world * e2e_val, "unit": "tokens/s",
+                "h2d_bytes_per_step": int(in_h.numel()) * 4, "d2h_bytes_per_step": B * n_new * 4},
+        "gpu_launches": args.steps * run.launches_per_step(),
         "clocks": clk,
         "wall_s": wall,
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if run.kind == "contiguous":
+        S = run.S
+        config["S"] = S
+        pre_ms = float(np.mean(t_pre))
+        pre_tflops = prefill_flops(m, B, S) / (pre_ms / 1e3) / 1e12
+        out["prefill_tok_s"] = world * B * S / (pre_ms / 1e3)
+        out["prefill_ms"] = pre_ms
+        out["roofline_prefill_phase"] = {"bound": "tensor", "achieved": pre_tflops, "peak": tf_burst,
+                                         "unit": "TFLOP/s", "frac": pre_tflops / tf_burst, "peak_kind": peak_kind,
+                                         "what": "prefill FLOPs / timed prefill phase"}
+    else:
+        config["context_lens"] = f"uniform in {wl['ctx']}, mean {float(np.mean(run.lens_np)):.0f}"
+        out["setup_prefill"] = {"tokens": run.prefill_tokens, "ms": run.prefill_ms,
+                                "tok_s": run.prefill_tokens / (run.prefill_ms / 1e3),
+                                "what": "varlen paged prefill of the contexts, one call per sequence (not in value)"}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and run.kind == "contiguous":
         v, sample, _ = oracle_generate_timed(wl, budget_s=15.0)
         out["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": cores(), "kind": "oracle", "sample": sample}
     ax.axon_free(model)

@@ -53,9 +53,19 @@ enum {
  * overlay; vLLM's PagedAttention manager, Sec. Related Work). */
 enum { AXON_KV_CONTIGUOUS = 0, AXON_KV_PAGED = 1 };
 
-/* Arithmetic mode: bf16 weights/activations with fp32 accumulation, or an
- * all-fp32 debug mode (Sec. Results: bf16 primary, fp32 fallback). */
-enum { AXON_BF16 = 0, AXON_FP32_DEBUG = 1 };
+/* Arithmetic mode (Sec. Results: bf16 primary, fp32 fallback):
+ *   AXON_BF16        bf16 weights, bf16 GEMM operands and KV cache, fp32
+ *                    accumulation, fp32 residual stream and logits;
+ *   AXON_FP32_DEBUG  everything fp32 (CUDA-core GEMMs), for checking;
+ *   AXON_FP16        the bf16 checkpoint converted exactly to fp16 (every
+ *                    bf16 value of magnitude 2^-14 .. 65504 is an fp16
+ *                    value), fp16 GEMM operands and KV cache, fp32
+ *                    accumulation and residual: same speed as AXON_BF16, 8x
+ *                    smaller operand rounding (10- vs 7-bit mantissa).
+ *                    Operands saturate at +-65504; a weight beyond that
+ *                    range makes axon_model_create return
+ *                    AXON_ERR_UNSUPPORTED. */
+enum { AXON_BF16 = 0, AXON_FP32_DEBUG = 1, AXON_FP16 = 2 };
 
 /* Element types of weight tensors handed to axon_model_create. */
 enum { AXON_DTYPE_BF16 = 0, AXON_DTYPE_F32 = 1 };
@@ -84,7 +94,7 @@ typedef struct axon_config {
   int32_t kv_layout;           /* AXON_KV_CONTIGUOUS or AXON_KV_PAGED */
   int32_t kv_block_size;       /* tokens per block: must be 16 */
   int32_t kv_num_blocks;       /* paged pool size in blocks (ignored if contiguous) */
-  int32_t precision;           /* AXON_BF16 or AXON_FP32_DEBUG */
+  int32_t precision;           /* AXON_BF16, AXON_FP16 or AXON_FP32_DEBUG */
 } axon_config;
 
 /* One named checkpoint tensor, HF Llama naming and [out, in] matrices, as a

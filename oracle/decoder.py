@@ -251,18 +251,23 @@ class Oracle:
     for the skeleton; Llama naming `model.layers.{i}.self_attn.q_proj.weight`
     as in the `_param(...)` lookups of the Python-overhead appendix).
 
-    weights: name -> array (float32 holding exact bf16 values, or float64).
+    weights: name -> array (float32 holding exact bf16 values, or float64),
+    or any mapping whose values numpy can widen.
     keep_f64: convert every matrix to float64 once (faster, 8 bytes/param);
-    otherwise each matmul widens its matrix on the fly.
+    otherwise the mapping is kept as given and each use widens its matrix
+    on the fly (for models whose float64 copy would not fit in memory).
     """
 
-    def __init__(self, cfg: DecoderConfig, weights: dict, keep_f64: bool = True):
+    def __init__(self, cfg: DecoderConfig, weights, keep_f64: bool = True):
         self.cfg = cfg
-        conv = (lambda a: np.asarray(a, dtype=np.float64)) if keep_f64 else (lambda a: np.asarray(a))
-        self.W = {k: conv(v) for k, v in weights.items()}
+        self.keep_f64 = keep_f64
+        if keep_f64:
+            self.W = {k: np.asarray(v, dtype=np.float64) for k, v in weights.items()}
+        else:
+            self.W = weights
 
     def _w(self, name):
-        return self.W[name]
+        return self.W[name] if self.keep_f64 else np.asarray(self.W[name], dtype=np.float64)
 
     def new_contiguous_cache(self, B, Tmax):
         c = self.cfg

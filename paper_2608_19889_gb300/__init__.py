@@ -25,7 +25,7 @@ AXON_ERR_CUDA = 6
 AXON_ERR_TIMEOUT = 7
 AXON_ERR_DEVICE_CHECK = 8
 AXON_KV_CONTIGUOUS, AXON_KV_PAGED = 0, 1
-AXON_BF16, AXON_FP32_DEBUG = 0, 1
+AXON_BF16, AXON_FP32_DEBUG, AXON_FP16 = 0, 1, 2
 AXON_DTYPE_BF16, AXON_DTYPE_F32 = 0, 1
 AXON_LOGITS_LAST, AXON_LOGITS_ALL = 0, 1
 

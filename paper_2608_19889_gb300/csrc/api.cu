@@ -50,6 +50,7 @@ struct axon_model {
   axon_config cfg{};
   int L = 0, D = 0, H = 0, G = 0, d = 0, F = 0, V = 0, Nqkv = 0;
   bool fp32 = false;
+  bool f16 = false;  // 16-bit operands are fp16 (AXON_FP16) rather than bf16
   size_t esz = 2;
   int device = 0;
   int num_sms = 148;
@@ -73,6 +74,7 @@ struct axon_model {
   int Pmax = 0;
   float* x = nullptr;
   void* a = nullptr;
+  void* a_lo = nullptr;  // fp16 mode: second term of the QKV input (x*g - a)
   float* ss = nullptr;
   void* q = nullptr;
   void* o = nullptr;
@@ -87,7 +89,7 @@ struct axon_model {
   int* attn_cnt = nullptr;
   int max_splits = 1;
   int* err = nullptr;
-  CUtensorMap t_a{}, t_o{}, t_u{};
+  CUtensorMap t_a{}, t_o{}, t_u{}, t_alo{};
   // decode graphs
   cudaStream_t cap_stream = nullptr;
   std::map<GraphKey, cudaGraphExec_t> graphs;
@@ -119,19 +121,29 @@ int dev_alloc(axon_model* m, void** p, size_t bytes) {
   return AXON_OK;
 }
 
-// dst[p][:] = src[rowmap[p]][:] with dtype conversion (bf16/f32 -> bf16/f32).
-__global__ void gather_rows_kernel(void* dst, int dst_f32, const void* src, int src_f32, const int* rowmap, int rows,
-                                   int cols) {
-  const int p = blockIdx.x;
-  if (p >= rows) return;
-  const long long sr = rowmap ? rowmap[p] : p;
+// Element types of repacked tensors.
+enum : int { DT_BF16 = 0, DT_F32 = 1, DT_F16 = 2 };
+
+// dst[p][:] = src[rowmap[p]][:] with dtype conversion (bf16/f32 -> bf16/f32/f16).
+// Values outside the finite fp16 range raise *overflow (fp16 destinations).
+__global__ void gather_rows_kernel(void* dst, int dst_dt, const void* src, int src_f32, const int* rowmap,
+                                   const int* dstmap, int rows, int cols, int* overflow) {
+  const int p0 = blockIdx.x;
+  if (p0 >= rows) return;
+  const long long sr = rowmap ? rowmap[p0] : p0;
+  const int p = dstmap ? dstmap[p0] : p0;
   for (int c = threadIdx.x; c < cols; c += blockDim.x) {
     const float v = src_f32 ? static_cast<const float*>(src)[sr * cols + c]
                             : __bfloat162float(static_cast<const bf16*>(src)[sr * cols + c]);
-    if (dst_f32)
-      static_cast<float*>(dst)[static_cast<long long>(p) * cols + c] = v;
-    else
-      static_cast<bf16*>(dst)[static_cast<long long>(p) * cols + c] = __float2bfloat16_rn(v);
+    const long long o = static_cast<long long>(p) * cols + c;
+    if (dst_dt == DT_F32) {
+      static_cast<float*>(dst)[o] = v;
+    } else if (dst_dt == DT_F16) {
+      if (!(fabsf(v) <= 65504.f)) atomicOr(overflow, 1);
+      static_cast<f16*>(dst)[o] = __float2half_rn(v);
+    } else {
+      static_cast<bf16*>(dst)[o] = __float2bfloat16_rn(v);
+    }
   }
 }
 
@@ -144,6 +156,9 @@ struct Builder {
   size_t staging_bytes = 0;
   int* d_rowmap = nullptr;
   size_t rowmap_cap = 0;
+  int* d_overflow = nullptr;
+  int* d_dstmap = nullptr;
+  size_t dstmap_cap = 0;
 
   const axon_tensor* find(const std::string& name) const {
     for (int i = 0; i < n; ++i)
@@ -175,9 +190,19 @@ struct Builder {
     CK(cudaMemcpyAsync(staging, t->data, bytes, cudaMemcpyDefault, st));
     return AXON_OK;
   }
-  int gather(void* dst, bool dst_f32, const axon_tensor* t, const std::vector<int>* rowmap, int rows, int cols) {
+  // dst_f32: fp32 destination; otherwise the model's 16-bit operand type.
+  // dstmap (optional): destination row of each gathered row.
+  int gather(void* dst, bool dst_f32, const axon_tensor* t, const std::vector<int>* rowmap, int rows, int cols,
+             const std::vector<int>* dstmap = nullptr) {
     int rc = stage(t, static_cast<size_t>(t->ndim == 2 ? t->shape[0] : 1) * cols);
     if (rc) return rc;
+    if (!d_overflow) {
+      if (cudaMalloc(&d_overflow, sizeof(int)) != cudaSuccess) {
+        cudaGetLastError();
+        return AXON_ERR_OOM;
+      }
+      CK(cudaMemsetAsync(d_overflow, 0, sizeof(int), st));
+    }
     const int* dm = nullptr;
     if (rowmap) {
       if (rowmap->size() > rowmap_cap) {
@@ -191,16 +216,34 @@ struct Builder {
       CK(cudaMemcpyAsync(d_rowmap, rowmap->data(), rowmap->size() * sizeof(int), cudaMemcpyHostToDevice, st));
       dm = d_rowmap;
     }
-    gather_rows_kernel<<<rows, 256, 0, st>>>(dst, dst_f32 ? 1 : 0, staging, t->dtype == AXON_DTYPE_F32 ? 1 : 0, dm,
-                                             rows, cols);
+    const int* ddm = nullptr;
+    if (dstmap) {
+      if (dstmap->size() > dstmap_cap) {
+        if (d_dstmap) cudaFree(d_dstmap);
+        if (cudaMalloc(&d_dstmap, dstmap->size() * sizeof(int)) != cudaSuccess) {
+          cudaGetLastError();
+          return AXON_ERR_OOM;
+        }
+        dstmap_cap = dstmap->size();
+      }
+      CK(cudaMemcpyAsync(d_dstmap, dstmap->data(), dstmap->size() * sizeof(int), cudaMemcpyHostToDevice, st));
+      ddm = d_dstmap;
+    }
+    const int dt = dst_f32 ? DT_F32 : (m->f16 ? DT_F16 : DT_BF16);
+    gather_rows_kernel<<<rows, 256, 0, st>>>(dst, dt, staging, t->dtype == AXON_DTYPE_F32 ? 1 : 0, dm, ddm, rows,
+                                             cols, d_overflow);
     CK(cudaGetLastError());
     // staging and rowmap are reused by the next call
     CK(cudaStreamSynchronize(st));
-    return AXON_OK;
+    int ovf = 0;
+    CK(cudaMemcpy(&ovf, d_overflow, sizeof(int), cudaMemcpyDeviceToHost));
+    return ovf ? AXON_ERR_UNSUPPORTED : AXON_OK;
   }
   ~Builder() {
     if (staging) cudaFree(staging);
     if (d_rowmap) cudaFree(d_rowmap);
+    if (d_overflow) cudaFree(d_overflow);
+    if (d_dstmap) cudaFree(d_dstmap);
   }
 };
 
@@ -210,7 +253,8 @@ int validate_config(const axon_config* c) {
       c->max_context <= 0)
     return AXON_ERR_INVALID_ARG;
   if (c->kv_layout != AXON_KV_CONTIGUOUS && c->kv_layout != AXON_KV_PAGED) return AXON_ERR_INVALID_ARG;
-  if (c->precision != AXON_BF16 && c->precision != AXON_FP32_DEBUG) return AXON_ERR_INVALID_ARG;
+  if (c->precision != AXON_BF16 && c->precision != AXON_FP32_DEBUG && c->precision != AXON_FP16)
+    return AXON_ERR_INVALID_ARG;
   if (c->kv_block_size != 16) return AXON_ERR_UNSUPPORTED;
   if (c->kv_layout == AXON_KV_PAGED && c->kv_num_blocks <= 0) return AXON_ERR_INVALID_ARG;
   if (c->num_attention_heads % c->num_key_value_heads) return AXON_ERR_UNSUPPORTED;
@@ -321,11 +365,30 @@ struct Prof {
     }
   }
 };
+// AXON_TRACE=1: name every launch on stderr and wait for it (debugging aid;
+// ignored while a stream is being captured).
+bool g_trace = false;
+cudaStream_t g_trace_stream = nullptr;
+const char* g_trace_name = "";
 inline void pbeg(Prof* p, const char* n) {
   if (p) p->begin(n);
+  if (g_trace) {
+    g_trace_name = n;
+    fprintf(stderr, "axon: launch %s\n", n);
+    fflush(stderr);
+  }
 }
 inline void pend(Prof* p, double bytes, double flops) {
   if (p) p->end(bytes, flops);
+  if (g_trace && g_trace_stream) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    cudaStreamIsCapturing(g_trace_stream, &cs);
+    if (cs == cudaStreamCaptureStatusNone) {
+      const cudaError_t e = cudaStreamSynchronize(g_trace_stream);
+      fprintf(stderr, "axon: done %s (%s)\n", g_trace_name, cudaGetErrorString(e));
+      fflush(stderr);
+    }
+  }
 }
 
 // One projection: picks the kernel for the mode and row count.
@@ -337,8 +400,11 @@ struct Proj {
   // the norm state a RESID producer leaves behind.
   // vmap: the weight's decode-projection TMA map; amaps: the activation
   // buffer's maps by token-box size (null: register-streaming GEMV).
+  // xg: fp16-mode decode consumers of a normed operand build it from the
+  // fp32 residual and this gain (see launch_gemv).
   NormState run(int kind, const void* W, const GemmMaps* maps, int N, int K, const void* act, long long act_stride,
-                int M, EpiArgs& ep, const CUtensorMap* vmap = nullptr, const CUtensorMap* amaps = nullptr) {
+                int M, EpiArgs& ep, const CUtensorMap* vmap = nullptr, const CUtensorMap* amaps = nullptr,
+                const float* xg = nullptr) {
     ep.M = M;
     ep.N = N;
     NormState ns;
@@ -348,13 +414,15 @@ struct Proj {
       ep.ticket = m->ticket;
       ns.rinv = true;
     }
-    if (gemv && !m->fp32 && vmap && amaps && m->use_tma_gemv) {
+    if (gemv && !m->fp32 && !m->f16 && vmap && amaps && m->use_tma_gemv) {
       const int tok = gemv_tma_tokens(M);
       const int idx = tok == 8 ? 0 : (tok == 16 ? 1 : (tok == 32 ? 2 : 3));
       rc = launch_gemv_tma(lc, kind, *vmap, amaps[idx], N, K, M, ep, m->tmawork);
       ns.parts = N / 16;
     } else if (gemv) {
-      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk);
+      const bool xs = m->f16 && xg && act == m->a;
+      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk, xs ? m->x : nullptr,
+                       xs ? xg : nullptr);
       ns.parts = N / 16;
     } else if (m->fp32) {
       rc = launch_gemm_simt(lc, kind, static_cast<const float*>(act), act_stride, static_cast<const float*>(W), M, N,
@@ -371,7 +439,8 @@ struct Proj {
 int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32_t* bt, int logits_mode, float* logits,
                     int32_t* next, cudaStream_t st, Prof* pf = nullptr) {
   const int M = B * S;
-  LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms};
+  LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms, m->f16};
+  g_trace_stream = st;
   const double es = static_cast<double>(m->esz);
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * m->H * m->d * es,
                wgu = 2.0 * m->F * m->D * es, wdn = static_cast<double>(m->D) * m->F * es,
@@ -380,7 +449,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
   const int D = m->D, Hd = m->H * m->d;
   pbeg(pf, "embed");
   CK(launch_embed(lc, m->fp32, m->embed, m->V, D, ids, M, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
-                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err));
+                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err, M > 64 ? m->a_lo : nullptr));
   pend(pf, static_cast<double>(M) * D * (es + 4 + es), 0);
   NormState ns;
   ns.rinv = true;
@@ -393,7 +462,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
     pbeg(pf, "prefill_qkv");
-    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, M, e);
+    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, M, e, nullptr, nullptr, w.g1);
     CK(pj.rc);
     pend(pf, wq + M * (D + m->Nqkv) * es, 2.0 * M * m->Nqkv * D);
 
@@ -421,7 +490,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     set_norm(m, ns, g);
     g.u_out = m->u;
     pbeg(pf, "prefill_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, M, g);
+    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, M, g, nullptr, nullptr, w.g2);
     CK(pj.rc);
     pend(pf, wgu + M * (D + m->F) * es, 2.0 * M * 2 * m->F * D);
 
@@ -432,6 +501,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
+    if (l + 1 < m->L && M > 64) dn.a_lo_out = m->a_lo;
     pbeg(pf, "prefill_down");
     ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, M, dn);
     CK(pj.rc);
@@ -459,7 +529,8 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     h.N = m->V;
     pbeg(pf, "prefill_lm_head");
     CK(launch_gemv(lc, EPI_LOGITS, m->fp32, m->head, m->V, D, static_cast<char*>(m->a) + off,
-                   static_cast<long long>(S) * D, B, h, m->splitk));
+                   static_cast<long long>(S) * D, B, h, m->splitk,
+                   m->f16 ? m->x + static_cast<size_t>(S - 1) * D : nullptr, m->f16 ? m->gf : nullptr));
     pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
     pbeg(pf, "finalize");
     CK(launch_finalize(lc, m->keys, B, 1, 0, B, next, nullptr));
@@ -471,7 +542,8 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt, float* logits,
                    int32_t* next, cudaStream_t st, Prof* pf = nullptr, double kv_tokens = 0,
                    float* attn_part = nullptr, int* attn_cnt = nullptr, int attn_rows_cap = 0) {
-  LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms};
+  LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms, m->f16};
+  g_trace_stream = st;
   Proj pj{m, lc};
   const int D = m->D, Hd = m->H * m->d;
   const double es = static_cast<double>(m->esz);
@@ -500,7 +572,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
     pbeg(pf, "decode_qkv");
-    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok);
+    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok, w.g1);
     CK(pj.rc);
     pend(pf, wq + B * (D + m->Nqkv) * es, 2.0 * B * m->Nqkv * D);
 
@@ -533,7 +605,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     set_norm(m, ns, g);
     g.u_out = m->u;
     pbeg(pf, "decode_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok);
+    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok, w.g2);
     CK(pj.rc);
     pend(pf, wgu + B * (D + m->F) * es, 2.0 * B * 2 * m->F * D);
 
@@ -558,7 +630,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   h.logits = logits;
   h.logits_stride = m->V;
   pbeg(pf, "decode_lm_head");
-  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok);
+  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok, m->gf);
   CK(pj.rc);
   pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
   pbeg(pf, "finalize");
@@ -640,10 +712,12 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->V = cfg->vocab_size;
   m->Nqkv = (m->H + 2 * m->G) * m->d;
   m->fp32 = cfg->precision == AXON_FP32_DEBUG;
+  m->f16 = cfg->precision == AXON_FP16;
   m->esz = m->fp32 ? 4 : 2;
   m->use_graphs = !env_flag("AXON_NO_GRAPH");
   m->use_pdl = !env_flag("AXON_NO_PDL");
   m->use_tma_gemv = env_flag("AXON_TMA_GEMV");
+  g_trace = env_flag("AXON_TRACE");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   auto fail = [&](int code) {
     cudaStreamSynchronize(st);
@@ -735,36 +809,14 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     // gate/up interleave: packed row r: chunk r/16, slots 0..7 gate, 8..15 up.
     if ((rc = dev_alloc(m, &w.wgu, static_cast<size_t>(2 * F) * D * es))) return fail(rc);
     {
-      // Build the interleaved matrix in two gathers over a [2F] row map whose
-      // entries index a virtual [gate; up] stack: stage gate and up into one
-      // contiguous buffer first.
-      const axon_tensor* tg = bl.find(p + "mlp.gate_proj.weight");
-      const axon_tensor* tu = bl.find(p + "mlp.up_proj.weight");
-      void* tmp = nullptr;
-      const size_t half = static_cast<size_t>(F) * D * es;
-      if (cudaMalloc(&tmp, 2 * half) != cudaSuccess) {
-        cudaGetLastError();
-        return fail(AXON_ERR_OOM);
+      // gate row j -> packed row (j/8)*16 + j%8, up row j -> (j/8)*16 + 8 + j%8
+      std::vector<int> to_gate(F), to_up(F);
+      for (int j = 0; j < F; ++j) {
+        to_gate[j] = (j >> 3) * 16 + (j & 7);
+        to_up[j] = (j >> 3) * 16 + 8 + (j & 7);
       }
-      int r1 = bl.gather(tmp, f32, tg, nullptr, F, D);
-      if (!r1) r1 = bl.gather(static_cast<char*>(tmp) + half, f32, tu, nullptr, F, D);
-      if (!r1) {
-        std::vector<int> imap(2 * F);
-        for (int r = 0; r < 2 * F; ++r) {
-          const int c = r >> 4, i = r & 15;
-          imap[r] = i < 8 ? c * 8 + i : F + c * 8 + (i - 8);
-        }
-        axon_tensor stack{};
-        stack.name = "gate_up";
-        stack.data = tmp;
-        stack.dtype = f32 ? AXON_DTYPE_F32 : AXON_DTYPE_BF16;
-        stack.ndim = 2;
-        stack.shape[0] = 2 * F;
-        stack.shape[1] = D;
-        r1 = bl.gather(w.wgu, f32, &stack, &imap, 2 * F, D);
-      }
-      cudaFree(tmp);
-      if (r1) return fail(r1);
+      if ((rc = bl.gather(w.wgu, f32, bl.find(p + "mlp.gate_proj.weight"), nullptr, F, D, &to_gate))) return fail(rc);
+      if ((rc = bl.gather(w.wgu, f32, bl.find(p + "mlp.up_proj.weight"), nullptr, F, D, &to_up))) return fail(rc);
     }
     if ((rc = dev_alloc(m, &w.wd, static_cast<size_t>(D) * F * es))) return fail(rc);
     if ((rc = bl.gather(w.wd, f32, bl.find(p + "mlp.down_proj.weight"), nullptr, D, F))) return fail(rc);
@@ -819,6 +871,10 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * D * 4))) return fail(rc);
   m->x = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &m->a, static_cast<size_t>(Mcap) * D * es))) return fail(rc);
+  if (m->f16) {
+    if ((rc = dev_alloc(m, &m->a_lo, static_cast<size_t>(Mcap) * D * es))) return fail(rc);
+    if (cudaMemsetAsync(m->a_lo, 0, static_cast<size_t>(Mcap) * D * es, st) != cudaSuccess) return fail(AXON_ERR_CUDA);
+  }
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * m->Pmax * 4))) return fail(rc);
   m->ss = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &m->q, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
@@ -871,32 +927,37 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
 
   // ---- TMA descriptors (bf16 tensor-core path)
   if (!f32) {
-    bool ok = make_tma_2d_bf16(&m->t_a, m->a, Mcap, D, 128) && make_tma_2d_bf16(&m->t_o, m->o, Mcap, Hd, 128) &&
-              make_tma_2d_bf16(&m->t_u, m->u, Mcap, F, 128);
+    bool ok = make_tma_2d_16(&m->t_a, m->a, Mcap, D, 128, m->f16) && make_tma_2d_16(&m->t_o, m->o, Mcap, Hd, 128, m->f16) &&
+              make_tma_2d_16(&m->t_u, m->u, Mcap, F, 128, m->f16);
+    if (ok && m->a_lo) ok = make_tma_2d_16(&m->t_alo, m->a_lo, Mcap, D, 128, m->f16);
     for (int l = 0; l < m->L && ok; ++l) {
       LayerW& w = m->layers[l];
       w.m_qkv.a = m->t_a;
-      ok = ok && make_tma_2d_bf16(&w.m_qkv.w, w.wqkv, m->Nqkv, D, 256);
+      ok = ok && make_tma_2d_16(&w.m_qkv.w, w.wqkv, m->Nqkv, D, 256, m->f16);
+      if (m->a_lo) {
+        w.m_qkv.a_lo = m->t_alo;
+        w.m_qkv.split = true;
+      }
       w.m_o.a = m->t_o;
-      ok = ok && make_tma_2d_bf16(&w.m_o.w, w.wo, D, Hd, 256);
+      ok = ok && make_tma_2d_16(&w.m_o.w, w.wo, D, Hd, 256, m->f16);
       w.m_gu.a = m->t_a;
-      ok = ok && make_tma_2d_bf16(&w.m_gu.w, w.wgu, 2 * F, D, 256);
+      ok = ok && make_tma_2d_16(&w.m_gu.w, w.wgu, 2 * F, D, 256, m->f16);
       w.m_d.a = m->t_u;
-      ok = ok && make_tma_2d_bf16(&w.m_d.w, w.wd, D, F, 256);
+      ok = ok && make_tma_2d_16(&w.m_d.w, w.wd, D, F, 256, m->f16);
     }
     m->m_head.a = m->t_a;
-    ok = ok && make_tma_2d_bf16(&m->m_head.w, m->head, V, D, 256);
+    ok = ok && make_tma_2d_16(&m->m_head.w, m->head, V, D, 256, m->f16);
     // decode projections: weight boxes of 128 rows, activation boxes of 8..64 token rows
     for (int l = 0; l < m->L && ok; ++l) {
       LayerW& w = m->layers[l];
-      ok = make_tma_2d_bf16(&w.v_qkv, w.wqkv, m->Nqkv, D, 128) && make_tma_2d_bf16(&w.v_o, w.wo, D, Hd, 128) &&
-           make_tma_2d_bf16(&w.v_gu, w.wgu, 2 * F, D, 128) && make_tma_2d_bf16(&w.v_d, w.wd, D, F, 128);
+      ok = make_tma_2d_16(&w.v_qkv, w.wqkv, m->Nqkv, D, 128, m->f16) && make_tma_2d_16(&w.v_o, w.wo, D, Hd, 128, m->f16) &&
+           make_tma_2d_16(&w.v_gu, w.wgu, 2 * F, D, 128, m->f16) && make_tma_2d_16(&w.v_d, w.wd, D, F, 128, m->f16);
     }
-    ok = ok && make_tma_2d_bf16(&m->v_head, m->head, V, D, 128);
+    ok = ok && make_tma_2d_16(&m->v_head, m->head, V, D, 128, m->f16);
     for (int i = 0; i < 4 && ok; ++i) {
       const uint32_t tok = 8u << i;
-      ok = make_tma_2d_bf16(&m->t_a_tok[i], m->a, Mcap, D, tok) && make_tma_2d_bf16(&m->t_o_tok[i], m->o, Mcap, Hd, tok) &&
-           make_tma_2d_bf16(&m->t_u_tok[i], m->u, Mcap, F, tok);
+      ok = make_tma_2d_16(&m->t_a_tok[i], m->a, Mcap, D, tok, m->f16) && make_tma_2d_16(&m->t_o_tok[i], m->o, Mcap, Hd, tok, m->f16) &&
+           make_tma_2d_16(&m->t_u_tok[i], m->u, Mcap, F, tok, m->f16);
     }
     if (!ok) return fail(AXON_ERR_CUDA);
   }

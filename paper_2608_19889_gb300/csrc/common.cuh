@@ -6,12 +6,14 @@
 
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda.h>
 #include <stdint.h>
 
 #define AXON_DEV __device__ __forceinline__
 
 typedef __nv_bfloat16 bf16;
+typedef __half f16;
 
 // Device error word bits (read by axon_check_device).
 enum : int {
@@ -32,11 +34,22 @@ AXON_DEV uint32_t pack_bf2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
 }
+// fp16 operands saturate at the largest finite half (NaN passes through).
+AXON_DEV float sat_half(float v) { return fabsf(v) > 65504.f ? copysignf(65504.f, v) : v; }
+AXON_DEV uint32_t pack_h2(float lo, float hi) {
+  __half2 h = __floats2half2_rn(sat_half(lo), sat_half(hi));
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+template <typename T> AXON_DEV uint32_t pack2(float lo, float hi);
+template <> AXON_DEV uint32_t pack2<bf16>(float lo, float hi) { return pack_bf2(lo, hi); }
+template <> AXON_DEV uint32_t pack2<f16>(float lo, float hi) { return pack_h2(lo, hi); }
 AXON_DEV float to_f(bf16 v) { return __bfloat162float(v); }
+AXON_DEV float to_f(f16 v) { return __half2float(v); }
 AXON_DEV float to_f(float v) { return v; }
 template <typename T> AXON_DEV T from_f(float v);
 template <> AXON_DEV float from_f<float>(float v) { return v; }
 template <> AXON_DEV bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+template <> AXON_DEV f16 from_f<f16>(float v) { return __float2half_rn(sat_half(v)); }
 
 // --------------------------------------------------------------- reductions
 AXON_DEV float warp_sum(float v) {
@@ -86,6 +99,18 @@ AXON_DEV void mma_bf16_16816(float* c, const uint32_t* a, const uint32_t* b) {
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
+
+AXON_DEV void mma_f16_16816(float* c, const uint32_t* a, const uint32_t* b) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+// m16n8k16 with fp32 accumulation on 16-bit operands of type T (bf16 or fp16).
+template <typename T> AXON_DEV void mma16816(float* c, const uint32_t* a, const uint32_t* b);
+template <> AXON_DEV void mma16816<bf16>(float* c, const uint32_t* a, const uint32_t* b) { mma_bf16_16816(c, a, b); }
+template <> AXON_DEV void mma16816<f16>(float* c, const uint32_t* a, const uint32_t* b) { mma_f16_16816(c, a, b); }
 
 AXON_DEV uint32_t smem_u32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
 
@@ -211,11 +236,15 @@ AXON_DEV uint64_t smem_desc_sw128(uint32_t addr) {
   d |= static_cast<uint64_t>(2u) << 61;                      // swizzle: 128B
   return d;
 }
-// Instruction descriptor: kind::f16, A=B=bf16, D=fp32, both K-major.
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+// Instruction descriptor: kind::f16, A=B=bf16 (ab_fmt 1) or fp16 (ab_fmt 0),
+// D=fp32, both K-major.
+__host__ __device__ constexpr uint32_t idesc_f32acc(int M, int N, uint32_t ab_fmt) {
   return (1u << 4)                                 // D format fp32
-         | (1u << 7)                               // A format bf16
-         | (1u << 10)                              // B format bf16
+         | (ab_fmt << 7)                           // A format
+         | (ab_fmt << 10)                          // B format
          | (static_cast<uint32_t>(N >> 3) << 17)   // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24);  // M / 16
 }
+template <typename T> struct MmaFmt;
+template <> struct MmaFmt<bf16> { static constexpr uint32_t v = 1; };
+template <> struct MmaFmt<f16> { static constexpr uint32_t v = 0; };

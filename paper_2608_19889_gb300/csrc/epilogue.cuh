@@ -53,6 +53,7 @@ struct EpiArgs {
   // RESID
   float* x;            // [M][N] residual (in/out)
   void* a_out;         // [M][N] x * gain
+  void* a_lo_out;      // optional [M][N]: x * gain - a_out (residual of the rounding), same type
   const float* gain;   // [N]
   float* ss_out;       // [M][ss_out_stride]
   int ss_out_stride;
@@ -111,6 +112,15 @@ AXON_DEV void store8<bf16>(bf16* dst, const float* v) {
   u.y = pack_bf2(v[2], v[3]);
   u.z = pack_bf2(v[4], v[5]);
   u.w = pack_bf2(v[6], v[7]);
+  *reinterpret_cast<uint4*>(dst) = u;
+}
+template <>
+AXON_DEV void store8<f16>(f16* dst, const float* v) {
+  uint4 u;
+  u.x = pack_h2(v[0], v[1]);
+  u.y = pack_h2(v[2], v[3]);
+  u.z = pack_h2(v[4], v[5]);
+  u.w = pack_h2(v[6], v[7]);
   *reinterpret_cast<uint4*>(dst) = u;
 }
 template <>
@@ -195,6 +205,16 @@ AXON_DEV float epi_resid16(const EpiArgs& e, int m, int n0, const float* v) {
   T* ap = reinterpret_cast<T*>(e.a_out) + static_cast<long long>(m) * e.N + n0;
   store8<T>(ap, ag);
   store8<T>(ap + 8, ag + 8);
+  if (e.a_lo_out) {
+    // second 16-bit term: what rounding a_out lost (split operand for the
+    // next QKV projection)
+    float lo[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) lo[i] = ag[i] - to_f(from_f<T>(ag[i]));
+    T* lp = reinterpret_cast<T*>(e.a_lo_out) + static_cast<long long>(m) * e.N + n0;
+    store8<T>(lp, lo);
+    store8<T>(lp + 8, lo + 8);
+  }
   return s;
 }
 

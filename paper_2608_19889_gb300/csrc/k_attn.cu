@@ -35,7 +35,7 @@ AXON_DEV uint32_t swz(uint32_t base, int tok, int ch) {
 // Copy one (block, kv head) tile of 16 x HD bf16 into swizzled shared memory
 // with `nthreads` cooperating threads starting at `tid`.
 template <int HD>
-AXON_DEV void stage_tile(uint32_t dst, const bf16* src, bool valid, int tid, int nthreads) {
+AXON_DEV void stage_tile(uint32_t dst, const uint16_t* src, bool valid, int tid, int nthreads) {
   constexpr int CH = HD / 8;
   for (int c = tid; c < 16 * CH; c += nthreads) {
     const int tok = c / CH, ch = c % CH;
@@ -44,7 +44,7 @@ AXON_DEV void stage_tile(uint32_t dst, const bf16* src, bool valid, int tid, int
 }
 
 template <int HD>
-AXON_DEV void load_q(uint32_t (&qa)[HD / 16][4], const bf16* row0, const bf16* row1, int q) {
+AXON_DEV void load_q(uint32_t (&qa)[HD / 16][4], const uint16_t* row0, const uint16_t* row1, int q) {
 #pragma unroll
   for (int kk = 0; kk < HD / 16; ++kk) {
     const int k = kk * 16 + 2 * q;
@@ -69,7 +69,7 @@ struct WarpState {
 
 // One 16-key tile: keys tok0 .. tok0+15; key t is visible to row r (r+8)
 // iff t <= lim0 (lim1).
-template <int HD>
+template <int HD, typename T16>
 AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16][4], WarpState<HD>& st, int tok0,
                           int lim0, int lim1, float sl2, int lane) {
   const int q = lane & 3;
@@ -83,8 +83,8 @@ AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16
     const int tok = (mi >> 1) * 8 + li, ch = 2 * kk + (mi & 1);
     ldsm_x4(kb, swz<HD>(ks, tok, ch));
     const uint32_t b0[2] = {kb[0], kb[1]}, b1[2] = {kb[2], kb[3]};
-    mma_bf16_16816(s[0], qa[kk], b0);
-    mma_bf16_16816(s[1], qa[kk], b1);
+    mma16816<T16>(s[0], qa[kk], b0);
+    mma16816<T16>(s[1], qa[kk], b1);
   }
   float mx0 = NEG_INF, mx1 = NEG_INF;
 #pragma unroll
@@ -127,16 +127,16 @@ AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16
     st.o[nd][2] *= a1;
     st.o[nd][3] *= a1;
   }
-  const uint32_t pa[4] = {pack_bf2(s[0][0], s[0][1]), pack_bf2(s[0][2], s[0][3]), pack_bf2(s[1][0], s[1][1]),
-                          pack_bf2(s[1][2], s[1][3])};
+  const uint32_t pa[4] = {pack2<T16>(s[0][0], s[0][1]), pack2<T16>(s[0][2], s[0][3]),
+                          pack2<T16>(s[1][0], s[1][1]), pack2<T16>(s[1][2], s[1][3])};
 #pragma unroll
   for (int nd2 = 0; nd2 < HD / 16; ++nd2) {
     uint32_t vb[4];
     const int tok = (mi & 1) * 8 + li, ch = 2 * nd2 + (mi >> 1);
     ldsm_x4_t(vb, swz<HD>(vs, tok, ch));
     const uint32_t b0[2] = {vb[0], vb[1]}, b1[2] = {vb[2], vb[3]};
-    mma_bf16_16816(st.o[2 * nd2], pa, b0);
-    mma_bf16_16816(st.o[2 * nd2 + 1], pa, b1);
+    mma16816<T16>(st.o[2 * nd2], pa, b0);
+    mma16816<T16>(st.o[2 * nd2 + 1], pa, b1);
   }
 }
 
@@ -148,7 +148,7 @@ AXON_DEV int block_of(const AttnArgs& p, int b, int j, bool& ok) {
 }
 
 // --------------------------------------------------------------- decode
-template <int HD>
+template <int HD, typename T16>
 __global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p) {
   extern __shared__ __align__(128) uint8_t sm[];
   constexpr int TILE = 16 * HD * 2;
@@ -172,15 +172,15 @@ __global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p)
   if (s >= n_used) return;
   const int jb = s * per, je = min(jb + per, nblk);
 
-  const bf16* qg = static_cast<const bf16*>(p.q) + (static_cast<long long>(b) * p.H + g * HPG) * HD;
+  const uint16_t* qg = static_cast<const uint16_t*>(p.q) + (static_cast<long long>(b) * p.H + g * HPG) * HD;
   uint32_t qa[HD / 16][4];
   load_q<HD>(qa, r < HPG ? qg + r * HD : nullptr, r + 8 < HPG ? qg + (r + 8) * HD : nullptr, q);
 
   WarpState<HD> st;
   st.init();
   const uint32_t wbase = smem_u32(sm) + warp * 4 * TILE;  // per warp: [stage][K | V]
-  const bf16* kp = static_cast<const bf16*>(p.k);
-  const bf16* vp = static_cast<const bf16*>(p.v);
+  const uint16_t* kp = static_cast<const uint16_t*>(p.k);
+  const uint16_t* vp = static_cast<const uint16_t*>(p.v);
   auto issue = [&](int j, int stg) {
     bool ok;
     const int blk = block_of(p, b, j, ok);
@@ -200,8 +200,8 @@ __global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p)
       cp_async_wait<0>();
     }
     __syncwarp();
-    attn_tile16<HD>(wbase + stg * 2 * TILE, wbase + stg * 2 * TILE + TILE, qa, st, j * 16, T - 1, T - 1,
-                    p.scale_log2, lane);
+    attn_tile16<HD, T16>(wbase + stg * 2 * TILE, wbase + stg * 2 * TILE + TILE, qa, st, j * 16, T - 1, T - 1,
+                         p.scale_log2, lane);
     __syncwarp();
     stg ^= 1;
   }
@@ -249,8 +249,8 @@ __global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p)
       }
     }
     if (n_used == 1) {
-      bf16* og = static_cast<bf16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
-      *og = __float2bfloat16_rn(L > 0.f ? O / L : 0.f);
+      T16* og = static_cast<T16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
+      *og = from_f<T16>(L > 0.f ? O / L : 0.f);
     } else {
       float* pr = part + (static_cast<long long>(s) * 16 + i) * rowlen;
       pr[dd] = O;
@@ -307,8 +307,8 @@ __global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p)
       O3 += cw[i][t + 3] * v3;
     }
     for (; t < n_used; ++t) O0 += cw[i][t] * __ldcg(pc + t * 16 * rowlen);
-    bf16* og = static_cast<bf16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
-    *og = __float2bfloat16_rn(((O0 + O1) + (O2 + O3)) * cinv[i]);
+    T16* og = static_cast<T16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
+    *og = from_f<T16>(((O0 + O1) + (O2 + O3)) * cinv[i]);
   }
   if (threadIdx.x == 0) p.counter[b * p.G + g] = 0;
 }
@@ -317,7 +317,7 @@ __global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p)
 // CTA: 4 warps x PW positions x (H/G) heads of one kv head g of sequence b;
 // key tiles staged 4 blocks (64 keys) at a time, double-buffered, shared by
 // the 4 warps.
-template <int HD>
+template <int HD, typename T16>
 __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   extern __shared__ __align__(128) uint8_t sm[];
   constexpr int TILE = 16 * HD * 2;
@@ -338,10 +338,12 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   int pos0, h0, pos1, h1;
   row_info(r, pos0, h0);
   row_info(r + 8, pos1, h1);
-  const bf16* qbase = static_cast<const bf16*>(p.q);
+  const uint16_t* qbase = static_cast<const uint16_t*>(p.q);
   const long long Hd = static_cast<long long>(p.H) * HD;
-  const bf16* qr0 = pos0 >= 0 ? qbase + (static_cast<long long>(b) * S + pos0) * Hd + (g * HPG + h0) * HD : nullptr;
-  const bf16* qr1 = pos1 >= 0 ? qbase + (static_cast<long long>(b) * S + pos1) * Hd + (g * HPG + h1) * HD : nullptr;
+  const uint16_t* qr0 =
+      pos0 >= 0 ? qbase + (static_cast<long long>(b) * S + pos0) * Hd + (g * HPG + h0) * HD : nullptr;
+  const uint16_t* qr1 =
+      pos1 >= 0 ? qbase + (static_cast<long long>(b) * S + pos1) * Hd + (g * HPG + h1) * HD : nullptr;
   uint32_t qa[HD / 16][4];
   load_q<HD>(qa, qr0, qr1, q);
 
@@ -353,8 +355,8 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   const int wfirst = p0 + warp * PW;
   const int wmax = min(wfirst + PW - 1, S - 1);
   const uint32_t base = smem_u32(sm);
-  const bf16* kp = static_cast<const bf16*>(p.k);
-  const bf16* vp = static_cast<const bf16*>(p.v);
+  const uint16_t* kp = static_cast<const uint16_t*>(p.k);
+  const uint16_t* vp = static_cast<const uint16_t*>(p.v);
   auto issue = [&](int stage_idx, int buf) {
     for (int jj = 0; jj < 4; ++jj) {
       const int j = stage_idx * 4 + jj;
@@ -383,7 +385,7 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
         const int j = sidx * 4 + jj;
         if (j >= nblk || j * 16 > wmax) break;
         const uint32_t t = base + buf * STAGE + jj * 2 * TILE;
-        attn_tile16<HD>(t, t + TILE, qa, st, j * 16, pos0, pos1, p.scale_log2, lane);
+        attn_tile16<HD, T16>(t, t + TILE, qa, st, j * 16, pos0, pos1, p.scale_log2, lane);
       }
     }
     __syncthreads();
@@ -393,17 +395,17 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   st.l0 += __shfl_xor_sync(0xffffffffu, st.l0, 2);
   st.l1 += __shfl_xor_sync(0xffffffffu, st.l1, 1);
   st.l1 += __shfl_xor_sync(0xffffffffu, st.l1, 2);
-  bf16* ob = static_cast<bf16*>(p.o);
+  T16* ob = static_cast<T16*>(p.o);
   const float inv0 = st.l0 > 0.f ? 1.f / st.l0 : 0.f, inv1 = st.l1 > 0.f ? 1.f / st.l1 : 0.f;
 #pragma unroll
   for (int nd = 0; nd < HD / 8; ++nd) {
     if (pos0 >= 0) {
-      bf16* d0 = ob + (static_cast<long long>(b) * S + pos0) * Hd + (g * HPG + h0) * HD + nd * 8 + 2 * q;
-      *reinterpret_cast<uint32_t*>(d0) = pack_bf2(st.o[nd][0] * inv0, st.o[nd][1] * inv0);
+      T16* d0 = ob + (static_cast<long long>(b) * S + pos0) * Hd + (g * HPG + h0) * HD + nd * 8 + 2 * q;
+      *reinterpret_cast<uint32_t*>(d0) = pack2<T16>(st.o[nd][0] * inv0, st.o[nd][1] * inv0);
     }
     if (pos1 >= 0) {
-      bf16* d1 = ob + (static_cast<long long>(b) * S + pos1) * Hd + (g * HPG + h1) * HD + nd * 8 + 2 * q;
-      *reinterpret_cast<uint32_t*>(d1) = pack_bf2(st.o[nd][2] * inv1, st.o[nd][3] * inv1);
+      T16* d1 = ob + (static_cast<long long>(b) * S + pos1) * Hd + (g * HPG + h1) * HD + nd * 8 + 2 * q;
+      *reinterpret_cast<uint32_t*>(d1) = pack2<T16>(st.o[nd][2] * inv1, st.o[nd][3] * inv1);
     }
   }
 }
@@ -478,7 +480,8 @@ constexpr size_t prefill_smem() { return 2 * 4 * 2 * 16 * HD * 2; }  // 2 stages
 template <int HD>
 cudaError_t decode_hd(const LaunchCtx& lc, const AttnArgs& a, int B) {
   const size_t smem = decode_smem<HD>();
-  return launch_k(lc, attn_decode_kernel<HD>, dim3(a.splits, a.G, B), dim3(DEC_WARPS * 32), smem, a);
+  if (lc.f16) return launch_k(lc, attn_decode_kernel<HD, f16>, dim3(a.splits, a.G, B), dim3(DEC_WARPS * 32), smem, a);
+  return launch_k(lc, attn_decode_kernel<HD, bf16>, dim3(a.splits, a.G, B), dim3(DEC_WARPS * 32), smem, a);
 }
 
 template <int HD>
@@ -487,21 +490,36 @@ cudaError_t prefill_hd(const LaunchCtx& lc, const AttnArgs& a, int B) {
   const int HPG = a.H / a.G;
   const int PW = 16 / HPG;
   const int PC = 4 * PW;
-  return launch_k(lc, attn_prefill_kernel<HD>, dim3((a.S + PC - 1) / PC, a.G, B), dim3(128), smem, a, PW);
+  const dim3 grid((a.S + PC - 1) / PC, a.G, B);
+  if (lc.f16) return launch_k(lc, attn_prefill_kernel<HD, f16>, grid, dim3(128), smem, a, PW);
+  return launch_k(lc, attn_prefill_kernel<HD, bf16>, grid, dim3(128), smem, a, PW);
 }
 
 }  // namespace
 
-cudaError_t prepare_attn_kernels() {
+namespace {
+template <typename T16>
+cudaError_t prepare_attn_t() {
   cudaError_t e = cudaSuccess;
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_decode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decode_smem<64>());
+    e = cudaFuncSetAttribute(attn_decode_kernel<64, T16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)decode_smem<64>());
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_decode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)decode_smem<128>());
+    e = cudaFuncSetAttribute(attn_decode_kernel<128, T16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)decode_smem<128>());
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_prefill_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)prefill_smem<64>());
+    e = cudaFuncSetAttribute(attn_prefill_kernel<64, T16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)prefill_smem<64>());
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_prefill_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)prefill_smem<128>());
+    e = cudaFuncSetAttribute(attn_prefill_kernel<128, T16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)prefill_smem<128>());
+  return e;
+}
+}  // namespace
+
+cudaError_t prepare_attn_kernels() {
+  cudaError_t e = prepare_attn_t<bf16>();
+  if (e == cudaSuccess) e = prepare_attn_t<f16>();
   return e;
 }
 

@@ -23,14 +23,22 @@
 
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4, GROUP_M = 8;
+constexpr int BM = 128, BN = 256, BK = 64, GROUP_M = 8;
 constexpr int A_BYTES = BM * BK * 2;  // 16 KB
 constexpr int B_BYTES = BN * BK * 2;  // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
 constexpr int NUM_THREADS = 192;
 constexpr uint32_t TMEM_COLS = 2 * BN;
+
+// SPLIT: the A operand is the sum of two 16-bit terms (hi + lo) and every
+// k-step issues two MMAs into the same accumulator (3 ring stages of 64 KB).
+template <bool SPLIT>
+struct GCfg {
+  static constexpr int STAGES = SPLIT ? 3 : 4;
+  static constexpr int A_TERMS = SPLIT ? 2 : 1;
+  static constexpr int STAGE_BYTES = A_TERMS * A_BYTES + B_BYTES;
+  static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
+};
 
 AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
   const int per_group = GROUP_M * num_n;
@@ -42,14 +50,18 @@ AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
   mb = first_m + (local - nb * gm);
 }
 
-template <int KIND>
+template <int KIND, typename T16, bool SPLIT>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, EpiArgs ep) {
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmAlo, int M, int N, int K, EpiArgs ep) {
+  using C = GCfg<SPLIT>;
+  constexpr int STAGES = C::STAGES;
+  constexpr int STAGE_BYTES = C::STAGE_BYTES;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t sA = base, sB = base + STAGES * A_BYTES;
+  // ring: [STAGES] A tiles, [STAGES] A_lo tiles (SPLIT), [STAGES] B tiles
+  const uint32_t sA = base, sAlo = base + STAGES * A_BYTES, sB = base + STAGES * A_BYTES * C::A_TERMS;
   const uint32_t bars = base + STAGES * STAGE_BYTES;
   const uint32_t tmem_slot = bars + 8 * (2 * STAGES + 4);
   const uint32_t* tmem_slot_ptr =
@@ -73,6 +85,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fence_proxy_async();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    if (SPLIT) tma_prefetch_desc(&tmAlo);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, TMEM_COLS);
@@ -103,6 +116,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           mbar_arrive_expect_tx(full_bar(s), STAGE_BYTES);
           tma_load_2d(sA + s * A_BYTES, &tmA, full_bar(s), kb * BK, mb * BM);
+          if (SPLIT) tma_load_2d(sAlo + s * A_BYTES, &tmAlo, full_bar(s), kb * BK, mb * BM);
           tma_load_2d(sB + s * B_BYTES, &tmB, full_bar(s), kb * BK, nb * BN);
         }
       }
@@ -110,7 +124,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      constexpr uint32_t idesc = idesc_f32acc(BM, BN, MmaFmt<T16>::v);
       int it = 0, lt = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++lt) {
@@ -132,6 +146,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K inside the swizzle atom
             tc_mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
+          if (SPLIT) {
+            const uint64_t ald = smem_desc_sw128(sAlo + s * A_BYTES);
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k) tc_mma_f16(d, ald + 2 * k, bd + 2 * k, idesc, 1u);
+          }
           tc_commit(empty_bar(s));
         }
         if (ok) tc_commit(accf_bar(buf));
@@ -169,11 +188,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(v[i]);
           if (KIND == EPI_QKV) {
-            epi_qkv16<bf16>(ep, m, n0, f, rinv);
+            epi_qkv16<T16>(ep, m, n0, f, rinv);
           } else if (KIND == EPI_RESID) {
-            ssum += epi_resid16<bf16>(ep, m, n0, f);
+            ssum += epi_resid16<T16>(ep, m, n0, f);
           } else if (KIND == EPI_SWIGLU) {
-            epi_swiglu16<bf16>(ep, m, n0, f, rinv);
+            epi_swiglu16<T16>(ep, m, n0, f, rinv);
           } else {
             const unsigned long long k = epi_logits16(ep, m, n0, f, rinv);
             best = k > best ? k : best;
@@ -207,55 +226,75 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int KIND>
+template <int KIND, typename T16, bool SPLIT>
 cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep) {
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const int grid = tiles < lc.num_sms ? tiles : lc.num_sms;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(NUM_THREADS);
-  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.dynamicSmemBytes = GCfg<SPLIT>::SMEM;
   cfg.stream = lc.stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = lc.pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND>, maps.a, maps.w, M, N, K, ep);
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT>, maps.a, maps.w, SPLIT ? maps.a_lo : maps.a, M, N,
+                            K, ep);
 }
 
 }  // namespace
 
-bool make_tma_2d_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+bool make_tma_2d_16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows, bool f16) {
   PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
   if (!fn || (reinterpret_cast<uintptr_t>(base) & 15) || ((cols * 2) & 15)) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
   cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  return fn(map, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+namespace {
+template <int KIND, typename T16, bool SPLIT>
+cudaError_t set_smem() {
+  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              GCfg<SPLIT>::SMEM);
+}
+template <typename T16>
+cudaError_t prepare_gemm_t() {
+  cudaError_t e = set_smem<EPI_QKV, T16, false>();
+  if (e == cudaSuccess) e = set_smem<EPI_QKV, T16, true>();
+  if (e == cudaSuccess) e = set_smem<EPI_RESID, T16, false>();
+  if (e == cudaSuccess) e = set_smem<EPI_SWIGLU, T16, false>();
+  if (e == cudaSuccess) e = set_smem<EPI_LOGITS, T16, false>();
+  return e;
+}
+template <typename T16>
+cudaError_t launch_t(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep) {
+  switch (kind) {
+    case EPI_QKV:
+      return maps.split ? launch_kind<EPI_QKV, T16, true>(lc, maps, M, N, K, ep)
+                        : launch_kind<EPI_QKV, T16, false>(lc, maps, M, N, K, ep);
+    case EPI_RESID: return launch_kind<EPI_RESID, T16, false>(lc, maps, M, N, K, ep);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false>(lc, maps, M, N, K, ep);
+    default: return launch_kind<EPI_LOGITS, T16, false>(lc, maps, M, N, K, ep);
+  }
+}
+}  // namespace
+
 cudaError_t prepare_gemm_kernels() {
-  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(gemm_tc_kernel<EPI_LOGITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  cudaError_t e = prepare_gemm_t<bf16>();
+  if (e == cudaSuccess) e = prepare_gemm_t<f16>();
   return e;
 }
 
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K,
                            const EpiArgs& ep) {
   if (M < 1 || N < 1 || K < BK || (K % BK)) return cudaErrorInvalidValue;
-  switch (kind) {
-    case EPI_QKV: return launch_kind<EPI_QKV>(lc, maps, M, N, K, ep);
-    case EPI_RESID: return launch_kind<EPI_RESID>(lc, maps, M, N, K, ep);
-    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU>(lc, maps, M, N, K, ep);
-    default: return launch_kind<EPI_LOGITS>(lc, maps, M, N, K, ep);
-  }
+  if (lc.f16) return launch_t<f16>(lc, kind, maps, M, N, K, ep);
+  return launch_t<bf16>(lc, kind, maps, M, N, K, ep);
 }

@@ -11,6 +11,8 @@
 // elements into the fragment slots in a fixed permutation that the token
 // operand mirrors. Partial sums meet in shared memory in a fixed warp order
 // (deterministic), then one thread per token runs the fused epilogue.
+#include <type_traits>
+
 #include "kernels.h"
 
 namespace {
@@ -56,10 +58,17 @@ AXON_DEV void finish_rinv(const EpiArgs& ep, int B, int nparts) {
   if (threadIdx.x == 0) *ep.ticket = 0;
 }
 
-template <int NT, int KIND>
-__global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __restrict__ W, int N, int K,
-                                                               const bf16* __restrict__ act, long long act_stride,
-                                                               int B, EpiArgs ep, SplitK sk) {
+// XS: the activation operand is formed in fp32 from the residual x and the
+// norm gain (x * gain, rows act_stride floats apart) and fed to the tensor
+// cores as two 16-bit terms (hi = round(x*gain), lo = round(x*gain - hi)),
+// two MMAs per k-step: the operand carries ~22 significant bits instead of
+// 11. (`act` is unused then.)
+template <int NT, int KIND, typename T16, bool XS>
+__global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const T16* __restrict__ W, int N, int K,
+                                                               const T16* __restrict__ act, long long act_stride,
+                                                               int B, EpiArgs ep, SplitK sk,
+                                                               const float* __restrict__ xres,
+                                                               const float* __restrict__ gain) {
   constexpr int TOK = NT * 8;
   __shared__ float red[GEMV_KW][16][TOK + 1];
   __shared__ float rinv_s[TOK];
@@ -75,38 +84,73 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __re
   const int per = (K >> 6) / sk.count;
   const int c_begin = blockIdx.y * per;
   const int nchunks = (blockIdx.y == sk.count - 1) ? (K >> 6) - c_begin : per;
-  const bf16* w0 = W + static_cast<long long>(row0) * K + 16 * q + c_begin * 64;
-  const bf16* w1 = W + static_cast<long long>(row1) * K + 16 * q + c_begin * 64;
+  const T16* w0 = W + static_cast<long long>(row0) * K + 16 * q + c_begin * 64;
+  const T16* w1 = W + static_cast<long long>(row1) * K + 16 * q + c_begin * 64;
 
   float acc[NT][4];
 #pragma unroll
   for (int t = 0; t < NT; ++t) acc[t][0] = acc[t][1] = acc[t][2] = acc[t][3] = 0.f;
 
-  const bf16* arow[NT];
+  const T16* arow[NT];
+  const float* xrow[NT];
   bool aval[NT];
 #pragma unroll
   for (int t = 0; t < NT; ++t) {
     const int tok = t * 8 + r;
     aval[t] = tok < B;
     arow[t] = act + static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q + c_begin * 64;
+    if (XS) xrow[t] = xres + static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q + c_begin * 64;
   }
+  const float* grow = XS ? gain + 16 * q + c_begin * 64 : nullptr;
 
   auto chunk = [&](int c, const uint4& wa0, const uint4& wa1, const uint4& wb0, const uint4& wb1) {
     const uint32_t A0[8] = {wa0.x, wa0.y, wa0.z, wa0.w, wa1.x, wa1.y, wa1.z, wa1.w};
     const uint32_t A1[8] = {wb0.x, wb0.y, wb0.z, wb0.w, wb1.x, wb1.y, wb1.z, wb1.w};
 #pragma unroll
     for (int t = 0; t < NT; ++t) {
-      uint4 x0 = make_uint4(0, 0, 0, 0), x1 = make_uint4(0, 0, 0, 0);
-      if (aval[t]) {
-        x0 = ld16(arow[t] + c * 64);
-        x1 = ld16(arow[t] + c * 64 + 8);
-      }
-      const uint32_t Bv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+      if (XS) {
+        float v[16];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t a[4] = {A0[2 * j], A1[2 * j], A0[2 * j + 1], A1[2 * j + 1]};
-        const uint32_t bb[2] = {Bv[2 * j], Bv[2 * j + 1]};
-        mma_bf16_16816(acc[t], a, bb);
+        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+        if (aval[t]) {
+#pragma unroll
+          for (int i = 0; i < 16; i += 4) {
+            const float4 xv = *reinterpret_cast<const float4*>(xrow[t] + c * 64 + i);
+            const float4 gv = *reinterpret_cast<const float4*>(grow + c * 64 + i);
+            v[i] = xv.x * gv.x;
+            v[i + 1] = xv.y * gv.y;
+            v[i + 2] = xv.z * gv.z;
+            v[i + 3] = xv.w * gv.w;
+          }
+        }
+        uint32_t Bh[8], Bl[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float h0 = to_f(from_f<T16>(v[2 * i])), h1 = to_f(from_f<T16>(v[2 * i + 1]));
+          Bh[i] = pack2<T16>(h0, h1);
+          Bl[i] = pack2<T16>(v[2 * i] - h0, v[2 * i + 1] - h1);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t a[4] = {A0[2 * j], A1[2 * j], A0[2 * j + 1], A1[2 * j + 1]};
+          const uint32_t bh[2] = {Bh[2 * j], Bh[2 * j + 1]};
+          const uint32_t bl[2] = {Bl[2 * j], Bl[2 * j + 1]};
+          mma16816<T16>(acc[t], a, bh);
+          mma16816<T16>(acc[t], a, bl);
+        }
+      } else {
+        uint4 x0 = make_uint4(0, 0, 0, 0), x1 = make_uint4(0, 0, 0, 0);
+        if (aval[t]) {
+          x0 = ld16(arow[t] + c * 64);
+          x1 = ld16(arow[t] + c * 64 + 8);
+        }
+        const uint32_t Bv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t a[4] = {A0[2 * j], A1[2 * j], A0[2 * j + 1], A1[2 * j + 1]};
+          const uint32_t bb[2] = {Bv[2 * j], Bv[2 * j + 1]};
+          mma16816<T16>(acc[t], a, bb);
+        }
       }
     }
   };
@@ -202,12 +246,12 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const bf16* __re
   }
   if (b < B) {
     if (KIND == EPI_QKV) {
-      epi_qkv16<bf16>(ep, b, n0, v, rinv_s[b]);
+      epi_qkv16<T16>(ep, b, n0, v, rinv_s[b]);
     } else if (KIND == EPI_RESID) {
-      const float s = epi_resid16<bf16>(ep, b, n0, v);
+      const float s = epi_resid16<T16>(ep, b, n0, v);
       ep.ss_out[static_cast<long long>(b) * ep.ss_out_stride + blockIdx.x] = s;
     } else if (KIND == EPI_SWIGLU) {
-      epi_swiglu16<bf16>(ep, b, n0, v, rinv_s[b]);
+      epi_swiglu16<T16>(ep, b, n0, v, rinv_s[b]);
     } else {
       const unsigned long long k = epi_logits16(ep, b, n0, v, rinv_s[b]);
       argmax_commit(ep.keys + b, k);
@@ -265,7 +309,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) embed_kernel(const T* __restrict__ E, int V, int D, const int* __restrict__ ids,
                                                     float* __restrict__ x, T* __restrict__ a,
                                                     const float* __restrict__ g, float* __restrict__ ss, int ss_stride,
-                                                    float* __restrict__ rinv, float eps, int* err) {
+                                                    float* __restrict__ rinv, float eps, int* err, T* __restrict__ a_lo) {
   __shared__ float red[8];
   grid_dep_launch();
   grid_dep_wait();
@@ -292,6 +336,12 @@ __global__ void __launch_bounds__(256) embed_kernel(const T* __restrict__ E, int
     reinterpret_cast<float4*>(xr + k)[0] = make_float4(v[0], v[1], v[2], v[3]);
     reinterpret_cast<float4*>(xr + k)[1] = make_float4(v[4], v[5], v[6], v[7]);
     store8<T>(ar + k, ag);
+    if (a_lo) {
+      float lo[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) lo[i] = ag[i] - to_f(from_f<T>(ag[i]));
+      store8<T>(a_lo + static_cast<long long>(m) * D + k, lo);
+    }
   }
   s = warp_sum(s);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
@@ -334,18 +384,47 @@ cudaError_t launch_k(const LaunchCtx& lc, K kernel, dim3 grid, dim3 block, size_
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
+template <int NT, typename T16>
+cudaError_t gemv_nt_t(const LaunchCtx& lc, int kind, const void* W, int N, int K, const void* act, long long st,
+                      int B, const EpiArgs& ep, SplitK sk, const float* x, const float* g) {
+  const dim3 grid((N + 15) / 16, sk.count), block(GEMV_KW * 32);
+  const T16* w = static_cast<const T16*>(W);
+  const T16* a = static_cast<const T16*>(act);
+  if constexpr (std::is_same<T16, f16>::value) {
+    if (x && g && kind != EPI_RESID) {
+      switch (kind) {
+        case EPI_QKV:
+          return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV, T16, true>, grid, block, 0, w, N, K, a, st, B, ep, sk, x,
+                          g);
+        case EPI_SWIGLU:
+          return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU, T16, true>, grid, block, 0, w, N, K, a, st, B, ep, sk, x,
+                          g);
+        default:
+          return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS, T16, true>, grid, block, 0, w, N, K, a, st, B, ep, sk, x,
+                          g);
+      }
+    }
+  }
+  const float* nx = nullptr;
+  switch (kind) {
+    case EPI_QKV:
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx, nx);
+    case EPI_RESID:
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_RESID, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx,
+                      nx);
+    case EPI_SWIGLU:
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx,
+                      nx);
+    default:
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx,
+                      nx);
+  }
+}
 template <int NT>
 cudaError_t gemv_nt(const LaunchCtx& lc, int kind, const void* W, int N, int K, const void* act, long long st, int B,
-                    const EpiArgs& ep, SplitK sk) {
-  const dim3 grid((N + 15) / 16, sk.count), block(GEMV_KW * 32);
-  const bf16* w = static_cast<const bf16*>(W);
-  const bf16* a = static_cast<const bf16*>(act);
-  switch (kind) {
-    case EPI_QKV: return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV>, grid, block, 0, w, N, K, a, st, B, ep, sk);
-    case EPI_RESID: return launch_k(lc, gemv_mma_kernel<NT, EPI_RESID>, grid, block, 0, w, N, K, a, st, B, ep, sk);
-    case EPI_SWIGLU: return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU>, grid, block, 0, w, N, K, a, st, B, ep, sk);
-    default: return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS>, grid, block, 0, w, N, K, a, st, B, ep, sk);
-  }
+                    const EpiArgs& ep, SplitK sk, const float* x, const float* g) {
+  if (lc.f16) return gemv_nt_t<NT, f16>(lc, kind, W, N, K, act, st, B, ep, sk, x, g);
+  return gemv_nt_t<NT, bf16>(lc, kind, W, N, K, act, st, B, ep, sk, nullptr, nullptr);
 }
 
 // Resident CTAs per SM of each projection instantiation (occupancy API),
@@ -383,7 +462,8 @@ SplitK choose_split(const LaunchCtx& lc, int nt_idx, int kind, int N, int K, con
 }  // namespace
 
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
-                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk) {
+                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk, const float* x,
+                        const float* g) {
   if (B < 1 || B > 64 || (K & 63) || N < 1) return cudaErrorInvalidValue;
   if (fp32) {
     const dim3 grid((N + 15) / 16), block(GEMV_KW * 32);
@@ -398,10 +478,10 @@ cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W,
   }
   const int nt_idx = B <= 8 ? 0 : (B <= 16 ? 1 : (B <= 32 ? 2 : 3));
   const SplitK sk = choose_split(lc, nt_idx, kind, N, K, wk);
-  if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
-  if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
-  if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
-  return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep, sk);
+  if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
+  if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
+  if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
+  return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
 }
 
 namespace {
@@ -410,13 +490,17 @@ cudaError_t occupancy_nt(int idx) {
   cudaError_t e = cudaSuccess;
   const int threads = GEMV_KW * 32;
   if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_QKV], gemv_mma_kernel<NT, EPI_QKV>, threads, 0);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_QKV], gemv_mma_kernel<NT, EPI_QKV, bf16, false>,
+                                                      threads, 0);
   if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_RESID], gemv_mma_kernel<NT, EPI_RESID>, threads, 0);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_RESID], gemv_mma_kernel<NT, EPI_RESID, bf16, false>,
+                                                      threads, 0);
   if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_SWIGLU], gemv_mma_kernel<NT, EPI_SWIGLU>, threads, 0);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_SWIGLU],
+                                                      gemv_mma_kernel<NT, EPI_SWIGLU, bf16, false>, threads, 0);
   if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_LOGITS], gemv_mma_kernel<NT, EPI_LOGITS>, threads, 0);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_LOGITS],
+                                                      gemv_mma_kernel<NT, EPI_LOGITS, bf16, false>, threads, 0);
   return e;
 }
 }  // namespace
@@ -430,12 +514,16 @@ cudaError_t prepare_gemv_kernels() {
 }
 
 cudaError_t launch_embed(const LaunchCtx& lc, bool fp32, const void* E, int V, int D, const int* ids, int M, float* x,
-                         void* a, const float* g, float* ss, int ss_stride, float* rinv, float eps, int* err) {
+                         void* a, const float* g, float* ss, int ss_stride, float* rinv, float eps, int* err,
+                         void* a_lo) {
   if (fp32)
     return launch_k(lc, embed_kernel<float>, dim3(M), dim3(256), 0, static_cast<const float*>(E), V, D, ids, x,
-                    static_cast<float*>(a), g, ss, ss_stride, rinv, eps, err);
+                    static_cast<float*>(a), g, ss, ss_stride, rinv, eps, err, static_cast<float*>(nullptr));
+  if (lc.f16)
+    return launch_k(lc, embed_kernel<f16>, dim3(M), dim3(256), 0, static_cast<const f16*>(E), V, D, ids, x,
+                    static_cast<f16*>(a), g, ss, ss_stride, rinv, eps, err, static_cast<f16*>(a_lo));
   return launch_k(lc, embed_kernel<bf16>, dim3(M), dim3(256), 0, static_cast<const bf16*>(E), V, D, ids, x,
-                  static_cast<bf16*>(a), g, ss, ss_stride, rinv, eps, err);
+                  static_cast<bf16*>(a), g, ss, ss_stride, rinv, eps, err, static_cast<bf16*>(a_lo));
 }
 
 cudaError_t launch_finalize(const LaunchCtx& lc, unsigned long long* keys, int n_keys, int key_stride, int key_offset,

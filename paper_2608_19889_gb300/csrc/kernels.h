@@ -13,6 +13,7 @@ struct LaunchCtx {
   cudaStream_t stream;
   bool pdl;
   int num_sms;
+  bool f16 = false;  // 16-bit operands are fp16 (else bf16); ignored in fp32 mode
 };
 
 // ---- decode projections (k_gemv.cu): out[b][n] = act[b] . W[n], B <= 64
@@ -30,8 +31,12 @@ struct SplitK {
   float* part;
   int* ticket;
 };
+// x, g (optional, fp16 mode, normed consumers): build the operand in fp32
+// as x * g from the residual rows (act_stride floats apart) and the gain,
+// fed as two fp16 terms; `act` is then not read.
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
-                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk);
+                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk,
+                        const float* x = nullptr, const float* g = nullptr);
 // Query occupancy of the projection kernels (once, before launches).
 cudaError_t prepare_gemv_kernels();
 
@@ -53,7 +58,8 @@ cudaError_t launch_gemv_tma(const LaunchCtx& lc, int kind, const CUtensorMap& w,
 // ---- embedding gather producing x, a = x * g and the row sum of squares.
 // rinv (optional): 1 / sqrt(mean(x^2) + eps) per row.
 cudaError_t launch_embed(const LaunchCtx& lc, bool fp32, const void* E, int V, int D, const int* ids, int M, float* x,
-                         void* a, const float* g, float* ss, int ss_stride, float* rinv, float eps, int* err);
+                         void* a, const float* g, float* ss, int ss_stride, float* rinv, float eps, int* err,
+                         void* a_lo = nullptr);
 
 // ---- greedy token from argmax keys; clears the keys; optionally advances
 // context lengths.
@@ -90,10 +96,12 @@ cudaError_t prepare_gemm_kernels();
 // ---- prefill projections (k_gemm.cu): tcgen05 + TMA persistent GEMM,
 // out[m][n] = A[m] . W[n], M x N x K with K % 64 == 0.
 struct GemmMaps {
-  CUtensorMap a;  // activations [rows][K] bf16, box 64 x 128
-  CUtensorMap w;  // weights [N][K] bf16, box 64 x 256
+  CUtensorMap a;     // activations [rows][K], box 64 x 128
+  CUtensorMap w;     // weights [N][K], box 64 x 256
+  CUtensorMap a_lo;  // second term of a split activation operand (used when split)
+  bool split = false;
 };
-bool make_tma_2d_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows);
+bool make_tma_2d_16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows, bool f16);
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep);
 
 // ---- fp32 debug projections (k_simt.cu): plain tiled CUDA-core GEMM with

@@ -37,12 +37,12 @@ def gpu_weights(shape: dict, seed: int = si.SEED_WEIGHTS):
 
 
 def create(shape, weights, max_batch, max_context, layout="contiguous", num_blocks=0, fp32=False,
-           max_prefill_tokens=0):
+           max_prefill_tokens=0, fp16=False):
     import paper_2608_19889_gb300 as ax
+    prec = ax.AXON_FP32_DEBUG if fp32 else (ax.AXON_FP16 if fp16 else ax.AXON_BF16)
     cfg = ax.make_config(shape, max_batch, max_context,
                          kv_layout=ax.AXON_KV_PAGED if layout == "paged" else ax.AXON_KV_CONTIGUOUS,
-                         kv_num_blocks=num_blocks, precision=ax.AXON_FP32_DEBUG if fp32 else ax.AXON_BF16,
-                         max_prefill_tokens=max_prefill_tokens)
+                         kv_num_blocks=num_blocks, precision=prec, max_prefill_tokens=max_prefill_tokens)
     return ax.axon_model_create(cfg, weights)
 
 

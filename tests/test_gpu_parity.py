@@ -104,13 +104,14 @@ def oracle_decode(o, cache, fed, ctx0):
     return np.stack(outs, 1)
 
 
+@pytest.mark.parametrize("prec", ["bf16", "fp16"])
 @pytest.mark.parametrize("shape,B,S", [(TINY, 2, 20), (TINY, 3, 45), (TINY128, 2, 33)])
-def test_tiny_prefill_all_positions_and_decode_gemv_path(shape, B, S):
+def test_tiny_prefill_all_positions_and_decode_gemv_path(shape, B, S, prec):
     """B*S <= 64: projections on the decode GEMV, attention on the prefill
     kernel; every position's logits, then 6 cached decode steps."""
     ax = _ax()
     w = gpu_weights(shape)
-    m = create(shape, w, max_batch=4, max_context=128)
+    m = create(shape, w, max_batch=4, max_context=128, fp16=prec == "fp16")
     try:
         ids = si.make_ids(B, S, shape["V"])
         lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_ALL, shape["V"])
@@ -126,12 +127,13 @@ def test_tiny_prefill_all_positions_and_decode_gemv_path(shape, B, S):
         ax.axon_free(m)
 
 
+@pytest.mark.parametrize("prec", ["bf16", "fp16"])
 @pytest.mark.parametrize("shape,B,S", [(TINY, 2, 100), (TINY128, 1, 300)])
-def test_tiny_prefill_tensor_core_path(shape, B, S):
+def test_tiny_prefill_tensor_core_path(shape, B, S, prec):
     """B*S > 64: projections on the tcgen05 GEMM (ragged 128-row tail)."""
     ax = _ax()
     w = gpu_weights(shape)
-    m = create(shape, w, max_batch=2, max_context=320)
+    m = create(shape, w, max_batch=2, max_context=320, fp16=prec == "fp16")
     try:
         ids = si.make_ids(B, S, shape["V"], seed=5)
         lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_ALL, shape["V"])
@@ -213,7 +215,7 @@ def test_fp32_debug_mode_relative_error():
         ax.axon_free(m)
 
 
-def _workload(name, n_check_steps=None):
+def _workload(name, n_check_steps=None, fp16=False):
     ax = _ax()
     wl = si.WORKLOADS[name]
     shape = si.MODEL_SHAPES[wl["model"]]
@@ -221,7 +223,7 @@ def _workload(name, n_check_steps=None):
     steps = n_new - 1 if n_check_steps is None else n_check_steps
     w = gpu_weights(shape)
     max_ctx = (S + n_new + 15) // 16 * 16
-    m = create(shape, w, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S)
+    m = create(shape, w, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S, fp16=fp16)
     try:
         ids = si.make_ids(B, S, shape["V"])
         lg, nxt = run_prefill(m, ids, ax.AXON_LOGITS_LAST, shape["V"])
@@ -247,3 +249,8 @@ def test_workload_135m():
 @pytest.mark.slow
 def test_workload_0_5b():
     _workload("0.5b_b1_s512_n128")
+
+
+@pytest.mark.slow
+def test_workload_0_5b_fp16_operands():
+    _workload("0.5b_b1_s512_n128", fp16=True)
