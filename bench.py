@@ -49,7 +49,7 @@ def decode_bytes_per_step(m, B, T_list):
     L, D, G, d, V = m["L"], m["D"], m["G"], m["d"], m["V"]
     small = (2 * L + 1) * D * 4 + (L * (m["H"] + 2 * G) * d * 4 if m["bias"] else 0)
     kv_tok = L * 2 * G * d * 2
-    kv_read = sum((t + 1) for t in T_list) * kv_tok
+    kv_read = sum(int(t) + 1 for t in T_list) * kv_tok
     kv_write = B * kv_tok
     return 2 * (lin + head) + small + kv_read + kv_write + B * V * 4
 
@@ -139,6 +139,44 @@ def oracle_generate_timed(wl, budget_s=20.0):
     sample = (f"prefill B={B} S={S} timed in full ({t_pre:.2f}s) + {n} of {wl['n_new']} decode steps "
               f"({per_step * 1e3:.1f} ms/step), remainder extrapolated")
     return B * wl["n_new"] / t_full, sample, n
+
+
+def kernel_source_sha():
+    """sha256 over the CUDA sources; a DRAM-traffic record taken from an ncu
+    capture is only valid for the sources it was taken on."""
+    import hashlib
+    d = os.path.join(os.path.dirname(os.path.abspath(__file__)), "paper_2608_19889_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in sorted(os.listdir(d)):
+        if f.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(d, f), "rb") as fh:
+                h.update(f.encode() + b"\0" + fh.read())
+    return h.hexdigest()
+
+
+def recorded_traffic(workload, precision, kind):
+    """DRAM bytes per launch of profiler kind `kind` from the committed ncu
+    summary profiles/dram_<workload>_<precision>.md (lines `traffic <kind>:
+    <bytes>` after a `source_sha256:` line), or None when there is none or
+    the CUDA sources changed since it was captured."""
+    p = os.path.join(os.path.dirname(os.path.abspath(__file__)), "profiles", f"dram_{workload}_{precision}.md")
+    if not os.path.exists(p):
+        return None
+    sha, rec = None, {}
+    with open(p) as fh:
+        for line in fh:
+            line = line.strip().strip("`")
+            if line.startswith("source_sha256:"):
+                sha = line.split(":", 1)[1].strip()
+            elif line.startswith("traffic ") and ":" in line:
+                k, v = line[len("traffic "):].split(":", 1)
+                try:
+                    rec[k.strip()] = float(v)
+                except ValueError:
+                    pass
+    if sha != kernel_source_sha():
+        return None
+    return rec.get(kind)
 
 
 def cores():
@@ -293,7 +331,7 @@ class PagedDecodeRun:
         return [list(self.lens_np), list(self.lens_np + self.n_new // 2), list(self.lens_np + self.n_new - 1)]
 
 
-def build_model(ax, torch, wl, m, st, layers=None, vocab=None):
+def build_model(ax, torch, wl, m, st, layers=None, vocab=None, precision=0):
     m = dict(m)
     if layers is not None:
         m["L"] = layers
@@ -309,11 +347,11 @@ def build_model(ax, torch, wl, m, st, layers=None, vocab=None):
         num_blocks = int(sum(-(-int(c) // 16) for c in caps)) + 64
         bt_np = si.make_block_table(caps, 16, max_ctx // 16, num_blocks)
         cfg = ax.make_config(m, max_batch=B, max_context=max_ctx, kv_layout=ax.AXON_KV_PAGED,
-                             kv_num_blocks=num_blocks, max_prefill_tokens=hi)
+                             kv_num_blocks=num_blocks, max_prefill_tokens=hi, precision=precision)
     else:
         B, S = wl["B"], wl["S"]
         max_ctx = (S + wl["n_new"] + 15) // 16 * 16
-        cfg = ax.make_config(m, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S)
+        cfg = ax.make_config(m, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S, precision=precision)
     with torch.cuda.stream(st):
         model = ax.axon_model_create(cfg, w, stream=st)
     del w
@@ -329,6 +367,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(si.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16"],
+                    help="operand type on the tensor cores; fp16 converts the bf16 checkpoint exactly and splits "
+                         "normalized activations into two fp16 terms (same weight bytes, same tensor rate)")
     ap.add_argument("--case", action="store_true",
                     help="profiling case: build the workload's model, run one prefill and --case-steps decode "
                          "steps, print nothing but a status line (for ncu)")
@@ -356,9 +397,10 @@ def main():
 
     wl = si.WORKLOADS[args.workload]
     st = torch.cuda.Stream()
+    prec = ax.AXON_FP16 if args.precision == "fp16" else ax.AXON_BF16
     model, m, lens, bt_np = build_model(ax, torch, wl, si.MODEL_SHAPES[wl["model"]], st,
                                         layers=args.case_layers if args.case else None,
-                                        vocab=args.case_vocab if args.case else None)
+                                        vocab=args.case_vocab if args.case else None, precision=prec)
     if wl["layout"] == "paged":
         run = PagedDecodeRun(ax, torch, model, m, wl, st, lens, bt_np)
     else:
@@ -466,7 +508,8 @@ def main():
         roof = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm}
     roof.update({"kernel": top_name, "launch_ms": per_launch_ms,
                  "per_launch_units": (top_bytes if roof["bound"] == "hbm" else top_flops) / top_n,
-                 "peak_kind": peak_kind, "traffic": None})
+                 "peak_kind": peak_kind,
+                 "traffic": recorded_traffic(args.workload, args.precision, top_name)})
     total_w = sum(x[0] for x in kinds)
     kernel_table = {k[1]: {"share_of_run": k[0] / total_w, "launch_ms": k[3] / k[2]} for k in kinds}
 
@@ -484,7 +527,7 @@ def main():
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "bf16",
+        "dtype": args.precision,
         "data": "synthetic (seeded random-init weights N(0,0.02), uniform random ids)",
         "config": config,
         "decode_tok_s": world * B * n_new / (dec_ms / 1e3),

@@ -74,7 +74,7 @@ struct axon_model {
   int Pmax = 0;
   float* x = nullptr;
   void* a = nullptr;
-  void* a_lo = nullptr;  // fp16 mode: second term of the QKV input (x*g - a)
+  void* a_lo = nullptr;  // fp16 mode: second term of the normed operand (x*g - a), same layout as a
   float* ss = nullptr;
   void* q = nullptr;
   void* o = nullptr;
@@ -400,11 +400,8 @@ struct Proj {
   // the norm state a RESID producer leaves behind.
   // vmap: the weight's decode-projection TMA map; amaps: the activation
   // buffer's maps by token-box size (null: register-streaming GEMV).
-  // xg: fp16-mode decode consumers of a normed operand build it from the
-  // fp32 residual and this gain (see launch_gemv).
   NormState run(int kind, const void* W, const GemmMaps* maps, int N, int K, const void* act, long long act_stride,
-                int M, EpiArgs& ep, const CUtensorMap* vmap = nullptr, const CUtensorMap* amaps = nullptr,
-                const float* xg = nullptr) {
+                int M, EpiArgs& ep, const CUtensorMap* vmap = nullptr, const CUtensorMap* amaps = nullptr) {
     ep.M = M;
     ep.N = N;
     NormState ns;
@@ -420,9 +417,10 @@ struct Proj {
       rc = launch_gemv_tma(lc, kind, *vmap, amaps[idx], N, K, M, ep, m->tmawork);
       ns.parts = N / 16;
     } else if (gemv) {
-      const bool xs = m->f16 && xg && act == m->a;
-      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk, xs ? m->x : nullptr,
-                       xs ? xg : nullptr);
+      // fp16 mode: consumers of the normed operand `a` also read its
+      // second term a_lo
+      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk,
+                       m->f16 && act == m->a ? m->a_lo : nullptr);
       ns.parts = N / 16;
     } else if (m->fp32) {
       rc = launch_gemm_simt(lc, kind, static_cast<const float*>(act), act_stride, static_cast<const float*>(W), M, N,
@@ -449,7 +447,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
   const int D = m->D, Hd = m->H * m->d;
   pbeg(pf, "embed");
   CK(launch_embed(lc, m->fp32, m->embed, m->V, D, ids, M, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
-                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err, M > 64 ? m->a_lo : nullptr));
+                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err, m->a_lo));
   pend(pf, static_cast<double>(M) * D * (es + 4 + es), 0);
   NormState ns;
   ns.rinv = true;
@@ -462,7 +460,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
     pbeg(pf, "prefill_qkv");
-    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, M, e, nullptr, nullptr, w.g1);
+    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, M, e);
     CK(pj.rc);
     pend(pf, wq + M * (D + m->Nqkv) * es, 2.0 * M * m->Nqkv * D);
 
@@ -478,6 +476,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     r.x = m->x;
     r.a_out = m->a;
     r.gain = w.g2;
+    r.a_lo_out = m->a_lo;
     r.ss_out = m->ss;
     r.ss_out_stride = m->Pmax;
     pbeg(pf, "prefill_o");
@@ -490,7 +489,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     set_norm(m, ns, g);
     g.u_out = m->u;
     pbeg(pf, "prefill_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, M, g, nullptr, nullptr, w.g2);
+    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, M, g);
     CK(pj.rc);
     pend(pf, wgu + M * (D + m->F) * es, 2.0 * M * 2 * m->F * D);
 
@@ -501,7 +500,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
-    if (l + 1 < m->L && M > 64) dn.a_lo_out = m->a_lo;
+    dn.a_lo_out = m->a_lo;
     pbeg(pf, "prefill_down");
     ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, M, dn);
     CK(pj.rc);
@@ -530,7 +529,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     pbeg(pf, "prefill_lm_head");
     CK(launch_gemv(lc, EPI_LOGITS, m->fp32, m->head, m->V, D, static_cast<char*>(m->a) + off,
                    static_cast<long long>(S) * D, B, h, m->splitk,
-                   m->f16 ? m->x + static_cast<size_t>(S - 1) * D : nullptr, m->f16 ? m->gf : nullptr));
+                   m->a_lo ? static_cast<char*>(m->a_lo) + off : nullptr));
     pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
     pbeg(pf, "finalize");
     CK(launch_finalize(lc, m->keys, B, 1, 0, B, next, nullptr));
@@ -552,7 +551,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
                whd = static_cast<double>(m->V) * m->D * es;
   pbeg(pf, "embed");
   CK(launch_embed(lc, m->fp32, m->embed, m->V, D, tokens, B, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
-                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err));
+                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err, m->a_lo));
   pend(pf, static_cast<double>(B) * D * (es + 4 + es), 0);
   NormState ns;
   ns.rinv = true;
@@ -572,7 +571,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
     pbeg(pf, "decode_qkv");
-    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok, w.g1);
+    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok);
     CK(pj.rc);
     pend(pf, wq + B * (D + m->Nqkv) * es, 2.0 * B * m->Nqkv * D);
 
@@ -592,6 +591,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     r.x = m->x;
     r.a_out = m->a;
     r.gain = w.g2;
+    r.a_lo_out = m->a_lo;
     r.ss_out = m->ss;
     r.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_o");
@@ -605,7 +605,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     set_norm(m, ns, g);
     g.u_out = m->u;
     pbeg(pf, "decode_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok, w.g2);
+    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok);
     CK(pj.rc);
     pend(pf, wgu + B * (D + m->F) * es, 2.0 * B * 2 * m->F * D);
 
@@ -615,6 +615,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     dn.x = m->x;
     dn.a_out = m->a;
     dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
+    dn.a_lo_out = m->a_lo;
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_down");
@@ -630,7 +631,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   h.logits = logits;
   h.logits_stride = m->V;
   pbeg(pf, "decode_lm_head");
-  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok, m->gf);
+  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok);
   CK(pj.rc);
   pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
   pbeg(pf, "finalize");

@@ -11,8 +11,6 @@
 // elements into the fragment slots in a fixed permutation that the token
 // operand mirrors. Partial sums meet in shared memory in a fixed warp order
 // (deterministic), then one thread per token runs the fused epilogue.
-#include <type_traits>
-
 #include "kernels.h"
 
 namespace {
@@ -58,17 +56,16 @@ AXON_DEV void finish_rinv(const EpiArgs& ep, int B, int nparts) {
   if (threadIdx.x == 0) *ep.ticket = 0;
 }
 
-// XS: the activation operand is formed in fp32 from the residual x and the
-// norm gain (x * gain, rows act_stride floats apart) and fed to the tensor
-// cores as two 16-bit terms (hi = round(x*gain), lo = round(x*gain - hi)),
-// two MMAs per k-step: the operand carries ~22 significant bits instead of
-// 11. (`act` is unused then.)
-template <int NT, int KIND, typename T16, bool XS>
+// LO: the activation operand is the sum of two 16-bit terms, act (the
+// rounded value) and act_lo (what that rounding lost, same layout), and
+// every k-step runs two MMAs into one accumulator: ~22 significant bits
+// per activation instead of 11. The MMAs run in every lane whatever the
+// token count (unused token slots feed zeros): mma.sync is warp-collective.
+template <int NT, int KIND, typename T16, bool LO>
 __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const T16* __restrict__ W, int N, int K,
                                                                const T16* __restrict__ act, long long act_stride,
                                                                int B, EpiArgs ep, SplitK sk,
-                                                               const float* __restrict__ xres,
-                                                               const float* __restrict__ gain) {
+                                                               const T16* __restrict__ act_lo) {
   constexpr int TOK = NT * 8;
   __shared__ float red[GEMV_KW][16][TOK + 1];
   __shared__ float rinv_s[TOK];
@@ -92,63 +89,45 @@ __global__ void __launch_bounds__(GEMV_KW * 32) gemv_mma_kernel(const T16* __res
   for (int t = 0; t < NT; ++t) acc[t][0] = acc[t][1] = acc[t][2] = acc[t][3] = 0.f;
 
   const T16* arow[NT];
-  const float* xrow[NT];
+  const T16* lrow[NT];
   bool aval[NT];
 #pragma unroll
   for (int t = 0; t < NT; ++t) {
     const int tok = t * 8 + r;
     aval[t] = tok < B;
-    arow[t] = act + static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q + c_begin * 64;
-    if (XS) xrow[t] = xres + static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q + c_begin * 64;
+    const long long off = static_cast<long long>(aval[t] ? tok : 0) * act_stride + 16 * q + c_begin * 64;
+    arow[t] = act + off;
+    lrow[t] = LO ? act_lo + off : nullptr;
   }
-  const float* grow = XS ? gain + 16 * q + c_begin * 64 : nullptr;
 
   auto chunk = [&](int c, const uint4& wa0, const uint4& wa1, const uint4& wb0, const uint4& wb1) {
     const uint32_t A0[8] = {wa0.x, wa0.y, wa0.z, wa0.w, wa1.x, wa1.y, wa1.z, wa1.w};
     const uint32_t A1[8] = {wb0.x, wb0.y, wb0.z, wb0.w, wb1.x, wb1.y, wb1.z, wb1.w};
 #pragma unroll
     for (int t = 0; t < NT; ++t) {
-      if (XS) {
-        float v[16];
+      uint4 x0 = make_uint4(0, 0, 0, 0), x1 = make_uint4(0, 0, 0, 0);
+      if (aval[t]) {
+        x0 = ld16(arow[t] + c * 64);
+        x1 = ld16(arow[t] + c * 64 + 8);
+      }
+      const uint32_t Bv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = 0.f;
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t a[4] = {A0[2 * j], A1[2 * j], A0[2 * j + 1], A1[2 * j + 1]};
+        const uint32_t bb[2] = {Bv[2 * j], Bv[2 * j + 1]};
+        mma16816<T16>(acc[t], a, bb);
+      }
+      if (LO) {
+        uint4 y0 = make_uint4(0, 0, 0, 0), y1 = make_uint4(0, 0, 0, 0);
         if (aval[t]) {
-#pragma unroll
-          for (int i = 0; i < 16; i += 4) {
-            const float4 xv = *reinterpret_cast<const float4*>(xrow[t] + c * 64 + i);
-            const float4 gv = *reinterpret_cast<const float4*>(grow + c * 64 + i);
-            v[i] = xv.x * gv.x;
-            v[i + 1] = xv.y * gv.y;
-            v[i + 2] = xv.z * gv.z;
-            v[i + 3] = xv.w * gv.w;
-          }
+          y0 = ld16(lrow[t] + c * 64);
+          y1 = ld16(lrow[t] + c * 64 + 8);
         }
-        uint32_t Bh[8], Bl[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const float h0 = to_f(from_f<T16>(v[2 * i])), h1 = to_f(from_f<T16>(v[2 * i + 1]));
-          Bh[i] = pack2<T16>(h0, h1);
-          Bl[i] = pack2<T16>(v[2 * i] - h0, v[2 * i + 1] - h1);
-        }
+        const uint32_t Bl[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const uint32_t a[4] = {A0[2 * j], A1[2 * j], A0[2 * j + 1], A1[2 * j + 1]};
-          const uint32_t bh[2] = {Bh[2 * j], Bh[2 * j + 1]};
-          const uint32_t bl[2] = {Bl[2 * j], Bl[2 * j + 1]};
-          mma16816<T16>(acc[t], a, bh);
-          mma16816<T16>(acc[t], a, bl);
-        }
-      } else {
-        uint4 x0 = make_uint4(0, 0, 0, 0), x1 = make_uint4(0, 0, 0, 0);
-        if (aval[t]) {
-          x0 = ld16(arow[t] + c * 64);
-          x1 = ld16(arow[t] + c * 64 + 8);
-        }
-        const uint32_t Bv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint32_t a[4] = {A0[2 * j], A1[2 * j], A0[2 * j + 1], A1[2 * j + 1]};
-          const uint32_t bb[2] = {Bv[2 * j], Bv[2 * j + 1]};
+          const uint32_t bb[2] = {Bl[2 * j], Bl[2 * j + 1]};
           mma16816<T16>(acc[t], a, bb);
         }
       }
@@ -384,47 +363,35 @@ cudaError_t launch_k(const LaunchCtx& lc, K kernel, dim3 grid, dim3 block, size_
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
-template <int NT, typename T16>
-cudaError_t gemv_nt_t(const LaunchCtx& lc, int kind, const void* W, int N, int K, const void* act, long long st,
-                      int B, const EpiArgs& ep, SplitK sk, const float* x, const float* g) {
+template <int NT, typename T16, bool LO>
+cudaError_t gemv_nt_lo(const LaunchCtx& lc, int kind, const T16* w, int N, int K, const T16* a, long long st, int B,
+                       const EpiArgs& ep, SplitK sk, const T16* al) {
   const dim3 grid((N + 15) / 16, sk.count), block(GEMV_KW * 32);
-  const T16* w = static_cast<const T16*>(W);
-  const T16* a = static_cast<const T16*>(act);
-  if constexpr (std::is_same<T16, f16>::value) {
-    if (x && g && kind != EPI_RESID) {
-      switch (kind) {
-        case EPI_QKV:
-          return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV, T16, true>, grid, block, 0, w, N, K, a, st, B, ep, sk, x,
-                          g);
-        case EPI_SWIGLU:
-          return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU, T16, true>, grid, block, 0, w, N, K, a, st, B, ep, sk, x,
-                          g);
-        default:
-          return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS, T16, true>, grid, block, 0, w, N, K, a, st, B, ep, sk, x,
-                          g);
-      }
-    }
-  }
-  const float* nx = nullptr;
   switch (kind) {
     case EPI_QKV:
-      return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx, nx);
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_QKV, T16, LO>, grid, block, 0, w, N, K, a, st, B, ep, sk, al);
     case EPI_RESID:
-      return launch_k(lc, gemv_mma_kernel<NT, EPI_RESID, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx,
-                      nx);
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_RESID, T16, LO>, grid, block, 0, w, N, K, a, st, B, ep, sk, al);
     case EPI_SWIGLU:
-      return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx,
-                      nx);
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_SWIGLU, T16, LO>, grid, block, 0, w, N, K, a, st, B, ep, sk, al);
     default:
-      return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS, T16, false>, grid, block, 0, w, N, K, a, st, B, ep, sk, nx,
-                      nx);
+      return launch_k(lc, gemv_mma_kernel<NT, EPI_LOGITS, T16, LO>, grid, block, 0, w, N, K, a, st, B, ep, sk, al);
   }
 }
 template <int NT>
 cudaError_t gemv_nt(const LaunchCtx& lc, int kind, const void* W, int N, int K, const void* act, long long st, int B,
-                    const EpiArgs& ep, SplitK sk, const float* x, const float* g) {
-  if (lc.f16) return gemv_nt_t<NT, f16>(lc, kind, W, N, K, act, st, B, ep, sk, x, g);
-  return gemv_nt_t<NT, bf16>(lc, kind, W, N, K, act, st, B, ep, sk, nullptr, nullptr);
+                    const EpiArgs& ep, SplitK sk, const void* act_lo) {
+  if (lc.f16) {
+    const f16* w = static_cast<const f16*>(W);
+    const f16* a = static_cast<const f16*>(act);
+    // The residual projections read attention / SwiGLU outputs, which have
+    // no second term.
+    if (act_lo && kind != EPI_RESID)
+      return gemv_nt_lo<NT, f16, true>(lc, kind, w, N, K, a, st, B, ep, sk, static_cast<const f16*>(act_lo));
+    return gemv_nt_lo<NT, f16, false>(lc, kind, w, N, K, a, st, B, ep, sk, nullptr);
+  }
+  return gemv_nt_lo<NT, bf16, false>(lc, kind, static_cast<const bf16*>(W), N, K, static_cast<const bf16*>(act), st, B,
+                                     ep, sk, nullptr);
 }
 
 // Resident CTAs per SM of each projection instantiation (occupancy API),
@@ -462,8 +429,8 @@ SplitK choose_split(const LaunchCtx& lc, int nt_idx, int kind, int N, int K, con
 }  // namespace
 
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
-                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk, const float* x,
-                        const float* g) {
+                        long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk,
+                        const void* act_lo) {
   if (B < 1 || B > 64 || (K & 63) || N < 1) return cudaErrorInvalidValue;
   if (fp32) {
     const dim3 grid((N + 15) / 16), block(GEMV_KW * 32);
@@ -478,29 +445,32 @@ cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W,
   }
   const int nt_idx = B <= 8 ? 0 : (B <= 16 ? 1 : (B <= 32 ? 2 : 3));
   const SplitK sk = choose_split(lc, nt_idx, kind, N, K, wk);
-  if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
-  if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
-  if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
-  return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep, sk, x, g);
+  if (B <= 8) return gemv_nt<1>(lc, kind, W, N, K, act, act_stride, B, ep, sk, act_lo);
+  if (B <= 16) return gemv_nt<2>(lc, kind, W, N, K, act, act_stride, B, ep, sk, act_lo);
+  if (B <= 32) return gemv_nt<4>(lc, kind, W, N, K, act, act_stride, B, ep, sk, act_lo);
+  return gemv_nt<8>(lc, kind, W, N, K, act, act_stride, B, ep, sk, act_lo);
 }
 
 namespace {
+// Resident CTAs per SM of a projection kind: the smaller of the plain bf16
+// variant and the fp16 split-operand variant (which holds more registers).
+template <int NT, int KIND>
+cudaError_t occupancy_kind(int idx) {
+  const int threads = GEMV_KW * 32;
+  int a = 0, b = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, gemv_mma_kernel<NT, KIND, bf16, false>, threads, 0);
+  b = a;
+  if (e == cudaSuccess && KIND != EPI_RESID)  // residual kinds never take the split operand
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, gemv_mma_kernel<NT, KIND, f16, true>, threads, 0);
+  g_resident[idx][KIND] = a < b ? a : b;
+  return e;
+}
 template <int NT>
 cudaError_t occupancy_nt(int idx) {
-  cudaError_t e = cudaSuccess;
-  const int threads = GEMV_KW * 32;
-  if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_QKV], gemv_mma_kernel<NT, EPI_QKV, bf16, false>,
-                                                      threads, 0);
-  if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_RESID], gemv_mma_kernel<NT, EPI_RESID, bf16, false>,
-                                                      threads, 0);
-  if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_SWIGLU],
-                                                      gemv_mma_kernel<NT, EPI_SWIGLU, bf16, false>, threads, 0);
-  if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g_resident[idx][EPI_LOGITS],
-                                                      gemv_mma_kernel<NT, EPI_LOGITS, bf16, false>, threads, 0);
+  cudaError_t e = occupancy_kind<NT, EPI_QKV>(idx);
+  if (e == cudaSuccess) e = occupancy_kind<NT, EPI_RESID>(idx);
+  if (e == cudaSuccess) e = occupancy_kind<NT, EPI_SWIGLU>(idx);
+  if (e == cudaSuccess) e = occupancy_kind<NT, EPI_LOGITS>(idx);
   return e;
 }
 }  // namespace

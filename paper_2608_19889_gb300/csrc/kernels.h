@@ -31,12 +31,11 @@ struct SplitK {
   float* part;
   int* ticket;
 };
-// x, g (optional, fp16 mode, normed consumers): build the operand in fp32
-// as x * g from the residual rows (act_stride floats apart) and the gain,
-// fed as two fp16 terms; `act` is then not read.
+// act_lo (optional, fp16 mode, ignored by the residual kinds): second term
+// of a split activation operand, same layout and stride as act.
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
                         long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk,
-                        const float* x = nullptr, const float* g = nullptr);
+                        const void* act_lo = nullptr);
 // Query occupancy of the projection kernels (once, before launches).
 cudaError_t prepare_gemv_kernels();
 
