@@ -368,7 +368,7 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(si.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16"],
-                    help="operand type on the tensor cores; fp16 converts the bf16 checkpoint exactly and splits "
+                    help="operand type on the tensor cores; fp16 converts the bf16 checkpoint to fp16 weights and splits "
                          "normalized activations into two fp16 terms (same weight bytes, same tensor rate)")
     ap.add_argument("--case", action="store_true",
                     help="profiling case: build the workload's model, run one prefill and --case-steps decode "

@@ -3,7 +3,7 @@ few layers (prefill through the tensor-core GEMM, B=64 paged decode), and
 the full-depth models on a short prompt. Slow (the float64 oracle does the
 same work on the host).
 
-These run in AXON_FP16 (bf16 checkpoint converted exactly to fp16 operands):
+These run in AXON_FP16 (the bf16 checkpoint converted to fp16 operands):
 at these widths the random-init logits have a standard deviation of 1.3-1.4,
 and rounding GEMM operands and the KV cache to bf16 alone moves the largest
 of the 128k-152k logits by ~0.06 (an exact float64 emulation of the bf16
