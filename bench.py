@@ -254,10 +254,6 @@ class GenerateRun:
     def generated_per_step(self):
         return self.B * self.n_new
 
-    def launches_per_step(self):
-        # embed + 5 per layer + LM head + finaliser, for the prefill and each decode step
-        return (5 * self.m["L"] + 3) * (1 + self.n_new)
-
     def profile_positions(self):
         return [[self.S] * self.B, [self.S + self.n_new // 2] * self.B, [self.S + self.n_new - 1] * self.B]
 
@@ -323,9 +319,6 @@ class PagedDecodeRun:
 
     def generated_per_step(self):
         return self.B * self.n_new
-
-    def launches_per_step(self):
-        return (5 * self.m["L"] + 3) * self.n_new
 
     def profile_positions(self):
         return [list(self.lens_np), list(self.lens_np + self.n_new // 2), list(self.lens_np + self.n_new - 1)]
@@ -484,7 +477,8 @@ def main():
     with torch.cuda.stream(st):
         if run.kind == "contiguous":
             prof_pre = ax.axon_profile_prefill(model, run.ids, next_tokens=run.tok, stream=st)
-        for pos in run.profile_positions():
+        positions = run.profile_positions()
+        for pos in positions:
             run.ctx.copy_(torch.tensor(pos, dtype=torch.int32))
             for e in ax.axon_profile_decode_step(model, run.tok, run.ctx, block_table=run.bt, next_tokens=run.tok,
                                                  stream=st):
@@ -492,6 +486,10 @@ def main():
                 for k in ("launches", "total_ms", "bytes", "flops"):
                     a[k] += e[k]
     torch.cuda.synchronize()
+    # Kernel launches per timed step, counted by the profiler on the same
+    # code path: one prefill (contiguous runs) + n_new decode steps.
+    dec_launches = sum(e["launches"] for e in prof_dec.values()) / len(positions)
+    launches_per_step = sum(e["launches"] for e in prof_pre) + n_new * dec_launches
     kinds = []  # (weight over the run, name, launches, ms, bytes, flops)
     for e in prof_pre:
         kinds.append((e["total_ms"], e["name"], e["launches"], e["total_ms"], e["bytes"], e["flops"]))
@@ -539,7 +537,7 @@ def main():
         "kernels": kernel_table,
         "e2e": {"value": world * e2e_val, "unit": "tokens/s",
                 "h2d_bytes_per_step": int(in_h.numel()) * 4, "d2h_bytes_per_step": B * n_new * 4},
-        "gpu_launches": args.steps * run.launches_per_step(),
+        "gpu_launches": int(round(args.steps * launches_per_step)),
         "clocks": clk,
         "wall_s": wall,
     }

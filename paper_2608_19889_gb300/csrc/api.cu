@@ -96,6 +96,12 @@ struct axon_model {
   bool use_graphs = true;
   bool use_pdl = true;
   bool use_tma_gemv = false;
+  // persistent decode step (B <= PERSIST_MAX_B): device layer table, grid
+  // barrier state, CTAs per launch (0: not available)
+  PersistLayer* players = nullptr;
+  CUtensorMap* pmaps = nullptr;  // [4L + 1] weight maps, box 256 x 16
+  PersistGrid* pgrid = nullptr;
+  int persist_ctas = 0;
 };
 
 namespace {
@@ -538,6 +544,57 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
   return AXON_OK;
 }
 
+bool persist_eligible(const axon_model* m, int B) {
+  return m->persist_ctas > 0 && !m->fp32 && B >= 1 && B <= PERSIST_MAX_B;
+}
+
+PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt,
+                         float* logits, int32_t* next, int splits, float* attn_part, int* attn_cnt) {
+  PersistArgs a;
+  memset(&a, 0, sizeof(a));
+  a.L = m->L;
+  a.D = m->D;
+  a.H = m->H;
+  a.G = m->G;
+  a.d = m->d;
+  a.F = m->F;
+  a.V = m->V;
+  a.Nqkv = m->Nqkv;
+  a.Pmax = m->Pmax;
+  a.B = B;
+  a.max_pos = m->cfg.max_context;
+  a.blocks_per_seq = m->blocks_per_seq;
+  a.num_blocks = static_cast<int>(m->num_blocks);
+  a.splits = splits;
+  a.eps = m->cfg.rms_norm_eps;
+  a.inv_D = 1.0f / static_cast<float>(m->D);
+  a.scale_log2 = static_cast<float>(1.0 / std::sqrt(static_cast<double>(m->d)) * 1.4426950408889634);
+  a.layers = m->players;
+  a.wmaps = m->pmaps;
+  a.embed = m->embed;
+  a.head = m->head;
+  a.gf = m->gf;
+  a.rope = m->rope;
+  a.x = m->x;
+  a.a = m->a;
+  a.a_lo = m->a_lo;
+  a.ss = m->ss;
+  a.q = m->q;
+  a.o = m->o;
+  a.u = m->u;
+  a.keys = m->keys;
+  a.attn_part = attn_part;
+  a.attn_cnt = attn_cnt;
+  a.err = m->err;
+  a.grid = m->pgrid;
+  a.tokens = tokens;
+  a.ctx = ctx;
+  a.block_table = bt;
+  a.logits = logits;
+  a.next = next;
+  return a;
+}
+
 int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt, float* logits,
                    int32_t* next, cudaStream_t st, Prof* pf = nullptr, double kv_tokens = 0,
                    float* attn_part = nullptr, int* attn_cnt = nullptr, int attn_rows_cap = 0) {
@@ -549,18 +606,30 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * Hd * es,
                wgu = 2.0 * m->F * m->D * es, wdn = static_cast<double>(m->D) * m->F * es,
                whd = static_cast<double>(m->V) * m->D * es;
-  pbeg(pf, "embed");
-  CK(launch_embed(lc, m->fp32, m->embed, m->V, D, tokens, B, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
-                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err, m->a_lo));
-  pend(pf, static_cast<double>(B) * D * (es + 4 + es), 0);
-  NormState ns;
-  ns.rinv = true;
   int splits = m->fp32 ? 1 : attn_decode_splits(B, m->G, m->blocks_per_seq, m->num_sms);
   if (attn_rows_cap > 0) {
     // caller-supplied merge scratch holds attn_rows_cap (sequence, kv head, split) slots
     const int cap = attn_rows_cap / (B * m->G);
     if (splits > cap) splits = cap < 1 ? 1 : cap;
   }
+  if (persist_eligible(m, B)) {
+    PersistArgs pa = persist_args(m, tokens, B, ctx, bt, logits, next, splits, attn_part ? attn_part : m->attn_part,
+                                  attn_cnt ? attn_cnt : m->attn_cnt);
+    pbeg(pf, "decode_persistent");
+    CK(launch_persist_decode(pa, m->d, m->f16, m->persist_ctas, st));
+    const double kvb = kv_tokens * 2.0 * m->G * m->d * es * m->L;
+    pend(pf, m->L * (wq + wo + wgu + wdn) + whd + kvb + B * (logits ? 4.0 * m->V : 0.0),
+         2.0 * B * (m->L * (static_cast<double>(m->Nqkv) * D + static_cast<double>(D) * Hd + 3.0 * m->F * D) +
+                    static_cast<double>(m->V) * D) +
+             4.0 * kv_tokens * m->H * m->d * m->L);
+    return AXON_OK;
+  }
+  pbeg(pf, "embed");
+  CK(launch_embed(lc, m->fp32, m->embed, m->V, D, tokens, B, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
+                  m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err, m->a_lo));
+  pend(pf, static_cast<double>(B) * D * (es + 4 + es), 0);
+  NormState ns;
+  ns.rinv = true;
   for (int l = 0; l < m->L; ++l) {
     const LayerW& w = m->layers[l];
     EpiArgs e = base_epi(m);
@@ -962,6 +1031,52 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     }
     if (!ok) return fail(AXON_ERR_CUDA);
   }
+  // ---- persistent decode step: layer table and grid barrier state
+  // opt-in (AXON_PERSIST=1) until it beats the multi-kernel step everywhere
+  if (!f32 && env_flag("AXON_PERSIST") && (m->d == 64 || m->d == 128)) {
+    const int per_sm = persist_ctas_per_sm(m->d, m->f16);
+    if (per_sm >= 1) {
+      std::vector<PersistLayer> pl(m->L);
+      for (int l = 0; l < m->L; ++l) {
+        const LayerW& w = m->layers[l];
+        PersistLayer& t = pl[l];
+        t.wqkv = w.wqkv;
+        t.bqkv = w.bqkv;
+        t.wo = w.wo;
+        t.wgu = w.wgu;
+        t.wd = w.wd;
+        t.g1 = w.g1;
+        t.g2 = w.g2;
+        t.gnext = l + 1 < m->L ? m->layers[l + 1].g1 : m->gf;
+        t.kc = static_cast<char*>(m->kpool) + static_cast<size_t>(l) * m->layer_kv_elems * m->esz;
+        t.vc = static_cast<char*>(m->vpool) + static_cast<size_t>(l) * m->layer_kv_elems * m->esz;
+      }
+      if ((rc = dev_alloc(m, &p, sizeof(PersistLayer) * (m->L > 0 ? m->L : 1)))) return fail(rc);
+      m->players = static_cast<PersistLayer*>(p);
+      if (m->L > 0 && cudaMemcpy(m->players, pl.data(), sizeof(PersistLayer) * m->L, cudaMemcpyHostToDevice) !=
+                          cudaSuccess)
+        return fail(AXON_ERR_CUDA);
+      std::vector<CUtensorMap> maps(4 * m->L + 1);
+      bool ok = true;
+      for (int l = 0; l < m->L && ok; ++l) {
+        const LayerW& w = m->layers[l];
+        ok = make_tma_2d_plain(&maps[4 * l + 0], w.wqkv, m->Nqkv, D, PERSIST_BOX_COLS, 16, m->f16) &&
+             make_tma_2d_plain(&maps[4 * l + 1], w.wo, D, Hd, PERSIST_BOX_COLS, 16, m->f16) &&
+             make_tma_2d_plain(&maps[4 * l + 2], w.wgu, 2 * F, D, PERSIST_BOX_COLS, 16, m->f16) &&
+             make_tma_2d_plain(&maps[4 * l + 3], w.wd, D, F, PERSIST_BOX_COLS, 16, m->f16);
+      }
+      ok = ok && make_tma_2d_plain(&maps[4 * m->L], m->head, V, D, PERSIST_BOX_COLS, 16, m->f16);
+      if (!ok) return fail(AXON_ERR_CUDA);
+      if ((rc = dev_alloc(m, &p, sizeof(CUtensorMap) * maps.size()))) return fail(rc);
+      m->pmaps = static_cast<CUtensorMap*>(p);
+      if (cudaMemcpy(m->pmaps, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice) != cudaSuccess)
+        return fail(AXON_ERR_CUDA);
+      if ((rc = dev_alloc(m, &p, sizeof(PersistGrid)))) return fail(rc);
+      m->pgrid = static_cast<PersistGrid*>(p);
+      if (cudaMemsetAsync(m->pgrid, 0, sizeof(PersistGrid), st) != cudaSuccess) return fail(AXON_ERR_CUDA);
+      m->persist_ctas = m->num_sms;  // one CTA per SM
+    }
+  }
   if (cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking) != cudaSuccess) return fail(AXON_ERR_CUDA);
   if (cudaStreamSynchronize(st) != cudaSuccess) return fail(AXON_ERR_CUDA);
   *out = m;
@@ -988,7 +1103,9 @@ int axon_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t*
   const bool paged = m->cfg.kv_layout == AXON_KV_PAGED;
   if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (!m->use_graphs) return enqueue_decode(m, d_tokens, B, d_context_lens, d_block_table, d_logits, d_next, st);
+  // The persistent step is a single launch: nothing for a graph to save.
+  if (!m->use_graphs || persist_eligible(m, B))
+    return enqueue_decode(m, d_tokens, B, d_context_lens, d_block_table, d_logits, d_next, st);
   const GraphKey key{B, d_tokens, d_context_lens, d_block_table, d_logits, d_next};
   auto it = m->graphs.find(key);
   if (it == m->graphs.end()) {

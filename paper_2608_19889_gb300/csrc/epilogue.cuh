@@ -189,7 +189,9 @@ AXON_DEV float epi_resid16(const EpiArgs& e, int m, int n0, const float* v) {
   float xn[16];
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
-    float4 t = *reinterpret_cast<const float4*>(xp + i);
+    // L2 read: the previous writer of this slice may be another SM of the
+    // same (persistent) kernel, whose writes L1 does not see.
+    float4 t = __ldcg(reinterpret_cast<const float4*>(xp + i));
     xn[i] = t.x + v[i];
     xn[i + 1] = t.y + v[i + 1];
     xn[i + 2] = t.z + v[i + 2];

@@ -101,9 +101,71 @@ struct GemmMaps {
   bool split = false;
 };
 bool make_tma_2d_16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows, bool f16);
+// Row-major [rows][cols] 16-bit matrix, box box_cols x box_rows, no swizzle
+// (dense rows in shared memory); out-of-range elements read as zero.
+bool make_tma_2d_plain(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
+                       uint32_t box_rows, bool f16);
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep);
 
 // ---- fp32 debug projections (k_simt.cu): plain tiled CUDA-core GEMM with
 // the same epilogues, any M.
 cudaError_t launch_gemm_simt(const LaunchCtx& lc, int kind, const float* A, long long a_stride, const float* W, int M,
                              int N, int K, const EpiArgs& ep);
+
+// ---- persistent decode step (k_persist.cu): one cooperative launch of one
+// CTA per SM runs a whole decode step for B <= PERSIST_MAX_B sequences.
+constexpr int PERSIST_MAX_B = 8;
+constexpr int PERSIST_BOX_COLS = 256;
+struct PersistLayer {
+  const void* wqkv;
+  const float* bqkv;  // or null
+  const void* wo;
+  const void* wgu;
+  const void* wd;
+  const float* g1;     // input norm gain
+  const float* g2;     // post-attention norm gain
+  const float* gnext;  // gain of the norm after this layer (next layer's g1, or the final norm)
+  void* kc;            // this layer's K pool
+  void* vc;            // this layer's V pool
+};
+// Grid barrier state: zero before a launch; the launch leaves it zero.
+struct PersistGrid {
+  unsigned count;
+  unsigned exit;
+  unsigned abort;
+  unsigned pad;
+};
+struct PersistArgs {
+  int L, D, H, G, d, F, V, Nqkv, Pmax, B;
+  int max_pos, blocks_per_seq, num_blocks, splits;
+  float eps, inv_D, scale_log2;
+  const PersistLayer* layers;  // device [L]
+  // device [4L + 1]: per layer the QKV, O, gate/up and down weights, then the
+  // LM head; box PERSIST_BOX_COLS x 16 rows, no swizzle
+  const CUtensorMap* wmaps;
+  const void* embed;
+  const void* head;
+  const float* gf;
+  const float2* rope;
+  float* x;
+  void* a;
+  void* a_lo;  // fp16 mode: second term of a
+  float* ss;   // norm partials [B][Pmax]
+  void* q;
+  void* o;
+  void* u;
+  unsigned long long* keys;
+  float* attn_part;
+  int* attn_cnt;
+  int* err;
+  PersistGrid* grid;
+  const int* tokens;
+  int* ctx;
+  const int* block_table;
+  float* logits;
+  int* next;
+};
+// Resident CTAs per SM of the kernel for this head_dim / type (0: not
+// available); also sets its shared-memory limit. Call before any launch.
+int persist_ctas_per_sm(int head_dim, bool use_f16);
+cudaError_t launch_persist_decode(const PersistArgs& a, int head_dim, bool use_f16, int nctas, cudaStream_t st);
