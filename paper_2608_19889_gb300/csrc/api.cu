@@ -75,6 +75,8 @@ struct axon_model {
   float* x = nullptr;
   void* a = nullptr;
   void* a_lo = nullptr;  // fp16 mode: second term of the normed operand (x*g - a), same layout as a
+  void* o_lo = nullptr;  // fp16 mode, decode: second terms of the attention output and the SwiGLU output
+  void* u_lo = nullptr;
   float* ss = nullptr;
   void* q = nullptr;
   void* o = nullptr;
@@ -401,6 +403,7 @@ inline void pend(Prof* p, double bytes, double flops) {
 struct Proj {
   const axon_model* m;
   LaunchCtx lc;
+  bool decode = false;  // o_lo / u_lo were written by this step's producers
   cudaError_t rc = cudaSuccess;
   // act: activation rows (row stride act_stride elements), M rows. Returns
   // the norm state a RESID producer leaves behind.
@@ -425,8 +428,13 @@ struct Proj {
     } else if (gemv) {
       // fp16 mode: consumers of the normed operand `a` also read its
       // second term a_lo
-      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk,
-                       m->f16 && act == m->a ? m->a_lo : nullptr);
+      const void* lo = nullptr;
+      if (m->f16) {
+        if (act == m->a) lo = m->a_lo;
+        else if (decode && act == m->o) lo = m->o_lo;
+        else if (decode && act == m->u) lo = m->u_lo;
+      }
+      rc = launch_gemv(lc, kind, m->fp32, W, N, K, act, act_stride, M, ep, m->splitk, lo);
       ns.parts = N / 16;
     } else if (m->fp32) {
       rc = launch_gemm_simt(lc, kind, static_cast<const float*>(act), act_stride, static_cast<const float*>(W), M, N,
@@ -582,6 +590,8 @@ PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int3
   a.q = m->q;
   a.o = m->o;
   a.u = m->u;
+  a.o_lo = m->o_lo;
+  a.u_lo = m->u_lo;
   a.keys = m->keys;
   a.attn_part = attn_part;
   a.attn_cnt = attn_cnt;
@@ -601,6 +611,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms, m->f16};
   g_trace_stream = st;
   Proj pj{m, lc};
+  pj.decode = true;
   const int D = m->D, Hd = m->H * m->d;
   const double es = static_cast<double>(m->esz);
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * Hd * es,
@@ -613,10 +624,25 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     if (splits > cap) splits = cap < 1 ? 1 : cap;
   }
   if (persist_eligible(m, B)) {
-    PersistArgs pa = persist_args(m, tokens, B, ctx, bt, logits, next, splits, attn_part ? attn_part : m->attn_part,
+    // Inside one launch a cross-CTA merge costs more than it saves at these
+    // lengths: split a sequence's keys only beyond 64 blocks (8 per warp).
+    int psplits = (m->blocks_per_seq + 63) / 64;
+    if (psplits > splits) psplits = splits;
+    PersistArgs pa = persist_args(m, tokens, B, ctx, bt, logits, next, psplits, attn_part ? attn_part : m->attn_part,
                                   attn_cnt ? attn_cnt : m->attn_cnt);
     pbeg(pf, "decode_persistent");
-    CK(launch_persist_decode(pa, m->d, m->f16, m->persist_ctas, st));
+    const cudaError_t pe = launch_persist_decode(pa, m->d, m->f16, m->persist_ctas, st);
+    if (pe == cudaErrorCooperativeLaunchTooLarge) {
+      // not every SM is free for a co-resident grid: take the launch chain
+      cudaGetLastError();
+      if (pf) {
+        cudaEventDestroy(pf->entries.back().a);
+        cudaEventDestroy(pf->entries.back().b);
+        pf->entries.pop_back();
+      }
+      goto launch_chain;
+    }
+    CK(pe);
     const double kvb = kv_tokens * 2.0 * m->G * m->d * es * m->L;
     pend(pf, m->L * (wq + wo + wgu + wdn) + whd + kvb + B * (logits ? 4.0 * m->V : 0.0),
          2.0 * B * (m->L * (static_cast<double>(m->Nqkv) * D + static_cast<double>(D) * Hd + 3.0 * m->F * D) +
@@ -624,6 +650,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
              4.0 * kv_tokens * m->H * m->d * m->L);
     return AXON_OK;
   }
+launch_chain:
   pbeg(pf, "embed");
   CK(launch_embed(lc, m->fp32, m->embed, m->V, D, tokens, B, m->x, m->a, m->L > 0 ? m->layers[0].g1 : m->gf, m->ss,
                   m->Pmax, m->rinv, m->cfg.rms_norm_eps, m->err, m->a_lo));
@@ -650,6 +677,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     at.splits = splits;
     at.part = attn_part ? attn_part : m->attn_part;
     at.counter = attn_cnt ? attn_cnt : m->attn_cnt;
+    at.o_lo = m->o_lo;
     pbeg(pf, "decode_attention");
     CK(launch_attn_decode(lc, m->fp32, at, B));
     pend(pf, kv_tokens * 2.0 * m->G * m->d * es + 2.0 * B * Hd * es, 4.0 * kv_tokens * m->H * m->d);
@@ -673,6 +701,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     g.ctx = ctx;
     set_norm(m, ns, g);
     g.u_out = m->u;
+    g.u_lo_out = m->u_lo;
     pbeg(pf, "decode_gateup");
     pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok);
     CK(pj.rc);
@@ -950,6 +979,10 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   if ((rc = dev_alloc(m, &m->q, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
   if ((rc = dev_alloc(m, &m->o, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
   if ((rc = dev_alloc(m, &m->u, static_cast<size_t>(Mcap) * F * es))) return fail(rc);
+  if (m->f16) {
+    if ((rc = dev_alloc(m, &m->o_lo, static_cast<size_t>(m->cfg.max_batch) * Hd * es))) return fail(rc);
+    if ((rc = dev_alloc(m, &m->u_lo, static_cast<size_t>(m->cfg.max_batch) * F * es))) return fail(rc);
+  }
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * 8))) return fail(rc);
   m->keys = static_cast<unsigned long long*>(p);
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * 4))) return fail(rc);
@@ -1032,8 +1065,8 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     if (!ok) return fail(AXON_ERR_CUDA);
   }
   // ---- persistent decode step: layer table and grid barrier state
-  // opt-in (AXON_PERSIST=1) until it beats the multi-kernel step everywhere
-  if (!f32 && env_flag("AXON_PERSIST") && (m->d == 64 || m->d == 128)) {
+  // default for B <= PERSIST_MAX_B; AXON_NO_PERSIST=1 keeps the launch chain
+  if (!f32 && !env_flag("AXON_NO_PERSIST") && (m->d == 64 || m->d == 128)) {
     const int per_sm = persist_ctas_per_sm(m->d, m->f16);
     if (per_sm >= 1) {
       std::vector<PersistLayer> pl(m->L);

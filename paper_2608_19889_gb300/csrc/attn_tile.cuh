@@ -168,12 +168,6 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
   if (s >= n_used) return;
   const int jb = s * per, je = min(jb + per, nblk);
 
-  const uint16_t* qg = static_cast<const uint16_t*>(p.q) + (static_cast<long long>(b) * p.H + g * HPG) * HD;
-  uint32_t qa[HD / 16][4];
-  load_q<HD>(qa, r < HPG ? qg + r * HD : nullptr, r + 8 < HPG ? qg + (r + 8) * HD : nullptr, q);
-
-  WarpState<HD> st;
-  st.init();
   const uint32_t wbase = smem_u32(sm) + warp * 4 * TILE;  // per warp: [stage][K | V]
   const uint16_t* kp = static_cast<const uint16_t*>(p.k);
   const uint16_t* vp = static_cast<const uint16_t*>(p.v);
@@ -185,8 +179,17 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
     stage_tile<HD>(wbase + stg * 2 * TILE + TILE, vp + off, ok, lane, 32);
     cp_async_commit();
   };
+  // The first key/value tile is requested before q is read: the two round
+  // trips overlap.
   int j = jb + warp, stg = 0;
   if (j < je) issue(j, 0);
+
+  const uint16_t* qg = static_cast<const uint16_t*>(p.q) + (static_cast<long long>(b) * p.H + g * HPG) * HD;
+  uint32_t qa[HD / 16][4];
+  load_q<HD>(qa, r < HPG ? qg + r * HD : nullptr, r + 8 < HPG ? qg + (r + 8) * HD : nullptr, q);
+
+  WarpState<HD> st;
+  st.init();
   for (; j < je; j += DEC_WARPS) {
     const int jn = j + DEC_WARPS;
     if (jn < je) {
@@ -246,7 +249,9 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
     }
     if (n_used == 1) {
       T16* og = static_cast<T16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
-      *og = from_f<T16>(L > 0.f ? O / L : 0.f);
+      const float ov = L > 0.f ? O / L : 0.f;
+      *og = from_f<T16>(ov);
+      if (p.o_lo) static_cast<T16*>(p.o_lo)[og - static_cast<T16*>(p.o)] = from_f<T16>(ov - to_f(from_f<T16>(ov)));
     } else {
       float* pr = part + (static_cast<long long>(s) * 16 + i) * rowlen;
       pr[dd] = O;
@@ -304,7 +309,9 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
     }
     for (; t < n_used; ++t) O0 += cw[i][t] * __ldcg(pc + t * 16 * rowlen);
     T16* og = static_cast<T16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
-    *og = from_f<T16>(((O0 + O1) + (O2 + O3)) * cinv[i]);
+    const float ov = ((O0 + O1) + (O2 + O3)) * cinv[i];
+    *og = from_f<T16>(ov);
+    if (p.o_lo) static_cast<T16*>(p.o_lo)[og - static_cast<T16*>(p.o)] = from_f<T16>(ov - to_f(from_f<T16>(ov)));
   }
   if (tid == 0) p.counter[b * p.G + g] = 0;
 }

@@ -62,7 +62,8 @@ struct EpiArgs {
   float* rinv_out;
   int* ticket;
   // SWIGLU
-  void* u_out;  // [M][N/2]
+  void* u_out;     // [M][N/2]
+  void* u_lo_out;  // optional [M][N/2]: u - u_out (second term of the down projection's operand)
   // LOGITS
   float* logits;  // [M][logits_stride] or null
   long long logits_stride;
@@ -229,6 +230,12 @@ AXON_DEV void epi_swiglu16(const EpiArgs& e, int m, int n0, const float* v, floa
   for (int i = 0; i < 8; ++i) u[i] = silu_f(v[i] * r) * (v[8 + i] * r);
   T* up = reinterpret_cast<T*>(e.u_out) + static_cast<long long>(m) * (e.N >> 1) + (n0 >> 1);
   store8<T>(up, u);
+  if (e.u_lo_out) {
+    float lo[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) lo[i] = u[i] - to_f(from_f<T>(u[i]));
+    store8<T>(reinterpret_cast<T*>(e.u_lo_out) + static_cast<long long>(m) * (e.N >> 1) + (n0 >> 1), lo);
+  }
 }
 
 // logits = r * v (columns >= N dropped); returns this chunk's argmax key.

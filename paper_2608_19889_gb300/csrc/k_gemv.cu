@@ -384,9 +384,7 @@ cudaError_t gemv_nt(const LaunchCtx& lc, int kind, const void* W, int N, int K, 
   if (lc.f16) {
     const f16* w = static_cast<const f16*>(W);
     const f16* a = static_cast<const f16*>(act);
-    // The residual projections read attention / SwiGLU outputs, which have
-    // no second term.
-    if (act_lo && kind != EPI_RESID)
+    if (act_lo)
       return gemv_nt_lo<NT, f16, true>(lc, kind, w, N, K, a, st, B, ep, sk, static_cast<const f16*>(act_lo));
     return gemv_nt_lo<NT, f16, false>(lc, kind, w, N, K, a, st, B, ep, sk, nullptr);
   }
@@ -460,7 +458,7 @@ cudaError_t occupancy_kind(int idx) {
   int a = 0, b = 0;
   cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, gemv_mma_kernel<NT, KIND, bf16, false>, threads, 0);
   b = a;
-  if (e == cudaSuccess && KIND != EPI_RESID)  // residual kinds never take the split operand
+  if (e == cudaSuccess)
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, gemv_mma_kernel<NT, KIND, f16, true>, threads, 0);
   g_resident[idx][KIND] = a < b ? a : b;
   return e;

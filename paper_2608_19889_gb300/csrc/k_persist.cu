@@ -115,13 +115,19 @@ AXON_DEV bool ring_wait(uint32_t bar, uint32_t parity, PersistGrid* g, volatile 
   }
 }
 
-// Grid-wide barrier of the consumer warps (the producer never takes part).
+AXON_DEV void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Grid-wide barrier of the consumer warps (the producer never takes part):
+// the CTA's writes are ordered before its arrival by the CTA barrier and the
+// release of the arrival (cumulative); the acquiring poll orders every later
+// read after all arrivals, and the closing CTA barrier passes that on.
 AXON_DEV void grid_sync(PersistGrid* g, unsigned& epoch, int tid, volatile int* s_abort, int* err) {
   consumer_sync();
   if (tid == 0) {
     ++epoch;
-    __threadfence();
-    atomicAdd(&g->count, 1u);
+    red_release_add(&g->count, 1u);
     const unsigned target = epoch * gridDim.x;
     if (!*s_abort) {
       const uint64_t t0 = global_ns();
@@ -141,7 +147,6 @@ AXON_DEV void grid_sync(PersistGrid* g, unsigned& epoch, int tid, volatile int* 
         }
       }
     }
-    __threadfence();
   }
   consumer_sync();
 }
@@ -555,6 +560,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       p.scale_log2 = A.scale_log2;
       p.part = A.attn_part;
       p.counter = A.attn_cnt;
+      p.o_lo = A.o_lo;
       p.err = A.err;
       const int items = A.splits * A.G * B;
       for (int it = blockIdx.x; it < items; it += gridDim.x) {
@@ -571,9 +577,9 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       e.a_out = A.a;
       e.a_lo_out = A.a_lo;
       e.gain = w.g2;
-      proj_phase<HD, EPI_RESID, T16, false>(R, cs, A, static_cast<const T16*>(w.wo), A.D, Hd,
-                                            static_cast<const T16*>(A.o), nullptr, Hd, e, red_base, rinv_s, best_s,
-                                            attn_sm, g, s_abort, tid);
+      proj_phase<HD, EPI_RESID, T16, LO>(R, cs, A, static_cast<const T16*>(w.wo), A.D, Hd,
+                                         static_cast<const T16*>(A.o), static_cast<const T16*>(A.o_lo), Hd, e,
+                                         red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
     }
     grid_sync(g, epoch, tid, s_abort, A.err);
     // gate/up + SwiGLU
@@ -581,6 +587,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       EpiArgs e = base_ep(A);
       e.N = 2 * A.F;
       e.u_out = A.u;
+      e.u_lo_out = A.u_lo;
       proj_phase<HD, EPI_SWIGLU, T16, LO>(R, cs, A, static_cast<const T16*>(w.wgu), 2 * A.F, A.D, a16, alo16, A.D, e,
                                           red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
     }
@@ -593,9 +600,9 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       e.a_out = A.a;
       e.a_lo_out = A.a_lo;
       e.gain = w.gnext;
-      proj_phase<HD, EPI_RESID, T16, false>(R, cs, A, static_cast<const T16*>(w.wd), A.D, A.F,
-                                            static_cast<const T16*>(A.u), nullptr, A.F, e, red_base, rinv_s, best_s,
-                                            attn_sm, g, s_abort, tid);
+      proj_phase<HD, EPI_RESID, T16, LO>(R, cs, A, static_cast<const T16*>(w.wd), A.D, A.F,
+                                         static_cast<const T16*>(A.u), static_cast<const T16*>(A.u_lo), A.F, e,
+                                         red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
     }
     grid_sync(g, epoch, tid, s_abort, A.err);
   }

@@ -31,7 +31,7 @@ struct SplitK {
   float* part;
   int* ticket;
 };
-// act_lo (optional, fp16 mode, ignored by the residual kinds): second term
+// act_lo (optional, fp16 mode): second term
 // of a split activation operand, same layout and stride as act.
 cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W, int N, int K, const void* act,
                         long long act_stride, int B, const EpiArgs& ep, const SplitKWork& wk,
@@ -81,6 +81,7 @@ struct AttnArgs {
   int splits;   // decode split-KV factor
   float scale_log2;
   float* part;  // decode partials
+  void* o_lo;   // optional [rows][H*d]: o minus its 16-bit rounding (decode, fp16 mode)
   int* counter;  // decode [B][G] tickets
   int* err;
 };
@@ -154,6 +155,8 @@ struct PersistArgs {
   void* q;
   void* o;
   void* u;
+  void* o_lo;  // fp16 mode: second terms of o and u
+  void* u_lo;
   unsigned long long* keys;
   float* attn_part;
   int* attn_cnt;

@@ -25,17 +25,17 @@ def _built():
 
 
 def _create(shape, w, persistent, **kw):
-    """Model with the persistent decode step switched on (AXON_PERSIST=1 at
-    creation) or off."""
-    old = os.environ.pop("AXON_PERSIST", None)
+    """Model with the persistent decode step (the default) or with the launch
+    chain (AXON_NO_PERSIST=1 at creation)."""
+    old = os.environ.pop("AXON_NO_PERSIST", None)
     try:
-        if persistent:
-            os.environ["AXON_PERSIST"] = "1"
+        if not persistent:
+            os.environ["AXON_NO_PERSIST"] = "1"
         return create(shape, w, **kw)
     finally:
-        os.environ.pop("AXON_PERSIST", None)
+        os.environ.pop("AXON_NO_PERSIST", None)
         if old is not None:
-            os.environ["AXON_PERSIST"] = old
+            os.environ["AXON_NO_PERSIST"] = old
 
 
 def _kinds(m, B, ctx0, bt=None):
