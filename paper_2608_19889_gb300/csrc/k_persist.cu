@@ -213,8 +213,9 @@ struct CState {
 template <int HD, typename T16, bool LO>
 AXON_DEV void load_stage(const Ring<HD>& R, CState& cs, const PersistArgs& A, PersistGrid* g, volatile int* s_abort,
                          int t, int spi, int K, int warp, int lane, int r, int q, bool tok_ok, bool staged,
-                         const uint8_t* act_sm, int pitch, const T16* arow, const T16* lrow, uint4& w0, uint4& w1,
-                         uint4& w2, uint4& w3, uint4& x0, uint4& x1, uint4& y0, uint4& y1, bool& on) {
+                         const uint8_t* act_sm, int pitch, const T16* xsrc, const T16* ysrc, int xrow_s, int yrow_s,
+                         bool want_y, uint4& w0, uint4& w1, uint4& w2, uint4& w3, uint4& x0, uint4& x1, uint4& y0,
+                         uint4& y1, bool& on) {
   constexpr int NS = PLayout<HD>::NS;
   const int k0 = (t % spi) * KC;
   const int kc = min(KC, K - k0);
@@ -232,19 +233,20 @@ AXON_DEV void load_stage(const Ring<HD>& R, CState& cs, const PersistArgs& A, Pe
     const int k = k0 + warp * 64;
     if (tok_ok) {
       if (staged) {
-        const uint32_t sa = smem_u32(act_sm) + r * pitch + (k + 16 * q) * 2;
+        const uint32_t sa = smem_u32(act_sm) + xrow_s * pitch + (k + 16 * q) * 2;
         x0 = lds16(sa);
         x1 = lds16(sa + 16);
-        if (LO) {
-          y0 = lds16(sa + A.B * pitch);
-          y1 = lds16(sa + A.B * pitch + 16);
+        if (LO && want_y) {
+          const uint32_t sb = smem_u32(act_sm) + yrow_s * pitch + (k + 16 * q) * 2;
+          y0 = lds16(sb);
+          y1 = lds16(sb + 16);
         }
       } else {
-        x0 = __ldcg(reinterpret_cast<const uint4*>(arow + k));
-        x1 = __ldcg(reinterpret_cast<const uint4*>(arow + k + 8));
-        if (LO) {
-          y0 = __ldcg(reinterpret_cast<const uint4*>(lrow + k));
-          y1 = __ldcg(reinterpret_cast<const uint4*>(lrow + k + 8));
+        x0 = __ldcg(reinterpret_cast<const uint4*>(xsrc + k));
+        x1 = __ldcg(reinterpret_cast<const uint4*>(xsrc + k + 8));
+        if (LO && want_y) {
+          y0 = __ldcg(reinterpret_cast<const uint4*>(ysrc + k));
+          y1 = __ldcg(reinterpret_cast<const uint4*>(ysrc + k + 8));
         }
       }
     }
@@ -312,9 +314,20 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
     rp = warp_sum(rp);
     if (lane == 0) rinv_s[warp] = 1.0f / sqrtf(rp * A.inv_D + A.eps);
   }
-  const bool tok_ok = r < B;
-  const T16* arow = act + static_cast<long long>(tok_ok ? r : 0) * act_stride + 16 * q;
-  const T16* lrow = LO ? act_lo + static_cast<long long>(tok_ok ? r : 0) * act_stride + 16 * q : nullptr;
+  // Token slot r of the MMA's N dimension normally holds token r (and, with
+  // the split operand, a second MMA set holds its second term). With B <= 4
+  // and the split operand the two terms share one MMA instead: slot 2b holds
+  // token b's first term and slot 2b+1 its second, and the reduction adds
+  // the two accumulator columns -- no extra MMA, no extra load.
+  const bool paired = LO && B <= 4;
+  const int tb = paired ? (r >> 1) : r;
+  const bool term_lo = paired && (r & 1);
+  const bool tok_ok = tb < B;
+  const int tsafe = tok_ok ? tb : 0;
+  const T16* xsrc = (term_lo ? act_lo : act) + static_cast<long long>(tsafe) * act_stride + 16 * q;
+  const T16* ysrc = LO ? act_lo + static_cast<long long>(tsafe) * act_stride + 16 * q : nullptr;
+  const int xrow_s = term_lo ? B + tsafe : tsafe, yrow_s = B + tsafe;
+  const bool want_y = LO && !paired;
 
   // Epilogues of the buffered items slot 0 .. nslots-1 (items i0 + slot * grid).
   auto flush = [&](int i0, int nslots) {
@@ -348,8 +361,8 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
     for (int t = 0; t < spi; ++t) {
       uint4 w0, w1, w2, w3, x0, x1, y0, y1;
       bool on;
-      load_stage<HD, T16, LO>(R, cs, A, g, s_abort, t, spi, K, warp, lane, r, q, tok_ok, staged, act_sm, pitch, arow,
-                              lrow, w0, w1, w2, w3, x0, x1, y0, y1, on);
+      load_stage<HD, T16, LO>(R, cs, A, g, s_abort, t, spi, K, warp, lane, r, q, tok_ok, staged, act_sm, pitch, xsrc,
+                              ysrc, xrow_s, yrow_s, want_y, w0, w1, w2, w3, x0, x1, y0, y1, on);
       if (on) {
         const uint32_t A0[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
         const uint32_t A1[8] = {w2.x, w2.y, w2.z, w2.w, w3.x, w3.y, w3.z, w3.w};
@@ -362,7 +375,7 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
           const uint32_t bb[2] = {Bv[2 * j], Bv[2 * j + 1]};
           mma16816<T16>(acc[j & 1], a, bb);
         }
-        if (LO) {
+        if (LO && want_y) {
           const uint32_t Bl[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
@@ -373,12 +386,17 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
         }
       }
     }
-    // Accumulator of lane (r, q): rows r, r+8 x tokens 2q, 2q+1.
+    // Accumulator of lane (r, q): rows r, r+8 x token slots 2q, 2q+1.
     float* red = red_base + cs.buf * RED_FLOATS;
-    red[(warp * 16 + r) * 9 + 2 * q] = acc[0][0] + acc[1][0];
-    red[(warp * 16 + r) * 9 + 2 * q + 1] = acc[0][1] + acc[1][1];
-    red[(warp * 16 + r + 8) * 9 + 2 * q] = acc[0][2] + acc[1][2];
-    red[(warp * 16 + r + 8) * 9 + 2 * q + 1] = acc[0][3] + acc[1][3];
+    if (paired) {  // slots 2q, 2q+1 = the two terms of token q
+      red[(warp * 16 + r) * 9 + q] = (acc[0][0] + acc[1][0]) + (acc[0][1] + acc[1][1]);
+      red[(warp * 16 + r + 8) * 9 + q] = (acc[0][2] + acc[1][2]) + (acc[0][3] + acc[1][3]);
+    } else {
+      red[(warp * 16 + r) * 9 + 2 * q] = acc[0][0] + acc[1][0];
+      red[(warp * 16 + r) * 9 + 2 * q + 1] = acc[0][1] + acc[1][1];
+      red[(warp * 16 + r + 8) * 9 + 2 * q] = acc[0][2] + acc[1][2];
+      red[(warp * 16 + r + 8) * 9 + 2 * q + 1] = acc[0][3] + acc[1][3];
+    }
     consumer_sync();
     if (tid < B * 16) {
       const int b = tid >> 4, rr = tid & 15;
