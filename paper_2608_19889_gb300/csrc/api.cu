@@ -34,6 +34,7 @@ struct LayerW {
   float* g1 = nullptr;
   float* g2 = nullptr;
   GemmMaps m_qkv{}, m_o{}, m_gu{}, m_d{};
+  GemmMaps m_qkv128{}, m_o128{}, m_gu128{}, m_d128{};  // the same with 128-row weight boxes
   CUtensorMap v_qkv{}, v_o{}, v_gu{}, v_d{};  // weight maps for the decode projections (box 64 x 128)
 };
 
@@ -60,7 +61,7 @@ struct axon_model {
   void* head = nullptr;
   float* gf = nullptr;
   std::vector<LayerW> layers;
-  GemmMaps m_head{};
+  GemmMaps m_head{}, m_head128{};
   CUtensorMap v_head{};
   // KV cache
   void* kpool = nullptr;
@@ -441,8 +442,9 @@ struct Proj {
                             K, ep);
       ns.parts = N / 16;
     } else {
-      rc = launch_gemm_tc(lc, kind, *maps, M, N, K, ep);
-      ns.parts = (N + 255) / 256;
+      const int tn = gemm_tile_n(lc, *maps, M, N);
+      rc = launch_gemm_tc(lc, kind, *maps, M, N, K, ep, tn);
+      ns.parts = (N + tn - 1) / tn;
     }
     return ns;
   }
@@ -1057,6 +1059,25 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
            make_tma_2d_16(&w.v_gu, w.wgu, 2 * F, D, 128, m->f16) && make_tma_2d_16(&w.v_d, w.wd, D, F, 128, m->f16);
     }
     ok = ok && make_tma_2d_16(&m->v_head, m->head, V, D, 128, m->f16);
+    // 128-wide output tiles reuse the 128-row weight boxes of the decode maps
+    for (int l = 0; l < m->L && ok; ++l) {
+      LayerW& w = m->layers[l];
+      w.m_qkv128 = w.m_qkv;
+      w.m_qkv128.w = w.v_qkv;
+      w.m_qkv.n128 = &w.m_qkv128;
+      w.m_o128 = w.m_o;
+      w.m_o128.w = w.v_o;
+      w.m_o.n128 = &w.m_o128;
+      w.m_gu128 = w.m_gu;
+      w.m_gu128.w = w.v_gu;
+      w.m_gu.n128 = &w.m_gu128;
+      w.m_d128 = w.m_d;
+      w.m_d128.w = w.v_d;
+      w.m_d.n128 = &w.m_d128;
+    }
+    m->m_head128 = m->m_head;
+    m->m_head128.w = m->v_head;
+    m->m_head.n128 = &m->m_head128;
     for (int i = 0; i < 4 && ok; ++i) {
       const uint32_t tok = 8u << i;
       ok = make_tma_2d_16(&m->t_a_tok[i], m->a, Mcap, D, tok, m->f16) && make_tma_2d_16(&m->t_o_tok[i], m->o, Mcap, Hd, tok, m->f16) &&

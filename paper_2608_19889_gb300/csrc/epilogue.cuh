@@ -130,10 +130,32 @@ AXON_DEV void store8<float>(float* dst, const float* v) {
   reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
 }
 
+// Global inputs of one QKV chunk: the RoPE (cos, sin) pairs of its 8
+// rotation frequencies at the row's position, and its 16 biases.
+struct QkvIn {
+  float2 cs[8];
+  float b[16];
+};
+
+AXON_DEV void load_qkv16(const EpiArgs& e, int m, int n0, QkvIn& in) {
+  const int Hd = e.H * e.d, Gd = e.G * e.d;
+  const int c = n0 < Hd ? n0 % e.d : (n0 < Hd + Gd ? (n0 - Hd) % e.d : (n0 - Hd - Gd) % e.d);
+  int b;
+  const int pos = row_seq_pos(e, m, b);
+  if (n0 < Hd + Gd) {
+    const int pc = min(max(pos, 0), e.max_pos - 1);
+    const float2* cs = e.rope + static_cast<long long>(pc) * (e.d >> 1) + (c >> 4) * 8;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) in.cs[i] = cs[i];
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i) in.b[i] = e.bias ? e.bias[n0 + i] : 0.f;
+}
+
 // q/k/v: scale by r, add bias, rotate q and k, store q to the q buffer and
-// k, v into the cache slot of (b, pos).
+// k, v into the cache slot of (b, pos). `in`: the chunk's loaded inputs.
 template <typename T>
-AXON_DEV void epi_qkv16(const EpiArgs& e, int m, int n0, const float* v, float r) {
+AXON_DEV void epi_qkv16x(const EpiArgs& e, int m, int n0, const float* v, float r, const QkvIn& in) {
   const int Hd = e.H * e.d, Gd = e.G * e.d;
   int region, head, c;
   if (n0 < Hd) {
@@ -149,22 +171,13 @@ AXON_DEV void epi_qkv16(const EpiArgs& e, int m, int n0, const float* v, float r
   float lo[8], hi[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    lo[i] = v[i] * r;
-    hi[i] = v[8 + i] * r;
-  }
-  if (e.bias) {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      lo[i] += e.bias[n0 + i];
-      hi[i] += e.bias[n0 + 8 + i];
-    }
+    lo[i] = v[i] * r + in.b[i];
+    hi[i] = v[8 + i] * r + in.b[8 + i];
   }
   if (region < 2) {
-    const int pc = min(max(pos, 0), e.max_pos - 1);
-    const float2* cs = e.rope + static_cast<long long>(pc) * half + j0;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const float2 t = cs[i];
+      const float2 t = in.cs[i];
       const float a = lo[i], bb = hi[i];
       lo[i] = a * t.x - bb * t.y;
       hi[i] = bb * t.x + a * t.y;
@@ -183,16 +196,22 @@ AXON_DEV void epi_qkv16(const EpiArgs& e, int m, int n0, const float* v, float r
   }
 }
 
-// x += v; a = x * gain; returns sum of x^2 over the 16 columns.
 template <typename T>
-AXON_DEV float epi_resid16(const EpiArgs& e, int m, int n0, const float* v) {
+AXON_DEV void epi_qkv16(const EpiArgs& e, int m, int n0, const float* v, float r) {
+  QkvIn in;
+  load_qkv16(e, m, n0, in);
+  epi_qkv16x<T>(e, m, n0, v, r, in);
+}
+
+// x += v; a = x * gain; returns sum of x^2 over the 16 columns. `xin`:
+// the 16 current residual values, already loaded by the caller.
+template <typename T>
+AXON_DEV float epi_resid16x(const EpiArgs& e, int m, int n0, const float* v, const float4* xin) {
   float* xp = e.x + static_cast<long long>(m) * e.N + n0;
   float xn[16];
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
-    // L2 read: the previous writer of this slice may be another SM of the
-    // same (persistent) kernel, whose writes L1 does not see.
-    float4 t = __ldcg(reinterpret_cast<const float4*>(xp + i));
+    const float4 t = xin[i >> 2];
     xn[i] = t.x + v[i];
     xn[i + 1] = t.y + v[i + 1];
     xn[i + 2] = t.z + v[i + 2];
@@ -219,6 +238,22 @@ AXON_DEV float epi_resid16(const EpiArgs& e, int m, int n0, const float* v) {
     store8<T>(lp + 8, lo + 8);
   }
   return s;
+}
+
+// Loads the 16 residual values of (m, n0..n0+15) from L2: the previous
+// writer of this slice may be another SM of the same (persistent) kernel,
+// whose writes L1 does not see.
+AXON_DEV void load_resid16(const EpiArgs& e, int m, int n0, float4* xin) {
+  const float* xp = e.x + static_cast<long long>(m) * e.N + n0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) xin[i] = __ldcg(reinterpret_cast<const float4*>(xp + 4 * i));
+}
+
+template <typename T>
+AXON_DEV float epi_resid16(const EpiArgs& e, int m, int n0, const float* v) {
+  float4 xin[4];
+  load_resid16(e, m, n0, xin);
+  return epi_resid16x<T>(e, m, n0, v, xin);
 }
 
 AXON_DEV float silu_f(float z) { return z / (1.0f + expf(-z)); }

@@ -43,7 +43,10 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, r = lane >> 2, q = lane & 3;
   const int HPG = p.H / p.G, S = p.S;
   const int PC = 4 * PW;
-  const int b = blockIdx.z, g = blockIdx.y, p0 = blockIdx.x * PC;
+  // grid (kv head, position block, sequence), position blocks counted down
+  // from the end: under the causal mask the last blocks carry the most keys,
+  // and dispatching them first keeps the tail of the launch short.
+  const int b = blockIdx.z, g = blockIdx.x, p0 = (gridDim.y - 1 - blockIdx.y) * PC;
   grid_dep_launch();
   grid_dep_wait();
 
@@ -206,7 +209,7 @@ cudaError_t prefill_hd(const LaunchCtx& lc, const AttnArgs& a, int B) {
   const int HPG = a.H / a.G;
   const int PW = 16 / HPG;
   const int PC = 4 * PW;
-  const dim3 grid((a.S + PC - 1) / PC, a.G, B);
+  const dim3 grid(a.G, (a.S + PC - 1) / PC, B);
   if (lc.f16) return launch_k(lc, attn_prefill_kernel<HD, f16>, grid, dim3(128), smem, a, PW);
   return launch_k(lc, attn_prefill_kernel<HD, bf16>, grid, dim3(128), smem, a, PW);
 }

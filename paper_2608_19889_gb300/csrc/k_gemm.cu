@@ -23,19 +23,23 @@
 
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, GROUP_M = 8;
+constexpr int BM = 128, BK = 64, GROUP_M = 8;
 constexpr int A_BYTES = BM * BK * 2;  // 16 KB
-constexpr int B_BYTES = BN * BK * 2;  // 32 KB
 constexpr int NUM_THREADS = 192;
-constexpr uint32_t TMEM_COLS = 2 * BN;
 
-// SPLIT: the A operand is the sum of two 16-bit terms (hi + lo) and every
-// k-step issues two MMAs into the same accumulator (3 ring stages of 64 KB).
-template <bool SPLIT>
+// BN_: columns of the output tile (256, or 128 where 256-wide tiles leave
+// the last wave mostly empty). SPLIT: the A operand is the sum of two
+// 16-bit terms (hi + lo) and every k-step issues two MMAs into the same
+// accumulator. The ring takes as many stages as fit in 200 KB, at most 6
+// (BN 256: 4, split 3; BN 128: 6, split 4).
+template <bool SPLIT, int BN_>
 struct GCfg {
-  static constexpr int STAGES = SPLIT ? 3 : 4;
+  static constexpr int BN = BN_;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
   static constexpr int A_TERMS = SPLIT ? 2 : 1;
   static constexpr int STAGE_BYTES = A_TERMS * A_BYTES + B_BYTES;
+  static constexpr int STAGES = (200 * 1024) / STAGE_BYTES > 6 ? 6 : (200 * 1024) / STAGE_BYTES;
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
   static constexpr int SMEM = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
 };
@@ -50,11 +54,14 @@ AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
   mb = first_m + (local - nb * gm);
 }
 
-template <int KIND, typename T16, bool SPLIT>
+template <int KIND, typename T16, bool SPLIT, int BN_>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmAlo, int M, int N, int K, EpiArgs ep) {
-  using C = GCfg<SPLIT>;
+  using C = GCfg<SPLIT, BN_>;
+  constexpr int BN = C::BN;
+  constexpr int B_BYTES = C::B_BYTES;
+  constexpr uint32_t TMEM_COLS = C::TMEM_COLS;
   constexpr int STAGES = C::STAGES;
   constexpr int STAGE_BYTES = C::STAGE_BYTES;
   extern __shared__ uint8_t smem_raw[];
@@ -177,8 +184,37 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       float ssum = 0.f;
       unsigned long long best = 0ull;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(q4 * 32) << 16) + buf * BN;
+      if (KIND == EPI_RESID) {
+        // 64 columns at a time: the 16 residual loads of a group are in
+        // flight together, and one TMEM wait covers 4 loads.
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 16) {
+        for (int c0 = 0; c0 < BN; c0 += 64) {
+          float4 xin[4][4];
+          if (mval) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              if (nb * BN + c0 + j * 16 < N) load_resid16(ep, m, nb * BN + c0 + j * 16, xin[j]);
+          }
+          uint32_t v[4][16];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) tmem_ld16(taddr + c0 + j * 16, v[j]);
+          tmem_wait_ld();
+          if (mval) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const int n0 = nb * BN + c0 + j * 16;
+              if (n0 < N) {
+                float f[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(v[j][i]);
+                ssum += epi_resid16x<T16>(ep, m, n0, f, xin[j]);
+              }
+            }
+          }
+        }
+      }
+#pragma unroll 1
+      for (int c = 0; c < BN && KIND != EPI_RESID; c += 16) {
         uint32_t v[16];
         tmem_ld16(taddr + c, v);
         tmem_wait_ld();
@@ -189,8 +225,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(v[i]);
           if (KIND == EPI_QKV) {
             epi_qkv16<T16>(ep, m, n0, f, rinv);
-          } else if (KIND == EPI_RESID) {
-            ssum += epi_resid16<T16>(ep, m, n0, f);
           } else if (KIND == EPI_SWIGLU) {
             epi_swiglu16<T16>(ep, m, n0, f, rinv);
           } else {
@@ -226,22 +260,22 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int KIND, typename T16, bool SPLIT>
+template <int KIND, typename T16, bool SPLIT, int BN>
 cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep) {
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const int grid = tiles < lc.num_sms ? tiles : lc.num_sms;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(NUM_THREADS);
-  cfg.dynamicSmemBytes = GCfg<SPLIT>::SMEM;
+  cfg.dynamicSmemBytes = GCfg<SPLIT, BN>::SMEM;
   cfg.stream = lc.stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = lc.pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT>, maps.a, maps.w, SPLIT ? maps.a_lo : maps.a, M, N,
-                            K, ep);
+  const GemmMaps& g = BN == 256 ? maps : *maps.n128;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN>, g.a, g.w, SPLIT ? g.a_lo : g.a, M, N, K, ep);
 }
 
 }  // namespace
@@ -272,10 +306,16 @@ bool make_tma_2d_plain(CUtensorMap* map, const void* base, uint64_t rows, uint64
 }
 
 namespace {
+template <int KIND, typename T16, bool SPLIT, int BN>
+cudaError_t set_smem1() {
+  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              GCfg<SPLIT, BN>::SMEM);
+}
 template <int KIND, typename T16, bool SPLIT>
 cudaError_t set_smem() {
-  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              GCfg<SPLIT>::SMEM);
+  cudaError_t e = set_smem1<KIND, T16, SPLIT, 256>();
+  if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128>();
+  return e;
 }
 template <typename T16>
 cudaError_t prepare_gemm_t() {
@@ -286,18 +326,30 @@ cudaError_t prepare_gemm_t() {
   if (e == cudaSuccess) e = set_smem<EPI_LOGITS, T16, false>();
   return e;
 }
-template <typename T16>
+template <typename T16, int BN>
 cudaError_t launch_t(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep) {
   switch (kind) {
     case EPI_QKV:
-      return maps.split ? launch_kind<EPI_QKV, T16, true>(lc, maps, M, N, K, ep)
-                        : launch_kind<EPI_QKV, T16, false>(lc, maps, M, N, K, ep);
-    case EPI_RESID: return launch_kind<EPI_RESID, T16, false>(lc, maps, M, N, K, ep);
-    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false>(lc, maps, M, N, K, ep);
-    default: return launch_kind<EPI_LOGITS, T16, false>(lc, maps, M, N, K, ep);
+      return maps.split ? launch_kind<EPI_QKV, T16, true, BN>(lc, maps, M, N, K, ep)
+                        : launch_kind<EPI_QKV, T16, false, BN>(lc, maps, M, N, K, ep);
+    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN>(lc, maps, M, N, K, ep);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN>(lc, maps, M, N, K, ep);
+    default: return launch_kind<EPI_LOGITS, T16, false, BN>(lc, maps, M, N, K, ep);
   }
 }
 }  // namespace
+
+// Output-tile width for an M x N product: 128 where 256-wide tiles leave
+// the last wave mostly idle (cost in column-waves: waves x width, plus a
+// per-tile overhead worth 16 columns), 256 otherwise.
+int gemm_tile_n(const LaunchCtx& lc, const GemmMaps& maps, int M, int N) {
+  if (!maps.n128) return 256;
+  const long long mt = (M + BM - 1) / BM;
+  const long long t256 = mt * ((N + 255) / 256), t128 = mt * ((N + 127) / 128);
+  const long long w256 = (t256 + lc.num_sms - 1) / lc.num_sms, w128 = (t128 + lc.num_sms - 1) / lc.num_sms;
+  const long long c256 = w256 * (256 + 16), c128 = w128 * (128 + 16);
+  return c128 * 100 < c256 * 85 ? 128 : 256;
+}
 
 cudaError_t prepare_gemm_kernels() {
   cudaError_t e = prepare_gemm_t<bf16>();
@@ -306,8 +358,13 @@ cudaError_t prepare_gemm_kernels() {
 }
 
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K,
-                           const EpiArgs& ep) {
+                           const EpiArgs& ep, int tile_n) {
   if (M < 1 || N < 1 || K < BK || (K % BK)) return cudaErrorInvalidValue;
-  if (lc.f16) return launch_t<f16>(lc, kind, maps, M, N, K, ep);
-  return launch_t<bf16>(lc, kind, maps, M, N, K, ep);
+  if (tile_n == 128) {
+    if (!maps.n128) return cudaErrorInvalidValue;
+    if (lc.f16) return launch_t<f16, 128>(lc, kind, maps, M, N, K, ep);
+    return launch_t<bf16, 128>(lc, kind, maps, M, N, K, ep);
+  }
+  if (lc.f16) return launch_t<f16, 256>(lc, kind, maps, M, N, K, ep);
+  return launch_t<bf16, 256>(lc, kind, maps, M, N, K, ep);
 }

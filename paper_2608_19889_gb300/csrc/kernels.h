@@ -97,16 +97,21 @@ cudaError_t prepare_gemm_kernels();
 // out[m][n] = A[m] . W[n], M x N x K with K % 64 == 0.
 struct GemmMaps {
   CUtensorMap a;     // activations [rows][K], box 64 x 128
-  CUtensorMap w;     // weights [N][K], box 64 x 256
+  CUtensorMap w;     // weights [N][K], box 64 x 256 (64 x 128 in the n128 set)
   CUtensorMap a_lo;  // second term of a split activation operand (used when split)
   bool split = false;
+  const GemmMaps* n128 = nullptr;  // the same operands with 128-row weight boxes (128-wide tiles), or null
 };
 bool make_tma_2d_16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows, bool f16);
 // Row-major [rows][cols] 16-bit matrix, box box_cols x box_rows, no swizzle
 // (dense rows in shared memory); out-of-range elements read as zero.
 bool make_tma_2d_plain(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
                        uint32_t box_rows, bool f16);
-cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep);
+// tile_n: 256 or 128 (from gemm_tile_n); the residual epilogue writes one
+// norm partial per row and tile, i.e. ceil(N / tile_n) of them.
+cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
+                           int tile_n = 256);
+int gemm_tile_n(const LaunchCtx& lc, const GemmMaps& maps, int M, int N);
 
 // ---- fp32 debug projections (k_simt.cu): plain tiled CUDA-core GEMM with
 // the same epilogues, any M.
