@@ -286,12 +286,32 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
   // ring stages then cost no L2 round trip. Falls back to L2 reads when
   // they do not fit next to the epilogue buffer (the attention staging
   // region is free during a projection phase).
+  // Residual phases also keep, per buffered item, the 16 x B residual
+  // values that its epilogue updates (prefetched, see below).
+  constexpr int PER_ITEM = (KIND == EPI_RESID ? 2 : 1) * 16 * 4;  // bytes per item and token
   const int pitch = K * 2 + 16;
   const int act_bytes = B * pitch * (LO ? 2 : 1);
-  const bool staged = act_bytes <= ATTN - 8 * B * 16 * 4;
-  float* vbuf = reinterpret_cast<float*>(act_sm + (staged ? ((act_bytes + 15) & ~15) : 0));
-  int cap = (ATTN - (staged ? ((act_bytes + 15) & ~15) : 0)) / (B * 16 * 4);
+  const bool staged = act_bytes <= ATTN - 8 * B * PER_ITEM;
+  const int act_off = staged ? ((act_bytes + 15) & ~15) : 0;
+  int cap = (ATTN - act_off) / (B * PER_ITEM);
   cap = cap > 64 ? 64 : cap;
+  float* vbuf = reinterpret_cast<float*>(act_sm + act_off);
+  float* xpre = vbuf + cap * B * 16;  // residual phases: [slot][token][16]
+  const int my_items = (n - i_first + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x);
+  // Residual phases: the residual slices of the next `cap` items go to
+  // shared memory (L2-only copies: they were written by other SMs before the
+  // phase barrier), in flight while the products run.
+  auto prefetch_x = [&](int first, int count) {
+    if (KIND != EPI_RESID) return;
+    const uint32_t dst = smem_u32(xpre);
+    for (int t = tid; t < count * B * 4; t += PCW * 32) {
+      const int slot = t / (B * 4), rem = t - slot * (B * 4), b = rem >> 2, piece = rem & 3;
+      const int item = first + slot * static_cast<int>(gridDim.x);
+      cp_async16(dst + ((slot * B + b) * 16 + piece * 4) * 4,
+                 A.x + static_cast<long long>(b) * A.D + item * 16 + piece * 4);
+    }
+    cp_async_commit();
+  };
   if (KIND == EPI_LOGITS && tid < B) best_s[tid] = 0ull;
   if (staged) {
     const int per_row = K >> 3;  // 16-byte pieces per row
@@ -307,13 +327,13 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
     cp_async_wait<0>();
   }
   consumer_sync();
-  // The norm scale of this phase's input: sum of the producer's partials.
-  if (KIND != EPI_RESID && warp < B) {
-    float rp = 0.f;
+  prefetch_x(i_first, my_items < cap ? my_items : cap);
+  // The norm scale of this phase's input: sum of the producer's partials,
+  // loads issued now and reduced before the first epilogue batch.
+  float rp = 0.f;
+  bool rinv_pending = KIND != EPI_RESID;
+  if (KIND != EPI_RESID && warp < B)
     for (int j = lane; j < A.Pmax; j += 32) rp += __ldcg(A.ss + warp * A.Pmax + j);
-    rp = warp_sum(rp);
-    if (lane == 0) rinv_s[warp] = 1.0f / sqrtf(rp * A.inv_D + A.eps);
-  }
   // Token slot r of the MMA's N dimension normally holds token r (and, with
   // the split operand, a second MMA set holds its second term). With B <= 4
   // and the split operand the two terms share one MMA instead: slot 2b holds
@@ -331,7 +351,13 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
 
   // Epilogues of the buffered items slot 0 .. nslots-1 (items i0 + slot * grid).
   auto flush = [&](int i0, int nslots) {
-    consumer_sync();  // sums of the last item visible
+    if (rinv_pending) {
+      rp = warp_sum(rp);
+      if (lane == 0 && warp < B) rinv_s[warp] = 1.0f / sqrtf(rp * A.inv_D + A.eps);
+      rinv_pending = false;
+    }
+    cp_async_wait<0>();  // this thread's residual prefetch
+    consumer_sync();     // sums of the last item, the prefetch and the norm scale visible
     unsigned long long best = 0ull;
     for (int t = tid; t < nslots * B; t += PCW * 32) {
       const int slot = t / B, b = t - slot * B;
@@ -343,7 +369,9 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
       if (KIND == EPI_QKV) {
         epi_qkv16<T16>(ep, b, n0, v, rinv_s[b]);
       } else if (KIND == EPI_RESID) {
-        A.ss[b * A.Pmax + item] = epi_resid16<T16>(ep, b, n0, v);
+        const float4* xp = reinterpret_cast<const float4*>(xpre + (slot * B + b) * 16);
+        const float4 xin[4] = {xp[0], xp[1], xp[2], xp[3]};
+        A.ss[b * A.Pmax + item] = epi_resid16x<T16>(ep, b, n0, v, xin);
       } else if (KIND == EPI_SWIGLU) {
         epi_swiglu16<T16>(ep, b, n0, v, rinv_s[b]);
       } else {
@@ -410,6 +438,8 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
       flush(i0, slot);
       i0 = i + static_cast<int>(gridDim.x);
       slot = 0;
+      const int left = (n - i0 + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x);
+      if (left > 0) prefetch_x(i0, left < cap ? left : cap);
     }
   }
   if (slot > 0) flush(i0, slot);
