@@ -160,8 +160,13 @@ int axon_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S,
  *   d_block_table   paged layout: [B, ceil(max_context/16)], else NULL.
  *   d_logits        [B, V] fp32 output, or NULL.
  *   d_next          [B] greedy next token; may alias d_tokens.
- * The step's launches are recorded once per (B, pointer set) into a CUDA
- * graph and replayed afterwards (set AXON_NO_GRAPH=1 to launch directly). */
+ * With B <= 8 (16-bit modes, head_dim 64 or 128) the whole step is one
+ * cooperative launch with one CTA per SM (the persistent decode step); if
+ * the device cannot hold that grid co-resident, or with AXON_NO_PERSIST=1
+ * set when the model was created, the step is a chain of 5L+3 kernels,
+ * recorded once per (B, pointer set) into a CUDA graph and replayed
+ * afterwards (AXON_NO_GRAPH=1: launched directly). Both paths compute the
+ * same operations; their fp32 summation orders differ. */
 int axon_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,
                      const int32_t* d_block_table, float* d_logits, int32_t* d_next, void* stream);
 
