@@ -405,6 +405,7 @@ struct Proj {
   const axon_model* m;
   LaunchCtx lc;
   bool decode = false;  // o_lo / u_lo were written by this step's producers
+  int gemv_max = 64;    // rows up to which the register-streaming GEMV runs (else the tcgen05 GEMM)
   cudaError_t rc = cudaSuccess;
   // act: activation rows (row stride act_stride elements), M rows. Returns
   // the norm state a RESID producer leaves behind.
@@ -415,7 +416,7 @@ struct Proj {
     ep.M = M;
     ep.N = N;
     NormState ns;
-    const bool gemv = M <= 64 || (!m->fp32 && maps == nullptr);
+    const bool gemv = M <= gemv_max || (!m->fp32 && maps == nullptr);
     if (gemv && kind == EPI_RESID) {
       ep.rinv_out = m->rinv;
       ep.ticket = m->ticket;
@@ -614,6 +615,10 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   g_trace_stream = st;
   Proj pj{m, lc};
   pj.decode = true;
+  // Above 32 tokens the GEMV's per-CTA re-reads of every activation row from
+  // L2 cost more than the weights; the tensor-core GEMM takes the 33..64
+  // tokens as one M tile and streams each weight tile once through TMA.
+  pj.gemv_max = 32;
   const int D = m->D, Hd = m->H * m->d;
   const double es = static_cast<double>(m->esz);
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * Hd * es,
@@ -669,7 +674,7 @@ launch_chain:
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
     pbeg(pf, "decode_qkv");
-    pj.run(EPI_QKV, w.wqkv, nullptr, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok);
+    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok);
     CK(pj.rc);
     pend(pf, wq + B * (D + m->Nqkv) * es, 2.0 * B * m->Nqkv * D);
 
@@ -694,7 +699,7 @@ launch_chain:
     r.ss_out = m->ss;
     r.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_o");
-    ns = pj.run(EPI_RESID, w.wo, nullptr, D, Hd, m->o, Hd, B, r, &w.v_o, m->t_o_tok);
+    ns = pj.run(EPI_RESID, w.wo, &w.m_o, D, Hd, m->o, Hd, B, r, &w.v_o, m->t_o_tok);
     CK(pj.rc);
     pend(pf, wo + B * (Hd * es + D * (8 + es)), 2.0 * B * D * Hd);
 
@@ -705,7 +710,7 @@ launch_chain:
     g.u_out = m->u;
     g.u_lo_out = m->u_lo;
     pbeg(pf, "decode_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, nullptr, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok);
+    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok);
     CK(pj.rc);
     pend(pf, wgu + B * (D + m->F) * es, 2.0 * B * 2 * m->F * D);
 
@@ -719,7 +724,7 @@ launch_chain:
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_down");
-    ns = pj.run(EPI_RESID, w.wd, nullptr, D, m->F, m->u, m->F, B, dn, &w.v_d, m->t_u_tok);
+    ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, B, dn, &w.v_d, m->t_u_tok);
     CK(pj.rc);
     pend(pf, wdn + B * (m->F * es + D * (8 + es)), 2.0 * B * D * m->F);
   }
@@ -731,7 +736,7 @@ launch_chain:
   h.logits = logits;
   h.logits_stride = m->V;
   pbeg(pf, "decode_lm_head");
-  pj.run(EPI_LOGITS, m->head, nullptr, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok);
+  pj.run(EPI_LOGITS, m->head, &m->m_head, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok);
   CK(pj.rc);
   pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
   pbeg(pf, "finalize");
