@@ -105,6 +105,7 @@ struct axon_model {
   CUtensorMap* pmaps = nullptr;  // [4L + 1] weight maps, box 256 x 16
   PersistGrid* pgrid = nullptr;
   int persist_ctas = 0;
+  int decode_gemv_max = 32;  // decode projections with more tokens take the tcgen05 GEMM (AXON_DECODE_GEMV_MAX)
 };
 
 namespace {
@@ -416,7 +417,11 @@ struct Proj {
     ep.M = M;
     ep.N = N;
     NormState ns;
-    const bool gemv = M <= gemv_max || (!m->fp32 && maps == nullptr);
+    // decode (gemv_max < 64): between 9 and gemv_max tokens the tcgen05 GEMM
+    // still wins where its 128-wide tiles cover every SM (gate/up, LM head)
+    const bool wide = gemv_max < 64 && M > 8 && maps != nullptr &&
+                      static_cast<long long>((N + 127) / 128) * ((M + 127) / 128) >= m->num_sms;
+    const bool gemv = (M <= gemv_max && !wide) || (!m->fp32 && maps == nullptr);
     if (gemv && kind == EPI_RESID) {
       ep.rinv_out = m->rinv;
       ep.ticket = m->ticket;
@@ -618,7 +623,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   // Above 32 tokens the GEMV's per-CTA re-reads of every activation row from
   // L2 cost more than the weights; the tensor-core GEMM takes the 33..64
   // tokens as one M tile and streams each weight tile once through TMA.
-  pj.gemv_max = 32;
+  pj.gemv_max = m->decode_gemv_max;
   const int D = m->D, Hd = m->H * m->d;
   const double es = static_cast<double>(m->esz);
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * Hd * es,
@@ -823,6 +828,10 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->use_graphs = !env_flag("AXON_NO_GRAPH");
   m->use_pdl = !env_flag("AXON_NO_PDL");
   m->use_tma_gemv = env_flag("AXON_TMA_GEMV");
+  if (const char* v = getenv("AXON_DECODE_GEMV_MAX")) {
+    const int t = atoi(v);
+    if (t >= 0 && t <= 64) m->decode_gemv_max = t;
+  }
   g_trace = env_flag("AXON_TRACE");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   auto fail = [&](int code) {
