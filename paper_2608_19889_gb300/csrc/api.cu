@@ -106,6 +106,7 @@ struct axon_model {
   PersistGrid* pgrid = nullptr;
   int persist_ctas = 0;
   int decode_gemv_max = 32;  // decode projections with more tokens take the tcgen05 GEMM (AXON_DECODE_GEMV_MAX)
+  GemmSplitK gemm_sk{};      // split-K workspace of the decode-sized tensor-core GEMMs
 };
 
 namespace {
@@ -417,11 +418,17 @@ struct Proj {
     ep.M = M;
     ep.N = N;
     NormState ns;
-    // decode (gemv_max < 64): between 9 and gemv_max tokens the tcgen05 GEMM
-    // still wins where its 128-wide tiles cover every SM (gate/up, LM head)
-    const bool wide = gemv_max < 64 && M > 8 && maps != nullptr &&
-                      static_cast<long long>((N + 127) / 128) * ((M + 127) / 128) >= m->num_sms;
-    const bool gemv = (M <= gemv_max && !wide) || (!m->fp32 && maps == nullptr);
+    // Decode (gemv_max < 64) above 8 tokens, measured choices:
+    //  * the tcgen05 GEMM where its 128-wide tiles cover every SM (gate/up,
+    //    LM head);
+    //  * the residual projections (O, down) on the split-K GEMM where the
+    //    parts stay cheap to sum: a long K (>= 8192) or at most 16 tokens;
+    //  * otherwise the GEMV up to gemv_max tokens, the plain GEMM above.
+    const bool dec = gemv_max < 64 && maps != nullptr && !m->fp32 && M > 8;
+    const bool wide = dec && static_cast<long long>((N + 127) / 128) * ((M + 127) / 128) >= m->num_sms;
+    const bool resid_split = dec && !wide && kind == EPI_RESID && (K >= 8192 || M <= 16) &&
+                             gemm_split_k(lc, M, N, K) > 1 && m->gemm_sk.ws != nullptr;
+    const bool gemv = (M <= gemv_max && !wide && !resid_split) || (!m->fp32 && maps == nullptr);
     if (gemv && kind == EPI_RESID) {
       ep.rinv_out = m->rinv;
       ep.ticket = m->ticket;
@@ -448,8 +455,11 @@ struct Proj {
                             K, ep);
       ns.parts = N / 16;
     } else {
-      const int tn = gemm_tile_n(lc, *maps, M, N);
-      rc = launch_gemm_tc(lc, kind, *maps, M, N, K, ep, tn);
+      int tn = gemm_tile_n(lc, *maps, M, N);
+      GemmSplitK sk = m->gemm_sk;
+      sk.ks = resid_split ? gemm_split_k(lc, M, N, K) : 1;
+      if (sk.ks > 1) tn = 256;
+      rc = launch_gemm_tc(lc, kind, *maps, M, N, K, ep, tn, &sk);
       ns.parts = (N + tn - 1) / tn;
     }
     return ns;
@@ -1027,6 +1037,17 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->splitk.ticket = static_cast<int*>(p);
   if (cudaMemsetAsync(m->splitk.ticket, 0, static_cast<size_t>(m->splitk.max_tiles) * 4, st) != cudaSuccess)
     return fail(AXON_ERR_CUDA);
+  if (!f32) {
+    // decode-sized tensor-core GEMMs with too few tiles split K (<= 128 rows)
+    const int nmax = std::max(std::max(m->Nqkv, 2 * F), std::max(D, V));
+    m->gemm_sk.max_tiles = (nmax + 255) / 256;
+    if ((rc = dev_alloc(m, &p, static_cast<size_t>(GEMM_MAX_UNITS) * 128 * 256 * 4))) return fail(rc);
+    m->gemm_sk.ws = static_cast<float*>(p);
+    if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->gemm_sk.max_tiles) * 4))) return fail(rc);
+    m->gemm_sk.tickets = static_cast<int*>(p);
+    if (cudaMemsetAsync(m->gemm_sk.tickets, 0, static_cast<size_t>(m->gemm_sk.max_tiles) * 4, st) != cudaSuccess)
+      return fail(AXON_ERR_CUDA);
+  }
   m->max_splits = 64;
   const int dec_b = cfg->max_batch < 64 ? cfg->max_batch : 64;
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(dec_b) * m->G * m->max_splits * 16 * (m->d + 2) * 4))) return fail(rc);

@@ -57,7 +57,8 @@ AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
 template <int KIND, typename T16, bool SPLIT, int BN_>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmAlo, int M, int N, int K, EpiArgs ep) {
+                   const __grid_constant__ CUtensorMap tmAlo, int M, int N, int K, EpiArgs ep, int ks, float* ws,
+                   int* tickets) {
   using C = GCfg<SPLIT, BN_>;
   constexpr int BN = C::BN;
   constexpr int B_BYTES = C::B_BYTES;
@@ -106,15 +107,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   grid_dep_wait();
   const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN;
   const int tiles = num_m * num_n, KB = K / BK;
+  // Work units: (tile, K split) pairs, the ks splits of a tile adjacent.
+  // ks > 1 only with one M tile (M <= BM): each unit leaves its partial tile
+  // in `ws` and the last of a tile's units to finish sums them.
+  const int units = tiles * ks;
 
   if (warp == 0) {
     if (lane == 0) {
       int it = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const int t = u / ks, sp = u - t * ks;
         int mb, nb;
         tile_coords(t, num_m, num_n, mb, nb);
-        for (int kb = 0; kb < KB; ++kb, ++it) {
+        const int kb1 = (sp + 1) * KB / ks;
+        for (int kb = sp * KB / ks; kb < kb1; ++kb, ++it) {
           const int s = it % STAGES;
           const uint32_t ph = (it / STAGES) & 1;
           if (!mbar_wait(empty_bar(s), ph ^ 1, ep.err)) {
@@ -134,13 +141,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       constexpr uint32_t idesc = idesc_f32acc(BM, BN, MmaFmt<T16>::v);
       int it = 0, lt = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++lt) {
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++lt) {
+        const int sp = u % ks;
+        const int kb0 = sp * KB / ks, kb1 = (sp + 1) * KB / ks;
         const int buf = lt & 1;
         const uint32_t aph = (lt >> 1) & 1;
         if (!mbar_wait(acce_bar(buf), aph ^ 1, ep.err)) break;
         tc_fence_after();
         const uint32_t d = tmem + buf * BN;
-        for (int kb = 0; kb < KB; ++kb, ++it) {
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % STAGES;
           const uint32_t ph = (it / STAGES) & 1;
           if (!mbar_wait(full_bar(s), ph, ep.err)) {
@@ -152,7 +161,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint64_t bd = smem_desc_sw128(sB + s * B_BYTES);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K inside the swizzle atom
-            tc_mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
+            tc_mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
           if (SPLIT) {
             const uint64_t ald = smem_desc_sw128(sAlo + s * A_BYTES);
 #pragma unroll
@@ -167,8 +176,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else {
     const int q4 = warp & 3;  // TMEM lane quarter this warp may read
     const int row = q4 * 32 + lane;
+    const int etid = threadIdx.x - 64;  // 0..127 over the 4 epilogue warps
+    __shared__ int s_last;
+    __shared__ float s_rinv[BM];
+    __shared__ float s_ssp[KIND == EPI_RESID ? BM : 1][KIND == EPI_RESID ? BN / 16 : 1];
     int lt = 0;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++lt) {
+      const int t = u / ks;
       int mb, nb;
       tile_coords(t, num_m, num_n, mb, nb);
       const int buf = lt & 1;
@@ -177,6 +191,77 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       __syncwarp();
       if (!got) break;
       tc_fence_after();
+      if (ks > 1) {
+        // 1. this unit's partial tile -> workspace (rows < M; mb == 0)
+        const uint32_t taddr = tmem + (static_cast<uint32_t>(q4 * 32) << 16) + buf * BN;
+        float* wp = ws + (static_cast<long long>(u) * BM + row) * BN;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 16) {
+          uint32_t v[16];
+          tmem_ld16(taddr + c, v);
+          tmem_wait_ld();
+          if (row < M) {
+#pragma unroll
+            for (int i = 0; i < 16; i += 4)
+              *reinterpret_cast<float4*>(wp + c + i) =
+                  make_float4(__uint_as_float(v[i]), __uint_as_float(v[i + 1]), __uint_as_float(v[i + 2]),
+                              __uint_as_float(v[i + 3]));
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(acce_bar(buf));
+        __threadfence();
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (etid == 0) s_last = (atomicAdd(tickets + t, 1) == ks - 1);
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (s_last) {
+          // 2. last unit of the tile: sum the ks partials in split order
+          // (deterministic) and run the epilogue, as (row, 16 columns) tasks
+          __threadfence();
+          if (KIND != EPI_RESID && etid < M) s_rinv[etid] = row_rinv(ep, etid);
+          asm volatile("bar.sync 1, 128;" ::: "memory");
+          constexpr int CH = BN / 16;
+          for (int task = etid; task < M * CH; task += 128) {
+            const int m = task / CH, c = (task - m * CH) * 16;
+            const int n0 = nb * BN + c;
+            if (n0 >= N) continue;
+            float f[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) f[i] = 0.f;
+            for (int sp = 0; sp < ks; ++sp) {
+              const float* pp = ws + ((static_cast<long long>(t) * ks + sp) * BM + m) * BN + c;
+#pragma unroll
+              for (int i = 0; i < 16; i += 4) {
+                const float4 a4 = __ldcg(reinterpret_cast<const float4*>(pp + i));
+                f[i] += a4.x;
+                f[i + 1] += a4.y;
+                f[i + 2] += a4.z;
+                f[i + 3] += a4.w;
+              }
+            }
+            if (KIND == EPI_QKV) {
+              epi_qkv16<T16>(ep, m, n0, f, s_rinv[m]);
+            } else if (KIND == EPI_RESID) {
+              s_ssp[m][c >> 4] = epi_resid16<T16>(ep, m, n0, f);
+            } else if (KIND == EPI_SWIGLU) {
+              epi_swiglu16<T16>(ep, m, n0, f, s_rinv[m]);
+            } else {
+              argmax_commit(ep.keys + m, epi_logits16(ep, m, n0, f, s_rinv[m]));
+            }
+          }
+          asm volatile("bar.sync 1, 128;" ::: "memory");
+          if (KIND == EPI_RESID && etid < M) {
+            // the row's norm partial for this 256-wide tile, chunks summed in order
+            // (as the unsplit tile would); chunks past N count zero
+            float ssum = 0.f;
+            for (int c = 0; c < BN / 16; ++c)
+              if (nb * BN + c * 16 < N) ssum += s_ssp[etid][c];
+            ep.ss_out[static_cast<long long>(etid) * ep.ss_out_stride + nb] = ssum;
+          }
+          if (etid == 0) tickets[t] = 0;
+        }
+        continue;
+      }
       const int m = mb * BM + row;
       const bool mval = m < M;
       float rinv = 1.f;
@@ -261,8 +346,9 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 template <int KIND, typename T16, bool SPLIT, int BN>
-cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep) {
-  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
+                        const GemmSplitK& sk) {
+  const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN) * sk.ks;
   const int grid = tiles < lc.num_sms ? tiles : lc.num_sms;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
@@ -275,7 +361,8 @@ cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N,
   cfg.attrs = attr;
   cfg.numAttrs = lc.pdl ? 1 : 0;
   const GemmMaps& g = BN == 256 ? maps : *maps.n128;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN>, g.a, g.w, SPLIT ? g.a_lo : g.a, M, N, K, ep);
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN>, g.a, g.w, SPLIT ? g.a_lo : g.a, M, N, K, ep,
+                            sk.ks, sk.ws, sk.tickets);
 }
 
 }  // namespace
@@ -327,14 +414,15 @@ cudaError_t prepare_gemm_t() {
   return e;
 }
 template <typename T16, int BN>
-cudaError_t launch_t(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep) {
+cudaError_t launch_t(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
+                     const GemmSplitK& sk) {
   switch (kind) {
     case EPI_QKV:
-      return maps.split ? launch_kind<EPI_QKV, T16, true, BN>(lc, maps, M, N, K, ep)
-                        : launch_kind<EPI_QKV, T16, false, BN>(lc, maps, M, N, K, ep);
-    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN>(lc, maps, M, N, K, ep);
-    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN>(lc, maps, M, N, K, ep);
-    default: return launch_kind<EPI_LOGITS, T16, false, BN>(lc, maps, M, N, K, ep);
+      return maps.split ? launch_kind<EPI_QKV, T16, true, BN>(lc, maps, M, N, K, ep, sk)
+                        : launch_kind<EPI_QKV, T16, false, BN>(lc, maps, M, N, K, ep, sk);
+    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN>(lc, maps, M, N, K, ep, sk);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN>(lc, maps, M, N, K, ep, sk);
+    default: return launch_kind<EPI_LOGITS, T16, false, BN>(lc, maps, M, N, K, ep, sk);
   }
 }
 }  // namespace
@@ -358,13 +446,34 @@ cudaError_t prepare_gemm_kernels() {
 }
 
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K,
-                           const EpiArgs& ep, int tile_n) {
+                           const EpiArgs& ep, int tile_n, const GemmSplitK* split) {
   if (M < 1 || N < 1 || K < BK || (K % BK)) return cudaErrorInvalidValue;
+  GemmSplitK sk;
+  if (split && split->ks > 1) {
+    // one M tile, 256-wide tiles, at most GEMM_MAX_UNITS units, at least one K block per unit
+    const int tiles = (N + 255) / 256;
+    if (M > BM || tile_n != 256 || !split->ws || !split->tickets || tiles * split->ks > GEMM_MAX_UNITS ||
+        split->ks > K / BK || tiles > split->max_tiles)
+      return cudaErrorInvalidValue;
+    sk = *split;
+  }
   if (tile_n == 128) {
     if (!maps.n128) return cudaErrorInvalidValue;
-    if (lc.f16) return launch_t<f16, 128>(lc, kind, maps, M, N, K, ep);
-    return launch_t<bf16, 128>(lc, kind, maps, M, N, K, ep);
+    if (lc.f16) return launch_t<f16, 128>(lc, kind, maps, M, N, K, ep, sk);
+    return launch_t<bf16, 128>(lc, kind, maps, M, N, K, ep, sk);
   }
-  if (lc.f16) return launch_t<f16, 256>(lc, kind, maps, M, N, K, ep);
-  return launch_t<bf16, 256>(lc, kind, maps, M, N, K, ep);
+  if (lc.f16) return launch_t<f16, 256>(lc, kind, maps, M, N, K, ep, sk);
+  return launch_t<bf16, 256>(lc, kind, maps, M, N, K, ep, sk);
+}
+
+int gemm_split_k(const LaunchCtx& lc, int M, int N, int K) {
+  if (M > BM) return 1;
+  const int tiles = (N + 255) / 256;
+  if (2 * tiles >= lc.num_sms) return 1;
+  int ks = lc.num_sms / tiles;
+  const int kmax = K / BK / 4;  // keep >= 4 K blocks per unit
+  if (ks > kmax) ks = kmax;
+  if (ks > 16) ks = 16;
+  if (tiles * ks > GEMM_MAX_UNITS) ks = GEMM_MAX_UNITS / tiles;
+  return ks < 2 ? 1 : ks;
 }

@@ -107,11 +107,26 @@ bool make_tma_2d_16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
 // (dense rows in shared memory); out-of-range elements read as zero.
 bool make_tma_2d_plain(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
                        uint32_t box_rows, bool f16);
+// Split-K mode of the GEMM for M <= 128 rows (decode): the K blocks are cut
+// into ks parts; each (256-wide tile, part) unit leaves its fp32 partial
+// tile in ws ([unit][128][256], rows < M written) and the last unit of a
+// tile to finish (ticket per tile, zero between launches, reset by that
+// unit; nobody waits) sums the parts in order and runs the epilogue.
+constexpr int GEMM_MAX_UNITS = 320;
+struct GemmSplitK {
+  int ks = 1;
+  float* ws = nullptr;       // GEMM_MAX_UNITS * 128 * 256 floats
+  int* tickets = nullptr;    // [max_tiles]
+  int max_tiles = 0;
+};
 // tile_n: 256 or 128 (from gemm_tile_n); the residual epilogue writes one
 // norm partial per row and tile, i.e. ceil(N / tile_n) of them.
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
-                           int tile_n = 256);
+                           int tile_n = 256, const GemmSplitK* split = nullptr);
 int gemm_tile_n(const LaunchCtx& lc, const GemmMaps& maps, int M, int N);
+// K split (1 = none) for a decode-sized M x N x K product whose 256-wide
+// tiles cannot fill half the GPU.
+int gemm_split_k(const LaunchCtx& lc, int M, int N, int K);
 
 // ---- fp32 debug projections (k_simt.cu): plain tiled CUDA-core GEMM with
 // the same epilogues, any M.
