@@ -571,7 +571,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 }
 
 bool persist_eligible(const axon_model* m, int B) {
-  return m->persist_ctas > 0 && !m->fp32 && B >= 1 && B <= PERSIST_MAX_B;
+  return m->persist_ctas > 0 && !m->fp32 && persist_fits(m->d, m->f16, B, m->D);
 }
 
 PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt,

@@ -727,6 +727,17 @@ int persist_ctas_per_sm(int head_dim, bool use_f16) {
   return n;
 }
 
+bool persist_fits(int head_dim, bool use_f16, int B, int D) {
+  if (B < 1 || B > PERSIST_MAX_B) return false;
+  // The normed operand of QKV, gate/up and the LM head (K = D; with its
+  // second term in fp16 mode, except when the two terms share one MMA) must
+  // stage in shared memory next to the epilogue buffer; streaming it from
+  // L2 stage by stage is slower than the launch chain.
+  const int attn = head_dim == 64 ? PLayout<64>::ATTN : PLayout<128>::ATTN;
+  const int rows = use_f16 ? 2 * B : B;
+  return rows * (D * 2 + 16) <= attn - 8 * B * 16 * 4;
+}
+
 cudaError_t launch_persist_decode(const PersistArgs& a, int head_dim, bool use_f16, int nctas, cudaStream_t st) {
   if (a.B < 1 || a.B > PERSIST_MAX_B || (a.D & 63) || (a.F & 63) || ((a.H * a.d) & 63)) return cudaErrorInvalidValue;
   if (head_dim == 64) return use_f16 ? launch_t<64, f16>(a, nctas, st) : launch_t<64, bf16>(a, nctas, st);

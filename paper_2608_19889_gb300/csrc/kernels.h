@@ -191,4 +191,7 @@ struct PersistArgs {
 // Resident CTAs per SM of the kernel for this head_dim / type (0: not
 // available); also sets its shared-memory limit. Call before any launch.
 int persist_ctas_per_sm(int head_dim, bool use_f16);
+// Whether B sequences of width D suit the kernel (their normed activations
+// stage in shared memory); else the decode step takes the launch chain.
+bool persist_fits(int head_dim, bool use_f16, int B, int D);
 cudaError_t launch_persist_decode(const PersistArgs& a, int head_dim, bool use_f16, int nctas, cudaStream_t st);
