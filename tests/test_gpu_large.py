@@ -6,10 +6,10 @@ same work on the host).
 These run in AXON_FP16 (the bf16 checkpoint converted to fp16 operands):
 at these widths the random-init logits have a standard deviation of 1.3-1.4,
 and rounding GEMM operands and the KV cache to bf16 alone moves the largest
-of the 128k-152k logits by ~0.06 (an exact float64 emulation of the bf16
-rounding points gives 0.058 for the two-layer 8B-width case below), above
-the 5e-2 bound. fp16 operands cut that rounding 8x. The bf16 mode is checked
-on the same case against that measured floor."""
+of the 128k-152k logits past the 5e-2 bound (about 0.06-0.07 on the
+two-layer 8B-width case below). fp16 operands cut that rounding 8x. The
+bf16 mode is run on the same case under a looser regression bound; parity
+at these widths is claimed for fp16 mode only."""
 import numpy as np
 import pytest
 
@@ -43,7 +43,7 @@ class LazyF32(dict):
         return super().__getitem__(k).float().numpy()
 
 
-BF16_FLOOR_8B_WIDTH = 8e-2  # bf16 operand rounding floor at 8B width (0.058 emulated) with margin
+BF16_FLOOR_8B_WIDTH = 8e-2  # regression bound for bf16 mode at 8B width (no parity claim; measured 0.057-0.073)
 
 
 @pytest.mark.parametrize("prec", ["fp16", "bf16"])
