@@ -1,0 +1,81 @@
+"""CPU checks of bench.py's accounting and of its reference-arm JSON line:
+the algorithmic byte and FLOP counts on shapes small enough to count by hand,
+the DRAM-traffic record lookup (valid only for the CUDA sources it was taken
+on), and `--impl reference` on the 135M workload."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+SHAPE = dict(L=2, D=64, H=4, G=2, d=16, F=96, V=100, bias=True)
+
+
+def test_model_bytes_counts_every_linear_weight():
+    lin, head = bench.model_bytes(SHAPE)
+    per_layer = (4 + 2 * 2) * 16 * 64 + 64 * 4 * 16 + 2 * 96 * 64 + 64 * 96
+    assert lin == 2 * per_layer
+    assert head == 100 * 64
+
+
+def test_decode_bytes_per_step_by_hand():
+    # B = 2 sequences whose new tokens sit at positions 5 and 9
+    lin, head = bench.model_bytes(SHAPE)
+    kv_tok = 2 * 2 * 2 * 16 * 2          # L * (K, V) * G * d * bf16
+    small = (2 * 2 + 1) * 64 * 4 + 2 * (4 + 2 * 2) * 16 * 4  # norm gains + qkv biases, fp32
+    want = 2 * (lin + head) + small + (6 + 10) * kv_tok + 2 * kv_tok + 2 * 100 * 4
+    assert bench.decode_bytes_per_step(SHAPE, 2, [5, 9]) == want
+
+
+def test_prefill_flops_by_hand():
+    lin, head = bench.model_bytes(SHAPE)
+    B, S = 3, 7
+    attn = 2 * B * 4 * 4 * 16 * S * (S + 1) / 2
+    assert bench.prefill_flops(SHAPE, B, S) == 2 * B * S * lin + attn + 2 * B * head
+
+
+def test_recorded_traffic_is_tied_to_the_sources(tmp_path, monkeypatch):
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    sha = bench.kernel_source_sha()
+    (prof / "dram_w_bf16.md").write_text(
+        "text\n```\nsource_sha256: %s\ntraffic decode_persistent: 12345\ntraffic prefill_qkv: 77\n```\n" % sha)
+    (prof / "dram_old_bf16.md").write_text("```\nsource_sha256: 0000\ntraffic decode_persistent: 1\n```\n")
+    real_dirname = os.path.dirname
+
+    def fake_dirname(p):
+        if p == os.path.abspath(bench.__file__):
+            return str(tmp_path)
+        return real_dirname(p)
+
+    monkeypatch.setattr(bench.os.path, "dirname", fake_dirname)
+    # the sha is computed over the real sources: point it back at the repository
+    monkeypatch.setattr(bench, "kernel_source_sha", lambda: sha)
+    assert bench.recorded_traffic("w", "bf16", "decode_persistent") == 12345.0
+    assert bench.recorded_traffic("w", "bf16", "prefill_qkv") == 77.0
+    assert bench.recorded_traffic("w", "bf16", "decode_o") is None
+    assert bench.recorded_traffic("old", "bf16", "decode_persistent") is None  # other sources
+    assert bench.recorded_traffic("missing", "bf16", "decode_persistent") is None
+
+
+def test_reference_arm_json_line():
+    out = subprocess.run(
+        [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1", "--warmup", "0",
+         "--workload", "135m_b1_s16_n16"],
+        capture_output=True, text=True, timeout=600, cwd=ROOT)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference"
+    assert line["metric"] == bench.METRIC
+    assert line["unit"] == "tokens/s" and line["value"] > 0
+    assert line["higher_is_better"] is True
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
+    assert line["config"]["workload"] == "135m_b1_s16_n16"
