@@ -218,6 +218,21 @@ def slot_of(block_table, b, p, block_size):
     return int(block_table[b][p // block_size]), int(p % block_size)
 
 
+class SeqSlot:
+    """One sequence's view of a batched cache: sequence slot `b` of `cache`
+    as if it were slot 0 (Cache.update / Cache.read of that sequence)."""
+
+    def __init__(self, cache, b):
+        self.cache = cache
+        self.b = int(b)
+
+    def write(self, l, b, pos, k, v):
+        self.cache.write(l, self.b, pos, k, v)
+
+    def read(self, l, b, T):
+        return self.cache.read(l, self.b, T)
+
+
 class PagedKV:
     """Paged cache: per layer a pool [num_blocks, block_size, G, d] and an
     integer block table [B, max_blocks] naming the pool block of each
@@ -325,6 +340,20 @@ class Oracle:
         context_lens[b]. Returns logits [B, V]."""
         tokens = np.asarray(tokens, dtype=np.int64).reshape(-1, 1)
         return self.forward(tokens, cache, context_lens)[:, 0, :]
+
+    def forward_varlen(self, chunks, cache, past_lens, last_only=True):
+        """Several sequences each append one chunk of new tokens of its own
+        length after past_lens[b] cached tokens -- a prompt, a further piece
+        of one, or a single decode token (Positions.position_ids with
+        past_length; Cache.update): sequence b's chunk runs through forward()
+        on that sequence's cache slot. Returns, per sequence, the logits of
+        the chunk's last token [V] (last_only) or of all its tokens [S_b, V]."""
+        out = []
+        for b, ch in enumerate(chunks):
+            ids = np.asarray(ch, dtype=np.int64).reshape(1, -1)
+            lg = self.forward(ids, SeqSlot(cache, b), [int(past_lens[b])], last_hidden_only=last_only)[0]
+            out.append(lg[-1] if last_only else lg)
+        return out
 
     def generate(self, prompt, n_new, cache, forced=None):
         """Greedy generation: prefill, then n_new - 1 decode steps feeding

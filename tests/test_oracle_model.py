@@ -184,3 +184,37 @@ def test_generate_teacher_forced_matches_free_running_when_forced_on_own_tokens(
     toks, logits = o.generate(ids, 4, o.new_contiguous_cache(1, 8))
     toks2, logits2 = o.generate(ids, 4, o.new_contiguous_cache(1, 8), forced=toks)
     assert np.array_equal(toks, toks2) and np.allclose(logits, logits2, rtol=1e-14, atol=1e-14)
+
+
+def test_varlen_equals_batched_forward_for_equal_lengths():
+    """forward_varlen over equal-length chunks is the batched forward."""
+    cfg, W = tiny_model()
+    o = od.Oracle(cfg, W)
+    ids = np.random.default_rng(3).integers(0, cfg.V, size=(3, 5))
+    c1 = o.new_contiguous_cache(3, 16)
+    ref = o.forward(ids, c1, [0, 0, 0])
+    c2 = o.new_contiguous_cache(3, 16)
+    got = o.forward_varlen([ids[b] for b in range(3)], c2, [0, 0, 0], last_only=False)
+    for b in range(3):
+        assert np.allclose(got[b], ref[b], rtol=0, atol=1e-12)
+
+
+def test_varlen_chunks_equal_one_prompt_and_mixed_decode():
+    """Prompts cut into chunks of different lengths (one of them a single
+    decode-like token) give the logits of the whole prompts, paged cache with
+    shuffled blocks included."""
+    cfg, W = tiny_model()
+    o = od.Oracle(cfg, W)
+    rng = np.random.default_rng(4)
+    lens = [7, 4, 9]
+    prompts = [rng.integers(0, cfg.V, size=n) for n in lens]
+    full = o.new_contiguous_cache(3, 16)
+    ref = [o.forward(p[None], od.SeqSlot(full, b), [0])[0] for b, p in enumerate(prompts)]
+    cut = [3, 3, 8]  # second sequence: last chunk is one token, like a decode step
+    bt = np.random.default_rng(5).permutation(3 * 4).reshape(3, 4)
+    for cache in (o.new_contiguous_cache(3, 16), o.new_paged_cache(12, 4, bt)):
+        first = o.forward_varlen([p[:c] for p, c in zip(prompts, cut)], cache, [0, 0, 0], last_only=False)
+        second = o.forward_varlen([p[c:] for p, c in zip(prompts, cut)], cache, cut, last_only=False)
+        for b in range(3):
+            assert np.allclose(first[b], ref[b][:cut[b]], rtol=0, atol=1e-12)
+            assert np.allclose(second[b], ref[b][cut[b]:], rtol=0, atol=1e-12)
