@@ -150,6 +150,45 @@ int axon_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S,
                  const int32_t* d_block_table, int32_t logits_mode, float* d_logits,
                  int32_t* d_next, void* stream);
 
+/* Variable-length batch: B sequences each append one chunk of new tokens
+ * after the tokens they already hold in the cache -- a whole prompt, the
+ * next piece of a long prompt (chunked prefill), or a single decode token
+ * -- packed row after row into one forward pass (Positions.position_ids
+ * with a per-sequence past_length and Cache.update, Sec. Built-In
+ * Libraries; the continuous batching of vLLM's PagedAttention manager,
+ * Sec. Related Work). Every chunk attends causally to its own sequence's
+ * cached tokens and to the earlier tokens of the chunk.
+ *   d_ids           [T] token ids, sequence b's chunk at rows
+ *                   cu_seqlens[b] .. cu_seqlens[b+1]-1.
+ *   B               1 .. max_batch; sequence b uses contiguous slot b, or
+ *                   the blocks named by row b of d_block_table.
+ *   T               total new tokens, B .. max_prefill_tokens.
+ *   d_cu_seqlens    [B+1] row offsets: cu[0] = 0, cu[B] = T, every chunk
+ *                   1 .. max_chunk tokens long.
+ *   d_context_lens  [B] IN/OUT: tokens already cached for sequence b (0 for
+ *                   a new prompt); chunk token i takes position
+ *                   context_lens[b] + i, which must stay below
+ *                   max_context. The call adds each chunk's length (in
+ *                   stream order, after all reads), so the next call --
+ *                   another chunk or axon_decode_step -- can follow
+ *                   without host work.
+ *   max_chunk       host bound on the longest chunk, 1 .. min(T,
+ *                   max_context); it sizes the attention grid.
+ *   d_block_table   paged layout: [B, ceil(max_context/16)], else NULL.
+ *   logits_mode     AXON_LOGITS_LAST: d_logits is [B, V], the last token of
+ *                   each chunk; AXON_LOGITS_ALL: d_logits is [T, V].
+ *   d_logits        fp32 output, or NULL.
+ *   d_next          [B] greedy next token after each chunk's last token
+ *                   (lowest index on ties), or NULL.
+ * Offsets and lengths are read on the device: inconsistent ones (cu not
+ * starting at 0, not ending at T, a chunk outside 1 .. max_chunk) or
+ * positions past max_context set the device error word
+ * (AXON_ERR_DEVICE_CHECK from axon_check_device) and the rows they affect
+ * are skipped. Cache slots at the chunk's positions are overwritten. */
+int axon_prefill_varlen(axon_model* m, const int32_t* d_ids, int32_t B, int32_t T, const int32_t* d_cu_seqlens,
+                        int32_t* d_context_lens, int32_t max_chunk, const int32_t* d_block_table,
+                        int32_t logits_mode, float* d_logits, int32_t* d_next, void* stream);
+
 /* One KV-cached greedy decode step for B sequences (generate loop, Sec.
  * Results; Cache.append in the appendix causal_lm listing).
  *   d_tokens        [B] the newest token of each sequence.

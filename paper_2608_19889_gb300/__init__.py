@@ -29,7 +29,7 @@ AXON_BF16, AXON_FP32_DEBUG, AXON_FP16 = 0, 1, 2
 AXON_DTYPE_BF16, AXON_DTYPE_F32 = 0, 1
 AXON_LOGITS_LAST, AXON_LOGITS_ALL = 0, 1
 
-EXPORTED = ["axon_model_create", "axon_prefill", "axon_decode_step", "axon_reset", "axon_check_device",
+EXPORTED = ["axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset", "axon_check_device",
             "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill", "axon_decode_step_noalloc",
             "axon_free", "axon_status_string"]
 
@@ -78,6 +78,7 @@ def lib() -> ctypes.CDLL:
         L.axon_model_create.argtypes = [ctypes.POINTER(axon_config), ctypes.POINTER(axon_tensor), i32, vp,
                                         ctypes.POINTER(vp)]
         L.axon_prefill.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp, vp]
+        L.axon_prefill_varlen.argtypes = [vp, vp, i32, i32, vp, vp, i32, vp, i32, vp, vp, vp]
         L.axon_decode_step.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
         L.axon_decode_step_noalloc.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
         L.axon_reset.argtypes = [vp]
@@ -90,7 +91,7 @@ def lib() -> ctypes.CDLL:
         L.axon_free.restype = None
         L.axon_status_string.argtypes = [ctypes.c_int]
         L.axon_status_string.restype = ctypes.c_char_p
-        for n in ("axon_model_create", "axon_prefill", "axon_decode_step", "axon_reset", "axon_check_device",
+        for n in ("axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset", "axon_check_device",
                   "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill",
                   "axon_decode_step_noalloc"):
             getattr(L, n).restype = ctypes.c_int
@@ -155,6 +156,19 @@ def axon_prefill(m, ids, block_table=None, logits_mode=AXON_LOGITS_LAST, logits=
     B, S = ids.shape
     _check("axon_prefill", lib().axon_prefill(m, _ptr(ids), B, S, _ptr(block_table), logits_mode, _ptr(logits),
                                               _ptr(next_tokens), _stream(stream)))
+
+
+def axon_prefill_varlen(m, ids, cu_seqlens, context_lens, max_chunk, block_table=None, logits_mode=AXON_LOGITS_LAST,
+                        logits=None, next_tokens=None, stream=None):
+    """ids: int32 [T] packed chunks; cu_seqlens: int32 [B+1] row offsets;
+    context_lens: int32 [B] tokens cached before each chunk (advanced by the
+    chunk lengths); max_chunk: host bound on the longest chunk. All device
+    tensors; outputs written into the given tensors."""
+    T = ids.shape[0]
+    B = cu_seqlens.shape[0] - 1
+    _check("axon_prefill_varlen", lib().axon_prefill_varlen(
+        m, _ptr(ids), B, T, _ptr(cu_seqlens), _ptr(context_lens), int(max_chunk), _ptr(block_table), logits_mode,
+        _ptr(logits), _ptr(next_tokens), _stream(stream)))
 
 
 def axon_decode_step(m, tokens, context_lens, block_table=None, logits=None, next_tokens=None, stream=None):

@@ -84,6 +84,12 @@ struct axon_model {
   void* u = nullptr;
   unsigned long long* keys = nullptr;
   float* rinv = nullptr;   // [Mcap] per-row inverse RMS from decode producers
+  // variable-length batches: (sequence, position) per row, and each chunk's
+  // last row of a (and a_lo) with its inverse RMS, gathered for the LM head
+  int2* rowmap = nullptr;     // [Mcap]
+  void* a_last = nullptr;     // [max_batch][D]
+  void* a_lo_last = nullptr;  // fp16 mode
+  float* rinv_last = nullptr;  // [max_batch]
   SplitKWork splitk{};     // decode projections' cross-CTA split-K workspace
   GemvTmaWork tmawork{};   // TMA stream-K decode projections' workspace
   CUtensorMap t_a_tok[4]{}, t_o_tok[4]{}, t_u_tok[4]{};  // activation maps, box 64 x {8,16,32,64} rows
@@ -466,10 +472,22 @@ struct Proj {
   }
 };
 
+// A variable-length batch (axon_prefill_varlen): sequence b's chunk is rows
+// cu[b] .. cu[b+1]-1 of the T packed rows, after ctx[b] cached tokens; ctx is
+// advanced by the chunk lengths at the end.
+struct VarlenBatch {
+  const int* cu;
+  int* ctx;
+  int T;
+  int max_chunk;
+};
+
 int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32_t* bt, int logits_mode, float* logits,
-                    int32_t* next, cudaStream_t st, Prof* pf = nullptr) {
-  const int M = B * S;
+                    int32_t* next, cudaStream_t st, Prof* pf = nullptr, const VarlenBatch* vl = nullptr) {
+  const int M = vl ? vl->T : B * S;
   LaunchCtx lc{st, m->use_pdl && !pf, m->num_sms, m->f16};
+  const int2* rowmap = vl ? m->rowmap : nullptr;
+  if (vl) CK(launch_varlen_rows(lc, vl->cu, vl->ctx, B, M, vl->max_chunk, m->cfg.max_context, m->rowmap, m->err));
   g_trace_stream = st;
   const double es = static_cast<double>(m->esz);
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * m->H * m->d * es,
@@ -487,6 +505,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     const LayerW& w = m->layers[l];
     EpiArgs e = base_epi(m);
     e.S = S;
+    e.rowmap = rowmap;
     set_norm(m, ns, e);
     e.bias = w.bqkv;
     e.q_out = m->q;
@@ -498,6 +517,13 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 
     AttnArgs at = base_attn(m, l, bt);
     at.S = S;
+    if (vl) {
+      at.S = vl->max_chunk;
+      at.cu = vl->cu;
+      at.past = vl->ctx;
+      at.rows = M;
+      at.rowmap = rowmap;
+    }
     pbeg(pf, "prefill_attention");
     CK(launch_attn_prefill(lc, m->fp32, at, B));
     pend(pf, static_cast<double>(M) * (m->H + 2 * m->G) * m->d * es + static_cast<double>(M) * Hd * es,
@@ -505,6 +531,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 
     EpiArgs r = base_epi(m);
     r.S = S;
+    r.rowmap = rowmap;
     r.x = m->x;
     r.a_out = m->a;
     r.gain = w.g2;
@@ -518,6 +545,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 
     EpiArgs g = base_epi(m);
     g.S = S;
+    g.rowmap = rowmap;
     set_norm(m, ns, g);
     g.u_out = m->u;
     pbeg(pf, "prefill_gateup");
@@ -527,6 +555,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 
     EpiArgs dn = base_epi(m);
     dn.S = S;
+    dn.rowmap = rowmap;
     dn.x = m->x;
     dn.a_out = m->a;
     dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
@@ -540,10 +569,38 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
   }
   EpiArgs h = base_epi(m);
   h.S = S;
+  h.rowmap = rowmap;
   h.keys = m->keys;
   h.logits = logits;
   h.logits_stride = m->V;
-  if (logits_mode == AXON_LOGITS_ALL) {
+  if (vl && logits_mode == AXON_LOGITS_ALL) {
+    set_norm(m, ns, h);
+    pj.run(EPI_LOGITS, m->head, &m->m_head, m->V, D, m->a, D, M, h);
+    CK(pj.rc);
+    CK(launch_finalize_varlen(lc, m->keys, M, vl->cu, 1, B, next, vl->ctx));
+  } else if (vl) {
+    // Last row of every chunk, gathered into B dense rows, then a GEMV of at
+    // most 64 rows at a time over the LM head.
+    const float* rv = ns.rinv ? m->rinv : nullptr;
+    CK(launch_gather_last(lc, vl->cu, B, M, m->a, m->a_lo, D * static_cast<int>(m->esz), rv, m->ss, m->Pmax,
+                          ns.parts, 1.0f / static_cast<float>(D), m->cfg.rms_norm_eps, m->a_last, m->a_lo_last,
+                          m->rinv_last));
+    for (int b0 = 0; b0 < B; b0 += 64) {
+      const int nb = std::min(64, B - b0);
+      EpiArgs hg = h;
+      hg.rowmap = nullptr;
+      hg.rinv = m->rinv_last + b0;
+      hg.rinv_stride = 1;
+      hg.M = nb;
+      hg.N = m->V;
+      hg.keys = m->keys + b0;
+      hg.logits = logits ? logits + static_cast<size_t>(b0) * m->V : nullptr;
+      const size_t off = static_cast<size_t>(b0) * D * m->esz;
+      CK(launch_gemv(lc, EPI_LOGITS, m->fp32, m->head, m->V, D, static_cast<char*>(m->a_last) + off, D, nb, hg,
+                     m->splitk, m->a_lo_last ? static_cast<char*>(m->a_lo_last) + off : nullptr));
+    }
+    CK(launch_finalize_varlen(lc, m->keys, B, vl->cu, 0, B, next, vl->ctx));
+  } else if (logits_mode == AXON_LOGITS_ALL) {
     set_norm(m, ns, h);
     pbeg(pf, "prefill_lm_head");
     pj.run(EPI_LOGITS, m->head, &m->m_head, m->V, D, m->a, D, M, h);
@@ -1013,6 +1070,12 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->keys = static_cast<unsigned long long*>(p);
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * 4))) return fail(rc);
   m->rinv = static_cast<float*>(p);
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * sizeof(int2)))) return fail(rc);
+  m->rowmap = static_cast<int2*>(p);
+  if ((rc = dev_alloc(m, &m->a_last, static_cast<size_t>(cfg->max_batch) * D * es))) return fail(rc);
+  if (m->f16 && (rc = dev_alloc(m, &m->a_lo_last, static_cast<size_t>(cfg->max_batch) * D * es))) return fail(rc);
+  if ((rc = dev_alloc(m, &p, static_cast<size_t>(cfg->max_batch) * 4))) return fail(rc);
+  m->rinv_last = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
   m->ticket = static_cast<int*>(p);
   {
@@ -1183,6 +1246,20 @@ int axon_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t S, cons
   if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
   return enqueue_prefill(m, d_ids, B, S, d_block_table, logits_mode, d_logits, d_next,
                          static_cast<cudaStream_t>(stream));
+}
+
+int axon_prefill_varlen(axon_model* m, const int32_t* d_ids, int32_t B, int32_t T, const int32_t* d_cu_seqlens,
+                        int32_t* d_context_lens, int32_t max_chunk, const int32_t* d_block_table, int32_t logits_mode,
+                        float* d_logits, int32_t* d_next, void* stream) {
+  if (!m || !d_ids || !d_cu_seqlens || !d_context_lens) return AXON_ERR_INVALID_ARG;
+  if (B < 1 || B > m->cfg.max_batch || T < B || T > m->cfg.max_prefill_tokens) return AXON_ERR_INVALID_ARG;
+  if (max_chunk < 1 || max_chunk > m->cfg.max_context || max_chunk > T) return AXON_ERR_INVALID_ARG;
+  if (logits_mode != AXON_LOGITS_LAST && logits_mode != AXON_LOGITS_ALL) return AXON_ERR_INVALID_ARG;
+  const bool paged = m->cfg.kv_layout == AXON_KV_PAGED;
+  if (paged != (d_block_table != nullptr)) return AXON_ERR_INVALID_ARG;
+  const VarlenBatch vl{d_cu_seqlens, d_context_lens, T, max_chunk};
+  return enqueue_prefill(m, d_ids, B, max_chunk, d_block_table, logits_mode, d_logits, d_next,
+                         static_cast<cudaStream_t>(stream), nullptr, &vl);
 }
 
 int axon_decode_step(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,

@@ -21,6 +21,7 @@ enum : int {
   DEVERR_BLOCK = 2,    // block-table entry outside [0, num_blocks)
   DEVERR_POS = 4,      // position outside [0, max_context)
   DEVERR_TIMEOUT = 8,  // a bounded mbarrier wait expired
+  DEVERR_SEQ = 16,     // variable-length batch: row offsets or cached lengths inconsistent
 };
 
 AXON_DEV void set_err(int* err, int bit) {

@@ -24,10 +24,12 @@ enum EpiKind : int { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LOGITS = 3 
 struct EpiArgs {
   int M;  // rows (tokens)
   int N;  // packed output columns
-  // row m -> (sequence b, position): decode (ctx != null): b = m,
+  // row m -> (sequence b, position): variable-length batch (rowmap !=
+  // null): (b, pos) = rowmap[m]; decode (ctx != null): b = m,
   // pos = ctx[m]; prefill: b = m / S, pos = m % S.
   int S;
   const int* ctx;
+  const int2* rowmap;
   int max_pos;
   // A-operand normalisation (QKV, SWIGLU, LOGITS): partial sums of squares
   // of the producer, ss_parts per row, rows ss_stride floats apart.
@@ -80,6 +82,11 @@ AXON_DEV float row_rinv(const EpiArgs& e, int m) {
 }
 
 AXON_DEV int row_seq_pos(const EpiArgs& e, int m, int& b) {
+  if (e.rowmap) {
+    const int2 r = e.rowmap[m];
+    b = r.x;
+    return r.y;
+  }
   if (e.ctx) {
     b = m;
     return e.ctx[m];

@@ -41,7 +41,7 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   constexpr int TILE = 16 * HD * 2;
   constexpr int STAGE = 4 * 2 * TILE;  // 4 blocks x (K, V)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, r = lane >> 2, q = lane & 3;
-  const int HPG = p.H / p.G, S = p.S;
+  const int HPG = p.H / p.G;
   const int PC = 4 * PW;
   // grid (kv head, position block, sequence), position blocks counted down
   // from the end: under the causal mask the last blocks carry the most keys,
@@ -49,32 +49,46 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   const int b = blockIdx.z, g = blockIdx.x, p0 = (gridDim.y - 1 - blockIdx.y) * PC;
   grid_dep_launch();
   grid_dep_wait();
+  // The sequence's chunk: rows row0 .. row0+S-1 of q / o, at positions
+  // past .. past+S-1 (a prompt from an empty cache: past = 0, row0 = b*S).
+  int S = p.S, row0 = b * p.S, past = 0;
+  if (p.cu) {
+    row0 = p.cu[b];
+    const int row1 = p.cu[b + 1];
+    past = p.past[b];
+    S = row1 - row0;
+    // inconsistent offsets (reported by the row-map kernel): no work
+    if (row0 < 0 || row1 > p.rows || S < 0 || S > p.S || past < 0 || past + S > p.blocks_per_seq * 16) S = 0;
+  }
+  if (p0 >= S) return;
 
+  // local index i of the chunk -> absolute position past + i (or -1: padding)
   auto row_info = [&](int i, int& pos, int& h) {
     const int pl = i / HPG;
     h = i - pl * HPG;
     pos = p0 + warp * PW + pl;
     if (i >= PW * HPG || pos >= S) pos = -1;
   };
-  int pos0, h0, pos1, h1;
-  row_info(r, pos0, h0);
-  row_info(r + 8, pos1, h1);
+  int i0, h0, i1, h1;
+  row_info(r, i0, h0);
+  row_info(r + 8, i1, h1);
+  const int pos0 = i0 >= 0 ? past + i0 : -1, pos1 = i1 >= 0 ? past + i1 : -1;
   const uint16_t* qbase = static_cast<const uint16_t*>(p.q);
   const long long Hd = static_cast<long long>(p.H) * HD;
   const uint16_t* qr0 =
-      pos0 >= 0 ? qbase + (static_cast<long long>(b) * S + pos0) * Hd + (g * HPG + h0) * HD : nullptr;
+      i0 >= 0 ? qbase + (static_cast<long long>(row0) + i0) * Hd + (g * HPG + h0) * HD : nullptr;
   const uint16_t* qr1 =
-      pos1 >= 0 ? qbase + (static_cast<long long>(b) * S + pos1) * Hd + (g * HPG + h1) * HD : nullptr;
+      i1 >= 0 ? qbase + (static_cast<long long>(row0) + i1) * Hd + (g * HPG + h1) * HD : nullptr;
   uint32_t qa[HD / 16][4];
   load_q<HD>(qa, qr0, qr1, q);
 
   WarpState<HD> st;
   st.init();
-  const int pend = min(p0 + PC, S);
+  const int pend = past + min(p0 + PC, S);  // keys 0 .. pend-1 are visible to some row
   const int nblk = (pend + 15) >> 4;
   const int nst = (nblk + 3) >> 2;
   const int wfirst = p0 + warp * PW;
-  const int wmax = min(wfirst + PW - 1, S - 1);
+  const int wmax = past + min(wfirst + PW - 1, S - 1);
   const uint32_t base = smem_u32(sm);
   const uint16_t* kp = static_cast<const uint16_t*>(p.k);
   const uint16_t* vp = static_cast<const uint16_t*>(p.v);
@@ -120,12 +134,12 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   const float inv0 = st.l0 > 0.f ? 1.f / st.l0 : 0.f, inv1 = st.l1 > 0.f ? 1.f / st.l1 : 0.f;
 #pragma unroll
   for (int nd = 0; nd < HD / 8; ++nd) {
-    if (pos0 >= 0) {
-      T16* d0 = ob + (static_cast<long long>(b) * S + pos0) * Hd + (g * HPG + h0) * HD + nd * 8 + 2 * q;
+    if (i0 >= 0) {
+      T16* d0 = ob + (static_cast<long long>(row0) + i0) * Hd + (g * HPG + h0) * HD + nd * 8 + 2 * q;
       *reinterpret_cast<uint32_t*>(d0) = pack2<T16>(st.o[nd][0] * inv0, st.o[nd][1] * inv0);
     }
-    if (pos1 >= 0) {
-      T16* d1 = ob + (static_cast<long long>(b) * S + pos1) * Hd + (g * HPG + h1) * HD + nd * 8 + 2 * q;
+    if (i1 >= 0) {
+      T16* d1 = ob + (static_cast<long long>(row0) + i1) * Hd + (g * HPG + h1) * HD + nd * 8 + 2 * q;
       *reinterpret_cast<uint32_t*>(d1) = pack2<T16>(st.o[nd][2] * inv1, st.o[nd][3] * inv1);
     }
   }
@@ -142,6 +156,10 @@ __global__ void __launch_bounds__(32) attn_f32_kernel(AttnArgs p, int decode) {
   if (decode) {
     b = m;
     pos = p.ctx[m];
+  } else if (p.rowmap) {
+    const int2 rm = p.rowmap[m];
+    b = rm.x;
+    pos = rm.y < 0 ? 0 : rm.y;  // unplaced row (already reported): any finite output
   } else {
     b = m / p.S;
     pos = m - b * p.S;
@@ -258,7 +276,7 @@ cudaError_t launch_attn_decode(const LaunchCtx& lc, bool fp32, const AttnArgs& a
 }
 
 cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B) {
-  if (fp32) return launch_k(lc, attn_f32_kernel, dim3(B * a.S, a.H), dim3(32), 0, a, 0);
+  if (fp32) return launch_k(lc, attn_f32_kernel, dim3(a.cu ? a.rows : B * a.S, a.H), dim3(32), 0, a, 0);
   if (a.H / a.G > 16) return cudaErrorInvalidValue;
   if (a.d == 64) return prefill_hd<64>(lc, a, B);
   if (a.d == 128) return prefill_hd<128>(lc, a, B);

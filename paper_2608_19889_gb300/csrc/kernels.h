@@ -65,6 +65,26 @@ cudaError_t launch_embed(const LaunchCtx& lc, bool fp32, const void* E, int V, i
 cudaError_t launch_finalize(const LaunchCtx& lc, unsigned long long* keys, int n_keys, int key_stride,
                             int key_offset, int B, int* next, int* ctx);
 
+// ---- variable-length batches (k_varlen.cu)
+// Row map of a packed batch: rowmap[m] = (sequence b, position past[b] + m -
+// cu[b]) for the T rows; checks cu (cu[0] = 0, non-decreasing, cu[B] = T,
+// chunks of 1 .. max_chunk rows) and past (>= 0, past + chunk <= max_pos),
+// setting DEVERR_SEQ / DEVERR_POS; a row it cannot place gets (0, -1).
+cudaError_t launch_varlen_rows(const LaunchCtx& lc, const int* cu, const int* past, int B, int T, int max_chunk,
+                               int max_pos, int2* rowmap, int* err);
+// Last row of each sequence's chunk gathered into dense [B] rows: the 16-bit
+// (or fp32) operand a (and its second term a_lo, fp16 mode) and the row's
+// inverse RMS, from either reduced rinv[row] or `parts` partial sums of
+// squares ss[row * ss_stride + i].
+cudaError_t launch_gather_last(const LaunchCtx& lc, const int* cu, int B, int T, const void* a, const void* a_lo,
+                               int row_bytes, const float* rinv, const float* ss, int ss_stride, int parts,
+                               float inv_D, float eps, void* a_out, void* a_lo_out, float* rinv_out);
+// Greedy token of each sequence from argmax keys (keys[b] when last_rows is
+// 0, else keys[cu[b+1]-1]), context lengths advanced by the chunk lengths
+// (optional), and the first n_keys keys cleared.
+cudaError_t launch_finalize_varlen(const LaunchCtx& lc, unsigned long long* keys, int n_keys, const int* cu,
+                                   int last_rows, int B, int* next, int* ctx);
+
 // ---- attention (k_attn.cu)
 struct AttnArgs {
   const void* q;  // [rows][H*d]
@@ -84,6 +104,13 @@ struct AttnArgs {
   void* o_lo;   // optional [rows][H*d]: o minus its 16-bit rounding (decode, fp16 mode)
   int* counter;  // decode [B][G] tickets
   int* err;
+  // Variable-length prefill (null otherwise): sequence b's chunk is rows
+  // cu[b] .. cu[b+1]-1 of q / o at positions past[b] + i; `rows` bounds
+  // the row offsets and S is the longest chunk (grid height).
+  const int* cu;
+  const int* past;
+  int rows;
+  const int2* rowmap;  // fp32 debug path: (sequence, position) per row
 };
 cudaError_t launch_attn_decode(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B);
 cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B);

@@ -49,6 +49,8 @@ def test_null_arguments_are_rejected_without_touching_the_device(built):
     assert lib.axon_model_create(None, None, 0, None, ctypes.byref(out)) == built.AXON_ERR_INVALID_ARG
     assert lib.axon_prefill(None, None, 1, 1, None, 0, None, None, None) == built.AXON_ERR_INVALID_ARG
     assert lib.axon_decode_step(None, None, 1, None, None, None, None, None) == built.AXON_ERR_INVALID_ARG
+    assert lib.axon_prefill_varlen(None, None, 1, 1, None, None, 1, None, 0, None, None, None) == \
+        built.AXON_ERR_INVALID_ARG
     lib.axon_free(None)
 
 
