@@ -55,6 +55,10 @@ READINGS = [
     "Greedy next token: argmax of the logits, lowest index on ties.",
     "KV cache: keys stored after RoPE; the paged overlay maps position p of "
     "sequence b to block_table[b][p // block_size], offset p % block_size.",
+    "Sliding window (the `window=` argument of causal_mask_for_input in the "
+    "appendix GPT-2 listing): with window W > 0 a query at position p sees "
+    "the keys at positions t with p - W < t <= p (itself and the W - 1 "
+    "before it); W = 0 means no window.",
 ]
 
 
@@ -75,12 +79,14 @@ class DecoderConfig:
     bias: bool  # attention_bias (q, k, v)
     theta: float  # rope_theta
     eps: float  # rms_norm_eps
+    window: int = 0  # sliding_window (0: none)
 
     @staticmethod
     def from_dict(c: dict) -> "DecoderConfig":
         return DecoderConfig(L=int(c["L"]), D=int(c["D"]), H=int(c["H"]), G=int(c["G"]),
                              d=int(c["d"]), F=int(c["F"]), V=int(c["V"]), tie=bool(c["tie"]),
-                             bias=bool(c["bias"]), theta=float(c["theta"]), eps=float(c["eps"]))
+                             bias=bool(c["bias"]), theta=float(c["theta"]), eps=float(c["eps"]),
+                             window=int(c.get("window", 0)))
 
 
 # ---------------------------------------------------------------------------
@@ -165,15 +171,21 @@ def attention_one_query(q, K, V, H, G):
     return o
 
 
-def causal_attention(q, K, V, q_pos, H, G):
+def causal_attention(q, K, V, q_pos, H, G, window=0):
     """Masking.causal_mask + Attention.attention for S queries of one sequence
-    (Sec. Built-In Libraries, attention and masking).
+    (Sec. Built-In Libraries, attention and masking; the `window=` argument
+    of causal_mask_for_input, appendix GPT-2 listing).
     q: [S, H, d] at positions q_pos [S]; K, V: [T, G, d] at positions 0..T-1.
-    Key t is visible to query i iff t <= q_pos[i]. Returns o: [S, H, d]."""
+    Key t is visible to query i iff t <= q_pos[i] and, with a window W > 0,
+    t > q_pos[i] - W. Returns o: [S, H, d]."""
     q = np.asarray(q, dtype=np.float64)
     S, _, d = q.shape
     T = K.shape[0]
-    keep = np.arange(T)[None, :] <= np.asarray(q_pos)[:, None]  # [S, T]
+    t = np.arange(T)[None, :]
+    p = np.asarray(q_pos)[:, None]
+    keep = t <= p  # [S, T]
+    if window > 0:
+        keep = keep & (t > p - window)
     o = np.empty_like(q)
     per = H // G
     for h in range(H):
@@ -318,7 +330,7 @@ class Oracle:
             for b in range(B):
                 cache.write(l, b, pos[b], k[b], v[b])
                 Kb, Vb = cache.read(l, b, int(pos[b, -1]) + 1)
-                o[b] = causal_attention(q[b], Kb, Vb, pos[b], c.H, c.G)
+                o[b] = causal_attention(q[b], Kb, Vb, pos[b], c.H, c.G, c.window)
             x = x + linear(o.reshape(B, S, c.H * c.d), self._w(p + "self_attn.o_proj.weight"))
             h2 = rmsnorm(x, self._w(p + "post_attention_layernorm.weight"), c.eps)
             u = swiglu(linear(h2, self._w(p + "mlp.gate_proj.weight")),

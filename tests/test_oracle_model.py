@@ -10,8 +10,8 @@ import synth_inputs as si
 from oracle import decoder as od
 
 
-def tiny_model(L=2, D=8, H=4, G=2, d=4, F=12, V=16, tie=False, bias=True, theta=100.0, eps=1e-5, seed=0):
-    m = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=bias, theta=theta, eps=eps)
+def tiny_model(L=2, D=8, H=4, G=2, d=4, F=12, V=16, tie=False, bias=True, theta=100.0, eps=1e-5, seed=0, window=0):
+    m = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=bias, theta=theta, eps=eps, window=window)
     w = si.weights_as_f32_numpy(si.make_weights(m, seed=seed))
     # Large-ish weights so that every term matters at tiny widths.
     w = {k: (v if k.endswith("layernorm.weight") or k == "model.norm.weight" else v * 20.0)
@@ -69,12 +69,14 @@ def _bf_forward(cfg, W, ids):
             o = []
             for hh in range(H):
                 g = hh * G // H
-                sc = [sum(qs[s][hh][j] * ks[t][g][j] for j in range(d)) / math.sqrt(d) for t in range(s + 1)]
+                # visible keys: t <= s, and with a window W only the last W of them
+                vis = [t for t in range(s + 1) if cfg.window == 0 or s - t < cfg.window]
+                sc = [sum(qs[s][hh][j] * ks[t][g][j] for j in range(d)) / math.sqrt(d) for t in vis]
                 mx = max(sc)
                 e = [math.exp(c - mx) for c in sc]
                 z = sum(e)
                 for j in range(d):
-                    o.append(sum(e[t] / z * vs[t][g][j] for t in range(s + 1)))
+                    o.append(sum(e[i] / z * vs[t][g][j] for i, t in enumerate(vis)))
             a = lin(o, W[p + "self_attn.o_proj.weight"])
             x1 = [xs[s][i] + a[i] for i in range(D)]
             h2 = rms(x1, W[p + "post_attention_layernorm.weight"])
@@ -88,9 +90,10 @@ def _bf_forward(cfg, W, ids):
     return [lin(rms(x, W["model.norm.weight"]), head) for x in xs]
 
 
-@pytest.mark.parametrize("tie,bias,H,G", [(False, True, 4, 2), (True, False, 2, 2), (False, False, 4, 1)])
-def test_oracle_matches_bruteforce_loops(tie, bias, H, G):
-    cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8)
+@pytest.mark.parametrize("tie,bias,H,G,window", [(False, True, 4, 2, 0), (True, False, 2, 2, 0), (False, False, 4, 1, 0),
+                                                 (False, True, 4, 2, 2), (True, False, 2, 2, 3)])
+def test_oracle_matches_bruteforce_loops(tie, bias, H, G, window):
+    cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8, window=window)
     ids = [3, 15, 0, 7, 7]
     ref = np.array(_bf_forward(cfg, W, ids))
     o = od.Oracle(cfg, W)
@@ -140,6 +143,23 @@ def test_incremental_decode_equals_full_recompute():
     for t in range(3, 8):
         step = o.decode_step(ids[:, t], cache, np.array([t, t]))
         assert np.allclose(step, full[:, t], rtol=1e-12, atol=1e-12)
+
+
+def test_sliding_window_decode_equals_full_recompute_and_differs_from_no_window():
+    cfg, W = tiny_model(window=3)
+    o = od.Oracle(cfg, W)
+    ids = np.array([[5, 1, 2, 11, 3, 8, 0, 14]])
+    full = o.prefill(ids, o.new_contiguous_cache(1, 8))
+    cache = o.new_contiguous_cache(1, 8)
+    o.prefill(ids[:, :2], cache)
+    for t in range(2, 8):
+        step = o.decode_step(ids[:, t], cache, np.array([t]))
+        assert np.allclose(step, full[:, t], rtol=1e-12, atol=1e-12)
+    cfg0, _ = tiny_model(window=0)
+    o0 = od.Oracle(cfg0, W)
+    none = o0.prefill(ids, o0.new_contiguous_cache(1, 8))
+    assert np.allclose(none[:, :3], full[:, :3], rtol=1e-12, atol=1e-12)  # the window covers positions 0..2
+    assert not np.allclose(none[:, 3:], full[:, 3:])
 
 
 def test_paged_cache_is_bit_identical_to_contiguous():

@@ -170,6 +170,52 @@ def test_causal_mask_ignores_future_keys():
     assert not np.allclose(o[3:], o2[3:])
 
 
+def test_window_one_sees_only_its_own_key():
+    S, H, G, d = 6, 4, 2, 8
+    q = RNG.normal(size=(S, H, d))
+    K = RNG.normal(size=(S, G, d))
+    V = RNG.normal(size=(S, G, d))
+    o = od.causal_attention(q, K, V, np.arange(S), H, G, window=1)
+    for i in range(S):
+        for h in range(H):
+            assert np.allclose(o[i, h], V[i, h // 2], atol=1e-15)
+
+
+def test_window_covering_the_context_is_no_window():
+    S, H, G, d = 7, 2, 1, 4
+    q = RNG.normal(size=(S, H, d))
+    K = RNG.normal(size=(S, G, d))
+    V = RNG.normal(size=(S, G, d))
+    full = od.causal_attention(q, K, V, np.arange(S), H, G)
+    for w in (S, S + 5):
+        assert np.array_equal(od.causal_attention(q, K, V, np.arange(S), H, G, window=w), full)
+
+
+def test_window_two_reduces_to_two_key_attention():
+    # query at position 4 with window 2 attends keys 3 and 4 only: the
+    # single-query attention over exactly those keys
+    S, H, G, d = 5, 2, 2, 8
+    q = RNG.normal(size=(S, H, d))
+    K = RNG.normal(size=(S, G, d))
+    V = RNG.normal(size=(S, G, d))
+    o = od.causal_attention(q, K, V, np.arange(S), H, G, window=2)
+    assert np.allclose(o[4], od.attention_one_query(q[4], K[3:5], V[3:5], H, G), atol=1e-14)
+    assert np.allclose(o[0], V[0][[0, 1]], atol=1e-15)  # position 0: only itself
+
+
+def test_window_ignores_keys_that_slid_out():
+    S, H, G, d, W = 9, 2, 1, 4, 3
+    q = RNG.normal(size=(S, H, d))
+    K = RNG.normal(size=(S, G, d))
+    V = RNG.normal(size=(S, G, d))
+    o = od.causal_attention(q, K, V, np.arange(S), H, G, window=W)
+    K2, V2 = K.copy(), V.copy()
+    K2[2], V2[2] = 50.0, -50.0  # visible to positions 2, 3, 4 only
+    o2 = od.causal_attention(q, K2, V2, np.arange(S), H, G, window=W)
+    assert np.array_equal(o[:2], o2[:2]) and np.array_equal(o[5:], o2[5:])
+    assert not np.allclose(o[2:5], o2[2:5])
+
+
 # ------------------------------------------------------------- integer helpers
 def test_slot_of_and_argmax_ties():
     bt = np.array([[7, 2, 9], [0, 5, 1]])
