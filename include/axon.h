@@ -95,6 +95,10 @@ typedef struct axon_config {
   int32_t kv_block_size;       /* tokens per block: must be 16 */
   int32_t kv_num_blocks;       /* paged pool size in blocks (ignored if contiguous) */
   int32_t precision;           /* AXON_BF16, AXON_FP16 or AXON_FP32_DEBUG */
+  int32_t sliding_window;      /* W > 0: a query at position p attends only to
+                                  keys p-W+1 .. p (the `window=` argument of
+                                  causal_mask_for_input, appendix GPT-2
+                                  listing); 0: full causal attention */
 } axon_config;
 
 /* One named checkpoint tensor, HF Llama naming and [out, in] matrices, as a

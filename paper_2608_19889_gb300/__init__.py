@@ -40,7 +40,7 @@ class axon_config(ctypes.Structure):
         "intermediate_size", "vocab_size", "tie_word_embeddings", "attention_bias")] + [
         ("rope_theta", ctypes.c_float), ("rms_norm_eps", ctypes.c_float)] + [
         (n, ctypes.c_int32) for n in ("max_batch", "max_context", "max_prefill_tokens", "kv_layout",
-                                      "kv_block_size", "kv_num_blocks", "precision")]
+                                      "kv_block_size", "kv_num_blocks", "precision", "sliding_window")]
 
 
 class axon_tensor(ctypes.Structure):
@@ -121,10 +121,11 @@ def axon_status_string(status: int) -> str:
 
 def make_config(m: dict, max_batch: int, max_context: int, kv_layout=AXON_KV_CONTIGUOUS, kv_num_blocks=0,
                 precision=AXON_BF16, max_prefill_tokens=0) -> axon_config:
-    """axon_config from a shape dict with keys L, D, H, G, d, F, V, tie, bias, theta, eps."""
+    """axon_config from a shape dict with keys L, D, H, G, d, F, V, tie, bias, theta, eps (and optionally
+    window, the sliding window; 0 or absent = none)."""
     return axon_config(m["L"], m["D"], m["H"], m["G"], m["d"], m["F"], m["V"], int(m["tie"]), int(m["bias"]),
                        float(m["theta"]), float(m["eps"]), max_batch, max_context, max_prefill_tokens, kv_layout, 16,
-                       kv_num_blocks, precision)
+                       kv_num_blocks, precision, int(m.get("window", 0)))
 
 
 def axon_model_create(cfg: axon_config, weights: dict, stream=None) -> ctypes.c_void_p:

@@ -273,6 +273,7 @@ int validate_config(const axon_config* c) {
   if (c->precision != AXON_BF16 && c->precision != AXON_FP32_DEBUG && c->precision != AXON_FP16)
     return AXON_ERR_INVALID_ARG;
   if (c->kv_block_size != 16) return AXON_ERR_UNSUPPORTED;
+  if (c->sliding_window < 0) return AXON_ERR_INVALID_ARG;
   if (c->kv_layout == AXON_KV_PAGED && c->kv_num_blocks <= 0) return AXON_ERR_INVALID_ARG;
   if (c->num_attention_heads % c->num_key_value_heads) return AXON_ERR_UNSUPPORTED;
   if (c->num_attention_heads / c->num_key_value_heads > 16) return AXON_ERR_UNSUPPORTED;
@@ -329,6 +330,7 @@ AttnArgs base_attn(const axon_model* m, int layer, const int* block_table) {
   a.G = m->G;
   a.d = m->d;
   a.scale_log2 = static_cast<float>(1.0 / std::sqrt(static_cast<double>(m->d)) * 1.4426950408889634);
+  a.window = m->cfg.sliding_window;
   a.err = m->err;
   return a;
 }
@@ -516,16 +518,10 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     pend(pf, wq + M * (D + m->Nqkv) * es, 2.0 * M * m->Nqkv * D);
 
     AttnArgs at = base_attn(m, l, bt);
-    at.S = S;
-    if (vl) {
-      at.S = vl->max_chunk;
-      at.cu = vl->cu;
-      at.past = vl->ctx;
-      at.rows = M;
-      at.rowmap = rowmap;
-    }
+    at.S = vl ? vl->max_chunk : S;
+    const AttnVarlen avl{vl ? vl->cu : nullptr, vl ? vl->ctx : nullptr, M, rowmap};
     pbeg(pf, "prefill_attention");
-    CK(launch_attn_prefill(lc, m->fp32, at, B));
+    CK(launch_attn_prefill(lc, m->fp32, at, B, vl ? &avl : nullptr));
     pend(pf, static_cast<double>(M) * (m->H + 2 * m->G) * m->d * es + static_cast<double>(M) * Hd * es,
          4.0 * B * m->H * m->d * (static_cast<double>(S) * (S + 1) / 2));
 
@@ -649,6 +645,7 @@ PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int3
   a.blocks_per_seq = m->blocks_per_seq;
   a.num_blocks = static_cast<int>(m->num_blocks);
   a.splits = splits;
+  a.window = m->cfg.sliding_window;
   a.eps = m->cfg.rms_norm_eps;
   a.inv_D = 1.0f / static_cast<float>(m->D);
   a.scale_log2 = static_cast<float>(1.0 / std::sqrt(static_cast<double>(m->d)) * 1.4426950408889634);

@@ -55,10 +55,11 @@ struct WarpState {
 };
 
 // One 16-key tile: keys tok0 .. tok0+15; key t is visible to row r (r+8)
-// iff t <= lim0 (lim1).
+// iff lo0 <= t <= lim0 (lo1 <= t <= lim1); lo is 0 without a sliding
+// window, else position - window + 1.
 template <int HD, typename T16>
 AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16][4], WarpState<HD>& st, int tok0,
-                          int lim0, int lim1, float sl2, int lane) {
+                          int lo0, int lim0, int lo1, int lim1, float sl2, int lane) {
   const int q = lane & 3;
   const int mi = lane >> 3, li = lane & 7;
   float s[2][4];
@@ -79,8 +80,8 @@ AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
       const int t = tok0 + nt * 8 + 2 * q + e;
-      s[nt][e] = (t <= lim0) ? s[nt][e] * sl2 : NEG_INF;
-      s[nt][2 + e] = (t <= lim1) ? s[nt][2 + e] * sl2 : NEG_INF;
+      s[nt][e] = (t <= lim0 && t >= lo0) ? s[nt][e] * sl2 : NEG_INF;
+      s[nt][2 + e] = (t <= lim1 && t >= lo1) ? s[nt][2 + e] * sl2 : NEG_INF;
       mx0 = fmaxf(mx0, s[nt][e]);
       mx1 = fmaxf(mx1, s[nt][2 + e]);
     }
@@ -161,12 +162,14 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
     T = tmax;
   }
   if (T < 1) T = 1;
-  const int nblk = (T + 15) >> 4;
+  // keys klo .. T-1: all of them, or the last `window`
+  const int klo = (p.window > 0 && T > p.window) ? T - p.window : 0;
+  const int jlo = klo >> 4, nblk = ((T + 15) >> 4) - jlo;
   // At least one block per warp; splits beyond the ones needed exit at once.
   const int per = max((nblk + p.splits - 1) / p.splits, DEC_WARPS);
   const int n_used = (nblk + per - 1) / per;
   if (s >= n_used) return;
-  const int jb = s * per, je = min(jb + per, nblk);
+  const int jb = jlo + s * per, je = min(jb + per, jlo + nblk);
 
   const uint32_t wbase = smem_u32(sm) + warp * 4 * TILE;  // per warp: [stage][K | V]
   const uint16_t* kp = static_cast<const uint16_t*>(p.k);
@@ -199,8 +202,8 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
       cp_async_wait<0>();
     }
     __syncwarp();
-    attn_tile16<HD, T16>(wbase + stg * 2 * TILE, wbase + stg * 2 * TILE + TILE, qa, st, j * 16, T - 1, T - 1,
-                         p.scale_log2, lane);
+    attn_tile16<HD, T16>(wbase + stg * 2 * TILE, wbase + stg * 2 * TILE + TILE, qa, st, j * 16, klo, T - 1, klo,
+                         T - 1, p.scale_log2, lane);
     __syncwarp();
     stg ^= 1;
   }

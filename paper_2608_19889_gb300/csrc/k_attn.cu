@@ -36,7 +36,7 @@ __global__ void __launch_bounds__(DEC_WARPS * 32) attn_decode_kernel(AttnArgs p)
 // key tiles staged 4 blocks (64 keys) at a time, double-buffered, shared by
 // the 4 warps.
 template <int HD, typename T16>
-__global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
+__global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW, AttnVarlen vl) {
   extern __shared__ __align__(128) uint8_t sm[];
   constexpr int TILE = 16 * HD * 2;
   constexpr int STAGE = 4 * 2 * TILE;  // 4 blocks x (K, V)
@@ -52,13 +52,13 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
   // The sequence's chunk: rows row0 .. row0+S-1 of q / o, at positions
   // past .. past+S-1 (a prompt from an empty cache: past = 0, row0 = b*S).
   int S = p.S, row0 = b * p.S, past = 0;
-  if (p.cu) {
-    row0 = p.cu[b];
-    const int row1 = p.cu[b + 1];
-    past = p.past[b];
+  if (vl.cu) {
+    row0 = vl.cu[b];
+    const int row1 = vl.cu[b + 1];
+    past = vl.past[b];
     S = row1 - row0;
     // inconsistent offsets (reported by the row-map kernel): no work
-    if (row0 < 0 || row1 > p.rows || S < 0 || S > p.S || past < 0 || past + S > p.blocks_per_seq * 16) S = 0;
+    if (row0 < 0 || row1 > vl.rows || S < 0 || S > p.S || past < 0 || past + S > p.blocks_per_seq * 16) S = 0;
   }
   if (p0 >= S) return;
 
@@ -84,18 +84,26 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
 
   WarpState<HD> st;
   st.init();
-  const int pend = past + min(p0 + PC, S);  // keys 0 .. pend-1 are visible to some row
-  const int nblk = (pend + 15) >> 4;
+  // Keys klo .. pend-1 are visible to some row of the CTA (klo > 0 only
+  // under a sliding window); staging starts at klo's block.
+  const int W = p.window;
+  const int pend = past + min(p0 + PC, S);
+  const int klo = (W > 0 && past + p0 >= W) ? past + p0 - W + 1 : 0;
+  const int jlo = klo >> 4;
+  const int nblk = ((pend + 15) >> 4) - jlo;
   const int nst = (nblk + 3) >> 2;
   const int wfirst = p0 + warp * PW;
   const int wmax = past + min(wfirst + PW - 1, S - 1);
+  // row lower limits (key index) and the warp's lowest one
+  const int lo0 = (W > 0 && pos0 >= W) ? pos0 - W + 1 : 0, lo1 = (W > 0 && pos1 >= W) ? pos1 - W + 1 : 0;
+  const int wlo = (W > 0 && past + wfirst >= W) ? past + wfirst - W + 1 : 0;
   const uint32_t base = smem_u32(sm);
   const uint16_t* kp = static_cast<const uint16_t*>(p.k);
   const uint16_t* vp = static_cast<const uint16_t*>(p.v);
   auto issue = [&](int stage_idx, int buf) {
     for (int jj = 0; jj < 4; ++jj) {
-      const int j = stage_idx * 4 + jj;
-      if (j >= nblk) break;
+      const int j = jlo + stage_idx * 4 + jj;
+      if (j >= jlo + nblk) break;
       bool ok;
       const int blk = block_of(p, b, j, ok);
       const long long off = (static_cast<long long>(blk) * p.G + g) * 16 * HD;
@@ -117,10 +125,11 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
     __syncthreads();
     if (wfirst < S) {
       for (int jj = 0; jj < 4; ++jj) {
-        const int j = sidx * 4 + jj;
-        if (j >= nblk || j * 16 > wmax) break;
+        const int j = jlo + sidx * 4 + jj;
+        if (j >= jlo + nblk || j * 16 > wmax) break;
+        if (j * 16 + 15 < wlo) continue;  // slid out of every row of this warp
         const uint32_t t = base + buf * STAGE + jj * 2 * TILE;
-        attn_tile16<HD, T16>(t, t + TILE, qa, st, j * 16, pos0, pos1, p.scale_log2, lane);
+        attn_tile16<HD, T16>(t, t + TILE, qa, st, j * 16, lo0, pos0, lo1, pos1, p.scale_log2, lane);
       }
     }
     __syncthreads();
@@ -147,7 +156,7 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW) {
 
 // ------------------------------------------------------- fp32 debug path
 // One warp per (row, query head): plain online softmax over visible keys.
-__global__ void __launch_bounds__(32) attn_f32_kernel(AttnArgs p, int decode) {
+__global__ void __launch_bounds__(32) attn_f32_kernel(AttnArgs p, int decode, AttnVarlen vl) {
   grid_dep_launch();
   grid_dep_wait();
   const int m = blockIdx.x, h = blockIdx.y, lane = threadIdx.x;
@@ -156,8 +165,8 @@ __global__ void __launch_bounds__(32) attn_f32_kernel(AttnArgs p, int decode) {
   if (decode) {
     b = m;
     pos = p.ctx[m];
-  } else if (p.rowmap) {
-    const int2 rm = p.rowmap[m];
+  } else if (vl.rowmap) {
+    const int2 rm = vl.rowmap[m];
     b = rm.x;
     pos = rm.y < 0 ? 0 : rm.y;  // unplaced row (already reported): any finite output
   } else {
@@ -175,7 +184,8 @@ __global__ void __launch_bounds__(32) attn_f32_kernel(AttnArgs p, int decode) {
   float mx = NEG_INF, l = 0.f;
   const float* kp = static_cast<const float*>(p.k);
   const float* vp = static_cast<const float*>(p.v);
-  for (int t = 0; t <= pos; ++t) {
+  const int t0 = (p.window > 0 && pos >= p.window) ? pos - p.window + 1 : 0;
+  for (int t = t0; t <= pos; ++t) {
     bool ok;
     const int blk = block_of(p, b, t >> 4, ok);
     if (!ok) continue;
@@ -222,14 +232,14 @@ cudaError_t decode_hd(const LaunchCtx& lc, const AttnArgs& a, int B) {
 }
 
 template <int HD>
-cudaError_t prefill_hd(const LaunchCtx& lc, const AttnArgs& a, int B) {
+cudaError_t prefill_hd(const LaunchCtx& lc, const AttnArgs& a, int B, const AttnVarlen& vl) {
   const size_t smem = prefill_smem<HD>();
   const int HPG = a.H / a.G;
   const int PW = 16 / HPG;
   const int PC = 4 * PW;
   const dim3 grid(a.G, (a.S + PC - 1) / PC, B);
-  if (lc.f16) return launch_k(lc, attn_prefill_kernel<HD, f16>, grid, dim3(128), smem, a, PW);
-  return launch_k(lc, attn_prefill_kernel<HD, bf16>, grid, dim3(128), smem, a, PW);
+  if (lc.f16) return launch_k(lc, attn_prefill_kernel<HD, f16>, grid, dim3(128), smem, a, PW, vl);
+  return launch_k(lc, attn_prefill_kernel<HD, bf16>, grid, dim3(128), smem, a, PW, vl);
 }
 
 }  // namespace
@@ -268,17 +278,18 @@ int attn_decode_splits(int B, int G, int max_blocks, int num_sms) {
 }
 
 cudaError_t launch_attn_decode(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B) {
-  if (fp32) return launch_k(lc, attn_f32_kernel, dim3(B, a.H), dim3(32), 0, a, 1);
+  if (fp32) return launch_k(lc, attn_f32_kernel, dim3(B, a.H), dim3(32), 0, a, 1, AttnVarlen{});
   if (a.H / a.G > 16) return cudaErrorInvalidValue;
   if (a.d == 64) return decode_hd<64>(lc, a, B);
   if (a.d == 128) return decode_hd<128>(lc, a, B);
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B) {
-  if (fp32) return launch_k(lc, attn_f32_kernel, dim3(a.cu ? a.rows : B * a.S, a.H), dim3(32), 0, a, 0);
+cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B, const AttnVarlen* vl) {
+  const AttnVarlen v = vl ? *vl : AttnVarlen{};
+  if (fp32) return launch_k(lc, attn_f32_kernel, dim3(vl ? v.rows : B * a.S, a.H), dim3(32), 0, a, 0, v);
   if (a.H / a.G > 16) return cudaErrorInvalidValue;
-  if (a.d == 64) return prefill_hd<64>(lc, a, B);
-  if (a.d == 128) return prefill_hd<128>(lc, a, B);
+  if (a.d == 64) return prefill_hd<64>(lc, a, B, v);
+  if (a.d == 128) return prefill_hd<128>(lc, a, B, v);
   return cudaErrorInvalidValue;
 }

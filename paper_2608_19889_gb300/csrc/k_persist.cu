@@ -605,6 +605,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       p.d = A.d;
       p.S = 1;
       p.splits = A.splits;
+      p.window = A.window;
       p.scale_log2 = A.scale_log2;
       p.part = A.attn_part;
       p.counter = A.attn_cnt;

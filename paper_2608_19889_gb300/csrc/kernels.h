@@ -99,21 +99,28 @@ struct AttnArgs {
   int H, G, d;
   int S;        // prefill prompt length
   int splits;   // decode split-KV factor
+  int window;   // sliding window: a query at position p sees keys p-window+1 .. p (0: no window)
   float scale_log2;
   float* part;  // decode partials
   void* o_lo;   // optional [rows][H*d]: o minus its 16-bit rounding (decode, fp16 mode)
   int* counter;  // decode [B][G] tickets
   int* err;
-  // Variable-length prefill (null otherwise): sequence b's chunk is rows
-  // cu[b] .. cu[b+1]-1 of q / o at positions past[b] + i; `rows` bounds
-  // the row offsets and S is the longest chunk (grid height).
+};
+// Variable-length prefill: sequence b's chunk is rows cu[b] .. cu[b+1]-1 of
+// q / o at positions past[b] + i; `rows` bounds the row offsets and the
+// AttnArgs' S is the longest chunk (grid height). Kept out of AttnArgs: the
+// decode kernels take AttnArgs by value and their register allocation
+// (measured 147 vs 128 per thread at head_dim 128) depends on its size.
+struct AttnVarlen {
   const int* cu;
   const int* past;
   int rows;
   const int2* rowmap;  // fp32 debug path: (sequence, position) per row
 };
 cudaError_t launch_attn_decode(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B);
-cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B);
+// vl: variable-length batch, or null (B sequences of a.S tokens from position 0)
+cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B,
+                                const AttnVarlen* vl = nullptr);
 int attn_decode_splits(int B, int G, int max_blocks, int num_sms);
 // Set kernel attributes (dynamic shared memory limits) once, before any
 // launch or graph capture.
@@ -185,7 +192,7 @@ struct PersistGrid {
 };
 struct PersistArgs {
   int L, D, H, G, d, F, V, Nqkv, Pmax, B;
-  int max_pos, blocks_per_seq, num_blocks, splits;
+  int max_pos, blocks_per_seq, num_blocks, splits, window;
   float eps, inv_D, scale_log2;
   const PersistLayer* layers;  // device [L]
   // device [4L + 1]: per layer the QKV, O, gate/up and down weights, then the
