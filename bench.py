@@ -258,10 +258,49 @@ class GenerateRun:
         return [[self.S] * self.B, [self.S + self.n_new // 2] * self.B, [self.S + self.n_new - 1] * self.B]
 
 
+PAGED_PREFILL_TOKENS = 16384  # rows per variable-length prefill call of the paged set-up
+
+
+def varlen_prefill_flops(m, calls):
+    """Algorithmic FLOPs of variable-length prefill calls; calls = list of
+    [(past, chunk)] per call: every new token through every linear, causal
+    attention of token past + i over past + i + 1 keys, the LM head on each
+    chunk's last token."""
+    lin, head = model_bytes(m)
+    total = 0.0
+    for chunks in calls:
+        T = sum(n for _, n in chunks)
+        keys = sum(n * past + n * (n + 1) / 2 for past, n in chunks)
+        total += 2 * T * lin + m["L"] * 4 * m["H"] * m["d"] * keys + 2 * len(chunks) * head
+    return total
+
+
+def plan_chunks(lens, budget):
+    """Chunked prefill schedule: sequences in order, cut into calls of at
+    most `budget` tokens; a sequence may continue in the next call. Returns
+    per call (first sequence, [(past, chunk) per sequence])."""
+    calls, cur, first, left = [], [], 0, budget
+    b, done = 0, 0
+    while b < len(lens):
+        n = min(int(lens[b]) - done, left)
+        if not cur:
+            first = b
+        cur.append((done, n))
+        done += n
+        left -= n
+        if done == int(lens[b]):
+            b, done = b + 1, 0
+        if left == 0 or b == len(lens):
+            calls.append((first, cur))
+            cur, left = [], budget
+    return calls
+
+
 class PagedDecodeRun:
     """Paged-cache workload: sequences with context lengths drawn from [lo, hi]
-    are prefilled one by one into a shuffled block pool (set-up, timed
-    separately); one step = n_new decode steps of the whole batch."""
+    are prefilled into a shuffled block pool by chunked variable-length
+    prefill calls of PAGED_PREFILL_TOKENS tokens (set-up, timed separately);
+    one step = n_new decode steps of the whole batch."""
 
     def __init__(self, ax, torch, model, m, wl, st, lens, bt_np):
         self.ax, self.torch, self.model, self.m, self.st = ax, torch, model, m, st
@@ -271,22 +310,36 @@ class PagedDecodeRun:
         self.bt = torch.from_numpy(bt_np).cuda()
         self.tok = torch.empty(self.B, dtype=torch.int32, device="cuda")
         self.first_tok = torch.empty(self.B, dtype=torch.int32, device="cuda")
-        self.ctx = torch.empty(self.B, dtype=torch.int32, device="cuda")
+        self.ctx = torch.zeros(self.B, dtype=torch.int32, device="cuda")
         self.logits = torch.empty(self.B, m["V"], device="cuda")
         self.kind = "paged"
-        # varlen prefill: one call per sequence on its block-table row
+        # chunked varlen prefill: each call covers consecutive sequences
+        # [first, first + n) -- block-table rows and context lengths are
+        # contiguous views -- with a piece of each
+        seqs = [si.make_ids(1, int(lens[b]), m["V"], seed=100 + b)[0] for b in range(self.B)]
+        self.calls = plan_chunks(lens, PAGED_PREFILL_TOKENS)
+        staged = []
+        for first, chunks in self.calls:
+            ids = np.concatenate([seqs[first + i][p:p + n] for i, (p, n) in enumerate(chunks)]).astype(np.int32)
+            cu = np.concatenate([[0], np.cumsum([n for _, n in chunks])]).astype(np.int32)
+            staged.append((first, len(chunks), max(n for _, n in chunks), torch.from_numpy(ids).cuda(),
+                           torch.from_numpy(cu).cuda()))
+        nxt = torch.empty(self.B, dtype=torch.int32, device="cuda")
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-        nxt = torch.empty(1, dtype=torch.int32, device="cuda")
+        torch.cuda.synchronize()
         with torch.cuda.stream(st):
             ev[0].record(st)
-            for b in range(self.B):
-                ids = torch.from_numpy(si.make_ids(1, int(lens[b]), m["V"], seed=100 + b)).cuda()
-                ax.axon_prefill(model, ids, block_table=self.bt[b:b + 1], next_tokens=nxt, stream=st)
-                self.first_tok[b:b + 1].copy_(nxt)
+            for first, n, mx, ids, cu in staged:
+                ax.axon_prefill_varlen(model, ids, cu, self.ctx[first:first + n], mx,
+                                       block_table=self.bt[first:first + n], next_tokens=nxt[:n], stream=st)
+                # a sequence continued by the next call gets its token there
+                self.first_tok[first:first + n].copy_(nxt[:n])
             ev[1].record(st)
         torch.cuda.synchronize()
+        assert np.array_equal(self.ctx.cpu().numpy(), lens), "chunked prefill left wrong context lengths"
         self.prefill_ms = ev[0].elapsed_time(ev[1])
         self.prefill_tokens = int(lens.sum())
+        self.prefill_flops = varlen_prefill_flops(m, [c for _, c in self.calls])
 
     def step(self, ev=None):
         ax, st = self.ax, self.st
@@ -340,7 +393,8 @@ def build_model(ax, torch, wl, m, st, layers=None, vocab=None, precision=0):
         num_blocks = int(sum(-(-int(c) // 16) for c in caps)) + 64
         bt_np = si.make_block_table(caps, 16, max_ctx // 16, num_blocks)
         cfg = ax.make_config(m, max_batch=B, max_context=max_ctx, kv_layout=ax.AXON_KV_PAGED,
-                             kv_num_blocks=num_blocks, max_prefill_tokens=hi, precision=precision)
+                             kv_num_blocks=num_blocks, max_prefill_tokens=PAGED_PREFILL_TOKENS,
+                             precision=precision)
     else:
         B, S = wl["B"], wl["S"]
         max_ctx = (S + wl["n_new"] + 15) // 16 * 16
@@ -553,9 +607,15 @@ def main():
                                          "what": "prefill FLOPs / timed prefill phase"}
     else:
         config["context_lens"] = f"uniform in {wl['ctx']}, mean {float(np.mean(run.lens_np)):.0f}"
-        out["setup_prefill"] = {"tokens": run.prefill_tokens, "ms": run.prefill_ms,
+        vl_tflops = run.prefill_flops / (run.prefill_ms / 1e3) / 1e12
+        out["setup_prefill"] = {"tokens": run.prefill_tokens, "ms": run.prefill_ms, "calls": len(run.calls),
                                 "tok_s": run.prefill_tokens / (run.prefill_ms / 1e3),
-                                "what": "varlen paged prefill of the contexts, one call per sequence (not in value)"}
+                                "roofline": {"bound": "tensor", "achieved": vl_tflops, "peak": tf_burst,
+                                             "unit": "TFLOP/s", "frac": vl_tflops / tf_burst,
+                                             "peak_kind": peak_kind},
+                                "what": f"chunked variable-length paged prefill of the contexts, "
+                                        f"{PAGED_PREFILL_TOKENS}-token calls, ids already on the device "
+                                        f"(not in value)"}
     if rank == 0 and world == 1 and not args.no_cpu_baseline and run.kind == "contiguous":
         v, sample, _ = oracle_generate_timed(wl, budget_s=15.0)
         out["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": cores(), "kind": "oracle", "sample": sample}

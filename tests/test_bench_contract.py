@@ -79,3 +79,26 @@ def test_reference_arm_json_line():
     assert line["e2e"] == {"value": line["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
                            "d2h_bytes_per_step": 0}
     assert line["config"]["workload"] == "135m_b1_s16_n16"
+
+
+def test_chunk_plan_covers_every_token_once_within_the_budget():
+    lens = [5, 3, 9, 2]
+    calls = bench.plan_chunks(lens, 6)
+    assert calls == [(0, [(0, 5), (0, 1)]), (1, [(1, 2), (0, 4)]), (2, [(4, 5), (0, 1)]), (3, [(1, 1)])]
+    got = {}
+    for first, chunks in calls:
+        assert sum(n for _, n in chunks) <= 6
+        for i, (past, n) in enumerate(chunks):
+            b = first + i
+            assert past == got.get(b, 0)  # each chunk continues where the last one stopped
+            got[b] = past + n
+    assert got == {0: 5, 1: 3, 2: 9, 3: 2}
+
+
+def test_varlen_prefill_flops_by_hand():
+    lin, head = bench.model_bytes(SHAPE)
+    # one whole prompt of 7 tokens counts like prefill_flops with B = 1
+    assert bench.varlen_prefill_flops(SHAPE, [[(0, 7)]]) == bench.prefill_flops(SHAPE, 1, 7)
+    # 3 new tokens after 4 cached ones attend 5 + 6 + 7 keys; a 1-token chunk after 9 attends 10
+    want = 2 * 4 * lin + 2 * 4 * 4 * 16 * (5 + 6 + 7 + 10) + 2 * 2 * head
+    assert bench.varlen_prefill_flops(SHAPE, [[(4, 3), (9, 1)]]) == want
