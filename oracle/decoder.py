@@ -43,7 +43,8 @@ READINGS = [
     "RMSNorm: y = x / sqrt(mean(x^2) + eps) * g; the gain multiplies the "
     "normalised vector (not 1+g); eps sits inside the square root.",
     "RoPE: rotate-half pairing (j, j + d/2), inv_freq_j = theta^(-2j/d), "
-    "angle = position * inv_freq_j, no frequency scaling.",
+    "angle = position * inv_freq_j; no frequency scaling unless configured "
+    "(next entry).",
     "Positions: the i-th new token of sequence b has position past_b + i, "
     "past_b = tokens already in the cache.",
     "GQA: query head h reads KV head floor(h / (H/G)) (contiguous groups).",
@@ -55,6 +56,12 @@ READINGS = [
     "Greedy next token: argmax of the logits, lowest index on ties.",
     "KV cache: keys stored after RoPE; the paged overlay maps position p of "
     "sequence b to block_table[b][p // block_size], offset p % block_size.",
+    "RoPE frequency scaling (Llama-3.1-family checkpoints; off unless "
+    "rope_factor > 0): with wavelength w_j = 2 pi / f_j and the original "
+    "context C, frequencies with w_j < C / high_freq_factor stay, those with "
+    "w_j > C / low_freq_factor are divided by the factor, and in between "
+    "f_j is blended linearly in t = (C / w_j - low) / (high - low): "
+    "(1 - t) f_j / factor + t f_j.",
     "Sliding window (the `window=` argument of causal_mask_for_input in the "
     "appendix GPT-2 listing): with window W > 0 a query at position p sees "
     "the keys at positions t with p - W < t <= p (itself and the W - 1 "
@@ -80,13 +87,24 @@ class DecoderConfig:
     theta: float  # rope_theta
     eps: float  # rms_norm_eps
     window: int = 0  # sliding_window (0: none)
+    # rope_scaling of Llama-3.1-family configs (rope_factor 0: none)
+    rope_factor: float = 0.0
+    rope_low: float = 1.0  # low_freq_factor
+    rope_high: float = 4.0  # high_freq_factor
+    rope_orig: int = 8192  # original_max_position_embeddings
 
     @staticmethod
     def from_dict(c: dict) -> "DecoderConfig":
         return DecoderConfig(L=int(c["L"]), D=int(c["D"]), H=int(c["H"]), G=int(c["G"]),
                              d=int(c["d"]), F=int(c["F"]), V=int(c["V"]), tie=bool(c["tie"]),
                              bias=bool(c["bias"]), theta=float(c["theta"]), eps=float(c["eps"]),
-                             window=int(c.get("window", 0)))
+                             window=int(c.get("window", 0)), rope_factor=float(c.get("rope_factor", 0.0)),
+                             rope_low=float(c.get("rope_low", 1.0)), rope_high=float(c.get("rope_high", 4.0)),
+                             rope_orig=int(c.get("rope_orig", 8192)))
+
+    def rope_scaling(self):
+        """(factor, low_freq_factor, high_freq_factor, original context), or None."""
+        return (self.rope_factor, self.rope_low, self.rope_high, self.rope_orig) if self.rope_factor > 0 else None
 
 
 # ---------------------------------------------------------------------------
@@ -111,14 +129,35 @@ def linear(x, W, b=None):
     return y
 
 
-def rope_inv_freq(d, theta):
+def rope_inv_freq(d, theta, scaling=None):
     """Positions (Sec. Built-In Libraries, positions and cache management):
-    rotary inverse frequencies theta^(-2j/d), j = 0 .. d/2-1."""
+    rotary inverse frequencies theta^(-2j/d), j = 0 .. d/2-1.
+
+    scaling = (factor, low_freq_factor, high_freq_factor, original context C)
+    applies the frequency-dependent stretch of Llama-3.1-family checkpoints
+    (one of the families the paper's benchmarks cover, Sec. Sub-4B Models):
+    each frequency's wavelength 2 pi / f is compared with C / high and
+    C / low; short wavelengths keep f, long ones take f / factor, and the
+    band between blends the two linearly in C / wavelength."""
     j = np.arange(d // 2, dtype=np.float64)
-    return np.power(float(theta), -2.0 * j / d)
+    f = np.power(float(theta), -2.0 * j / d)
+    if scaling is None:
+        return f
+    factor, low, high, C = (float(v) for v in scaling)
+    wavelen = 2.0 * math.pi / f
+    out = np.empty_like(f)
+    for i in range(f.shape[0]):
+        if wavelen[i] < C / high:  # high frequency: unchanged
+            out[i] = f[i]
+        elif wavelen[i] > C / low:  # low frequency: stretched by the factor
+            out[i] = f[i] / factor
+        else:  # between: linear blend in C / wavelength
+            t = (C / wavelen[i] - low) / (high - low)
+            out[i] = (1.0 - t) * f[i] / factor + t * f[i]
+    return out
 
 
-def rope(x, pos, theta):
+def rope(x, pos, theta, scaling=None):
     """Rotary embedding applied by `rope_apply` (Table 6 call counts) with the
     rotate-half pairing: for j < d/2,
         out_j       = x_j cos(p f_j) - x_{j+d/2} sin(p f_j)
@@ -126,7 +165,7 @@ def rope(x, pos, theta):
     x: [..., d]; pos broadcasts against x[..., 0]."""
     x = np.asarray(x, dtype=np.float64)
     d = x.shape[-1]
-    f = rope_inv_freq(d, theta)
+    f = rope_inv_freq(d, theta, scaling)
     ang = np.asarray(pos, dtype=np.float64)[..., None] * f
     c, s = np.cos(ang), np.sin(ang)
     x1, x2 = x[..., : d // 2], x[..., d // 2:]
@@ -324,8 +363,8 @@ class Oracle:
             q = linear(h, self._w(p + "self_attn.q_proj.weight"), bq).reshape(B, S, c.H, c.d)
             k = linear(h, self._w(p + "self_attn.k_proj.weight"), bk).reshape(B, S, c.G, c.d)
             v = linear(h, self._w(p + "self_attn.v_proj.weight"), bv).reshape(B, S, c.G, c.d)
-            q = rope(q, pos[:, :, None], c.theta)
-            k = rope(k, pos[:, :, None], c.theta)
+            q = rope(q, pos[:, :, None], c.theta, c.rope_scaling())
+            k = rope(k, pos[:, :, None], c.theta, c.rope_scaling())
             o = np.empty((B, S, c.H, c.d))
             for b in range(B):
                 cache.write(l, b, pos[b], k[b], v[b])

@@ -162,6 +162,23 @@ def test_sliding_window_decode_equals_full_recompute_and_differs_from_no_window(
     assert not np.allclose(none[:, 3:], full[:, 3:])
 
 
+def test_rope_scaling_changes_only_positions_beyond_zero_and_factor_one_is_off():
+    base = dict(L=2, D=8, H=4, G=2, d=4, F=12, V=16, tie=False, bias=True, theta=100.0, eps=1e-5)
+    _, W = tiny_model()
+    ids = np.array([[5, 1, 2, 11, 3, 8]])
+
+    def run(extra):
+        o = od.Oracle(od.DecoderConfig.from_dict(dict(base, **extra)), W)
+        return o.prefill(ids, o.new_contiguous_cache(1, 8))
+
+    plain = run({})
+    assert np.allclose(run(dict(rope_factor=1.0, rope_low=1.0, rope_high=4.0, rope_orig=64)), plain,
+                       rtol=1e-12, atol=1e-12)
+    scaled = run(dict(rope_factor=8.0, rope_low=1.0, rope_high=4.0, rope_orig=64))
+    assert np.allclose(scaled[:, 0], plain[:, 0], rtol=1e-12, atol=1e-12)  # position 0: no rotation at all
+    assert not np.allclose(scaled[:, 1:], plain[:, 1:])
+
+
 def test_paged_cache_is_bit_identical_to_contiguous():
     cfg, W = tiny_model()
     o = od.Oracle(cfg, W)

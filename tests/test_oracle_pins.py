@@ -77,6 +77,40 @@ def test_rope_dot_depends_only_on_relative_position():
 
 
 # ------------------------------------------------------------ SiLU / softmax
+LLAMA31 = (8.0, 1.0, 4.0, 8192)  # factor, low_freq_factor, high_freq_factor, original context
+
+
+def test_rope_scaling_factor_one_is_no_scaling():
+    f = od.rope_inv_freq(128, 5e5)
+    for low, high in [(1.0, 4.0), (2.0, 3.0)]:
+        assert np.allclose(od.rope_inv_freq(128, 5e5, (1.0, low, high, 8192)), f, rtol=1e-15, atol=0)
+
+
+def test_rope_scaling_bands_at_their_closed_form_edges():
+    d, theta = 128, 5e5
+    factor, low, high, C = LLAMA31
+    f = od.rope_inv_freq(d, theta)
+    g = od.rope_inv_freq(d, theta, LLAMA31)
+    # wavelength 2 pi theta^(2j/d) < C/high  <=>  j < (d/2) ln(C / (2 pi high)) / ln(theta)
+    n_keep = math.ceil((d / 2) * math.log(C / (2 * math.pi * high)) / math.log(theta))
+    n_stretch_from = math.floor((d / 2) * math.log(C / (2 * math.pi * low)) / math.log(theta)) + 1
+    assert 0 < n_keep < n_stretch_from < d // 2
+    assert np.array_equal(g[:n_keep], f[:n_keep])
+    assert np.allclose(g[n_stretch_from:], f[n_stretch_from:] / factor, rtol=1e-15, atol=0)
+    mid = g[n_keep:n_stretch_from] / f[n_keep:n_stretch_from]
+    assert np.all((mid < 1.0) & (mid > 1.0 / factor))
+
+
+def test_rope_scaling_ratio_is_continuous_and_monotone_in_wavelength():
+    # 1024 frequencies: the ratio scaled / unscaled falls from 1 to 1/factor
+    # without a jump at either band edge (a reversed blend jumps by 7/8)
+    g = od.rope_inv_freq(2048, 5e5, LLAMA31)
+    r = g / od.rope_inv_freq(2048, 5e5)
+    assert r[0] == 1.0 and abs(r[-1] - 1 / 8) < 1e-15
+    assert np.all(np.diff(r) <= 1e-15)
+    assert np.max(np.abs(np.diff(r))) < 0.05
+
+
 def test_silu_matches_library_logistic():
     z = np.linspace(-40, 40, 801)
     assert np.allclose(od.silu(z), z * expit(z), rtol=1e-14, atol=1e-300)
