@@ -99,6 +99,16 @@ typedef struct axon_config {
                                   keys p-W+1 .. p (the `window=` argument of
                                   causal_mask_for_input, appendix GPT-2
                                   listing); 0: full causal attention */
+  /* RoPE frequency scaling of Llama-3.1-family checkpoints (HF
+   * rope_scaling {"rope_type": "llama3", ...}); rope_scaling_factor 0 =
+   * none. A rotary frequency f with wavelength w = 2 pi / f is kept when
+   * w < original / high_freq_factor, divided by the factor when
+   * w > original / low_freq_factor, and blended linearly in
+   * t = (original / w - low) / (high - low) between: (1-t) f / factor + t f. */
+  float rope_scaling_factor;
+  float rope_low_freq_factor;
+  float rope_high_freq_factor;
+  int32_t rope_original_max_position;
 } axon_config;
 
 /* One named checkpoint tensor, HF Llama naming and [out, in] matrices, as a

@@ -40,7 +40,9 @@ class axon_config(ctypes.Structure):
         "intermediate_size", "vocab_size", "tie_word_embeddings", "attention_bias")] + [
         ("rope_theta", ctypes.c_float), ("rms_norm_eps", ctypes.c_float)] + [
         (n, ctypes.c_int32) for n in ("max_batch", "max_context", "max_prefill_tokens", "kv_layout",
-                                      "kv_block_size", "kv_num_blocks", "precision", "sliding_window")]
+                                      "kv_block_size", "kv_num_blocks", "precision", "sliding_window")] + [
+        (n, ctypes.c_float) for n in ("rope_scaling_factor", "rope_low_freq_factor", "rope_high_freq_factor")] + [
+        ("rope_original_max_position", ctypes.c_int32)]
 
 
 class axon_tensor(ctypes.Structure):
@@ -122,10 +124,12 @@ def axon_status_string(status: int) -> str:
 def make_config(m: dict, max_batch: int, max_context: int, kv_layout=AXON_KV_CONTIGUOUS, kv_num_blocks=0,
                 precision=AXON_BF16, max_prefill_tokens=0) -> axon_config:
     """axon_config from a shape dict with keys L, D, H, G, d, F, V, tie, bias, theta, eps (and optionally
-    window, the sliding window; 0 or absent = none)."""
+    window, the sliding window, and rope_factor / rope_low / rope_high / rope_orig, the RoPE frequency
+    scaling; 0 or absent = none)."""
     return axon_config(m["L"], m["D"], m["H"], m["G"], m["d"], m["F"], m["V"], int(m["tie"]), int(m["bias"]),
                        float(m["theta"]), float(m["eps"]), max_batch, max_context, max_prefill_tokens, kv_layout, 16,
-                       kv_num_blocks, precision, int(m.get("window", 0)))
+                       kv_num_blocks, precision, int(m.get("window", 0)), float(m.get("rope_factor", 0.0)),
+                       float(m.get("rope_low", 1.0)), float(m.get("rope_high", 4.0)), int(m.get("rope_orig", 8192)))
 
 
 def axon_model_create(cfg: axon_config, weights: dict, stream=None) -> ctypes.c_void_p:

@@ -112,6 +112,7 @@ struct axon_model {
   PersistGrid* pgrid = nullptr;
   int persist_ctas = 0;
   int decode_gemv_max = 32;  // decode projections with more tokens take the tcgen05 GEMM (AXON_DECODE_GEMV_MAX)
+  int persist_split_blocks = 16;  // persistent step: key blocks per split-KV item (AXON_PERSIST_SPLIT_BLOCKS)
   GemmSplitK gemm_sk{};      // split-K workspace of the decode-sized tensor-core GEMMs
 };
 
@@ -274,6 +275,11 @@ int validate_config(const axon_config* c) {
     return AXON_ERR_INVALID_ARG;
   if (c->kv_block_size != 16) return AXON_ERR_UNSUPPORTED;
   if (c->sliding_window < 0) return AXON_ERR_INVALID_ARG;
+  if (c->rope_scaling_factor < 0.f) return AXON_ERR_INVALID_ARG;
+  if (c->rope_scaling_factor > 0.f &&
+      (c->rope_original_max_position <= 0 || c->rope_low_freq_factor <= 0.f ||
+       c->rope_high_freq_factor <= c->rope_low_freq_factor))
+    return AXON_ERR_INVALID_ARG;
   if (c->kv_layout == AXON_KV_PAGED && c->kv_num_blocks <= 0) return AXON_ERR_INVALID_ARG;
   if (c->num_attention_heads % c->num_key_value_heads) return AXON_ERR_UNSUPPORTED;
   if (c->num_attention_heads / c->num_key_value_heads > 16) return AXON_ERR_UNSUPPORTED;
@@ -700,9 +706,14 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     if (splits > cap) splits = cap < 1 ? 1 : cap;
   }
   if (persist_eligible(m, B)) {
-    // Inside one launch a cross-CTA merge costs more than it saves at these
-    // lengths: split a sequence's keys only beyond 64 blocks (8 per warp).
-    int psplits = (m->blocks_per_seq + 63) / 64;
+    // Inside one launch a cross-CTA merge costs more than it saves up to 64
+    // key blocks (8 per warp; measured at 40 blocks, head_dim 64: 0.743 ms
+    // per step unsplit, 0.775-0.790 ms split). Beyond that the keys split
+    // into items of persist_split_blocks blocks (80 blocks, head_dim 128:
+    // 3.170 ms per step in items of 16, 3.239 ms in items of 64).
+    int psplits = m->blocks_per_seq > 64
+                      ? (m->blocks_per_seq + m->persist_split_blocks - 1) / m->persist_split_blocks
+                      : 1;
     if (psplits > splits) psplits = splits;
     PersistArgs pa = persist_args(m, tokens, B, ctx, bt, logits, next, psplits, attn_part ? attn_part : m->attn_part,
                                   attn_cnt ? attn_cnt : m->attn_cnt);
@@ -892,6 +903,10 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->use_graphs = !env_flag("AXON_NO_GRAPH");
   m->use_pdl = !env_flag("AXON_NO_PDL");
   m->use_tma_gemv = env_flag("AXON_TMA_GEMV");
+  if (const char* v = getenv("AXON_PERSIST_SPLIT_BLOCKS")) {
+    const int t = atoi(v);
+    if (t >= 8 && t <= 4096) m->persist_split_blocks = t;
+  }
   if (const char* v = getenv("AXON_DECODE_GEMV_MAX")) {
     const int t = atoi(v);
     if (t >= 0 && t <= 64) m->decode_gemv_max = t;
@@ -1022,14 +1037,30 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
       cudaMemsetAsync(m->vpool, 0, kv_bytes, st) != cudaSuccess)
     return fail(AXON_ERR_CUDA);
 
-  // ---- RoPE table in double precision: (cos, sin)(p * theta^(-2j/d))
+  // ---- RoPE table in double precision: (cos, sin)(p * f_j), f_j =
+  // theta^(-2j/d), stretched per band when frequency scaling is configured
   {
     const int half = m->d / 2;
+    std::vector<double> freq(half);
+    for (int j = 0; j < half; ++j) {
+      double f = std::pow(static_cast<double>(cfg->rope_theta), -2.0 * j / m->d);
+      if (cfg->rope_scaling_factor > 0.f) {
+        const double factor = cfg->rope_scaling_factor, lo = cfg->rope_low_freq_factor,
+                     hi = cfg->rope_high_freq_factor, C = cfg->rope_original_max_position;
+        const double w = 2.0 * 3.14159265358979323846 / f;
+        if (w > C / lo) {
+          f = f / factor;
+        } else if (w >= C / hi) {
+          const double t = (C / w - lo) / (hi - lo);
+          f = (1.0 - t) * f / factor + t * f;
+        }
+      }
+      freq[j] = f;
+    }
     std::vector<float2> tab(static_cast<size_t>(cfg->max_context) * half);
     for (int pos = 0; pos < cfg->max_context; ++pos)
       for (int j = 0; j < half; ++j) {
-        const double f = std::pow(static_cast<double>(cfg->rope_theta), -2.0 * j / m->d);
-        const double ang = pos * f;
+        const double ang = pos * freq[j];
         tab[static_cast<size_t>(pos) * half + j] = make_float2(static_cast<float>(std::cos(ang)),
                                                                static_cast<float>(std::sin(ang)));
       }

@@ -117,3 +117,25 @@ def test_persistent_decode_paged_cache(prec):
         assert ax.axon_check_device(m)[0] == 0
     finally:
         ax.axon_free(m)
+
+
+@pytest.mark.parametrize("shape", [TINY, TINY128])
+def test_persistent_decode_split_kv_long_context(shape):
+    """A context of more than 64 key blocks: the persistent step splits each
+    sequence's keys into items of 16 blocks and merges them across CTAs."""
+    ax = _ax()
+    B, S, max_ctx = 2, 1100, 1152  # 72 key blocks of capacity: 5 splits
+    w = gpu_weights(shape)
+    m = _create(shape, w, True, max_batch=B, max_context=max_ctx, max_prefill_tokens=B * S)
+    try:
+        assert "decode_persistent" in _kinds(m, B, [max_ctx - 2] * B)
+        ids = si.make_ids(B, S, shape["V"], seed=17)
+        _, nxt = run_prefill(m, ids, ax.AXON_LOGITS_LAST, shape["V"])
+        dl, fed = decode_steps(m, nxt, [S] * B, 6, shape["V"])
+        o = oracle_for(shape, w)
+        cache = o.new_contiguous_cache(B, max_ctx)
+        o.prefill(ids, cache, last_only=True)
+        check(dl, oracle_decode(o, cache, fed, [S] * B), what=f"persistent split-KV decode d={shape['d']}")
+        assert ax.axon_check_device(m)[0] == 0
+    finally:
+        ax.axon_free(m)
