@@ -186,6 +186,23 @@ def cores():
         return os.cpu_count()
 
 
+def max_over_ranks(ms, dist, device):
+    """The slowest rank's time: every replica's timed region is bracketed by
+    barriers, and the job is done when the last replica is."""
+    if dist is None:
+        return float(ms)
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank, world, ms):
+    """Units all replicas processed (each rank runs the full workload on its
+    own GPU, weak scaling) per second of the slowest rank."""
+    return world * units_per_rank / (ms / 1e3)
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return
@@ -494,11 +511,7 @@ def main():
     t_pre = [e[0].elapsed_time(e[1]) for e in ev]
     t_dec = [e[1].elapsed_time(e[2]) for e in ev]
     t_step = [e[0].elapsed_time(e[2]) for e in ev]
-    ms = float(np.mean(t_step))
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(np.mean(t_step), dist, "cuda")
 
     # ---- end to end through the public API with host buffers: inputs copied in
     # from pinned memory, generated tokens copied out, inside the timed region.
@@ -517,11 +530,11 @@ def main():
             e2e_ev[1].record(st)
             e2e_ev[1].synchronize()
             e2e_ms.append(e2e_ev[0].elapsed_time(e2e_ev[1]))
-    e2e_val = run.generated_per_step() / (float(np.mean(e2e_ms)) / 1e3)
+    e2e_val = whole_job_rate(run.generated_per_step(), world, max_over_ranks(np.mean(e2e_ms), dist, "cuda"))
 
     hbm, tf_burst, tf_sus, peak_kind = read_peaks()
     dec_bytes = sum(decode_bytes_per_step(m, B, T) for T in run.decode_positions())
-    dec_ms = float(np.mean(t_dec))
+    dec_ms = max_over_ranks(np.mean(t_dec), dist, "cuda")
     dec_gbs = dec_bytes / (dec_ms / 1e3) / 1e9
 
     # ---- per-kernel timing (CUDA events around each launch, no graph) of
@@ -570,7 +583,7 @@ def main():
               "l2": "inputs larger than L2 (weights " + f"{2 * sum(model_bytes(m)) / 1e9:.2f} GB > 129 MB)"}
     out = {
         "metric": METRIC,
-        "value": world * run.generated_per_step() / (ms / 1e3),
+        "value": whole_job_rate(run.generated_per_step(), world, ms),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
@@ -582,14 +595,14 @@ def main():
         "dtype": args.precision,
         "data": "synthetic (seeded random-init weights N(0,0.02), uniform random ids)",
         "config": config,
-        "decode_tok_s": world * B * n_new / (dec_ms / 1e3),
+        "decode_tok_s": whole_job_rate(B * n_new, world, dec_ms),
         "decode_ms": dec_ms,
         "roofline": roof,
         "roofline_decode_step": {"bound": "hbm", "achieved": dec_gbs, "peak": hbm, "unit": "GB/s",
                                  "frac": dec_gbs / hbm, "peak_kind": peak_kind,
                                  "what": "all decode bytes (weights + KV + logits) / timed decode phase"},
         "kernels": kernel_table,
-        "e2e": {"value": world * e2e_val, "unit": "tokens/s",
+        "e2e": {"value": e2e_val, "unit": "tokens/s",
                 "h2d_bytes_per_step": int(in_h.numel()) * 4, "d2h_bytes_per_step": B * n_new * 4},
         "gpu_launches": int(round(args.steps * launches_per_step)),
         "clocks": clk,
@@ -598,9 +611,9 @@ def main():
     if run.kind == "contiguous":
         S = run.S
         config["S"] = S
-        pre_ms = float(np.mean(t_pre))
+        pre_ms = max_over_ranks(np.mean(t_pre), dist, "cuda")
         pre_tflops = prefill_flops(m, B, S) / (pre_ms / 1e3) / 1e12
-        out["prefill_tok_s"] = world * B * S / (pre_ms / 1e3)
+        out["prefill_tok_s"] = whole_job_rate(B * S, world, pre_ms)
         out["prefill_ms"] = pre_ms
         out["roofline_prefill_phase"] = {"bound": "tensor", "achieved": pre_tflops, "peak": tf_burst,
                                          "unit": "TFLOP/s", "frac": pre_tflops / tf_burst, "peak_kind": peak_kind,
