@@ -51,7 +51,9 @@ READINGS = [
     "Attention scale 1/sqrt(d), causal mask keeps keys with position <= "
     "query position, softmax with max subtraction.",
     "Biases: q, k, v only (when attention_bias); never on o, gate, up, down.",
-    "SwiGLU: silu(h Wg^T) * (h Wu^T), silu(z) = z / (1 + exp(-z)).",
+    "SwiGLU: silu(h Wg^T) * (h Wu^T), silu(z) = z / (1 + exp(-z)); with "
+    "hidden_act gelu_tanh the gate takes gelu_new, 0.5 z (1 + tanh(sqrt(2/pi) "
+    "(z + 0.044715 z^3))), the GELU of the GPT-2 listing.",
     "LM head: logits = rmsnorm(x) Whead^T with Whead = embedding when tied.",
     "Greedy next token: argmax of the logits, lowest index on ties.",
     "KV cache: keys stored after RoPE; the paged overlay maps position p of "
@@ -92,6 +94,7 @@ class DecoderConfig:
     rope_low: float = 1.0  # low_freq_factor
     rope_high: float = 4.0  # high_freq_factor
     rope_orig: int = 8192  # original_max_position_embeddings
+    act: str = "silu"  # hidden_act of the gated MLP: "silu" or "gelu_tanh"
 
     @staticmethod
     def from_dict(c: dict) -> "DecoderConfig":
@@ -100,7 +103,7 @@ class DecoderConfig:
                              bias=bool(c["bias"]), theta=float(c["theta"]), eps=float(c["eps"]),
                              window=int(c.get("window", 0)), rope_factor=float(c.get("rope_factor", 0.0)),
                              rope_low=float(c.get("rope_low", 1.0)), rope_high=float(c.get("rope_high", 4.0)),
-                             rope_orig=int(c.get("rope_orig", 8192)))
+                             rope_orig=int(c.get("rope_orig", 8192)), act=str(c.get("act", "silu")))
 
     def rope_scaling(self):
         """(factor, low_freq_factor, high_freq_factor, original context), or None."""
@@ -179,10 +182,20 @@ def silu(z):
         return z / (1.0 + np.exp(-z))
 
 
-def swiglu(gate, up):
+def gelu_tanh(z):
+    """Activations.gelu_new (appendix GPT-2 listing; Sec. Built-In Libraries,
+    activations), the tanh form of GELU:
+    0.5 z (1 + tanh(sqrt(2/pi) (z + 0.044715 z^3)))."""
+    z = np.asarray(z, dtype=np.float64)
+    return 0.5 * z * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (z + 0.044715 * z ** 3)))
+
+
+def swiglu(gate, up, act="silu"):
     """Act.swiglu between NN.linear@up and NN.linear@down (appendix, function
-    application listing): silu(gate) * up."""
-    return silu(gate) * np.asarray(up, dtype=np.float64)
+    application listing): silu(gate) * up; with act="gelu_tanh" the gate
+    goes through gelu_new instead (the gated-GELU MLP)."""
+    a = gelu_tanh(gate) if act == "gelu_tanh" else silu(gate)
+    return a * np.asarray(up, dtype=np.float64)
 
 
 def softmax(s, axis=-1):
@@ -373,7 +386,7 @@ class Oracle:
             x = x + linear(o.reshape(B, S, c.H * c.d), self._w(p + "self_attn.o_proj.weight"))
             h2 = rmsnorm(x, self._w(p + "post_attention_layernorm.weight"), c.eps)
             u = swiglu(linear(h2, self._w(p + "mlp.gate_proj.weight")),
-                       linear(h2, self._w(p + "mlp.up_proj.weight")))
+                       linear(h2, self._w(p + "mlp.up_proj.weight")), c.act)
             x = x + linear(u, self._w(p + "mlp.down_proj.weight"))
         if last_hidden_only:
             x = x[:, -1:, :]

@@ -10,8 +10,9 @@ import synth_inputs as si
 from oracle import decoder as od
 
 
-def tiny_model(L=2, D=8, H=4, G=2, d=4, F=12, V=16, tie=False, bias=True, theta=100.0, eps=1e-5, seed=0, window=0):
-    m = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=bias, theta=theta, eps=eps, window=window)
+def tiny_model(L=2, D=8, H=4, G=2, d=4, F=12, V=16, tie=False, bias=True, theta=100.0, eps=1e-5, seed=0, window=0,
+               act="silu"):
+    m = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=bias, theta=theta, eps=eps, window=window, act=act)
     w = si.weights_as_f32_numpy(si.make_weights(m, seed=seed))
     # Large-ish weights so that every term matters at tiny widths.
     w = {k: (v if k.endswith("layernorm.weight") or k == "model.norm.weight" else v * 20.0)
@@ -82,7 +83,11 @@ def _bf_forward(cfg, W, ids):
             h2 = rms(x1, W[p + "post_attention_layernorm.weight"])
             gt = lin(h2, W[p + "mlp.gate_proj.weight"])
             up = lin(h2, W[p + "mlp.up_proj.weight"])
-            u = [gt[i] / (1.0 + math.exp(-gt[i])) * up[i] for i in range(F)]
+            if cfg.act == "gelu_tanh":
+                c = math.sqrt(2.0 / math.pi)
+                u = [0.5 * gt[i] * (1.0 + math.tanh(c * (gt[i] + 0.044715 * gt[i] ** 3))) * up[i] for i in range(F)]
+            else:
+                u = [gt[i] / (1.0 + math.exp(-gt[i])) * up[i] for i in range(F)]
             dn = lin(u, W[p + "mlp.down_proj.weight"])
             new_x.append([x1[i] + dn[i] for i in range(D)])
         xs = new_x
@@ -90,10 +95,11 @@ def _bf_forward(cfg, W, ids):
     return [lin(rms(x, W["model.norm.weight"]), head) for x in xs]
 
 
-@pytest.mark.parametrize("tie,bias,H,G,window", [(False, True, 4, 2, 0), (True, False, 2, 2, 0), (False, False, 4, 1, 0),
-                                                 (False, True, 4, 2, 2), (True, False, 2, 2, 3)])
-def test_oracle_matches_bruteforce_loops(tie, bias, H, G, window):
-    cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8, window=window)
+@pytest.mark.parametrize("tie,bias,H,G,window,act", [(False, True, 4, 2, 0, "silu"), (True, False, 2, 2, 0, "silu"),
+                                                     (False, False, 4, 1, 0, "silu"), (False, True, 4, 2, 2, "silu"),
+                                                     (True, False, 2, 2, 3, "silu"), (False, True, 4, 2, 0, "gelu_tanh")])
+def test_oracle_matches_bruteforce_loops(tie, bias, H, G, window, act):
+    cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8, window=window, act=act)
     ids = [3, 15, 0, 7, 7]
     ref = np.array(_bf_forward(cfg, W, ids))
     o = od.Oracle(cfg, W)

@@ -120,6 +120,25 @@ def test_silu_matches_library_logistic():
     assert np.allclose(od.swiglu(g, u), g * expit(g) * u, rtol=1e-14)
 
 
+def test_gelu_tanh_against_exact_gelu_and_its_identities():
+    from scipy.special import erf
+    z = np.linspace(-8, 8, 4001)
+    g = od.gelu_tanh(z)
+    exact = 0.5 * z * (1 + erf(z / math.sqrt(2)))  # GELU from the normal CDF
+    assert np.max(np.abs(g - exact)) < 1e-3  # the tanh form approximates it closely...
+    assert np.max(np.abs(g - exact)) > 1e-5  # ...but is not it
+    assert np.allclose(g - od.gelu_tanh(-z), z, atol=1e-13)  # gelu(z) - gelu(-z) = z
+    assert od.gelu_tanh(0.0) == 0.0
+    assert abs(od.gelu_tanh(1.0) - 0.5 * (1 + math.tanh(math.sqrt(2 / math.pi) * 1.044715))) < 1e-15
+
+
+def test_gated_mlp_activation_choice():
+    gate = RNG.normal(size=(3, 5))
+    up = RNG.normal(size=(3, 5))
+    assert np.allclose(od.swiglu(gate, up), gate * expit(gate) * up, atol=1e-15)
+    assert np.allclose(od.swiglu(gate, up, "gelu_tanh"), od.gelu_tanh(gate) * up, atol=1e-15)
+
+
 def test_softmax_rows_sum_to_one_and_shift_invariant():
     s = RNG.normal(size=(4, 33)) * 10
     a = od.softmax(s)
