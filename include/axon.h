@@ -67,6 +67,11 @@ enum { AXON_KV_CONTIGUOUS = 0, AXON_KV_PAGED = 1 };
  *                    AXON_ERR_UNSUPPORTED. */
 enum { AXON_BF16 = 0, AXON_FP32_DEBUG = 1, AXON_FP16 = 2 };
 
+/* Gate activation of the gated MLP (Activations built-ins, Sec. Built-In
+ * Libraries): silu (SwiGLU, Llama / Qwen / Mistral) or the tanh form of
+ * GELU, gelu_new of the appendix GPT-2 listing (gated GELU). */
+enum { AXON_ACT_SILU = 0, AXON_ACT_GELU_TANH = 1 };
+
 /* Element types of weight tensors handed to axon_model_create. */
 enum { AXON_DTYPE_BF16 = 0, AXON_DTYPE_F32 = 1 };
 
@@ -109,6 +114,7 @@ typedef struct axon_config {
   float rope_low_freq_factor;
   float rope_high_freq_factor;
   int32_t rope_original_max_position;
+  int32_t hidden_act;          /* AXON_ACT_SILU or AXON_ACT_GELU_TANH: u = act(h W_gate^T) * (h W_up^T) */
 } axon_config;
 
 /* One named checkpoint tensor, HF Llama naming and [out, in] matrices, as a

@@ -276,6 +276,7 @@ int validate_config(const axon_config* c) {
   if (c->kv_block_size != 16) return AXON_ERR_UNSUPPORTED;
   if (c->sliding_window < 0) return AXON_ERR_INVALID_ARG;
   if (c->rope_scaling_factor < 0.f) return AXON_ERR_INVALID_ARG;
+  if (c->hidden_act != AXON_ACT_SILU && c->hidden_act != AXON_ACT_GELU_TANH) return AXON_ERR_INVALID_ARG;
   if (c->rope_scaling_factor > 0.f &&
       (c->rope_original_max_position <= 0 || c->rope_low_freq_factor <= 0.f ||
        c->rope_high_freq_factor <= c->rope_low_freq_factor))
@@ -313,6 +314,7 @@ EpiArgs base_epi(const axon_model* m) {
   e.max_pos = m->cfg.max_context;
   e.inv_D = 1.0f / static_cast<float>(m->D);
   e.eps = m->cfg.rms_norm_eps;
+  e.act = m->cfg.hidden_act;
   e.H = m->H;
   e.G = m->G;
   e.d = m->d;
@@ -653,6 +655,7 @@ PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int3
   a.splits = splits;
   a.window = m->cfg.sliding_window;
   a.eps = m->cfg.rms_norm_eps;
+  a.act = m->cfg.hidden_act;
   a.inv_D = 1.0f / static_cast<float>(m->D);
   a.scale_log2 = static_cast<float>(1.0 / std::sqrt(static_cast<double>(m->d)) * 1.4426950408889634);
   a.layers = m->players;

@@ -20,6 +20,8 @@
 #include "common.cuh"
 
 enum EpiKind : int { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LOGITS = 3 };
+// Gate activation of the gated MLP (axon_config.hidden_act).
+enum ActKind : int { ACT_SILU = 0, ACT_GELU_TANH = 1 };
 
 struct EpiArgs {
   int M;  // rows (tokens)
@@ -66,6 +68,7 @@ struct EpiArgs {
   // SWIGLU
   void* u_out;     // [M][N/2]
   void* u_lo_out;  // optional [M][N/2]: u - u_out (second term of the down projection's operand)
+  int act;         // gate activation: ACT_SILU or ACT_GELU_TANH
   // LOGITS
   float* logits;  // [M][logits_stride] or null
   long long logits_stride;
@@ -263,13 +266,21 @@ AXON_DEV float epi_resid16(const EpiArgs& e, int m, int n0, const float* v) {
   return epi_resid16x<T>(e, m, n0, v, xin);
 }
 
-AXON_DEV float silu_f(float z) { return z / (1.0f + expf(-z)); }
+// Both gate activations are z * sigmoid(k(z)): silu with k(z) = z, and
+// gelu_new, 0.5 z (1 + tanh(sqrt(2/pi) (z + 0.044715 z^3))), with
+// k(z) = 2 sqrt(2/pi) (z + 0.044715 z^3), since (1 + tanh(a)) / 2 =
+// sigmoid(2a).
+AXON_DEV float gate_act(float z, bool gelu) {
+  const float k = gelu ? 1.5957691216057308f * fmaf(0.044715f * z, z * z, z) : z;
+  return z / (1.0f + expf(-k));
+}
 
 template <typename T>
 AXON_DEV void epi_swiglu16(const EpiArgs& e, int m, int n0, const float* v, float r) {
   float u[8];
+  const bool gelu = e.act == ACT_GELU_TANH;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) u[i] = silu_f(v[i] * r) * (v[8 + i] * r);
+  for (int i = 0; i < 8; ++i) u[i] = gate_act(v[i] * r, gelu) * (v[8 + i] * r);
   T* up = reinterpret_cast<T*>(e.u_out) + static_cast<long long>(m) * (e.N >> 1) + (n0 >> 1);
   store8<T>(up, u);
   if (e.u_lo_out) {

@@ -455,6 +455,7 @@ AXON_DEV EpiArgs base_ep(const PersistArgs& A) {
   e.max_pos = A.max_pos;
   e.inv_D = A.inv_D;
   e.eps = A.eps;
+  e.act = A.act;
   e.H = A.H;
   e.G = A.G;
   e.d = A.d;

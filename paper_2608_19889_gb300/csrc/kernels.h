@@ -192,7 +192,7 @@ struct PersistGrid {
 };
 struct PersistArgs {
   int L, D, H, G, d, F, V, Nqkv, Pmax, B;
-  int max_pos, blocks_per_seq, num_blocks, splits, window;
+  int max_pos, blocks_per_seq, num_blocks, splits, window, act;
   float eps, inv_D, scale_log2;
   const PersistLayer* layers;  // device [L]
   // device [4L + 1]: per layer the QKV, O, gate/up and down weights, then the
