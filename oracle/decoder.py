@@ -64,6 +64,10 @@ READINGS = [
     "w_j > C / low_freq_factor are divided by the factor, and in between "
     "f_j is blended linearly in t = (C / w_j - low) / (high - low): "
     "(1 - t) f_j / factor + t f_j.",
+    "qk-norm (Qwen3-family layers, off unless configured): after the q and "
+    "k projections (and biases), each head's d values go through the same "
+    "RMSNorm as the hidden state, with gains q_norm / k_norm of length d, "
+    "before RoPE.",
     "Sliding window (the `window=` argument of causal_mask_for_input in the "
     "appendix GPT-2 listing): with window W > 0 a query at position p sees "
     "the keys at positions t with p - W < t <= p (itself and the W - 1 "
@@ -95,6 +99,7 @@ class DecoderConfig:
     rope_high: float = 4.0  # high_freq_factor
     rope_orig: int = 8192  # original_max_position_embeddings
     act: str = "silu"  # hidden_act of the gated MLP: "silu" or "gelu_tanh"
+    qk_norm: bool = False  # per-head RMSNorm of q and k before RoPE (Qwen3-family layers)
 
     @staticmethod
     def from_dict(c: dict) -> "DecoderConfig":
@@ -103,7 +108,8 @@ class DecoderConfig:
                              bias=bool(c["bias"]), theta=float(c["theta"]), eps=float(c["eps"]),
                              window=int(c.get("window", 0)), rope_factor=float(c.get("rope_factor", 0.0)),
                              rope_low=float(c.get("rope_low", 1.0)), rope_high=float(c.get("rope_high", 4.0)),
-                             rope_orig=int(c.get("rope_orig", 8192)), act=str(c.get("act", "silu")))
+                             rope_orig=int(c.get("rope_orig", 8192)), act=str(c.get("act", "silu")),
+                             qk_norm=bool(c.get("qk_norm", False)))
 
     def rope_scaling(self):
         """(factor, low_freq_factor, high_freq_factor, original context), or None."""
@@ -376,6 +382,9 @@ class Oracle:
             q = linear(h, self._w(p + "self_attn.q_proj.weight"), bq).reshape(B, S, c.H, c.d)
             k = linear(h, self._w(p + "self_attn.k_proj.weight"), bk).reshape(B, S, c.G, c.d)
             v = linear(h, self._w(p + "self_attn.v_proj.weight"), bv).reshape(B, S, c.G, c.d)
+            if c.qk_norm:  # NN.rmsnorm over each head's d values, gains q_norm / k_norm
+                q = rmsnorm(q, self._w(p + "self_attn.q_norm.weight"), c.eps)
+                k = rmsnorm(k, self._w(p + "self_attn.k_norm.weight"), c.eps)
             q = rope(q, pos[:, :, None], c.theta, c.rope_scaling())
             k = rope(k, pos[:, :, None], c.theta, c.rope_scaling())
             o = np.empty((B, S, c.H, c.d))

@@ -47,7 +47,8 @@ SEED_WEIGHTS, SEED_IDS, SEED_CTX, SEED_BLOCKS = 0, 1, 2, 3
 
 
 def weight_shapes(m: dict) -> dict:
-    """HF Llama parameter names and shapes ([out, in] for matrices)."""
+    """HF Llama parameter names and shapes ([out, in] for matrices); with
+    qk_norm, the per-head q and k RMSNorm gains of Qwen3-family layers."""
     L, D, H, G, d, F, V = (m[k] for k in ("L", "D", "H", "G", "d", "F", "V"))
     shapes = {"model.embed_tokens.weight": (V, D)}
     for l in range(L):
@@ -60,6 +61,9 @@ def weight_shapes(m: dict) -> dict:
             shapes[p + "self_attn.q_proj.bias"] = (H * d,)
             shapes[p + "self_attn.k_proj.bias"] = (G * d,)
             shapes[p + "self_attn.v_proj.bias"] = (G * d,)
+        if m.get("qk_norm"):
+            shapes[p + "self_attn.q_norm.weight"] = (d,)
+            shapes[p + "self_attn.k_norm.weight"] = (d,)
         shapes[p + "self_attn.o_proj.weight"] = (D, H * d)
         shapes[p + "post_attention_layernorm.weight"] = (D,)
         shapes[p + "mlp.gate_proj.weight"] = (F, D)
@@ -84,7 +88,7 @@ def make_weights(m: dict, seed: int = SEED_WEIGHTS, device="cpu") -> dict:
         g.manual_seed(_tensor_seed(seed, name))
         t = torch.empty(shape, dtype=torch.float32, device=device)
         t.normal_(0.0, 0.02, generator=g)
-        if name.endswith("layernorm.weight") or name == "model.norm.weight":
+        if name.endswith(("layernorm.weight", "q_norm.weight", "k_norm.weight")) or name == "model.norm.weight":
             t += 1.0
         out[name] = t.to(torch.bfloat16)
     return out

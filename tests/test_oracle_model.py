@@ -11,11 +11,13 @@ from oracle import decoder as od
 
 
 def tiny_model(L=2, D=8, H=4, G=2, d=4, F=12, V=16, tie=False, bias=True, theta=100.0, eps=1e-5, seed=0, window=0,
-               act="silu"):
-    m = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=bias, theta=theta, eps=eps, window=window, act=act)
+               act="silu", qk_norm=False):
+    m = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=bias, theta=theta, eps=eps, window=window, act=act,
+             qk_norm=qk_norm)
     w = si.weights_as_f32_numpy(si.make_weights(m, seed=seed))
     # Large-ish weights so that every term matters at tiny widths.
-    w = {k: (v if k.endswith("layernorm.weight") or k == "model.norm.weight" else v * 20.0)
+    w = {k: (v if k.endswith(("layernorm.weight", "q_norm.weight", "k_norm.weight")) or k == "model.norm.weight"
+             else v * 20.0)
          for k, v in w.items()}
     return od.DecoderConfig.from_dict(m), w
 
@@ -62,8 +64,13 @@ def _bf_forward(cfg, W, ids):
             q = lin(h, W[p + "self_attn.q_proj.weight"], W.get(p + "self_attn.q_proj.bias"))
             k = lin(h, W[p + "self_attn.k_proj.weight"], W.get(p + "self_attn.k_proj.bias"))
             v = lin(h, W[p + "self_attn.v_proj.weight"], W.get(p + "self_attn.v_proj.bias"))
-            qs.append([rot(q[hh * d:(hh + 1) * d], s) for hh in range(H)])
-            ks.append([rot(k[g * d:(g + 1) * d], s) for g in range(G)])
+            qh = [q[hh * d:(hh + 1) * d] for hh in range(H)]
+            kh = [k[g * d:(g + 1) * d] for g in range(G)]
+            if cfg.qk_norm:
+                qh = [rms(v_, W[p + "self_attn.q_norm.weight"]) for v_ in qh]
+                kh = [rms(v_, W[p + "self_attn.k_norm.weight"]) for v_ in kh]
+            qs.append([rot(v_, s) for v_ in qh])
+            ks.append([rot(v_, s) for v_ in kh])
             vs.append([v[g * d:(g + 1) * d] for g in range(G)])
         new_x = []
         for s in range(S):
@@ -95,11 +102,12 @@ def _bf_forward(cfg, W, ids):
     return [lin(rms(x, W["model.norm.weight"]), head) for x in xs]
 
 
-@pytest.mark.parametrize("tie,bias,H,G,window,act", [(False, True, 4, 2, 0, "silu"), (True, False, 2, 2, 0, "silu"),
-                                                     (False, False, 4, 1, 0, "silu"), (False, True, 4, 2, 2, "silu"),
-                                                     (True, False, 2, 2, 3, "silu"), (False, True, 4, 2, 0, "gelu_tanh")])
-def test_oracle_matches_bruteforce_loops(tie, bias, H, G, window, act):
-    cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8, window=window, act=act)
+@pytest.mark.parametrize("tie,bias,H,G,window,act,qkn", [
+    (False, True, 4, 2, 0, "silu", False), (True, False, 2, 2, 0, "silu", False), (False, False, 4, 1, 0, "silu", False),
+    (False, True, 4, 2, 2, "silu", False), (True, False, 2, 2, 3, "silu", False),
+    (False, True, 4, 2, 0, "gelu_tanh", False), (False, True, 4, 2, 0, "silu", True)])
+def test_oracle_matches_bruteforce_loops(tie, bias, H, G, window, act, qkn):
+    cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8, window=window, act=act, qk_norm=qkn)
     ids = [3, 15, 0, 7, 7]
     ref = np.array(_bf_forward(cfg, W, ids))
     o = od.Oracle(cfg, W)
@@ -183,6 +191,36 @@ def test_rope_scaling_changes_only_positions_beyond_zero_and_factor_one_is_off()
     scaled = run(dict(rope_factor=8.0, rope_low=1.0, rope_high=4.0, rope_orig=64))
     assert np.allclose(scaled[:, 0], plain[:, 0], rtol=1e-12, atol=1e-12)  # position 0: no rotation at all
     assert not np.allclose(scaled[:, 1:], plain[:, 1:])
+
+
+def test_qk_norm_makes_logits_invariant_to_the_scale_of_q_and_k_projections():
+    # per-head RMSNorm of q and k removes any positive scale of their
+    # projections (bias off, eps negligible against the scaled norms)
+    cfg, W = tiny_model(qk_norm=True, bias=False, eps=1e-12)
+    ids = np.array([[5, 1, 2, 11, 3, 8]])
+    o = od.Oracle(cfg, W)
+    base = o.prefill(ids, o.new_contiguous_cache(1, 8))
+    W2 = dict(W)
+    for l in range(cfg.L):
+        W2[f"model.layers.{l}.self_attn.q_proj.weight"] = W[f"model.layers.{l}.self_attn.q_proj.weight"] * 7.0
+        W2[f"model.layers.{l}.self_attn.k_proj.weight"] = W[f"model.layers.{l}.self_attn.k_proj.weight"] * 0.25
+    o2 = od.Oracle(cfg, W2)
+    assert np.allclose(o2.prefill(ids, o2.new_contiguous_cache(1, 8)), base, rtol=1e-10, atol=1e-10)
+    cfg0, _ = tiny_model(qk_norm=False, bias=False, eps=1e-12)  # without it the scale matters
+    a = od.Oracle(cfg0, W).prefill(ids, od.Oracle(cfg0, W).new_contiguous_cache(1, 8))
+    b = od.Oracle(cfg0, W2).prefill(ids, od.Oracle(cfg0, W2).new_contiguous_cache(1, 8))
+    assert not np.allclose(a, b)
+
+
+def test_qk_norm_decode_equals_full_recompute():
+    cfg, W = tiny_model(qk_norm=True)
+    o = od.Oracle(cfg, W)
+    ids = np.array([[5, 1, 2, 11, 3, 8, 0, 14]])
+    full = o.prefill(ids, o.new_contiguous_cache(1, 8))
+    cache = o.new_contiguous_cache(1, 8)
+    o.prefill(ids[:, :3], cache)
+    for t in range(3, 8):
+        assert np.allclose(o.decode_step(ids[:, t], cache, np.array([t])), full[:, t], rtol=1e-12, atol=1e-12)
 
 
 def test_paged_cache_is_bit_identical_to_contiguous():
