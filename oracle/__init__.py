@@ -10,6 +10,9 @@ built-in operation it restates. The paper names the operations (NN.rmsnorm,
 NN.linear, Attention.attention with grouped-query heads, Positions with
 past_length, Cache.update/append, Act.swiglu) but prints no formulas for them;
 the readings taken where it is silent are listed in `decoder.READINGS`.
+`gpt2` holds the GPT-2 causal LM of the paper's complete model definition
+(LayerNorm, learned positions, fused biased projections, gelu_new MLP), with
+its own READINGS.
 """
 from .decoder import (  # noqa: F401
     DecoderConfig,

@@ -75,6 +75,44 @@ def weight_shapes(m: dict) -> dict:
     return shapes
 
 
+def gpt2_weight_shapes(c: dict) -> dict:
+    """HF GPT-2 parameter names and shapes (the appendix's complete model):
+    `transpose=true` matrices stored [in, out]; keys L, D, V, P (positions)."""
+    L, D, V, P = int(c["L"]), int(c["D"]), int(c["V"]), int(c["P"])
+    s = {"transformer.wte.weight": (V, D), "transformer.wpe.weight": (P, D)}
+    for l in range(L):
+        p = f"transformer.h.{l}."
+        for ln in ("ln_1", "ln_2"):
+            s[p + ln + ".weight"] = (D,)
+            s[p + ln + ".bias"] = (D,)
+        s[p + "attn.c_attn.weight"] = (D, 3 * D)
+        s[p + "attn.c_attn.bias"] = (3 * D,)
+        s[p + "attn.c_proj.weight"] = (D, D)
+        s[p + "attn.c_proj.bias"] = (D,)
+        s[p + "mlp.c_fc.weight"] = (D, 4 * D)
+        s[p + "mlp.c_fc.bias"] = (4 * D,)
+        s[p + "mlp.c_proj.weight"] = (4 * D, D)
+        s[p + "mlp.c_proj.bias"] = (D,)
+    s["transformer.ln_f.weight"] = (D,)
+    s["transformer.ln_f.bias"] = (D,)
+    return s
+
+
+def make_gpt2_weights(c: dict, seed: int = SEED_WEIGHTS, device="cpu") -> dict:
+    """bf16 GPT-2 tensors by HF name: LayerNorm gains 1 + N(0, 0.02), every
+    other tensor (matrices, embeddings, biases) N(0, 0.02)."""
+    out = {}
+    for name, shape in gpt2_weight_shapes(c).items():
+        g = torch.Generator(device=device)
+        g.manual_seed(_tensor_seed(seed, name))
+        t = torch.empty(shape, dtype=torch.float32, device=device)
+        t.normal_(0.0, 0.02, generator=g)
+        if ".ln_" in name and name.endswith(".weight"):
+            t += 1.0
+        out[name] = t.to(torch.bfloat16)
+    return out
+
+
 def _tensor_seed(seed: int, name: str) -> int:
     return (seed * 1_000_003 + zlib.crc32(name.encode())) & 0x7FFF_FFFF_FFFF
 
