@@ -69,3 +69,33 @@ def test_config_struct_layout_matches_header():
         fields += [p.strip(",") for p in " ".join(parts[1:]).split(",")]
     assert [f[0] for f in ax.axon_config._fields_] == [f.strip() for f in fields]
     assert names
+
+
+def test_invalid_configs_are_rejected_before_any_device_work(built):
+    """axon_model_create validates the config on the host before its first
+    CUDA call, so every rejection below runs without a GPU."""
+    import ctypes as C
+    ax = built
+    shape = dict(L=1, D=128, H=4, G=2, d=64, F=192, V=100, tie=True, bias=False, theta=1e4, eps=1e-5)
+    cases = [
+        (dict(sliding_window=-1), ax.AXON_ERR_INVALID_ARG),
+        (dict(hidden_act=5), ax.AXON_ERR_INVALID_ARG),
+        (dict(rope_scaling_factor=8.0, rope_low_freq_factor=4.0, rope_high_freq_factor=1.0,
+              rope_original_max_position=8192), ax.AXON_ERR_INVALID_ARG),
+        (dict(rope_scaling_factor=-1.0), ax.AXON_ERR_INVALID_ARG),
+        (dict(precision=7), ax.AXON_ERR_INVALID_ARG),
+        (dict(kv_layout=ax.AXON_KV_PAGED, kv_num_blocks=0), ax.AXON_ERR_INVALID_ARG),
+        (dict(head_dim=96), ax.AXON_ERR_UNSUPPORTED),
+        (dict(num_key_value_heads=3), ax.AXON_ERR_UNSUPPORTED),
+        (dict(kv_block_size=32), ax.AXON_ERR_UNSUPPORTED),
+        (dict(max_context=100), ax.AXON_ERR_UNSUPPORTED),
+        (dict(hidden_size=100), ax.AXON_ERR_UNSUPPORTED),
+    ]
+    for change, want in cases:
+        cfg = ax.make_config(shape, max_batch=2, max_context=128)
+        for k, v in change.items():
+            setattr(cfg, k, v)
+        out = C.c_void_p(1234)
+        rc = ax.lib().axon_model_create(C.byref(cfg), None, 0, None, C.byref(out))
+        assert rc == want, (change, rc)
+        assert out.value is None, change
