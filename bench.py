@@ -41,22 +41,35 @@ def model_bytes(m):
     return lin, V * D
 
 
+def keys_seen(pos, window):
+    """Keys a query at position pos attends to: pos + 1, or at most the
+    sliding window."""
+    return pos + 1 if not window else min(pos + 1, window)
+
+
+def keys_seen_by_run(past, n, window):
+    """Sum of keys_seen over positions past .. past + n - 1."""
+    if not window:
+        return n * past + n * (n + 1) / 2
+    return sum(keys_seen(p, window) for p in range(past, past + n))
+
+
 def decode_bytes_per_step(m, B, T_list):
     """Algorithmic HBM bytes of one decode step: every weight once (bf16),
-    norms/biases, KV read of all cached tokens + the new token, KV write,
-    fp32 logits write."""
+    norms/biases, KV read of the keys each new token sees (all cached tokens
+    + itself, or its sliding window), KV write, fp32 logits write."""
     lin, head = model_bytes(m)
     L, D, G, d, V = m["L"], m["D"], m["G"], m["d"], m["V"]
     small = (2 * L + 1) * D * 4 + (L * (m["H"] + 2 * G) * d * 4 if m["bias"] else 0)
     kv_tok = L * 2 * G * d * 2
-    kv_read = sum(int(t) + 1 for t in T_list) * kv_tok
+    kv_read = sum(keys_seen(int(t), m.get("window", 0)) for t in T_list) * kv_tok
     kv_write = B * kv_tok
     return 2 * (lin + head) + small + kv_read + kv_write + B * V * 4
 
 
 def prefill_flops(m, B, S):
     lin, head = model_bytes(m)
-    attn = m["L"] * B * 4 * m["H"] * m["d"] * S * (S + 1) / 2
+    attn = m["L"] * B * 4 * m["H"] * m["d"] * keys_seen_by_run(0, S, m.get("window", 0))
     return 2 * B * S * lin + attn + 2 * B * head
 
 
@@ -287,7 +300,7 @@ def varlen_prefill_flops(m, calls):
     total = 0.0
     for chunks in calls:
         T = sum(n for _, n in chunks)
-        keys = sum(n * past + n * (n + 1) / 2 for past, n in chunks)
+        keys = sum(keys_seen_by_run(past, n, m.get("window", 0)) for past, n in chunks)
         total += 2 * T * lin + m["L"] * 4 * m["H"] * m["d"] * keys + 2 * len(chunks) * head
     return total
 

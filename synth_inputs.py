@@ -30,6 +30,9 @@ MODEL_SHAPES = {
     "0.5b": dict(L=24, D=896, H=14, G=2, d=64, F=4864, V=151936, tie=True, bias=True, theta=1e6, eps=1e-6),
     "8b": dict(L=32, D=4096, H=32, G=8, d=128, F=14336, V=128256, tie=False, bias=False, theta=5e5, eps=1e-5),
     "32b": dict(L=64, D=5120, H=40, G=8, d=128, F=27648, V=152064, tie=False, bias=True, theta=1e6, eps=1e-6),
+    # Mistral-shaped 7B: the Llama block with a 4096-token sliding window
+    "7b_swa": dict(L=32, D=4096, H=32, G=8, d=128, F=14336, V=32000, tie=False, bias=False, theta=1e4, eps=1e-5,
+                   window=4096),
 }
 
 # Workloads: prompt batch and length, decode steps, cache layout.
@@ -41,6 +44,8 @@ WORKLOADS = {
     "8b_paged_b64_ctx512-4096_n128": dict(model="8b", B=64, ctx=(512, 4096), n_new=128, layout="paged"),
     "32b_b1_s2048_n256": dict(model="32b", B=1, S=2048, n_new=256, layout="contiguous"),
     "32b_b16_s2048_n256": dict(model="32b", B=16, S=2048, n_new=256, layout="contiguous"),
+    # prompt twice the window: the window bounds prefill attention and every decode step's keys
+    "7b_swa_b1_s8192_n256": dict(model="7b_swa", B=1, S=8192, n_new=256, layout="contiguous"),
 }
 
 SEED_WEIGHTS, SEED_IDS, SEED_CTX, SEED_BLOCKS = 0, 1, 2, 3

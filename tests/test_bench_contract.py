@@ -102,3 +102,16 @@ def test_varlen_prefill_flops_by_hand():
     # 3 new tokens after 4 cached ones attend 5 + 6 + 7 keys; a 1-token chunk after 9 attends 10
     want = 2 * 4 * lin + 2 * 4 * 4 * 16 * (5 + 6 + 7 + 10) + 2 * 2 * head
     assert bench.varlen_prefill_flops(SHAPE, [[(4, 3), (9, 1)]]) == want
+
+
+def test_sliding_window_counts_only_the_visible_keys():
+    W = dict(SHAPE, window=3)
+    lin, head = bench.model_bytes(SHAPE)
+    kv_tok = 2 * 2 * 2 * 16 * 2
+    # new tokens at positions 5 and 1: 3 and 2 keys visible
+    assert bench.decode_bytes_per_step(W, 2, [5, 1]) - bench.decode_bytes_per_step(SHAPE, 2, [5, 1]) == \
+        (3 + 2 - 6 - 2) * kv_tok
+    # a 7-token prompt sees 1 + 2 + 3 + 3 + 3 + 3 + 3 keys
+    assert bench.prefill_flops(W, 1, 7) == 2 * 7 * lin + 2 * 4 * 4 * 16 * 18 + 2 * head
+    assert bench.varlen_prefill_flops(W, [[(4, 3)]]) == 2 * 3 * lin + 2 * 4 * 4 * 16 * 9 + 2 * head
+    assert bench.keys_seen_by_run(4, 3, 0) == 5 + 6 + 7
