@@ -280,11 +280,13 @@ def test_varlen_equals_batched_forward_for_equal_lengths():
         assert np.allclose(got[b], ref[b], rtol=0, atol=1e-12)
 
 
-def test_varlen_chunks_equal_one_prompt_and_mixed_decode():
+@pytest.mark.parametrize("window", [0, 2, 5])
+def test_varlen_chunks_equal_one_prompt_and_mixed_decode(window):
     """Prompts cut into chunks of different lengths (one of them a single
     decode-like token) give the logits of the whole prompts, paged cache with
-    shuffled blocks included."""
-    cfg, W = tiny_model()
+    shuffled blocks included; under a sliding window narrower and wider than
+    the chunks too."""
+    cfg, W = tiny_model(window=window)
     o = od.Oracle(cfg, W)
     rng = np.random.default_rng(4)
     lens = [7, 4, 9]
