@@ -1,0 +1,130 @@
+"""Loading a Hugging Face checkpoint directory into the C ABI's inputs.
+
+The model definition and "a standard safetensors checkpoint" go in (Fig. 1;
+appendix "A Complete Model Definition"). This module reads the two files a
+checkpoint directory holds for that:
+
+* `config.json` -> the shape dict that `make_config` takes (HF key names);
+* `*.safetensors` (one file, or shards listed by
+  `model.safetensors.index.json`) -> {HF tensor name: torch tensor}, parsed
+  here directly: an 8-byte little-endian header length, a JSON header of
+  {name: {dtype, shape, data_offsets}}, then the raw little-endian bytes.
+
+Only what `axon_model_create` accepts is returned: bf16 and fp32 tensors pass
+through; fp16 tensors are widened to fp32 (exact). Host memory only; the
+create call copies and repacks on the device.
+"""
+from __future__ import annotations
+
+import json
+import os
+import struct
+
+import numpy as np
+
+_DTYPES = {"BF16": (np.uint16, 2), "F16": (np.float16, 2), "F32": (np.float32, 4)}
+
+
+def read_safetensors(path: str, names=None) -> dict:
+    """{name: torch tensor} of one .safetensors file (bf16 / fp16 / fp32),
+    optionally restricted to `names`."""
+    import torch
+    with open(path, "rb") as f:
+        (n,) = struct.unpack("<Q", f.read(8))
+        header = json.loads(f.read(n).decode("utf-8"))
+        base = 8 + n
+        out = {}
+        for name, meta in header.items():
+            if name == "__metadata__" or (names is not None and name not in names):
+                continue
+            dt = meta["dtype"]
+            if dt not in _DTYPES:
+                raise ValueError(f"{path}: tensor {name} has unsupported dtype {dt}")
+            np_t, size = _DTYPES[dt]
+            start, end = meta["data_offsets"]
+            shape = tuple(int(s) for s in meta["shape"])
+            count = int(np.prod(shape)) if shape else 1
+            if end - start != count * size:
+                raise ValueError(f"{path}: tensor {name}: {end - start} bytes for shape {shape}")
+            f.seek(base + start)
+            arr = np.frombuffer(f.read(end - start), dtype=np.dtype(np_t).newbyteorder("<")).reshape(shape)
+            if dt == "BF16":
+                t = torch.from_numpy(arr.astype(np.uint16).view(np.int16).copy()).view(torch.bfloat16)
+            else:  # fp16 widens exactly; fp32 passes through
+                t = torch.from_numpy(arr.astype(np.float32))
+            out[name] = t
+    return out
+
+
+def read_checkpoint(directory: str) -> dict:
+    """Every tensor of a checkpoint directory: `model.safetensors`, or the
+    shards named by `model.safetensors.index.json`."""
+    index = os.path.join(directory, "model.safetensors.index.json")
+    if os.path.exists(index):
+        with open(index) as f:
+            weight_map = json.load(f)["weight_map"]
+        out = {}
+        for shard in sorted(set(weight_map.values())):
+            names = {k for k, v in weight_map.items() if v == shard}
+            out.update(read_safetensors(os.path.join(directory, shard), names))
+        return out
+    single = os.path.join(directory, "model.safetensors")
+    if not os.path.exists(single):
+        raise FileNotFoundError(f"{directory}: no model.safetensors or model.safetensors.index.json")
+    return read_safetensors(single)
+
+
+def shape_from_hf_config(c: dict) -> dict:
+    """The shape dict of `make_config` from an HF config.json of a
+    Llama-family decoder (Llama, Mistral, Qwen2, SmolLM, ...). Raises on a
+    model this library does not implement."""
+    mt = c.get("model_type", "llama")
+    if mt not in ("llama", "mistral", "qwen2"):
+        raise ValueError(f"model_type {mt!r} is not a Llama-family decoder this library implements")
+    H = int(c["num_attention_heads"])
+    D = int(c["hidden_size"])
+    shape = dict(L=int(c["num_hidden_layers"]), D=D, H=H, G=int(c.get("num_key_value_heads", H)),
+                 d=int(c.get("head_dim") or D // H), F=int(c["intermediate_size"]), V=int(c["vocab_size"]),
+                 tie=bool(c.get("tie_word_embeddings", False)),
+                 bias=bool(c.get("attention_bias", mt == "qwen2")),
+                 theta=float(c.get("rope_theta", 10000.0)), eps=float(c.get("rms_norm_eps", 1e-6)))
+    if c.get("mlp_bias"):
+        raise ValueError("MLP biases are not implemented")
+    act = c.get("hidden_act", "silu")
+    if act in ("gelu_pytorch_tanh", "gelu_new"):
+        shape["act"] = "gelu_tanh"
+    elif act != "silu":
+        raise ValueError(f"hidden_act {act!r} is not implemented")
+    window = c.get("sliding_window")
+    if window and mt == "mistral":
+        shape["window"] = int(window)
+    elif window and c.get("use_sliding_window", False):
+        # Qwen2 windows the layers from max_window_layers on
+        first = int(c.get("max_window_layers", 0))
+        if 0 < first < shape["L"]:
+            raise ValueError("a sliding window on only some layers is not implemented")
+        if first <= 0:
+            shape["window"] = int(window)
+    rs = c.get("rope_scaling")
+    if rs:
+        kind = rs.get("rope_type", rs.get("type"))
+        if kind != "llama3":
+            raise ValueError(f"rope_scaling {kind!r} is not implemented")
+        shape.update(rope_factor=float(rs["factor"]), rope_low=float(rs["low_freq_factor"]),
+                     rope_high=float(rs["high_freq_factor"]),
+                     rope_orig=int(rs["original_max_position_embeddings"]))
+    return shape
+
+
+def load_model(directory: str, max_batch: int, max_context: int, **config_kw):
+    """(model handle, shape dict) from a checkpoint directory: the config is
+    read, the tensors are read to host memory, and axon_model_create copies
+    them to the device. config_kw go to make_config (layout, precision, ...)."""
+    from . import axon_model_create, make_config
+    with open(os.path.join(directory, "config.json")) as f:
+        shape = shape_from_hf_config(json.load(f))
+    weights = read_checkpoint(directory)
+    if shape["tie"]:
+        weights.pop("lm_head.weight", None)
+    cfg = make_config(shape, max_batch=max_batch, max_context=max_context, **config_kw)
+    return axon_model_create(cfg, weights), shape

@@ -1,0 +1,122 @@
+"""Checkpoint loading on the host: the hand-written safetensors reader (single
+file and sharded index, bf16 / fp16 / fp32) against tensors written here, and
+the HF config.json mapping of the Llama-family variants the kernels implement."""
+import json
+import struct
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import synth_inputs as si  # noqa: E402
+from paper_2608_19889_gb300 import checkpoint as ck  # noqa: E402
+
+
+def _write_safetensors(path, tensors):
+    """Minimal writer: header of dtype / shape / byte offsets, then the data."""
+    header, blobs, off = {}, [], 0
+    for name, t in tensors.items():
+        if t.dtype == torch.bfloat16:
+            raw, dt = t.view(torch.int16).numpy().astype("<i2").tobytes(), "BF16"
+        elif t.dtype == torch.float16:
+            raw, dt = t.numpy().astype("<f2").tobytes(), "F16"
+        else:
+            raw, dt = t.numpy().astype("<f4").tobytes(), "F32"
+        header[name] = {"dtype": dt, "shape": list(t.shape), "data_offsets": [off, off + len(raw)]}
+        blobs.append(raw)
+        off += len(raw)
+    header["__metadata__"] = {"format": "pt"}
+    h = json.dumps(header).encode()
+    with open(path, "wb") as f:
+        f.write(struct.pack("<Q", len(h)))
+        f.write(h)
+        for b in blobs:
+            f.write(b)
+
+
+def test_reader_returns_the_written_tensors_in_every_dtype(tmp_path):
+    g = torch.Generator().manual_seed(0)
+    ts = {"a.bf16": torch.randn(3, 5, generator=g).to(torch.bfloat16),
+          "b.f16": torch.randn(7, generator=g).to(torch.float16),
+          "c.f32": torch.randn(2, 2, 2, generator=g)}
+    _write_safetensors(tmp_path / "x.safetensors", ts)
+    got = ck.read_safetensors(str(tmp_path / "x.safetensors"))
+    assert set(got) == set(ts)
+    assert got["a.bf16"].dtype == torch.bfloat16 and torch.equal(got["a.bf16"], ts["a.bf16"])
+    assert got["b.f16"].dtype == torch.float32 and torch.equal(got["b.f16"], ts["b.f16"].float())  # exact widening
+    assert torch.equal(got["c.f32"], ts["c.f32"])
+
+
+def test_sharded_checkpoint_reads_every_tensor_once(tmp_path):
+    m = dict(L=2, D=64, H=4, G=2, d=16, F=96, V=50, tie=False, bias=True, theta=1e4, eps=1e-5)
+    w = si.make_weights(m)
+    names = sorted(w)
+    shards = {"model-00001-of-00002.safetensors": names[: len(names) // 2],
+              "model-00002-of-00002.safetensors": names[len(names) // 2:]}
+    weight_map = {}
+    for shard, ns in shards.items():
+        _write_safetensors(tmp_path / shard, {n: w[n] for n in ns})
+        weight_map.update({n: shard for n in ns})
+    with open(tmp_path / "model.safetensors.index.json", "w") as f:
+        json.dump({"metadata": {}, "weight_map": weight_map}, f)
+    got = ck.read_checkpoint(str(tmp_path))
+    assert set(got) == set(si.weight_shapes(m))
+    assert all(torch.equal(got[n], w[n]) for n in names)
+
+
+def test_truncated_tensor_is_rejected(tmp_path):
+    _write_safetensors(tmp_path / "x.safetensors", {"a": torch.zeros(4)})
+    raw = bytearray((tmp_path / "x.safetensors").read_bytes())
+    (n,) = struct.unpack("<Q", raw[:8])
+    hdr = json.loads(raw[8:8 + n])
+    hdr["a"]["shape"] = [5]  # 20 bytes expected, 16 stored
+    h = json.dumps(hdr).encode()
+    (tmp_path / "y.safetensors").write_bytes(struct.pack("<Q", len(h)) + h + raw[8 + n:])
+    with pytest.raises(ValueError):
+        ck.read_safetensors(str(tmp_path / "y.safetensors"))
+
+
+LLAMA31 = {"model_type": "llama", "num_hidden_layers": 32, "hidden_size": 4096, "num_attention_heads": 32,
+           "num_key_value_heads": 8, "intermediate_size": 14336, "vocab_size": 128256, "rope_theta": 500000.0,
+           "rms_norm_eps": 1e-5, "tie_word_embeddings": False, "hidden_act": "silu",
+           "rope_scaling": {"rope_type": "llama3", "factor": 8.0, "low_freq_factor": 1.0, "high_freq_factor": 4.0,
+                            "original_max_position_embeddings": 8192}}
+
+
+def test_llama_config_with_rope_scaling():
+    s = ck.shape_from_hf_config(LLAMA31)
+    assert (s["L"], s["D"], s["H"], s["G"], s["d"], s["F"], s["V"]) == (32, 4096, 32, 8, 128, 14336, 128256)
+    assert s["tie"] is False and s["bias"] is False and s["theta"] == 5e5 and s["eps"] == 1e-5
+    assert (s["rope_factor"], s["rope_low"], s["rope_high"], s["rope_orig"]) == (8.0, 1.0, 4.0, 8192)
+    assert "window" not in s and s.get("act", "silu") == "silu"
+
+
+def test_qwen2_has_qkv_bias_and_mistral_its_window():
+    q = dict(LLAMA31, model_type="qwen2", rope_scaling=None, tie_word_embeddings=True, use_sliding_window=False,
+             sliding_window=32768)
+    s = ck.shape_from_hf_config(q)
+    assert s["bias"] is True and s["tie"] is True and "window" not in s
+    m = dict(LLAMA31, model_type="mistral", rope_scaling=None, sliding_window=4096)
+    assert ck.shape_from_hf_config(m)["window"] == 4096
+    assert "window" not in ck.shape_from_hf_config(dict(m, sliding_window=None))
+    qw = dict(q, use_sliding_window=True, sliding_window=4096)
+    assert ck.shape_from_hf_config(dict(qw, max_window_layers=0))["window"] == 4096  # every layer windowed
+    assert "window" not in ck.shape_from_hf_config(dict(qw, max_window_layers=32))  # no layer windowed
+
+
+def test_gelu_gate_and_unsupported_configs():
+    assert ck.shape_from_hf_config(dict(LLAMA31, rope_scaling=None, hidden_act="gelu_pytorch_tanh"))["act"] == \
+        "gelu_tanh"
+    for bad in (dict(LLAMA31, model_type="gpt2"), dict(LLAMA31, hidden_act="relu"),
+                dict(LLAMA31, rope_scaling={"rope_type": "yarn", "factor": 4.0}), dict(LLAMA31, mlp_bias=True),
+                dict(LLAMA31, model_type="qwen2", use_sliding_window=True, sliding_window=4096,
+                     max_window_layers=28)):
+        with pytest.raises(ValueError):
+            ck.shape_from_hf_config(bad)
+
+
+def test_head_dim_defaults_to_width_over_heads():
+    c = {k: v for k, v in LLAMA31.items() if k != "rope_scaling"}
+    assert ck.shape_from_hf_config(c)["d"] == 128
+    assert ck.shape_from_hf_config(dict(c, head_dim=64))["d"] == 64
