@@ -30,9 +30,9 @@ AXON_DTYPE_BF16, AXON_DTYPE_F32 = 0, 1
 AXON_LOGITS_LAST, AXON_LOGITS_ALL = 0, 1
 AXON_ACT_SILU, AXON_ACT_GELU_TANH = 0, 1
 
-EXPORTED = ["axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset", "axon_check_device",
-            "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill", "axon_decode_step_noalloc",
-            "axon_free", "axon_status_string"]
+EXPORTED = ["axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset",
+            "axon_check_device", "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill",
+            "axon_decode_step_noalloc", "axon_free", "axon_status_string"]
 
 
 class axon_config(ctypes.Structure):
@@ -94,8 +94,8 @@ def lib() -> ctypes.CDLL:
         L.axon_free.restype = None
         L.axon_status_string.argtypes = [ctypes.c_int]
         L.axon_status_string.restype = ctypes.c_char_p
-        for n in ("axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset", "axon_check_device",
-                  "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill",
+        for n in ("axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset",
+                  "axon_check_device", "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill",
                   "axon_decode_step_noalloc"):
             getattr(L, n).restype = ctypes.c_int
         _lib = L

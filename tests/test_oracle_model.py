@@ -103,8 +103,8 @@ def _bf_forward(cfg, W, ids):
 
 
 @pytest.mark.parametrize("tie,bias,H,G,window,act,qkn", [
-    (False, True, 4, 2, 0, "silu", False), (True, False, 2, 2, 0, "silu", False), (False, False, 4, 1, 0, "silu", False),
-    (False, True, 4, 2, 2, "silu", False), (True, False, 2, 2, 3, "silu", False),
+    (False, True, 4, 2, 0, "silu", False), (True, False, 2, 2, 0, "silu", False),
+    (False, False, 4, 1, 0, "silu", False), (False, True, 4, 2, 2, "silu", False), (True, False, 2, 2, 3, "silu", False),
     (False, True, 4, 2, 0, "gelu_tanh", False), (False, True, 4, 2, 0, "silu", True)])
 def test_oracle_matches_bruteforce_loops(tie, bias, H, G, window, act, qkn):
     cfg, W = tiny_model(tie=tie, bias=bias, H=H, G=G, d=4, D=8, window=window, act=act, qk_norm=qkn)
