@@ -295,10 +295,13 @@ int axon_profile_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t
  * allocated per call. It calls no cudaMalloc, cudaFree or graph
  * instantiation.
  *   Limits: B * num_key_value_heads <= 256 and head_dim <= 128, else
- *   AXON_ERR_UNSUPPORTED; bf16 precision only (AXON_ERR_UNSUPPORTED in
- *   AXON_FP32_DEBUG).
- *   First call on a device: resolves the array's device address (with that
- *   device current) -- make that first call before any stream capture.
+ *   AXON_ERR_UNSUPPORTED; the 16-bit modes AXON_BF16 and AXON_FP16 only
+ *   (AXON_ERR_UNSUPPORTED in AXON_FP32_DEBUG). The attention keeps at most
+ *   256 / (B * num_key_value_heads) key splits per sequence and kv head.
+ *   First call on a device (and the first after the device's context was
+ *   torn down, e.g. by cudaDeviceReset): resolves the array's device address
+ *   in the current context, with that device current -- make that first
+ *   call before any stream capture.
  *   Every call shares the one array and clears the parts that must start
  *   at zero: calls that overlap on the GPU (different streams, or several
  *   models at once) race on it and must be serialised by the caller.

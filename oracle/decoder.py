@@ -362,10 +362,12 @@ class Oracle:
         c = self.cfg
         return PagedKV(c.L, num_blocks, block_size, c.G, c.d, block_table)
 
-    def forward(self, ids, cache, past_lens, last_hidden_only=False):
+    def forward(self, ids, cache, past_lens, last_hidden_only=False, rows=None):
         """One pass over new tokens ids [B, S] whose sequence b already holds
         past_lens[b] cached tokens. Writes their K, V into the cache
-        (Cache.update / Cache.append) and returns logits [B, S, V]."""
+        (Cache.update / Cache.append) and returns logits [B, S, V]; with
+        `rows` (indices into the S new tokens) only those positions go
+        through the final norm and LM head: logits [B, len(rows), V]."""
         c = self.cfg
         ids = np.asarray(ids, dtype=np.int64)
         B, S = ids.shape
@@ -399,14 +401,16 @@ class Oracle:
             x = x + linear(u, self._w(p + "mlp.down_proj.weight"))
         if last_hidden_only:
             x = x[:, -1:, :]
+        elif rows is not None:
+            x = x[:, np.asarray(rows, dtype=np.int64), :]
         head = self._w("model.embed_tokens.weight") if c.tie else self._w("lm_head.weight")
         return linear(rmsnorm(x, self._w("model.norm.weight"), c.eps), head)
 
-    def prefill(self, ids, cache, last_only=False):
-        """Prompt pass from an empty cache; logits for every position, or for
-        the last one only."""
+    def prefill(self, ids, cache, last_only=False, rows=None):
+        """Prompt pass from an empty cache; logits for every position, for
+        the last one only, or for the positions listed in `rows`."""
         B = np.asarray(ids).shape[0]
-        return self.forward(ids, cache, np.zeros(B, dtype=np.int64), last_hidden_only=last_only)
+        return self.forward(ids, cache, np.zeros(B, dtype=np.int64), last_hidden_only=last_only, rows=rows)
 
     def decode_step(self, tokens, cache, context_lens):
         """One KV-cached decode step: token b enters at position

@@ -76,6 +76,7 @@ struct axon_model {
   float* x = nullptr;
   void* a = nullptr;
   void* a_lo = nullptr;  // fp16 mode: second term of the normed operand (x*g - a), same layout as a
+  void* q_lo = nullptr;  // 16-bit modes, decode: second term of q (rows 8..15 of the attention tiles)
   void* o_lo = nullptr;  // fp16 mode, decode: second terms of the attention output and the SwiGLU output
   void* u_lo = nullptr;
   float* ss = nullptr;
@@ -91,8 +92,6 @@ struct axon_model {
   void* a_lo_last = nullptr;  // fp16 mode
   float* rinv_last = nullptr;  // [max_batch]
   SplitKWork splitk{};     // decode projections' cross-CTA split-K workspace
-  GemvTmaWork tmawork{};   // TMA stream-K decode projections' workspace
-  CUtensorMap t_a_tok[4]{}, t_o_tok[4]{}, t_u_tok[4]{};  // activation maps, box 64 x {8,16,32,64} rows
   int* ticket = nullptr;   // last-CTA counter of the residual producers
   float* attn_part = nullptr;
   int* attn_cnt = nullptr;
@@ -104,7 +103,6 @@ struct axon_model {
   std::map<GraphKey, cudaGraphExec_t> graphs;
   bool use_graphs = true;
   bool use_pdl = true;
-  bool use_tma_gemv = false;
   // persistent decode step (B <= PERSIST_MAX_B): device layer table, grid
   // barrier state, CTAs per launch (0: not available)
   PersistLayer* players = nullptr;
@@ -427,10 +425,8 @@ struct Proj {
   cudaError_t rc = cudaSuccess;
   // act: activation rows (row stride act_stride elements), M rows. Returns
   // the norm state a RESID producer leaves behind.
-  // vmap: the weight's decode-projection TMA map; amaps: the activation
-  // buffer's maps by token-box size (null: register-streaming GEMV).
   NormState run(int kind, const void* W, const GemmMaps* maps, int N, int K, const void* act, long long act_stride,
-                int M, EpiArgs& ep, const CUtensorMap* vmap = nullptr, const CUtensorMap* amaps = nullptr) {
+                int M, EpiArgs& ep) {
     ep.M = M;
     ep.N = N;
     NormState ns;
@@ -450,12 +446,7 @@ struct Proj {
       ep.ticket = m->ticket;
       ns.rinv = true;
     }
-    if (gemv && !m->fp32 && !m->f16 && vmap && amaps && m->use_tma_gemv) {
-      const int tok = gemv_tma_tokens(M);
-      const int idx = tok == 8 ? 0 : (tok == 16 ? 1 : (tok == 32 ? 2 : 3));
-      rc = launch_gemv_tma(lc, kind, *vmap, amaps[idx], N, K, M, ep, m->tmawork);
-      ns.parts = N / 16;
-    } else if (gemv) {
+    if (gemv) {
       // fp16 mode: consumers of the normed operand `a` also read its
       // second term a_lo
       const void* lo = nullptr;
@@ -631,8 +622,10 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
   return AXON_OK;
 }
 
+// The persistent step's attention always pairs q's two terms in one MMA
+// tile, which needs at most 8 query heads per kv head.
 bool persist_eligible(const axon_model* m, int B) {
-  return m->persist_ctas > 0 && !m->fp32 && persist_fits(m->d, m->f16, B, m->D);
+  return m->persist_ctas > 0 && !m->fp32 && m->H / m->G <= 8 && persist_fits(m->d, m->f16, B, m->D);
 }
 
 PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt,
@@ -669,6 +662,7 @@ PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int3
   a.a_lo = m->a_lo;
   a.ss = m->ss;
   a.q = m->q;
+  a.q_lo = m->q_lo;
   a.o = m->o;
   a.u = m->u;
   a.o_lo = m->o_lo;
@@ -755,9 +749,10 @@ launch_chain:
     set_norm(m, ns, e);
     e.bias = w.bqkv;
     e.q_out = m->q;
+    e.q_lo_out = m->q_lo;
     kv_layout_args(m, l, bt, e);
     pbeg(pf, "decode_qkv");
-    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, B, e, &w.v_qkv, m->t_a_tok);
+    pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, B, e);
     CK(pj.rc);
     pend(pf, wq + B * (D + m->Nqkv) * es, 2.0 * B * m->Nqkv * D);
 
@@ -768,6 +763,7 @@ launch_chain:
     at.part = attn_part ? attn_part : m->attn_part;
     at.counter = attn_cnt ? attn_cnt : m->attn_cnt;
     at.o_lo = m->o_lo;
+    at.q_lo = m->q_lo;
     pbeg(pf, "decode_attention");
     CK(launch_attn_decode(lc, m->fp32, at, B));
     pend(pf, kv_tokens * 2.0 * m->G * m->d * es + 2.0 * B * Hd * es, 4.0 * kv_tokens * m->H * m->d);
@@ -782,7 +778,7 @@ launch_chain:
     r.ss_out = m->ss;
     r.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_o");
-    ns = pj.run(EPI_RESID, w.wo, &w.m_o, D, Hd, m->o, Hd, B, r, &w.v_o, m->t_o_tok);
+    ns = pj.run(EPI_RESID, w.wo, &w.m_o, D, Hd, m->o, Hd, B, r);
     CK(pj.rc);
     pend(pf, wo + B * (Hd * es + D * (8 + es)), 2.0 * B * D * Hd);
 
@@ -793,7 +789,7 @@ launch_chain:
     g.u_out = m->u;
     g.u_lo_out = m->u_lo;
     pbeg(pf, "decode_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, B, g, &w.v_gu, m->t_a_tok);
+    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, B, g);
     CK(pj.rc);
     pend(pf, wgu + B * (D + m->F) * es, 2.0 * B * 2 * m->F * D);
 
@@ -807,7 +803,7 @@ launch_chain:
     dn.ss_out = m->ss;
     dn.ss_out_stride = m->Pmax;
     pbeg(pf, "decode_down");
-    ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, B, dn, &w.v_d, m->t_u_tok);
+    ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, B, dn);
     CK(pj.rc);
     pend(pf, wdn + B * (m->F * es + D * (8 + es)), 2.0 * B * D * m->F);
   }
@@ -819,7 +815,7 @@ launch_chain:
   h.logits = logits;
   h.logits_stride = m->V;
   pbeg(pf, "decode_lm_head");
-  pj.run(EPI_LOGITS, m->head, &m->m_head, m->V, D, m->a, D, B, h, &m->v_head, m->t_a_tok);
+  pj.run(EPI_LOGITS, m->head, &m->m_head, m->V, D, m->a, D, B, h);
   CK(pj.rc);
   pend(pf, whd + B * (D * es + (logits ? 4.0 * m->V : 0.0)), 2.0 * B * m->V * D);
   pbeg(pf, "finalize");
@@ -905,7 +901,6 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->esz = m->fp32 ? 4 : 2;
   m->use_graphs = !env_flag("AXON_NO_GRAPH");
   m->use_pdl = !env_flag("AXON_NO_PDL");
-  m->use_tma_gemv = env_flag("AXON_TMA_GEMV");
   if (const char* v = getenv("AXON_PERSIST_SPLIT_BLOCKS")) {
     const int t = atoi(v);
     if (t >= 8 && t <= 4096) m->persist_split_blocks = t;
@@ -927,7 +922,7 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, m->device);
   if (major < 10) return fail(AXON_ERR_UNSUPPORTED);
   if (prepare_attn_kernels() != cudaSuccess || prepare_gemm_kernels() != cudaSuccess ||
-      prepare_gemv_tma_kernels() != cudaSuccess || prepare_gemv_kernels() != cudaSuccess)
+      prepare_gemv_kernels() != cudaSuccess)
     return fail(AXON_ERR_CUDA);
 
   Builder bl{m, weights, n_weights, st};
@@ -1093,6 +1088,10 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   if ((rc = dev_alloc(m, &m->q, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
   if ((rc = dev_alloc(m, &m->o, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
   if ((rc = dev_alloc(m, &m->u, static_cast<size_t>(Mcap) * F * es))) return fail(rc);
+  if (!f32) {
+    const size_t rows = static_cast<size_t>(cfg->max_batch < 64 ? cfg->max_batch : 64);
+    if ((rc = dev_alloc(m, &m->q_lo, rows * Hd * es))) return fail(rc);
+  }
   if (m->f16) {
     if ((rc = dev_alloc(m, &m->o_lo, static_cast<size_t>(m->cfg.max_batch) * Hd * es))) return fail(rc);
     if ((rc = dev_alloc(m, &m->u_lo, static_cast<size_t>(m->cfg.max_batch) * F * es))) return fail(rc);
@@ -1109,20 +1108,6 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->rinv_last = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
   m->ticket = static_cast<int*>(p);
-  {
-    int maxn = V;
-    if (2 * F > maxn) maxn = 2 * F;
-    if (m->Nqkv > maxn) maxn = m->Nqkv;
-    m->tmawork.max_row_blocks = (maxn + 127) / 128;
-    m->tmawork.max_grid = m->num_sms;
-    if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->num_sms) * 2 * 128 * 64 * 4))) return fail(rc);
-    m->tmawork.part = static_cast<float*>(p);
-    if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->tmawork.max_row_blocks) * 8 * 4 + 64))) return fail(rc);
-    m->tmawork.slice_ticket = static_cast<int*>(p);
-    m->tmawork.rinv_ticket = m->tmawork.slice_ticket + static_cast<size_t>(m->tmawork.max_row_blocks) * 8;
-    if (cudaMemsetAsync(p, 0, static_cast<size_t>(m->tmawork.max_row_blocks) * 8 * 4 + 64, st) != cudaSuccess)
-      return fail(AXON_ERR_CUDA);
-  }
   m->splitk.max_tiles = 1024;
   m->splitk.max_ctas = 2048;
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(m->splitk.max_ctas) * 16 * 64 * 4))) return fail(rc);
@@ -1207,11 +1192,6 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     m->m_head128 = m->m_head;
     m->m_head128.w = m->v_head;
     m->m_head.n128 = &m->m_head128;
-    for (int i = 0; i < 4 && ok; ++i) {
-      const uint32_t tok = 8u << i;
-      ok = make_tma_2d_16(&m->t_a_tok[i], m->a, Mcap, D, tok, m->f16) && make_tma_2d_16(&m->t_o_tok[i], m->o, Mcap, Hd, tok, m->f16) &&
-           make_tma_2d_16(&m->t_u_tok[i], m->u, Mcap, F, tok, m->f16);
-    }
     if (!ok) return fail(AXON_ERR_CUDA);
   }
   // ---- persistent decode step: layer table and grid barrier state

@@ -7,6 +7,8 @@
 
 #include <math.h>
 
+#include <type_traits>
+
 #include "kernels.h"
 
 namespace {
@@ -57,7 +59,15 @@ struct WarpState {
 // One 16-key tile: keys tok0 .. tok0+15; key t is visible to row r (r+8)
 // iff lo0 <= t <= lim0 (lo1 <= t <= lim1); lo is 0 without a sliding
 // window, else position - window + 1.
-template <int HD, typename T16>
+//
+// PAIRED (decode with at most 8 query heads per kv head, whose rows 8..15
+// would be padding): row r + 8 carries the second 16-bit term of row r's
+// query instead of another head. The score of row r is the sum of the two
+// rows' products, and the probabilities enter the P.V product the same way
+// -- their 16-bit rounding in row r, what it lost in row r + 8 -- so both
+// accumulator rows add up to head r's output (folded by the caller). The
+// second terms cost no extra MMA. Only row r's softmax state is used.
+template <int HD, typename T16, bool PAIRED = false>
 AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16][4], WarpState<HD>& st, int tok0,
                           int lo0, int lim0, int lo1, int lim1, float sl2, int lane) {
   const int q = lane & 3;
@@ -74,6 +84,13 @@ AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16
     mma16816<T16>(s[0], qa[kk], b0);
     mma16816<T16>(s[1], qa[kk], b1);
   }
+  if (PAIRED) {
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt) {
+      s[nt][0] += s[nt][2];
+      s[nt][1] += s[nt][3];
+    }
+  }
   float mx0 = NEG_INF, mx1 = NEG_INF;
 #pragma unroll
   for (int nt = 0; nt < 2; ++nt) {
@@ -81,39 +98,55 @@ AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16
     for (int e = 0; e < 2; ++e) {
       const int t = tok0 + nt * 8 + 2 * q + e;
       s[nt][e] = (t <= lim0 && t >= lo0) ? s[nt][e] * sl2 : NEG_INF;
-      s[nt][2 + e] = (t <= lim1 && t >= lo1) ? s[nt][2 + e] * sl2 : NEG_INF;
       mx0 = fmaxf(mx0, s[nt][e]);
-      mx1 = fmaxf(mx1, s[nt][2 + e]);
+      if (!PAIRED) {
+        s[nt][2 + e] = (t <= lim1 && t >= lo1) ? s[nt][2 + e] * sl2 : NEG_INF;
+        mx1 = fmaxf(mx1, s[nt][2 + e]);
+      }
     }
   }
   mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
   mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-  const float nm0 = fmaxf(st.m0, mx0), nm1 = fmaxf(st.m1, mx1);
+  if (!PAIRED) {
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+  }
+  const float nm0 = fmaxf(st.m0, mx0), nm1 = PAIRED ? NEG_INF : fmaxf(st.m1, mx1);
   const float base0 = (nm0 == NEG_INF) ? 0.f : nm0, base1 = (nm1 == NEG_INF) ? 0.f : nm1;
-  const float a0 = exp2f(st.m0 - base0), a1 = exp2f(st.m1 - base1);
+  const float a0 = exp2f(st.m0 - base0), a1 = PAIRED ? a0 : exp2f(st.m1 - base1);
   float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
   for (int nt = 0; nt < 2; ++nt) {
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
       s[nt][e] = exp2f(s[nt][e] - base0);
-      s[nt][2 + e] = exp2f(s[nt][2 + e] - base1);
       ps0 += s[nt][e];
-      ps1 += s[nt][2 + e];
+      if (!PAIRED) {
+        s[nt][2 + e] = exp2f(s[nt][2 + e] - base1);
+        ps1 += s[nt][2 + e];
+      }
     }
   }
   st.l0 = st.l0 * a0 + ps0;
-  st.l1 = st.l1 * a1 + ps1;
   st.m0 = nm0;
-  st.m1 = nm1;
+  if (!PAIRED) {
+    st.l1 = st.l1 * a1 + ps1;
+    st.m1 = nm1;
+  }
 #pragma unroll
   for (int nd = 0; nd < HD / 8; ++nd) {
     st.o[nd][0] *= a0;
     st.o[nd][1] *= a0;
     st.o[nd][2] *= a1;
     st.o[nd][3] *= a1;
+  }
+  if (PAIRED) {
+    // row r + 8: what the 16-bit rounding of row r's probabilities lost
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt) {
+      s[nt][2] = s[nt][0] - to_f(from_f<T16>(s[nt][0]));
+      s[nt][3] = s[nt][1] - to_f(from_f<T16>(s[nt][1]));
+    }
   }
   const uint32_t pa[4] = {pack2<T16>(s[0][0], s[0][1]), pack2<T16>(s[0][2], s[0][3]),
                           pack2<T16>(s[1][0], s[1][1]), pack2<T16>(s[1][2], s[1][3])};
@@ -126,6 +159,20 @@ AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16
     mma16816<T16>(st.o[2 * nd2], pa, b0);
     mma16816<T16>(st.o[2 * nd2 + 1], pa, b1);
   }
+}
+
+// After the last PAIRED tile: add row r + 8's partial output into row r and
+// leave row r + 8 empty.
+template <int HD>
+AXON_DEV void fold_paired(WarpState<HD>& st) {
+#pragma unroll
+  for (int nd = 0; nd < HD / 8; ++nd) {
+    st.o[nd][0] += st.o[nd][2];
+    st.o[nd][1] += st.o[nd][3];
+    st.o[nd][2] = st.o[nd][3] = 0.f;
+  }
+  st.m1 = NEG_INF;
+  st.l1 = 0.f;
 }
 
 AXON_DEV int block_of(const AttnArgs& p, int b, int j, bool& ok) {
@@ -149,7 +196,10 @@ AXON_DEV void dec_sync() {
 // by DEC_WARPS warps (thread `tid` of them) with `sm` as staging memory
 // (decode_smem<HD>() bytes). Reads of q and of the merge partials bypass L1:
 // they may have been written by another SM earlier in the same kernel.
-template <int HD, typename T16, bool NAMED>
+// PAIR = 1: the caller guarantees a second term of q and at most 8 query
+// heads per kv head, so only the paired tile loop is compiled; PAIR = 0:
+// chosen at run time.
+template <int HD, typename T16, bool NAMED, int PAIR = 0>
 AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* sm, int tid) {
   constexpr int TILE = 16 * HD * 2;
   const int warp = tid >> 5, lane = tid & 31, r = lane >> 2, q = lane & 3;
@@ -187,25 +237,42 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
   int j = jb + warp, stg = 0;
   if (j < je) issue(j, 0);
 
-  const uint16_t* qg = static_cast<const uint16_t*>(p.q) + (static_cast<long long>(b) * p.H + g * HPG) * HD;
+  // With a second term of q and at most 8 query heads per kv head, rows
+  // r + 8 of the MMA tiles carry the second terms (attn_tile16, PAIRED).
+  const long long qoff = (static_cast<long long>(b) * p.H + g * HPG) * HD;
+  const uint16_t* qg = static_cast<const uint16_t*>(p.q) + qoff;
+  const bool paired = PAIR == 1 || (p.q_lo != nullptr && HPG <= 8);
+  const uint16_t* qg1 = paired ? static_cast<const uint16_t*>(p.q_lo) + qoff + r * HD : qg + (r + 8) * HD;
   uint32_t qa[HD / 16][4];
-  load_q<HD>(qa, r < HPG ? qg + r * HD : nullptr, r + 8 < HPG ? qg + (r + 8) * HD : nullptr, q);
+  load_q<HD>(qa, r < HPG ? qg + r * HD : nullptr, (paired ? r : r + 8) < HPG ? qg1 : nullptr, q);
 
   WarpState<HD> st;
   st.init();
-  for (; j < je; j += DEC_WARPS) {
-    const int jn = j + DEC_WARPS;
-    if (jn < je) {
-      issue(jn, stg ^ 1);
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
+  auto run_tiles = [&](auto paired_tag) {
+    constexpr bool PAIRED = decltype(paired_tag)::value;
+    for (; j < je; j += DEC_WARPS) {
+      const int jn = j + DEC_WARPS;
+      if (jn < je) {
+        issue(jn, stg ^ 1);
+        cp_async_wait<1>();
+      } else {
+        cp_async_wait<0>();
+      }
+      __syncwarp();
+      attn_tile16<HD, T16, PAIRED>(wbase + stg * 2 * TILE, wbase + stg * 2 * TILE + TILE, qa, st, j * 16, klo, T - 1,
+                                   klo, T - 1, p.scale_log2, lane);
+      __syncwarp();
+      stg ^= 1;
     }
-    __syncwarp();
-    attn_tile16<HD, T16>(wbase + stg * 2 * TILE, wbase + stg * 2 * TILE + TILE, qa, st, j * 16, klo, T - 1, klo,
-                         T - 1, p.scale_log2, lane);
-    __syncwarp();
-    stg ^= 1;
+    if (PAIRED) fold_paired<HD>(st);
+  };
+  if constexpr (PAIR == 1) {
+    run_tiles(std::true_type{});
+  } else {
+    if (paired)
+      run_tiles(std::true_type{});
+    else
+      run_tiles(std::false_type{});
   }
   st.l0 += __shfl_xor_sync(0xffffffffu, st.l0, 1);
   st.l0 += __shfl_xor_sync(0xffffffffu, st.l0, 2);

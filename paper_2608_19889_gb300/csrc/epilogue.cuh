@@ -48,6 +48,7 @@ struct EpiArgs {
   const float2* rope;  // [max_pos][d/2] (cos, sin)
   int H, G, d;
   void* q_out;  // [M][H*d]
+  void* q_lo_out;  // optional [M][H*d] (decode): q - q_out, the second 16-bit term of q
   void* k_cache;  // this layer's pool [num_blocks][G][16][d]
   void* v_cache;
   const int* block_table;  // paged: [B][bt_stride]; null = contiguous
@@ -194,9 +195,22 @@ AXON_DEV void epi_qkv16x(const EpiArgs& e, int m, int n0, const float* v, float 
     }
   }
   if (region == 0) {
-    T* dst = reinterpret_cast<T*>(e.q_out) + static_cast<long long>(m) * Hd + head * e.d + j0;
+    const long long qo = static_cast<long long>(m) * Hd + head * e.d + j0;
+    T* dst = reinterpret_cast<T*>(e.q_out) + qo;
     store8<T>(dst, lo);
     store8<T>(dst + half, hi);
+    if (e.q_lo_out) {
+      // what the 16-bit rounding of q lost: the decode attention multiplies
+      // both terms with the keys
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        lo[i] -= to_f(from_f<T>(lo[i]));
+        hi[i] -= to_f(from_f<T>(hi[i]));
+      }
+      T* ld = reinterpret_cast<T*>(e.q_lo_out) + qo;
+      store8<T>(ld, lo);
+      store8<T>(ld + half, hi);
+    }
   } else {
     const long long off = kv_offset(e, b, pos, head);
     if (off < 0) return;

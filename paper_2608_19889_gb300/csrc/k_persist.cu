@@ -578,6 +578,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       e.N = A.Nqkv;
       e.bias = w.bqkv;
       e.q_out = A.q;
+      e.q_lo_out = A.q_lo;
       e.k_cache = w.kc;
       e.v_cache = w.vc;
       e.block_table = A.block_table;
@@ -611,11 +612,12 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       p.part = A.attn_part;
       p.counter = A.attn_cnt;
       p.o_lo = A.o_lo;
+      p.q_lo = A.q_lo;
       p.err = A.err;
       const int items = A.splits * A.G * B;
       for (int it = blockIdx.x; it < items; it += gridDim.x) {
         const int s = it % A.splits, gg = (it / A.splits) % A.G, b = it / (A.splits * A.G);
-        attn_decode_item<HD, T16, true>(p, s, gg, b, attn_sm, tid);
+        attn_decode_item<HD, T16, true, 1>(p, s, gg, b, attn_sm, tid);
       }
     }
     grid_sync(g, epoch, tid, s_abort, A.err);

@@ -39,20 +39,6 @@ cudaError_t launch_gemv(const LaunchCtx& lc, int kind, bool fp32, const void* W,
 // Query occupancy of the projection kernels (once, before launches).
 cudaError_t prepare_gemv_kernels();
 
-// ---- decode projections, TMA-fed persistent stream-K variant
-// (k_gemv_tma.cu). W map: box 64 x 128 rows; activation map: box 64 x
-// gemv_tma_tokens(B) rows of a row-contiguous [rows][K] buffer.
-struct GemvTmaWork {
-  float* part;        // [max_grid][2][128][64]
-  int* slice_ticket;  // [max_row_blocks][8], zeroed once
-  int* rinv_ticket;   // [1], zeroed once
-  int max_grid;
-  int max_row_blocks;
-};
-int gemv_tma_tokens(int B);
-cudaError_t prepare_gemv_tma_kernels();
-cudaError_t launch_gemv_tma(const LaunchCtx& lc, int kind, const CUtensorMap& w, const CUtensorMap& a, int N, int K,
-                            int B, const EpiArgs& ep, const GemvTmaWork& wk);
 
 // ---- embedding gather producing x, a = x * g and the row sum of squares.
 // rinv (optional): 1 / sqrt(mean(x^2) + eps) per row.
@@ -103,6 +89,7 @@ struct AttnArgs {
   float scale_log2;
   float* part;  // decode partials
   void* o_lo;   // optional [rows][H*d]: o minus its 16-bit rounding (decode, fp16 mode)
+  const void* q_lo;  // optional [rows][H*d]: q minus its 16-bit rounding (decode)
   int* counter;  // decode [B][G] tickets
   int* err;
 };
@@ -207,6 +194,7 @@ struct PersistArgs {
   void* a_lo;  // fp16 mode: second term of a
   float* ss;   // norm partials [B][Pmax]
   void* q;
+  void* q_lo;  // second term of q (16-bit modes)
   void* o;
   void* u;
   void* o_lo;  // fp16 mode: second terms of o and u

@@ -11,6 +11,7 @@
 // The array lives in every device that loads this library, for the life of
 // the process: NOALLOC_ROWS merge slots of (16 head rows x (head_dim + 2))
 // floats plus one ticket per (sequence, kv head), about 2.1 MB.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -34,11 +35,34 @@ constexpr int NOALLOC_PART_FLOATS = NOALLOC_ROWS * 16 * (NOALLOC_MAX_HEAD_DIM + 
 // followed by the per-(sequence, kv head) tickets that pick the merging CTA.
 static __device__ __align__(256) float g_noalloc_scratch[NOALLOC_PART_FLOATS + NOALLOC_ROWS];
 
-// Device address of g_noalloc_scratch per device, resolved once per device
-// with that device current (in host code the symbol's name is only a
-// host-side stand-in, never a device address).
+// Device address of g_noalloc_scratch per device, resolved with that device
+// current (in host code the symbol's name is only a host-side stand-in, never
+// a device address). The address belongs to the context the module was
+// loaded into: after cudaDeviceReset (or any teardown of the primary
+// context) the module is loaded again, possibly elsewhere, so each entry
+// remembers its context and is resolved again when the current one differs.
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  }
+  return fn;
+}
+
+struct Resolved {
+  CUcontext ctx = nullptr;
+  float* addr = nullptr;
+};
 std::mutex g_mu;
-float* g_addr[64] = {};
+Resolved g_addr[64];
 
 float* scratch_on_current_device(int* status) {
   int dev = -1;
@@ -47,17 +71,27 @@ float* scratch_on_current_device(int* status) {
     return nullptr;
   }
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_addr[dev]) {
+  CtxGetCurrentFn get = ctx_get_current();
+  CUcontext ctx = nullptr;
+  if (!get || get(&ctx) != CUDA_SUCCESS) {
+    *status = AXON_ERR_CUDA;
+    return nullptr;
+  }
+  Resolved& r = g_addr[dev];
+  if (!r.addr || !ctx || r.ctx != ctx) {
+    // cudaGetSymbolAddress also binds the device's primary context to this
+    // thread when nothing is bound yet; the context is read again after it
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) {
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p || get(&ctx) != CUDA_SUCCESS || !ctx) {
       cudaGetLastError();
       *status = AXON_ERR_CUDA;
       return nullptr;
     }
-    g_addr[dev] = static_cast<float*>(p);
+    r.addr = static_cast<float*>(p);
+    r.ctx = ctx;
   }
   *status = AXON_OK;
-  return g_addr[dev];
+  return r.addr;
 }
 
 }  // namespace

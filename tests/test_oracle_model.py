@@ -115,6 +115,19 @@ def test_oracle_matches_bruteforce_loops(tie, bias, H, G, window, act, qkn):
     assert np.allclose(got, ref, rtol=1e-12, atol=1e-12)
 
 
+def test_selected_rows_match_bruteforce_loops_at_those_positions():
+    """prefill(rows=...) returns exactly the listed positions' logits (the
+    large-shape GPU checks compare sampled rows through it)."""
+    cfg, W = tiny_model()
+    ids = [3, 15, 0, 7, 7, 2]
+    ref = np.array(_bf_forward(cfg, W, ids))
+    o = od.Oracle(cfg, W)
+    rows = [4, 0, 5]
+    got = o.prefill(np.array([ids]), o.new_contiguous_cache(1, 8), rows=rows)[0]
+    assert got.shape == (3, cfg.V)
+    assert np.allclose(got, ref[rows], rtol=1e-12, atol=1e-12)
+
+
 # ------------------------------------------------------------- special cases
 def test_zero_layers_is_norm_then_head():
     cfg, W = tiny_model(L=0)
