@@ -115,6 +115,11 @@ typedef struct axon_config {
   float rope_high_freq_factor;
   int32_t rope_original_max_position;
   int32_t hidden_act;          /* AXON_ACT_SILU or AXON_ACT_GELU_TANH: u = act(h W_gate^T) * (h W_up^T) */
+  int32_t qk_norm;             /* 1: each head's q and k (after the projection and its bias) go
+                                  through RMSNorm over their head_dim values, with rms_norm_eps and
+                                  the gains model.layers.{i}.self_attn.{q,k}_norm.weight [head_dim],
+                                  before RoPE (Qwen3-family layers); 0: none. Decode then always
+                                  takes the launch chain. */
 } axon_config;
 
 /* One named checkpoint tensor, HF Llama naming and [out, in] matrices, as a
@@ -128,6 +133,7 @@ typedef struct axon_config {
  *   model.layers.{i}.post_attention_layernorm.weight[D]
  *   model.layers.{i}.mlp.{gate,up}_proj.weight      [F, D]
  *   model.layers.{i}.mlp.down_proj.weight           [D, F]
+ *   model.layers.{i}.self_attn.{q,k}_norm.weight    [d] (if qk_norm)
  *   model.norm.weight                               [D]
  *   lm_head.weight                                  [V, D] (absent if tied)
  * `data` may be a host or a device pointer (unified addressing); it is

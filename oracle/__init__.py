@@ -31,4 +31,6 @@ from .decoder import (  # noqa: F401
     slot_of,
     Oracle,
     argmax_lowest,
+    moe_route,
+    topk_lowest,
 )

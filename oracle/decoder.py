@@ -68,6 +68,14 @@ READINGS = [
     "k projections (and biases), each head's d values go through the same "
     "RMSNorm as the hidden state, with gains q_norm / k_norm of length d, "
     "before RoPE.",
+    "Mixture of experts (the MoE built-ins: MoE.softmax_topk_router and "
+    "grouped experts; off unless n_experts > 0): layers from first_dense on "
+    "replace the MLP by p = softmax(h Wr^T) over the E experts, the top_k "
+    "experts by p (lowest index on ties), weights p of those (divided by "
+    "their sum when norm_topk), y = sum_j w_j * swiglu-MLP_e_j(h), plus the "
+    "shared experts' SwiGLU MLP of width n_shared * F_e when n_shared > 0 "
+    "(DeepSeek-MoE layout; HF names mlp.gate, mlp.experts.{e}.*, "
+    "mlp.shared_experts.*).",
     "Sliding window (the `window=` argument of causal_mask_for_input in the "
     "appendix GPT-2 listing): with window W > 0 a query at position p sees "
     "the keys at positions t with p - W < t <= p (itself and the W - 1 "
@@ -100,6 +108,13 @@ class DecoderConfig:
     rope_orig: int = 8192  # original_max_position_embeddings
     act: str = "silu"  # hidden_act of the gated MLP: "silu" or "gelu_tanh"
     qk_norm: bool = False  # per-head RMSNorm of q and k before RoPE (Qwen3-family layers)
+    # mixture of experts (n_experts 0: every layer has the dense MLP)
+    n_experts: int = 0  # E routed experts
+    top_k: int = 0  # experts per token
+    moe_F: int = 0  # intermediate size of one expert
+    n_shared: int = 0  # shared experts (one dense MLP of width n_shared * moe_F)
+    first_dense: int = 0  # leading layers that keep the dense MLP (width F)
+    norm_topk: bool = False  # divide the top-k weights by their sum
 
     @staticmethod
     def from_dict(c: dict) -> "DecoderConfig":
@@ -109,7 +124,13 @@ class DecoderConfig:
                              window=int(c.get("window", 0)), rope_factor=float(c.get("rope_factor", 0.0)),
                              rope_low=float(c.get("rope_low", 1.0)), rope_high=float(c.get("rope_high", 4.0)),
                              rope_orig=int(c.get("rope_orig", 8192)), act=str(c.get("act", "silu")),
-                             qk_norm=bool(c.get("qk_norm", False)))
+                             qk_norm=bool(c.get("qk_norm", False)), n_experts=int(c.get("n_experts", 0)),
+                             top_k=int(c.get("top_k", 0)), moe_F=int(c.get("moe_F", 0)),
+                             n_shared=int(c.get("n_shared", 0)), first_dense=int(c.get("first_dense", 0)),
+                             norm_topk=bool(c.get("norm_topk", False)))
+
+    def is_moe_layer(self, l: int) -> bool:
+        return self.n_experts > 0 and l >= self.first_dense
 
     def rope_scaling(self):
         """(factor, low_freq_factor, high_freq_factor, original context), or None."""
@@ -202,6 +223,28 @@ def swiglu(gate, up, act="silu"):
     goes through gelu_new instead (the gated-GELU MLP)."""
     a = gelu_tanh(gate) if act == "gelu_tanh" else silu(gate)
     return a * np.asarray(up, dtype=np.float64)
+
+
+def topk_lowest(p, k):
+    """Indices of the k largest entries along the last axis, largest first;
+    among equal entries the lower index comes first."""
+    p = np.asarray(p)
+    return np.argsort(-p, axis=-1, kind="stable")[..., :k]
+
+
+def moe_route(h, Wr, top_k, norm_topk, forced=None):
+    """MoE.softmax_topk_router (Sec. Built-In Libraries, specialised
+    modules listing): router probabilities p = softmax(h Wr^T) over the
+    experts, the top_k experts by p and their weights (divided by their sum
+    when norm_topk). h: [T, D]; Wr: [E, D]. With `forced` [T, k] the given
+    experts are taken instead of the top_k (teacher-forced routing).
+    Returns (experts [T, k], weights [T, k], p [T, E])."""
+    p = softmax(linear(h, Wr), axis=-1)
+    idx = topk_lowest(p, top_k) if forced is None else np.asarray(forced, dtype=np.int64)
+    w = np.take_along_axis(p, idx, axis=-1)
+    if norm_topk:
+        w = w / np.sum(w, axis=-1, keepdims=True)
+    return idx, w, p
 
 
 def softmax(s, axis=-1):
@@ -350,6 +393,11 @@ class Oracle:
             self.W = {k: np.asarray(v, dtype=np.float64) for k, v in weights.items()}
         else:
             self.W = weights
+        # MoE: per-layer expert choices to use instead of the router's top-k
+        # ({layer: [tokens, k]} for the rows of the next forward), and the
+        # routing each MoE layer took in the last forward
+        self.forced_routing = None
+        self.last_routing = {}
 
     def _w(self, name):
         return self.W[name] if self.keep_f64 else np.asarray(self.W[name], dtype=np.float64)
@@ -396,15 +444,41 @@ class Oracle:
                 o[b] = causal_attention(q[b], Kb, Vb, pos[b], c.H, c.G, c.window)
             x = x + linear(o.reshape(B, S, c.H * c.d), self._w(p + "self_attn.o_proj.weight"))
             h2 = rmsnorm(x, self._w(p + "post_attention_layernorm.weight"), c.eps)
-            u = swiglu(linear(h2, self._w(p + "mlp.gate_proj.weight")),
-                       linear(h2, self._w(p + "mlp.up_proj.weight")), c.act)
-            x = x + linear(u, self._w(p + "mlp.down_proj.weight"))
+            if c.is_moe_layer(l):
+                forced = None if self.forced_routing is None else self.forced_routing[l]
+                x = x + self.moe_mlp(h2.reshape(B * S, c.D), p, forced).reshape(B, S, c.D)
+            else:
+                u = swiglu(linear(h2, self._w(p + "mlp.gate_proj.weight")),
+                           linear(h2, self._w(p + "mlp.up_proj.weight")), c.act)
+                x = x + linear(u, self._w(p + "mlp.down_proj.weight"))
         if last_hidden_only:
             x = x[:, -1:, :]
         elif rows is not None:
             x = x[:, np.asarray(rows, dtype=np.int64), :]
         head = self._w("model.embed_tokens.weight") if c.tie else self._w("lm_head.weight")
         return linear(rmsnorm(x, self._w("model.norm.weight"), c.eps), head)
+
+    def moe_mlp(self, h, p, forced=None):
+        """Mixture-of-experts MLP of one layer for rows h [T, D]: each token
+        goes through its routed experts one at a time (the per-expert loop
+        the paper's compiler rewrites into stacked experts), weighted by its
+        router weights, plus the shared experts. Records the routing in
+        self.last_routing[p]."""
+        c = self.cfg
+        idx, w, prob = moe_route(h, self._w(p + "mlp.gate.weight"), c.top_k, c.norm_topk, forced)
+        self.last_routing[p] = (idx, w, prob)
+        y = np.zeros_like(h)
+        for t in range(h.shape[0]):
+            for j in range(idx.shape[1]):
+                e = f"{p}mlp.experts.{int(idx[t, j])}."
+                u = swiglu(linear(h[t], self._w(e + "gate_proj.weight")), linear(h[t], self._w(e + "up_proj.weight")),
+                           c.act)
+                y[t] += w[t, j] * linear(u, self._w(e + "down_proj.weight"))
+        if c.n_shared:
+            s = p + "mlp.shared_experts."
+            u = swiglu(linear(h, self._w(s + "gate_proj.weight")), linear(h, self._w(s + "up_proj.weight")), c.act)
+            y = y + linear(u, self._w(s + "down_proj.weight"))
+        return y
 
     def prefill(self, ids, cache, last_only=False, rows=None):
         """Prompt pass from an empty cache; logits for every position, for

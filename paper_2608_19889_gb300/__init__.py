@@ -43,7 +43,7 @@ class axon_config(ctypes.Structure):
         (n, ctypes.c_int32) for n in ("max_batch", "max_context", "max_prefill_tokens", "kv_layout",
                                       "kv_block_size", "kv_num_blocks", "precision", "sliding_window")] + [
         (n, ctypes.c_float) for n in ("rope_scaling_factor", "rope_low_freq_factor", "rope_high_freq_factor")] + [
-        ("rope_original_max_position", ctypes.c_int32), ("hidden_act", ctypes.c_int32)]
+        ("rope_original_max_position", ctypes.c_int32), ("hidden_act", ctypes.c_int32), ("qk_norm", ctypes.c_int32)]
 
 
 class axon_tensor(ctypes.Structure):
@@ -126,12 +126,13 @@ def make_config(m: dict, max_batch: int, max_context: int, kv_layout=AXON_KV_CON
                 precision=AXON_BF16, max_prefill_tokens=0) -> axon_config:
     """axon_config from a shape dict with keys L, D, H, G, d, F, V, tie, bias, theta, eps (and optionally
     window, the sliding window, rope_factor / rope_low / rope_high / rope_orig, the RoPE frequency
-    scaling, 0 or absent = none; act, "silu" (default) or "gelu_tanh")."""
+    scaling, 0 or absent = none; act, "silu" (default) or "gelu_tanh"; qk_norm, per-head RMSNorm of q and k)."""
     return axon_config(m["L"], m["D"], m["H"], m["G"], m["d"], m["F"], m["V"], int(m["tie"]), int(m["bias"]),
                        float(m["theta"]), float(m["eps"]), max_batch, max_context, max_prefill_tokens, kv_layout, 16,
                        kv_num_blocks, precision, int(m.get("window", 0)), float(m.get("rope_factor", 0.0)),
                        float(m.get("rope_low", 1.0)), float(m.get("rope_high", 4.0)), int(m.get("rope_orig", 8192)),
-                       AXON_ACT_GELU_TANH if m.get("act", "silu") == "gelu_tanh" else AXON_ACT_SILU)
+                       AXON_ACT_GELU_TANH if m.get("act", "silu") == "gelu_tanh" else AXON_ACT_SILU,
+                       int(bool(m.get("qk_norm", False))))
 
 
 def axon_model_create(cfg: axon_config, weights: dict, stream=None) -> ctypes.c_void_p:

@@ -33,6 +33,8 @@ struct LayerW {
   void* wd = nullptr;
   float* g1 = nullptr;
   float* g2 = nullptr;
+  float* qn = nullptr;  // qk-norm gains [d] (null when off)
+  float* kn = nullptr;
   GemmMaps m_qkv{}, m_o{}, m_gu{}, m_d{};
   GemmMaps m_qkv128{}, m_o128{}, m_gu128{}, m_d128{};  // the same with 128-row weight boxes
   CUtensorMap v_qkv{}, v_o{}, v_gu{}, v_d{};  // weight maps for the decode projections (box 64 x 128)
@@ -85,6 +87,7 @@ struct axon_model {
   void* u = nullptr;
   unsigned long long* keys = nullptr;
   float* rinv = nullptr;   // [Mcap] per-row inverse RMS from decode producers
+  float* qk_raw = nullptr;  // qk-norm: [Mcap][H + G][d] fp32 q and k before the norm
   // variable-length batches: (sequence, position) per row, and each chunk's
   // last row of a (and a_lo) with its inverse RMS, gathered for the LM head
   int2* rowmap = nullptr;     // [Mcap]
@@ -111,6 +114,9 @@ struct axon_model {
   int persist_ctas = 0;
   int decode_gemv_max = 32;  // decode projections with more tokens take the tcgen05 GEMM (AXON_DECODE_GEMV_MAX)
   int persist_split_blocks = 16;  // persistent step: key blocks per split-KV item (AXON_PERSIST_SPLIT_BLOCKS)
+  // decode attention grid budget in CTAs (AXON_ATTN_TARGET_CTAS; 0: the
+  // split count with the smallest estimated makespan)
+  int attn_target_ctas = 0;
   GemmSplitK gemm_sk{};      // split-K workspace of the decode-sized tensor-core GEMMs
 };
 
@@ -275,6 +281,7 @@ int validate_config(const axon_config* c) {
   if (c->sliding_window < 0) return AXON_ERR_INVALID_ARG;
   if (c->rope_scaling_factor < 0.f) return AXON_ERR_INVALID_ARG;
   if (c->hidden_act != AXON_ACT_SILU && c->hidden_act != AXON_ACT_GELU_TANH) return AXON_ERR_INVALID_ARG;
+  if (c->qk_norm != 0 && c->qk_norm != 1) return AXON_ERR_INVALID_ARG;
   if (c->rope_scaling_factor > 0.f &&
       (c->rope_original_max_position <= 0 || c->rope_low_freq_factor <= 0.f ||
        c->rope_high_freq_factor <= c->rope_low_freq_factor))
@@ -339,6 +346,14 @@ AttnArgs base_attn(const axon_model* m, int layer, const int* block_table) {
   a.window = m->cfg.sliding_window;
   a.err = m->err;
   return a;
+}
+
+// qk-norm inputs of a QKV epilogue (left null when the model has none).
+void set_qk_norm(const axon_model* m, const LayerW& w, EpiArgs& e) {
+  if (!m->cfg.qk_norm) return;
+  e.qk_raw = m->qk_raw;
+  e.qn_gain = w.qn;
+  e.kn_gain = w.kn;
 }
 
 // Which form the next norm's scale is available in after a producer: the
@@ -511,10 +526,16 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     e.bias = w.bqkv;
     e.q_out = m->q;
     kv_layout_args(m, l, bt, e);
+    set_qk_norm(m, w, e);
     pbeg(pf, "prefill_qkv");
     pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, M, e);
     CK(pj.rc);
     pend(pf, wq + M * (D + m->Nqkv) * es, 2.0 * M * m->Nqkv * D);
+    if (e.qk_raw) {
+      pbeg(pf, "prefill_qk_norm");
+      CK(launch_qk_norm_rope(lc, m->fp32, e, M));
+      pend(pf, static_cast<double>(M) * (m->H + m->G) * m->d * (4 + es), 0);
+    }
 
     AttnArgs at = base_attn(m, l, bt);
     at.S = vl ? vl->max_chunk : S;
@@ -623,9 +644,12 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 }
 
 // The persistent step's attention always pairs q's two terms in one MMA
-// tile, which needs at most 8 query heads per kv head.
+// tile, which needs at most 8 query heads per kv head; qk-norm needs a
+// kernel of its own between QKV and attention, so those models decode on
+// the launch chain.
 bool persist_eligible(const axon_model* m, int B) {
-  return m->persist_ctas > 0 && !m->fp32 && m->H / m->G <= 8 && persist_fits(m->d, m->f16, B, m->D);
+  return m->persist_ctas > 0 && !m->fp32 && !m->cfg.qk_norm && m->H / m->G <= 8 &&
+         persist_fits(m->d, m->f16, B, m->D);
 }
 
 PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt,
@@ -696,12 +720,15 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * Hd * es,
                wgu = 2.0 * m->F * m->D * es, wdn = static_cast<double>(m->D) * m->F * es,
                whd = static_cast<double>(m->V) * m->D * es;
-  int splits = m->fp32 ? 1 : attn_decode_splits(B, m->G, m->blocks_per_seq, m->num_sms);
+  // merge slots per (sequence, kv head): the model's partial buffer, or the
+  // caller-supplied scratch of attn_rows_cap (sequence, kv head, split) slots
+  int cap = m->max_splits;
   if (attn_rows_cap > 0) {
-    // caller-supplied merge scratch holds attn_rows_cap (sequence, kv head, split) slots
-    const int cap = attn_rows_cap / (B * m->G);
-    if (splits > cap) splits = cap < 1 ? 1 : cap;
+    const int c = attn_rows_cap / (B * m->G);
+    cap = c < 1 ? 1 : (c < cap ? c : cap);
   }
+  int splits = m->fp32 ? 1 : attn_decode_splits(B, m->G, m->blocks_per_seq, m->num_sms, m->attn_target_ctas);
+  if (splits > cap) splits = cap;
   if (persist_eligible(m, B)) {
     // Inside one launch a cross-CTA merge costs more than it saves up to 64
     // key blocks (8 per warp; measured at 40 blocks, head_dim 64: 0.743 ms
@@ -711,7 +738,7 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     int psplits = m->blocks_per_seq > 64
                       ? (m->blocks_per_seq + m->persist_split_blocks - 1) / m->persist_split_blocks
                       : 1;
-    if (psplits > splits) psplits = splits;
+    if (psplits > cap) psplits = cap;
     PersistArgs pa = persist_args(m, tokens, B, ctx, bt, logits, next, psplits, attn_part ? attn_part : m->attn_part,
                                   attn_cnt ? attn_cnt : m->attn_cnt);
     pbeg(pf, "decode_persistent");
@@ -751,10 +778,16 @@ launch_chain:
     e.q_out = m->q;
     e.q_lo_out = m->q_lo;
     kv_layout_args(m, l, bt, e);
+    set_qk_norm(m, w, e);
     pbeg(pf, "decode_qkv");
     pj.run(EPI_QKV, w.wqkv, &w.m_qkv, m->Nqkv, D, m->a, D, B, e);
     CK(pj.rc);
     pend(pf, wq + B * (D + m->Nqkv) * es, 2.0 * B * m->Nqkv * D);
+    if (e.qk_raw) {
+      pbeg(pf, "decode_qk_norm");
+      CK(launch_qk_norm_rope(lc, m->fp32, e, B));
+      pend(pf, static_cast<double>(B) * (m->H + m->G) * m->d * (4 + es), 0);
+    }
 
     AttnArgs at = base_attn(m, l, bt);
     at.ctx = ctx;
@@ -918,6 +951,11 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   };
   if (cudaGetDevice(&m->device) != cudaSuccess) return fail(AXON_ERR_CUDA);
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
+  m->attn_target_ctas = 0;
+  if (const char* v = getenv("AXON_ATTN_TARGET_CTAS")) {
+    const int t = atoi(v);
+    if (t >= 1 && t <= 1 << 20) m->attn_target_ctas = t;
+  }
   int major = 0;
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, m->device);
   if (major < 10) return fail(AXON_ERR_UNSUPPORTED);
@@ -942,6 +980,10 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     if ((rc = bl.check(bl.find(p + "mlp.gate_proj.weight"), F, D))) return fail(rc);
     if ((rc = bl.check(bl.find(p + "mlp.up_proj.weight"), F, D))) return fail(rc);
     if ((rc = bl.check(bl.find(p + "mlp.down_proj.weight"), D, F))) return fail(rc);
+    if (cfg->qk_norm) {
+      if ((rc = bl.check(bl.find(p + "self_attn.q_norm.weight"), m->d, -1))) return fail(rc);
+      if ((rc = bl.check(bl.find(p + "self_attn.k_norm.weight"), m->d, -1))) return fail(rc);
+    }
     if (cfg->attention_bias) {
       if ((rc = bl.check(bl.find(p + "self_attn.q_proj.bias"), Hd, -1))) return fail(rc);
       if ((rc = bl.check(bl.find(p + "self_attn.k_proj.bias"), Gd, -1))) return fail(rc);
@@ -1021,6 +1063,16 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     if ((rc = bl.gather(w.g1, true, bl.find(p + "input_layernorm.weight"), nullptr, 1, D))) return fail(rc);
     if ((rc = bl.gather(w.g2, true, bl.find(p + "post_attention_layernorm.weight"), nullptr, 1, D)))
       return fail(rc);
+    if (cfg->qk_norm) {
+      void* qn = nullptr;
+      void* kn = nullptr;
+      if ((rc = dev_alloc(m, &qn, m->d * 4))) return fail(rc);
+      if ((rc = dev_alloc(m, &kn, m->d * 4))) return fail(rc);
+      w.qn = static_cast<float*>(qn);
+      w.kn = static_cast<float*>(kn);
+      if ((rc = bl.gather(w.qn, true, bl.find(p + "self_attn.q_norm.weight"), nullptr, 1, m->d))) return fail(rc);
+      if ((rc = bl.gather(w.kn, true, bl.find(p + "self_attn.k_norm.weight"), nullptr, 1, m->d))) return fail(rc);
+    }
   }
 
   // ---- KV cache: pools [L][num_blocks][G][16][d]
@@ -1102,6 +1154,10 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->rinv = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * sizeof(int2)))) return fail(rc);
   m->rowmap = static_cast<int2*>(p);
+  if (cfg->qk_norm) {
+    if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * (m->H + m->G) * m->d * 4))) return fail(rc);
+    m->qk_raw = static_cast<float*>(p);
+  }
   if ((rc = dev_alloc(m, &m->a_last, static_cast<size_t>(cfg->max_batch) * D * es))) return fail(rc);
   if (m->f16 && (rc = dev_alloc(m, &m->a_lo_last, static_cast<size_t>(cfg->max_batch) * D * es))) return fail(rc);
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(cfg->max_batch) * 4))) return fail(rc);

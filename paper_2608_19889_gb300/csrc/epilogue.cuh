@@ -49,6 +49,13 @@ struct EpiArgs {
   int H, G, d;
   void* q_out;  // [M][H*d]
   void* q_lo_out;  // optional [M][H*d] (decode): q - q_out, the second 16-bit term of q
+  // qk-norm (null when off): q and k leave the epilogue unrotated and
+  // unrounded, [M][H + G][d] fp32 (natural dimension order), for the
+  // kernel that normalises each head, applies the gains and RoPE and stores
+  // them (launch_qk_norm_rope); v is stored as usual.
+  float* qk_raw;
+  const float* qn_gain;  // [d]
+  const float* kn_gain;  // [d]
   void* k_cache;  // this layer's pool [num_blocks][G][16][d]
   void* v_cache;
   const int* block_table;  // paged: [B][bt_stride]; null = contiguous
@@ -184,6 +191,15 @@ AXON_DEV void epi_qkv16x(const EpiArgs& e, int m, int n0, const float* v, float 
   for (int i = 0; i < 8; ++i) {
     lo[i] = v[i] * r + in.b[i];
     hi[i] = v[8 + i] * r + in.b[8 + i];
+  }
+  if (region < 2 && e.qk_raw) {
+    float* raw = e.qk_raw + (static_cast<long long>(m) * (e.H + e.G) + (region == 0 ? head : e.H + head)) * e.d + j0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      raw[i] = lo[i];
+      raw[half + i] = hi[i];
+    }
+    return;
   }
   if (region < 2) {
 #pragma unroll

@@ -270,11 +270,33 @@ cudaError_t prepare_attn_kernels() {
   return e;
 }
 
-int attn_decode_splits(int B, int G, int max_blocks, int num_sms) {
-  int want = (2 * num_sms + B * G - 1) / (B * G);
-  if (want > max_blocks) want = max_blocks;
-  if (want > 64) want = 64;
-  return want < 1 ? 1 : want;
+int attn_decode_splits(int B, int G, int max_blocks, int num_sms, int target_ctas) {
+  const int bg = B * G;
+  const int smax = max_blocks < 64 ? max_blocks : 64;
+  if (target_ctas > 0) {  // explicit grid budget
+    const int want = target_ctas / bg;
+    return want < 1 ? 1 : (want > smax ? smax : want);
+  }
+  // B x G CTAs already cover every SM: no split (with ragged contexts,
+  // measured on 64 sequences of 512-4096 tokens, one split beats two).
+  if (bg >= num_sms) return 1;
+  // One resident CTA per SM (128 KB of staging): choose the split count with
+  // the smallest makespan, waves x (key blocks per split + a per-CTA cost of
+  // about 4 blocks), where a split holds at least one block per warp.
+  int best = 1;
+  long long best_cost = -1;
+  for (int s = 1; s <= smax; ++s) {
+    const int per = max((max_blocks + s - 1) / s, DEC_WARPS);
+    const int used = (max_blocks + per - 1) / per;
+    if (used < s) break;  // further splits would exit at once
+    const long long waves = (static_cast<long long>(bg) * used + num_sms - 1) / num_sms;
+    const long long cost = waves * (per + 4);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = s;
+    }
+  }
+  return best;
 }
 
 cudaError_t launch_attn_decode(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B) {

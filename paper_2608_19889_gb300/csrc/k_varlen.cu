@@ -87,6 +87,54 @@ __global__ void __launch_bounds__(1024) finalize_varlen_kernel(unsigned long lon
   for (int j = threadIdx.x; j < n_keys; j += blockDim.x) keys[j] = 0ull;
 }
 
+// qk-norm of Qwen3-family layers (the RMSNorm built-in applied to each
+// head's d values of q and k before RoPE): one warp per (row, head); heads
+// 0 .. H-1 are q, H .. H+G-1 are k. Reads the QKV epilogue's fp32 values,
+// sums their squares in a fixed order, scales by 1 / sqrt(mean + eps) and
+// the gains, rotates the (j, j + d/2) pairs, and stores q (with its second
+// 16-bit term when q_lo_out is set) or k into the row's cache slot: one
+// rounding, as without the norm.
+template <typename T>
+__global__ void __launch_bounds__(32) qk_norm_rope_kernel(EpiArgs e) {
+  grid_dep_launch();
+  grid_dep_wait();
+  const int m = blockIdx.x, h = blockIdx.y, lane = threadIdx.x;
+  const int d = e.d, half = d >> 1;
+  const float* x = e.qk_raw + (static_cast<long long>(m) * (e.H + e.G) + h) * d;
+  float ss = 0.f;
+  for (int i = lane; i < d; i += 32) ss += x[i] * x[i];
+  ss = warp_sum(ss);
+  const float r = 1.0f / sqrtf(ss / static_cast<float>(d) + e.eps);
+  const bool is_q = h < e.H;
+  const float* gn = is_q ? e.qn_gain : e.kn_gain;
+  int b;
+  const int pos = row_seq_pos(e, m, b);
+  T* dst;
+  T* dlo = nullptr;
+  if (is_q) {
+    const long long off = (static_cast<long long>(m) * e.H + h) * d;
+    dst = static_cast<T*>(e.q_out) + off;
+    if (e.q_lo_out) dlo = static_cast<T*>(e.q_lo_out) + off;
+  } else {
+    const long long off = kv_offset(e, b, pos, h - e.H);
+    if (off < 0) return;  // reported where v was stored
+    dst = static_cast<T*>(e.k_cache) + off;
+  }
+  const float2* cs = e.rope + static_cast<long long>(min(max(pos, 0), e.max_pos - 1)) * half;
+  for (int j = lane; j < half; j += 32) {
+    const float a = x[j] * r * gn[j], bb = x[j + half] * r * gn[j + half];
+    const float2 t = cs[j];
+    const float o0 = a * t.x - bb * t.y, o1 = bb * t.x + a * t.y;
+    const T h0 = from_f<T>(o0), h1 = from_f<T>(o1);
+    dst[j] = h0;
+    dst[j + half] = h1;
+    if (dlo) {
+      dlo[j] = from_f<T>(o0 - to_f(h0));
+      dlo[j + half] = from_f<T>(o1 - to_f(h1));
+    }
+  }
+}
+
 template <typename K, typename... Args>
 cudaError_t launch_k(const LaunchCtx& lc, K kernel, dim3 grid, dim3 block, Args... args) {
   cudaLaunchConfig_t cfg = {};
@@ -122,4 +170,12 @@ cudaError_t launch_gather_last(const LaunchCtx& lc, const int* cu, int B, int T,
 cudaError_t launch_finalize_varlen(const LaunchCtx& lc, unsigned long long* keys, int n_keys, const int* cu,
                                    int last_rows, int B, int* next, int* ctx) {
   return launch_k(lc, finalize_varlen_kernel, dim3(1), dim3(1024), keys, n_keys, cu, last_rows, B, next, ctx);
+}
+
+cudaError_t launch_qk_norm_rope(const LaunchCtx& lc, bool fp32, const EpiArgs& e, int rows) {
+  if (rows < 1 || !e.qk_raw || !e.qn_gain || !e.kn_gain) return cudaErrorInvalidValue;
+  const dim3 grid(rows, e.H + e.G);
+  if (fp32) return launch_k(lc, qk_norm_rope_kernel<float>, grid, dim3(32), e);
+  if (lc.f16) return launch_k(lc, qk_norm_rope_kernel<f16>, grid, dim3(32), e);
+  return launch_k(lc, qk_norm_rope_kernel<bf16>, grid, dim3(32), e);
 }

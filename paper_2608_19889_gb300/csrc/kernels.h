@@ -71,6 +71,12 @@ cudaError_t launch_gather_last(const LaunchCtx& lc, const int* cu, int B, int T,
 cudaError_t launch_finalize_varlen(const LaunchCtx& lc, unsigned long long* keys, int n_keys, const int* cu,
                                    int last_rows, int B, int* next, int* ctx);
 
+// ---- qk-norm (k_varlen.cu): q and k of `rows` rows from e.qk_raw,
+// normalised per head, scaled by the gains, rotated and stored (q, its second
+// term when e.q_lo_out is set, k into the cache slot of the row's position);
+// e is the QKV launch's epilogue argument block.
+cudaError_t launch_qk_norm_rope(const LaunchCtx& lc, bool fp32, const EpiArgs& e, int rows);
+
 // ---- attention (k_attn.cu)
 struct AttnArgs {
   const void* q;  // [rows][H*d]
@@ -108,7 +114,10 @@ cudaError_t launch_attn_decode(const LaunchCtx& lc, bool fp32, const AttnArgs& a
 // vl: variable-length batch, or null (B sequences of a.S tokens from position 0)
 cudaError_t launch_attn_prefill(const LaunchCtx& lc, bool fp32, const AttnArgs& a, int B,
                                 const AttnVarlen* vl = nullptr);
-int attn_decode_splits(int B, int G, int max_blocks, int num_sms);
+// Key splits of the decode attention (1 .. min(max_blocks, 64)): the count
+// with the smallest estimated makespan over num_sms SMs, or, with
+// target_ctas > 0, as many as keep B x G x splits within that many CTAs.
+int attn_decode_splits(int B, int G, int max_blocks, int num_sms, int target_ctas);
 // Set kernel attributes (dynamic shared memory limits) once, before any
 // launch or graph capture.
 cudaError_t prepare_attn_kernels();

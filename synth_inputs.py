@@ -30,6 +30,11 @@ MODEL_SHAPES = {
     "0.5b": dict(L=24, D=896, H=14, G=2, d=64, F=4864, V=151936, tie=True, bias=True, theta=1e6, eps=1e-6),
     "8b": dict(L=32, D=4096, H=32, G=8, d=128, F=14336, V=128256, tie=False, bias=False, theta=5e5, eps=1e-5),
     "32b": dict(L=64, D=5120, H=40, G=8, d=128, F=27648, V=152064, tie=False, bias=True, theta=1e6, eps=1e-6),
+    # DeepSeek-MoE-16B-shaped: 28 layers, the first dense, the rest with 64
+    # routed experts (6 per token, weights not renormalised) and 2 shared
+    # experts of width 1408 each; multi-head attention, head_dim 128
+    "moe16b": dict(L=28, D=2048, H=16, G=16, d=128, F=10944, V=102400, tie=False, bias=False, theta=1e4,
+                   eps=1e-6, n_experts=64, top_k=6, moe_F=1408, n_shared=2, first_dense=1, norm_topk=False),
     # Mistral-shaped 7B: the Llama block with a 4096-token sliding window
     "7b_swa": dict(L=32, D=4096, H=32, G=8, d=128, F=14336, V=32000, tie=False, bias=False, theta=1e4, eps=1e-5,
                    window=4096),
@@ -53,7 +58,10 @@ SEED_WEIGHTS, SEED_IDS, SEED_CTX, SEED_BLOCKS = 0, 1, 2, 3
 
 def weight_shapes(m: dict) -> dict:
     """HF Llama parameter names and shapes ([out, in] for matrices); with
-    qk_norm, the per-head q and k RMSNorm gains of Qwen3-family layers."""
+    qk_norm, the per-head q and k RMSNorm gains of Qwen3-family layers; with
+    n_experts > 0, layers from first_dense on carry a mixture-of-experts MLP
+    in the DeepSeek-MoE naming (router mlp.gate, routed mlp.experts.{e}.*,
+    shared mlp.shared_experts.*)."""
     L, D, H, G, d, F, V = (m[k] for k in ("L", "D", "H", "G", "d", "F", "V"))
     shapes = {"model.embed_tokens.weight": (V, D)}
     for l in range(L):
@@ -71,6 +79,20 @@ def weight_shapes(m: dict) -> dict:
             shapes[p + "self_attn.k_norm.weight"] = (d,)
         shapes[p + "self_attn.o_proj.weight"] = (D, H * d)
         shapes[p + "post_attention_layernorm.weight"] = (D,)
+        if m.get("n_experts", 0) and l >= m.get("first_dense", 0):
+            E, Fe, ns = m["n_experts"], m["moe_F"], m.get("n_shared", 0)
+            shapes[p + "mlp.gate.weight"] = (E, D)
+            for e in range(E):
+                q = f"{p}mlp.experts.{e}."
+                shapes[q + "gate_proj.weight"] = (Fe, D)
+                shapes[q + "up_proj.weight"] = (Fe, D)
+                shapes[q + "down_proj.weight"] = (D, Fe)
+            if ns:
+                q = p + "mlp.shared_experts."
+                shapes[q + "gate_proj.weight"] = (ns * Fe, D)
+                shapes[q + "up_proj.weight"] = (ns * Fe, D)
+                shapes[q + "down_proj.weight"] = (D, ns * Fe)
+            continue
         shapes[p + "mlp.gate_proj.weight"] = (F, D)
         shapes[p + "mlp.up_proj.weight"] = (F, D)
         shapes[p + "mlp.down_proj.weight"] = (D, F)

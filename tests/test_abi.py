@@ -80,6 +80,7 @@ def test_invalid_configs_are_rejected_before_any_device_work(built):
     cases = [
         (dict(sliding_window=-1), ax.AXON_ERR_INVALID_ARG),
         (dict(hidden_act=5), ax.AXON_ERR_INVALID_ARG),
+        (dict(qk_norm=2), ax.AXON_ERR_INVALID_ARG),
         (dict(rope_scaling_factor=8.0, rope_low_freq_factor=4.0, rope_high_freq_factor=1.0,
               rope_original_max_position=8192), ax.AXON_ERR_INVALID_ARG),
         (dict(rope_scaling_factor=-1.0), ax.AXON_ERR_INVALID_ARG),

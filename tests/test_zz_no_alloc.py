@@ -11,17 +11,22 @@ array owned by the library.
 
 Each case below is chosen so that the attention really splits the keys, and
 so really writes and merges partial states in that shared array:
-  * launch chain (B > 8), 10 key splits per (sequence, kv head), the same
-    count as the regular step: results must be bit-identical;
-  * launch chain with more splits than the fixed array holds: the step keeps
-    256 / (B * kv heads) = 8 of the regular step's 10 (94 key blocks in
-    splits of 12 instead of 10), so the fp32 merge order and the 16-bit
-    rounding of the attention output differ;
+  * launch chain (B > 8) over 10 key blocks of capacity: 2 key splits per
+    (sequence, kv head), the same count as the regular step, so results must
+    be bit-identical;
+  * launch chain with more splits than the fixed array holds: the model is
+    created with a grid budget of 1024 attention CTAs (AXON_ATTN_TARGET_CTAS),
+    which gives the regular step 32 splits of its 128 blocks of capacity; the
+    fixed array keeps 256 / (B * kv heads) = 8, so the 94 blocks of context
+    fall into 8 splits of 12 blocks instead of 12 splits of 8, and the fp32
+    merge order and the 16-bit rounding of the attention output differ;
   * the persistent single-launch step (B <= 8) over more than 64 key blocks,
     which it cuts into items of 16 blocks: 5 splits, bit-identical.
 The second call checks that what the first call left in the shared array
 does not leak into its result. This file is collected last so a failure
 here comes after every other test."""
+import os
+
 import numpy as np
 import pytest
 
@@ -33,11 +38,12 @@ pytestmark = pytest.mark.gpu
 
 SHAPE = dict(L=2, D=256, H=8, G=2, d=128, F=320, V=1000, tie=False, bias=True, theta=1e4, eps=1e-5)
 
-# (case, B, prompt length, max_context, bit-identical to the regular step)
+# (case, B, prompt length, max_context, bit-identical to the regular step,
+#  attention grid budget at creation or None)
 CASES = [
-    ("chain_10_splits", 12, 140, 160, True),
-    ("chain_splits_clamped", 16, 1500, 2048, False),
-    ("persistent_5_splits", 2, 1100, 1280, True),
+    ("chain_2_splits", 12, 140, 160, True, None),
+    ("chain_splits_clamped", 16, 1500, 2048, False, 1024),
+    ("persistent_5_splits", 2, 1100, 1280, True, None),
 ]
 
 
@@ -50,12 +56,20 @@ def _built():
 
 
 @pytest.mark.parametrize("prec", ["bf16", "fp16"])
-@pytest.mark.parametrize("case,B,S,max_ctx,identical", CASES)
-def test_noalloc_decode_two_calls(case, B, S, max_ctx, identical, prec):
+@pytest.mark.parametrize("case,B,S,max_ctx,identical,target", CASES)
+def test_noalloc_decode_two_calls(case, B, S, max_ctx, identical, target, prec):
     import paper_2608_19889_gb300 as ax
     V = SHAPE["V"]
     w = gpu_weights(SHAPE)
-    m = create(SHAPE, w, max_batch=B, max_context=max_ctx, fp16=prec == "fp16")
+    old = os.environ.pop("AXON_ATTN_TARGET_CTAS", None)
+    try:
+        if target:
+            os.environ["AXON_ATTN_TARGET_CTAS"] = str(target)
+        m = create(SHAPE, w, max_batch=B, max_context=max_ctx, fp16=prec == "fp16")
+    finally:
+        os.environ.pop("AXON_ATTN_TARGET_CTAS", None)
+        if old is not None:
+            os.environ["AXON_ATTN_TARGET_CTAS"] = old
     try:
         ids = si.make_ids(B, S, V, seed=11)
         tok = torch.empty(B, dtype=torch.int32, device="cuda")
