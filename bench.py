@@ -35,10 +35,44 @@ METRIC = "decode & prefill tokens/s on 1 GB300; % of HBM / BF16 tensor roofline"
 DEFAULT_WORKLOAD = "32b_b16_s2048_n256"
 
 
-def model_bytes(m):
+def moe_layers(m):
+    """Layers with a mixture-of-experts MLP."""
+    return max(0, m["L"] - m.get("first_dense", 0)) if m.get("n_experts", 0) else 0
+
+
+def expected_active_experts(m, tokens):
+    """Distinct experts that `tokens` tokens route to when each picks top_k
+    of E uniformly: E (1 - (1 - k/E)^tokens). The algorithmic expert bytes
+    of a decode step; the routing itself is decided on the device."""
+    E, k = m["n_experts"], m["top_k"]
+    return E * (1.0 - (1.0 - k / E) ** tokens)
+
+
+def model_bytes(m, active_experts=None):
+    """(linear weight elements, LM head elements). Mixture-of-experts layers
+    count the router, the shared experts and `active_experts` routed experts
+    (all E when None)."""
     L, D, H, G, d, F, V = (m[k] for k in ("L", "D", "H", "G", "d", "F", "V"))
-    lin = L * ((H + 2 * G) * d * D + D * H * d + 2 * F * D + D * F)
+    attn = (H + 2 * G) * d * D + D * H * d
+    Lm = moe_layers(m)
+    lin = L * attn + (L - Lm) * 3 * F * D
+    if Lm:
+        E, Fe = m["n_experts"], m["moe_F"]
+        act = E if active_experts is None else active_experts
+        lin += Lm * (E * D + 3 * m.get("n_shared", 0) * Fe * D + act * 3 * Fe * D)
     return lin, V * D
+
+
+def linear_flops_per_token(m):
+    """2 x the weight elements one token multiplies: attention projections,
+    dense MLPs, and in MoE layers the router, the shared experts and top_k
+    routed experts."""
+    L, D, H, G, d, F = (m[k] for k in ("L", "D", "H", "G", "d", "F"))
+    Lm = moe_layers(m)
+    per = L * ((H + 2 * G) * d * D + D * H * d) + (L - Lm) * 3 * F * D
+    if Lm:
+        per += Lm * (m["n_experts"] * D + 3 * (m.get("n_shared", 0) + m["top_k"]) * m["moe_F"] * D)
+    return 2 * per
 
 
 def keys_seen(pos, window):
@@ -58,9 +92,10 @@ def decode_bytes_per_step(m, B, T_list):
     """Algorithmic HBM bytes of one decode step: every weight once (bf16),
     norms/biases, KV read of the keys each new token sees (all cached tokens
     + itself, or its sliding window), KV write, fp32 logits write."""
-    lin, head = model_bytes(m)
+    lin, head = model_bytes(m, expected_active_experts(m, B) if moe_layers(m) else None)
     L, D, G, d, V = m["L"], m["D"], m["G"], m["d"], m["V"]
     small = (2 * L + 1) * D * 4 + (L * (m["H"] + 2 * G) * d * 4 if m["bias"] else 0)
+    small += moe_layers(m) * m.get("n_experts", 0) * D * 2  # fp32 routers counted in bf16 above
     kv_tok = L * 2 * G * d * 2
     kv_read = sum(keys_seen(int(t), m.get("window", 0)) for t in T_list) * kv_tok
     kv_write = B * kv_tok
@@ -68,9 +103,9 @@ def decode_bytes_per_step(m, B, T_list):
 
 
 def prefill_flops(m, B, S):
-    lin, head = model_bytes(m)
+    _, head = model_bytes(m)
     attn = m["L"] * B * 4 * m["H"] * m["d"] * keys_seen_by_run(0, S, m.get("window", 0))
-    return 2 * B * S * lin + attn + 2 * B * head
+    return B * S * linear_flops_per_token(m) + attn + 2 * B * head
 
 
 def tensor_peak(burst, sustained, phase_ms):
@@ -188,15 +223,19 @@ def oracle_one_layer_timed(wl, n_dec=2):
     on the values). Returns (generated tokens/s, sample description)."""
     from oracle import decoder as od
     m = si.MODEL_SHAPES[wl["model"]]
-    L, V = m["L"], m["V"]
-    m1 = dict(m, L=1)
+    V = m["V"]
+    # the layer timed is a typical one: with a mixture of experts, the first
+    # layer after the leading dense ones (which the base run includes)
+    base = m.get("first_dense", 0) if m.get("n_experts", 0) else 0
+    L = m["L"] - base
+    m1 = dict(m, L=base + 1)
     w = si.make_weights(m1, device="cpu")
     W = si.weights_as_f32_numpy(w)
     del w
     o1 = od.Oracle(od.DecoderConfig.from_dict(m1), W, keep_f64=True)
     del W
-    # L = 0 on the same float64 arrays (no copy: they are float64 already)
-    o0 = od.Oracle(od.DecoderConfig.from_dict(dict(m, L=0)), o1.W, keep_f64=False)
+    # the base layers only, on the same float64 arrays (no copy)
+    o0 = od.Oracle(od.DecoderConfig.from_dict(dict(m, L=base)), o1.W, keep_f64=False)
     B, n_new = wl["B"], wl["n_new"]
     tok = si.make_ids(1, B, V, seed=7)[0]
 
@@ -216,13 +255,14 @@ def oracle_one_layer_timed(wl, n_dec=2):
         num_blocks = int(sum(-(-int(c) // 16) for c in caps)) + 64
         bt = si.make_block_table(caps, 16, max_ctx // 16, num_blocks)
         c1 = o1.new_paged_cache(num_blocks, 16, bt)
-        c1.K[0].fill(0.01)
-        c1.V[0].fill(0.01)
+        for li in range(len(c1.K)):
+            c1.K[li].fill(0.01)
+            c1.V[li].fill(0.01)
         c0 = o0.new_paged_cache(num_blocks, 16, bt)
         d1 = decode_time(o1, c1, lens)
         d0 = decode_time(o0, c0, lens)
         per_step = d0 + L * max(d1 - d0, 0.0)
-        sample = (f"one full-width layer + embedding/norm/LM head, extrapolated by L={L}: {n_dec} decode steps of "
+        sample = (f"one full-width layer + embedding/norm/LM head{" + " + str(base) + " leading dense layer(s)" if base else ""}, extrapolated by {L} layers: {n_dec} decode steps of "
                   f"B={B} over a paged cache at contexts {lo}..{hi} (K/V contents constant, timing only): "
                   f"{d1:.2f}s/step with the layer, {d0:.2f}s/step without")
         return B * n_new / (n_new * per_step), sample
@@ -232,8 +272,9 @@ def oracle_one_layer_timed(wl, n_dec=2):
     p1, _ = _timed(lambda: o1.prefill(ids, c1, last_only=True))
     p0, _ = _timed(lambda: o0.prefill(ids, o0.new_contiguous_cache(1, S), last_only=True))
     cB = o1.new_contiguous_cache(B, S + n_dec)
-    cB.K[0][:, :S] = c1.K[0][0]
-    cB.V[0][:, :S] = c1.V[0][0]
+    for li in range(len(cB.K)):
+        cB.K[li][:, :S] = c1.K[li][0]
+        cB.V[li][:, :S] = c1.V[li][0]
     del c1
     lens = np.full(B, S)
     d1 = decode_time(o1, cB, lens)
@@ -241,7 +282,8 @@ def oracle_one_layer_timed(wl, n_dec=2):
     t_pre = B * (p0 + L * max(p1 - p0, 0.0))
     per_step = d0 + L * max(d1 - d0, 0.0)
     t_full = t_pre + n_new * per_step
-    sample = (f"one full-width layer + embedding/norm/LM head, extrapolated by L={L}: prefill of 1 x {S} tokens "
+    sample = (f"one full-width layer + embedding/norm/LM head{' + ' + str(base) + ' leading dense layer(s)' if base else ''}, "
+              f"extrapolated by {L} layers: prefill of 1 x {S} tokens "
               f"({p1:.2f}s with the layer, {p0:.2f}s without; x B={B}) + {n_dec} decode steps of B={B} at context "
               f"{S} ({d1:.3f}s/step with the layer, {d0:.3f}s/step without); generate = prefill + {n_new} steps")
     return B * n_new / t_full, sample
@@ -402,12 +444,12 @@ def varlen_prefill_flops(m, calls):
     [(past, chunk)] per call: every new token through every linear, causal
     attention of token past + i over past + i + 1 keys, the LM head on each
     chunk's last token."""
-    lin, head = model_bytes(m)
+    _, head = model_bytes(m)
     total = 0.0
     for chunks in calls:
         T = sum(n for _, n in chunks)
         keys = sum(keys_seen_by_run(past, n, m.get("window", 0)) for past, n in chunks)
-        total += 2 * T * lin + m["L"] * 4 * m["H"] * m["d"] * keys + 2 * len(chunks) * head
+        total += T * linear_flops_per_token(m) + m["L"] * 4 * m["H"] * m["d"] * keys + 2 * len(chunks) * head
     return total
 
 

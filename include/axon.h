@@ -120,6 +120,23 @@ typedef struct axon_config {
                                   the gains model.layers.{i}.self_attn.{q,k}_norm.weight [head_dim],
                                   before RoPE (Qwen3-family layers); 0: none. Decode then always
                                   takes the launch chain. */
+  /* Mixture of experts (the MoE built-ins: softmax top-k router, grouped
+   * experts; DeepSeek-MoE layout). n_routed_experts E > 0: layers from
+   * first_k_dense_replace on replace the MLP by
+   *   p = softmax(h W_router^T) over the E experts (fp32 router),
+   *   the num_experts_per_tok experts with the largest p (lowest index on
+   *   ties), weights p (divided by their sum when norm_topk_prob),
+   *   y = sum_j w_j * SwiGLU-MLP_j(h) + SwiGLU-MLP_shared(h),
+   * with experts of width moe_intermediate_size and, when
+   * n_shared_experts > 0, one shared MLP of width n_shared_experts *
+   * moe_intermediate_size. E <= 256, 1 <= num_experts_per_tok <= min(8, E),
+   * 16-bit modes only; decode takes the launch chain. */
+  int32_t n_routed_experts;
+  int32_t num_experts_per_tok;
+  int32_t moe_intermediate_size;
+  int32_t n_shared_experts;
+  int32_t first_k_dense_replace;
+  int32_t norm_topk_prob;
 } axon_config;
 
 /* One named checkpoint tensor, HF Llama naming and [out, in] matrices, as a
@@ -134,6 +151,15 @@ typedef struct axon_config {
  *   model.layers.{i}.mlp.{gate,up}_proj.weight      [F, D]
  *   model.layers.{i}.mlp.down_proj.weight           [D, F]
  *   model.layers.{i}.self_attn.{q,k}_norm.weight    [d] (if qk_norm)
+ *   mixture-of-experts layers (i >= first_k_dense_replace when
+ *   n_routed_experts > 0) carry instead of mlp.{gate,up,down}_proj:
+ *   model.layers.{i}.mlp.gate.weight                [E, D] (router)
+ *   model.layers.{i}.mlp.experts.{e}.{gate,up}_proj.weight [Fe, D]
+ *   model.layers.{i}.mlp.experts.{e}.down_proj.weight      [D, Fe]
+ *   model.layers.{i}.mlp.shared_experts.{gate,up}_proj.weight [Fs, D]
+ *   model.layers.{i}.mlp.shared_experts.down_proj.weight   [D, Fs]
+ *     (Fe = moe_intermediate_size, Fs = n_shared_experts * Fe; shared only
+ *     when n_shared_experts > 0)
  *   model.norm.weight                               [D]
  *   lm_head.weight                                  [V, D] (absent if tied)
  * `data` may be a host or a device pointer (unified addressing); it is
@@ -315,6 +341,19 @@ int axon_profile_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t
  * differ from it by floating-point rounding of the merge. */
 int axon_decode_step_noalloc(axon_model* m, const int32_t* d_tokens, int32_t B, int32_t* d_context_lens,
                              const int32_t* d_block_table, float* d_logits, int32_t* d_next, void* stream);
+
+/* Inspection hook for mixture-of-experts models (the routing is decided on
+ * the device; tests compare it with the oracle's). With d_experts non-NULL,
+ * every later prefill or decode pass writes, for each MoE layer l and each
+ * of its first `rows` token rows t (in the pass's row order: b * S + s for
+ * axon_prefill, b for axon_decode_step, packed rows for
+ * axon_prefill_varlen), the chosen experts in rank order into
+ * d_experts[(l * rows + t) * num_experts_per_tok + j] (int32, device
+ * memory owned by the caller, L * rows * num_experts_per_tok entries;
+ * rows of dense layers are not written). NULL turns recording off.
+ * AXON_ERR_UNSUPPORTED for models without experts. Decode graphs recorded
+ * before the call are dropped. */
+int axon_moe_routing_record(axon_model* m, int32_t* d_experts, int32_t rows);
 
 /* Release everything the model owns. NULL is a no-op. */
 void axon_free(axon_model* m);

@@ -32,7 +32,7 @@ AXON_ACT_SILU, AXON_ACT_GELU_TANH = 0, 1
 
 EXPORTED = ["axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset",
             "axon_check_device", "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill",
-            "axon_decode_step_noalloc", "axon_free", "axon_status_string"]
+            "axon_decode_step_noalloc", "axon_moe_routing_record", "axon_free", "axon_status_string"]
 
 
 class axon_config(ctypes.Structure):
@@ -43,7 +43,9 @@ class axon_config(ctypes.Structure):
         (n, ctypes.c_int32) for n in ("max_batch", "max_context", "max_prefill_tokens", "kv_layout",
                                       "kv_block_size", "kv_num_blocks", "precision", "sliding_window")] + [
         (n, ctypes.c_float) for n in ("rope_scaling_factor", "rope_low_freq_factor", "rope_high_freq_factor")] + [
-        ("rope_original_max_position", ctypes.c_int32), ("hidden_act", ctypes.c_int32), ("qk_norm", ctypes.c_int32)]
+        ("rope_original_max_position", ctypes.c_int32), ("hidden_act", ctypes.c_int32), ("qk_norm", ctypes.c_int32)] + [
+        (n, ctypes.c_int32) for n in ("n_routed_experts", "num_experts_per_tok", "moe_intermediate_size",
+                                      "n_shared_experts", "first_k_dense_replace", "norm_topk_prob")]
 
 
 class axon_tensor(ctypes.Structure):
@@ -84,6 +86,7 @@ def lib() -> ctypes.CDLL:
         L.axon_prefill_varlen.argtypes = [vp, vp, i32, i32, vp, vp, i32, vp, i32, vp, vp, vp]
         L.axon_decode_step.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
         L.axon_decode_step_noalloc.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
+        L.axon_moe_routing_record.argtypes = [vp, vp, i32]
         L.axon_reset.argtypes = [vp]
         L.axon_check_device.argtypes = [vp, vp, p_i32]
         L.axon_kv_view_get.argtypes = [vp, ctypes.POINTER(axon_kv_view)]
@@ -96,7 +99,7 @@ def lib() -> ctypes.CDLL:
         L.axon_status_string.restype = ctypes.c_char_p
         for n in ("axon_model_create", "axon_prefill", "axon_prefill_varlen", "axon_decode_step", "axon_reset",
                   "axon_check_device", "axon_kv_view_get", "axon_profile_decode_step", "axon_profile_prefill",
-                  "axon_decode_step_noalloc"):
+                  "axon_decode_step_noalloc", "axon_moe_routing_record"):
             getattr(L, n).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -126,13 +129,16 @@ def make_config(m: dict, max_batch: int, max_context: int, kv_layout=AXON_KV_CON
                 precision=AXON_BF16, max_prefill_tokens=0) -> axon_config:
     """axon_config from a shape dict with keys L, D, H, G, d, F, V, tie, bias, theta, eps (and optionally
     window, the sliding window, rope_factor / rope_low / rope_high / rope_orig, the RoPE frequency
-    scaling, 0 or absent = none; act, "silu" (default) or "gelu_tanh"; qk_norm, per-head RMSNorm of q and k)."""
+    scaling, 0 or absent = none; act, "silu" (default) or "gelu_tanh"; qk_norm, per-head RMSNorm of q and k;
+    n_experts, top_k, moe_F, n_shared, first_dense, norm_topk: the mixture-of-experts MLP)."""
     return axon_config(m["L"], m["D"], m["H"], m["G"], m["d"], m["F"], m["V"], int(m["tie"]), int(m["bias"]),
                        float(m["theta"]), float(m["eps"]), max_batch, max_context, max_prefill_tokens, kv_layout, 16,
                        kv_num_blocks, precision, int(m.get("window", 0)), float(m.get("rope_factor", 0.0)),
                        float(m.get("rope_low", 1.0)), float(m.get("rope_high", 4.0)), int(m.get("rope_orig", 8192)),
                        AXON_ACT_GELU_TANH if m.get("act", "silu") == "gelu_tanh" else AXON_ACT_SILU,
-                       int(bool(m.get("qk_norm", False))))
+                       int(bool(m.get("qk_norm", False))), int(m.get("n_experts", 0)), int(m.get("top_k", 0)),
+                       int(m.get("moe_F", 0)), int(m.get("n_shared", 0)), int(m.get("first_dense", 0)),
+                       int(bool(m.get("norm_topk", False))))
 
 
 def axon_model_create(cfg: axon_config, weights: dict, stream=None) -> ctypes.c_void_p:
@@ -184,6 +190,12 @@ def axon_decode_step(m, tokens, context_lens, block_table=None, logits=None, nex
     B = tokens.shape[0]
     _check("axon_decode_step", lib().axon_decode_step(m, _ptr(tokens), B, _ptr(context_lens), _ptr(block_table),
                                                       _ptr(logits), _ptr(next_tokens), _stream(stream)))
+
+
+def axon_moe_routing_record(m, experts=None, rows=0):
+    """experts: int32 device tensor [L, rows, k] that later passes fill with
+    each MoE layer's chosen experts (see include/axon.h), or None to stop."""
+    _check("axon_moe_routing_record", lib().axon_moe_routing_record(m, _ptr(experts), int(rows)))
 
 
 def axon_decode_step_noalloc(m, tokens, context_lens, block_table=None, logits=None, next_tokens=None, stream=None):

@@ -17,7 +17,7 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libaxon_gb300.so")
 SOURCES = ["api.cu", "k_gemv.cu", "k_attn.cu", "k_gemm.cu", "k_simt.cu", "k_persist.cu",
-           "k_varlen.cu", "noalloc.cu"]
+           "k_varlen.cu", "k_moe.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr", "-I" + INCLUDE]
 

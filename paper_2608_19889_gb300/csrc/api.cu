@@ -35,6 +35,15 @@ struct LayerW {
   float* g2 = nullptr;
   float* qn = nullptr;  // qk-norm gains [d] (null when off)
   float* kn = nullptr;
+  int Fl = 0;  // width of the layer's dense SwiGLU MLP (the shared experts' in a MoE layer; 0: none)
+  // mixture of experts: fp32 router [E][D]; the experts stacked as one
+  // [E * 2Fe][D] gate/up tensor (each expert's rows interleaved in 16-row
+  // chunks like the dense one) and one [E * D][Fe] down tensor
+  bool moe = false;
+  float* router = nullptr;
+  void* wgu_e = nullptr;
+  void* wd_e = nullptr;
+  GemmMaps m_gu_e{}, m_d_e{}, m_gu_e128{}, m_d_e128{};
   GemmMaps m_qkv{}, m_o{}, m_gu{}, m_d{};
   GemmMaps m_qkv128{}, m_o128{}, m_gu128{}, m_d128{};  // the same with 128-row weight boxes
   CUtensorMap v_qkv{}, v_o{}, v_gu{}, v_d{};  // weight maps for the decode projections (box 64 x 128)
@@ -100,7 +109,7 @@ struct axon_model {
   int* attn_cnt = nullptr;
   int max_splits = 1;
   int* err = nullptr;
-  CUtensorMap t_a{}, t_o{}, t_u{}, t_alo{};
+  CUtensorMap t_a{}, t_o{}, t_alo{};
   // decode graphs
   cudaStream_t cap_stream = nullptr;
   std::map<GraphKey, cudaGraphExec_t> graphs;
@@ -118,6 +127,26 @@ struct axon_model {
   // split count with the smallest estimated makespan)
   int attn_target_ctas = 0;
   GemmSplitK gemm_sk{};      // split-K workspace of the decode-sized tensor-core GEMMs
+  // mixture of experts: routing and sorted-row workspace for up to Mcap
+  // tokens (R_cap sorted rows)
+  bool moe = false;
+  int E = 0, topk = 0, Fe = 0;
+  long long R_cap = 0;
+  int* moe_topk_idx = nullptr;
+  float* moe_topk_w = nullptr;
+  int* moe_slot_row = nullptr;
+  int* moe_row_tok = nullptr;
+  float* moe_row_w = nullptr;
+  int* moe_mb_expert = nullptr;
+  int* moe_nmb = nullptr;
+  float* moe_ones = nullptr;  // [1] = 1.0: the sorted operand is already normalised
+  void* moe_h = nullptr;      // [Mcap][D]
+  void* moe_a_sorted = nullptr;
+  void* moe_u_sorted = nullptr;
+  float* moe_y_sorted = nullptr;
+  CUtensorMap t_asorted{}, t_usorted{};
+  int32_t* moe_record = nullptr;  // axon_moe_routing_record: [L][record_rows][k], or null
+  int moe_record_rows = 0;
 };
 
 namespace {
@@ -130,6 +159,12 @@ namespace {
         fprintf(stderr, "axon: %s failed: %s (%s:%d)\n", #call, cudaGetErrorString(e_), __FILE__, __LINE__); \
       return AXON_ERR_CUDA;                                                         \
     }                                                                               \
+  } while (0)
+
+#define CK_RC(expr)        \
+  do {                     \
+    const int rc_ = (expr); \
+    if (rc_) return rc_;    \
   } while (0)
 
 int dev_alloc(axon_model* m, void** p, size_t bytes) {
@@ -282,6 +317,17 @@ int validate_config(const axon_config* c) {
   if (c->rope_scaling_factor < 0.f) return AXON_ERR_INVALID_ARG;
   if (c->hidden_act != AXON_ACT_SILU && c->hidden_act != AXON_ACT_GELU_TANH) return AXON_ERR_INVALID_ARG;
   if (c->qk_norm != 0 && c->qk_norm != 1) return AXON_ERR_INVALID_ARG;
+  if (c->n_routed_experts < 0 || c->n_shared_experts < 0 || c->first_k_dense_replace < 0 ||
+      (c->norm_topk_prob != 0 && c->norm_topk_prob != 1))
+    return AXON_ERR_INVALID_ARG;
+  if (c->n_routed_experts > 0) {
+    if (c->num_experts_per_tok < 1 || c->num_experts_per_tok > 8 || c->num_experts_per_tok > c->n_routed_experts ||
+        c->moe_intermediate_size <= 0 || c->first_k_dense_replace > c->num_hidden_layers)
+      return AXON_ERR_INVALID_ARG;
+    if (c->n_routed_experts > MOE_MAX_EXPERTS || c->moe_intermediate_size % 64 || c->hidden_size % 128 ||
+        c->precision == AXON_FP32_DEBUG)
+      return AXON_ERR_UNSUPPORTED;
+  }
   if (c->rope_scaling_factor > 0.f &&
       (c->rope_original_max_position <= 0 || c->rope_low_freq_factor <= 0.f ||
        c->rope_high_freq_factor <= c->rope_low_freq_factor))
@@ -488,6 +534,137 @@ struct Proj {
   }
 };
 
+// Expected number of distinct experts that T tokens route to when each
+// picks k of E experts uniformly: E * (1 - (1 - k/E)^T). The algorithmic
+// expert-weight bytes of a mixture-of-experts step (the routing itself is
+// known only on the device).
+double expected_active_experts(int E, int k, int T) {
+  return E * (1.0 - std::pow(1.0 - static_cast<double>(k) / E, static_cast<double>(T)));
+}
+
+MoeArgs moe_args(const axon_model* m, const LayerW& w) {
+  MoeArgs a;
+  memset(&a, 0, sizeof(a));
+  a.D = m->D;
+  a.E = m->E;
+  a.k = m->topk;
+  a.norm_topk = m->cfg.norm_topk_prob;
+  a.act = m->a;
+  a.act_lo = m->a_lo;
+  a.act_stride = m->D;
+  a.router = w.router;
+  a.h_hi = m->moe_h;
+  a.topk_idx = m->moe_topk_idx;
+  a.topk_w = m->moe_topk_w;
+  a.slot_row = m->moe_slot_row;
+  a.row_tok = m->moe_row_tok;
+  a.row_w = m->moe_row_w;
+  a.mb_expert = m->moe_mb_expert;
+  a.n_mblocks = m->moe_nmb;
+  a.a_sorted = m->moe_a_sorted;
+  a.y_sorted = m->moe_y_sorted;
+  a.err = m->err;
+  return a;
+}
+
+// The MLP half of layer l, after the O projection left the operand
+// a = x * g2 with norm state ns: the dense SwiGLU MLP, or the mixture of
+// experts -- routing, the stable sort into expert segments, the grouped
+// expert GEMMs (gate/up + SwiGLU, down scaled by the routing weight), the
+// combine into the residual -- followed by the shared experts' MLP when the
+// layer has one. `row` carries the row -> (sequence, position) map of the
+// pass (S, rowmap or ctx); `decode` selects the decode projections' second
+// SwiGLU term and the profiler names. Updates ns to the next operand's
+// norm state.
+int enqueue_mlp(axon_model* m, int l, Proj& pj, const LaunchCtx& lc, Prof* pf, const EpiArgs& row, int M,
+                bool decode, NormState& ns) {
+  const LayerW& w = m->layers[l];
+  const int D = m->D;
+  const double es = static_cast<double>(m->esz);
+  const float* gnext = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
+  if (w.moe) {
+    const int E = m->E, k = m->topk, Fe = m->Fe;
+    const int R = static_cast<int>(m->R_cap);
+    const double act = expected_active_experts(E, k, M);
+    MoeArgs ma = moe_args(m, w);
+    if (m->moe_record) {
+      ma.record = m->moe_record + static_cast<size_t>(l) * m->moe_record_rows * k;
+      ma.record_rows = m->moe_record_rows;
+    }
+    EpiArgs nx = base_epi(m);
+    set_norm(m, ns, nx);
+    pbeg(pf, decode ? "decode_moe_route" : "prefill_moe_route");
+    CK(launch_moe_route(lc, ma, M, nx));
+    CK(launch_moe_plan(lc, ma, M));
+    CK(launch_moe_gather(lc, ma));
+    pend(pf, static_cast<double>(E) * D * 4 + M * D * (2 * es + es * k), 2.0 * M * E * D);
+    // tile width: 128 when the experts' blocks alone leave most SMs idle
+    const int tn = (static_cast<long long>(M) * k * ((D + 255) / 256) < m->num_sms) ? 128 : 256;
+    GemmGroup grp;
+    grp.mb_expert = m->moe_mb_expert;
+    grp.n_mblocks = m->moe_nmb;
+    grp.row_valid = m->moe_row_tok;
+    EpiArgs g = base_epi(m);
+    g.M = R;
+    g.N = 2 * Fe;
+    g.u_out = m->moe_u_sorted;
+    g.rinv = m->moe_ones;  // the sorted rows are normalised already
+    g.rinv_stride = 0;
+    pbeg(pf, decode ? "decode_moe_gateup" : "prefill_moe_gateup");
+    CK(launch_gemm_tc(lc, EPI_SWIGLU, w.m_gu_e, R, 2 * Fe, D, g, tn, nullptr, &grp));
+    pend(pf, act * 2.0 * Fe * D * es + M * k * (D + Fe) * es, 2.0 * M * k * 2 * Fe * D);
+    EpiArgs dn = base_epi(m);
+    dn.M = R;
+    dn.N = D;
+    dn.y_out = m->moe_y_sorted;
+    dn.row_w = m->moe_row_w;
+    pbeg(pf, decode ? "decode_moe_down" : "prefill_moe_down");
+    CK(launch_gemm_tc(lc, EPI_ROWSCALE, w.m_d_e, R, D, Fe, dn, tn, nullptr, &grp));
+    pend(pf, act * static_cast<double>(D) * Fe * es + M * k * (Fe * es + D * 4.0), 2.0 * M * k * D * Fe);
+    EpiArgs cb = base_epi(m);
+    cb.M = M;
+    cb.N = D;
+    cb.x = m->x;
+    if (!w.Fl) {  // no shared experts: the combine is the layer's residual producer
+      cb.a_out = m->a;
+      cb.a_lo_out = m->a_lo;
+      cb.gain = gnext;
+      cb.ss_out = m->ss;
+      cb.ss_out_stride = m->Pmax;
+    }
+    pbeg(pf, decode ? "decode_moe_combine" : "prefill_moe_combine");
+    CK(launch_moe_combine(lc, ma, M, cb));
+    pend(pf, M * (k * D * 4.0 + D * (8.0 + (w.Fl ? 0 : es))), 0);
+    if (!w.Fl) {
+      ns.rinv = false;
+      ns.parts = D / 16;
+      return AXON_OK;
+    }
+  }
+  const int Fl = w.Fl;
+  EpiArgs g = row;
+  set_norm(m, ns, g);
+  g.u_out = m->u;
+  if (decode) g.u_lo_out = m->u_lo;
+  pbeg(pf, decode ? "decode_gateup" : "prefill_gateup");
+  pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * Fl, D, m->a, D, M, g);
+  CK(pj.rc);
+  pend(pf, 2.0 * Fl * D * es + M * (D + Fl) * es, 2.0 * M * 2 * Fl * D);
+
+  EpiArgs dn = row;
+  dn.x = m->x;
+  dn.a_out = m->a;
+  dn.gain = gnext;
+  dn.a_lo_out = m->a_lo;
+  dn.ss_out = m->ss;
+  dn.ss_out_stride = m->Pmax;
+  pbeg(pf, decode ? "decode_down" : "prefill_down");
+  ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, Fl, m->u, Fl, M, dn);
+  CK(pj.rc);
+  pend(pf, static_cast<double>(D) * Fl * es + M * (Fl * es + D * (8 + es)), 2.0 * M * D * Fl);
+  return AXON_OK;
+}
+
 // A variable-length batch (axon_prefill_varlen): sequence b's chunk is rows
 // cu[b] .. cu[b+1]-1 of the T packed rows, after ctx[b] cached tokens; ctx is
 // advanced by the chunk lengths at the end.
@@ -507,7 +684,6 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
   g_trace_stream = st;
   const double es = static_cast<double>(m->esz);
   const double wq = static_cast<double>(m->Nqkv) * m->D * es, wo = static_cast<double>(m->D) * m->H * m->d * es,
-               wgu = 2.0 * m->F * m->D * es, wdn = static_cast<double>(m->D) * m->F * es,
                whd = static_cast<double>(m->V) * m->D * es;
   Proj pj{m, lc};
   const int D = m->D, Hd = m->H * m->d;
@@ -559,29 +735,10 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
     CK(pj.rc);
     pend(pf, wo + M * (Hd * es + D * (8 + es)), 2.0 * M * D * Hd);
 
-    EpiArgs g = base_epi(m);
-    g.S = S;
-    g.rowmap = rowmap;
-    set_norm(m, ns, g);
-    g.u_out = m->u;
-    pbeg(pf, "prefill_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, M, g);
-    CK(pj.rc);
-    pend(pf, wgu + M * (D + m->F) * es, 2.0 * M * 2 * m->F * D);
-
-    EpiArgs dn = base_epi(m);
-    dn.S = S;
-    dn.rowmap = rowmap;
-    dn.x = m->x;
-    dn.a_out = m->a;
-    dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
-    dn.ss_out = m->ss;
-    dn.ss_out_stride = m->Pmax;
-    dn.a_lo_out = m->a_lo;
-    pbeg(pf, "prefill_down");
-    ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, M, dn);
-    CK(pj.rc);
-    pend(pf, wdn + M * (m->F * es + D * (8 + es)), 2.0 * M * D * m->F);
+    EpiArgs row = base_epi(m);
+    row.S = S;
+    row.rowmap = rowmap;
+    CK_RC(enqueue_mlp(m, l, pj, lc, pf, row, M, false, ns));
   }
   EpiArgs h = base_epi(m);
   h.S = S;
@@ -645,10 +802,10 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 
 // The persistent step's attention always pairs q's two terms in one MMA
 // tile, which needs at most 8 query heads per kv head; qk-norm needs a
-// kernel of its own between QKV and attention, so those models decode on
-// the launch chain.
+// kernel of its own between QKV and attention and mixture-of-experts layers
+// their routing kernels, so those models decode on the launch chain.
 bool persist_eligible(const axon_model* m, int B) {
-  return m->persist_ctas > 0 && !m->fp32 && !m->cfg.qk_norm && m->H / m->G <= 8 &&
+  return m->persist_ctas > 0 && !m->fp32 && !m->cfg.qk_norm && !m->moe && m->H / m->G <= 8 &&
          persist_fits(m->d, m->f16, B, m->D);
 }
 
@@ -815,30 +972,10 @@ launch_chain:
     CK(pj.rc);
     pend(pf, wo + B * (Hd * es + D * (8 + es)), 2.0 * B * D * Hd);
 
-    EpiArgs g = base_epi(m);
-    g.S = 1;
-    g.ctx = ctx;
-    set_norm(m, ns, g);
-    g.u_out = m->u;
-    g.u_lo_out = m->u_lo;
-    pbeg(pf, "decode_gateup");
-    pj.run(EPI_SWIGLU, w.wgu, &w.m_gu, 2 * m->F, D, m->a, D, B, g);
-    CK(pj.rc);
-    pend(pf, wgu + B * (D + m->F) * es, 2.0 * B * 2 * m->F * D);
-
-    EpiArgs dn = base_epi(m);
-    dn.S = 1;
-    dn.ctx = ctx;
-    dn.x = m->x;
-    dn.a_out = m->a;
-    dn.gain = (l + 1 < m->L) ? m->layers[l + 1].g1 : m->gf;
-    dn.a_lo_out = m->a_lo;
-    dn.ss_out = m->ss;
-    dn.ss_out_stride = m->Pmax;
-    pbeg(pf, "decode_down");
-    ns = pj.run(EPI_RESID, w.wd, &w.m_d, D, m->F, m->u, m->F, B, dn);
-    CK(pj.rc);
-    pend(pf, wdn + B * (m->F * es + D * (8 + es)), 2.0 * B * D * m->F);
+    EpiArgs row = base_epi(m);
+    row.S = 1;
+    row.ctx = ctx;
+    CK_RC(enqueue_mlp(m, l, pj, lc, pf, row, B, true, ns));
   }
   EpiArgs h = base_epi(m);
   h.S = 1;
@@ -977,9 +1114,26 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     if ((rc = bl.check(bl.find(p + "self_attn.k_proj.weight"), Gd, D))) return fail(rc);
     if ((rc = bl.check(bl.find(p + "self_attn.v_proj.weight"), Gd, D))) return fail(rc);
     if ((rc = bl.check(bl.find(p + "self_attn.o_proj.weight"), D, Hd))) return fail(rc);
-    if ((rc = bl.check(bl.find(p + "mlp.gate_proj.weight"), F, D))) return fail(rc);
-    if ((rc = bl.check(bl.find(p + "mlp.up_proj.weight"), F, D))) return fail(rc);
-    if ((rc = bl.check(bl.find(p + "mlp.down_proj.weight"), D, F))) return fail(rc);
+    if (cfg->n_routed_experts > 0 && l >= cfg->first_k_dense_replace) {
+      const int E = cfg->n_routed_experts, Fe = cfg->moe_intermediate_size, Fs = cfg->n_shared_experts * Fe;
+      if ((rc = bl.check(bl.find(p + "mlp.gate.weight"), E, D))) return fail(rc);
+      for (int e = 0; e < E; ++e) {
+        const std::string q = p + "mlp.experts." + std::to_string(e) + ".";
+        if ((rc = bl.check(bl.find(q + "gate_proj.weight"), Fe, D))) return fail(rc);
+        if ((rc = bl.check(bl.find(q + "up_proj.weight"), Fe, D))) return fail(rc);
+        if ((rc = bl.check(bl.find(q + "down_proj.weight"), D, Fe))) return fail(rc);
+      }
+      if (Fs) {
+        const std::string q = p + "mlp.shared_experts.";
+        if ((rc = bl.check(bl.find(q + "gate_proj.weight"), Fs, D))) return fail(rc);
+        if ((rc = bl.check(bl.find(q + "up_proj.weight"), Fs, D))) return fail(rc);
+        if ((rc = bl.check(bl.find(q + "down_proj.weight"), D, Fs))) return fail(rc);
+      }
+    } else {
+      if ((rc = bl.check(bl.find(p + "mlp.gate_proj.weight"), F, D))) return fail(rc);
+      if ((rc = bl.check(bl.find(p + "mlp.up_proj.weight"), F, D))) return fail(rc);
+      if ((rc = bl.check(bl.find(p + "mlp.down_proj.weight"), D, F))) return fail(rc);
+    }
     if (cfg->qk_norm) {
       if ((rc = bl.check(bl.find(p + "self_attn.q_norm.weight"), m->d, -1))) return fail(rc);
       if ((rc = bl.check(bl.find(p + "self_attn.k_norm.weight"), m->d, -1))) return fail(rc);
@@ -1041,19 +1195,42 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     if ((rc = dev_alloc(m, &w.wo, static_cast<size_t>(D) * Hd * es))) return fail(rc);
     if ((rc = bl.gather(w.wo, f32, bl.find(p + "self_attn.o_proj.weight"), nullptr, D, Hd))) return fail(rc);
     // gate/up interleave: packed row r: chunk r/16, slots 0..7 gate, 8..15 up.
-    if ((rc = dev_alloc(m, &w.wgu, static_cast<size_t>(2 * F) * D * es))) return fail(rc);
-    {
-      // gate row j -> packed row (j/8)*16 + j%8, up row j -> (j/8)*16 + 8 + j%8
-      std::vector<int> to_gate(F), to_up(F);
-      for (int j = 0; j < F; ++j) {
+    // gate row j -> packed row (j/8)*16 + j%8, up row j -> (j/8)*16 + 8 + j%8
+    auto pack_mlp = [&](const std::string& q, int width, void* gu, void* dn) {
+      std::vector<int> to_gate(width), to_up(width);
+      for (int j = 0; j < width; ++j) {
         to_gate[j] = (j >> 3) * 16 + (j & 7);
         to_up[j] = (j >> 3) * 16 + 8 + (j & 7);
       }
-      if ((rc = bl.gather(w.wgu, f32, bl.find(p + "mlp.gate_proj.weight"), nullptr, F, D, &to_gate))) return fail(rc);
-      if ((rc = bl.gather(w.wgu, f32, bl.find(p + "mlp.up_proj.weight"), nullptr, F, D, &to_up))) return fail(rc);
+      int r = bl.gather(gu, f32, bl.find(q + "gate_proj.weight"), nullptr, width, D, &to_gate);
+      if (!r) r = bl.gather(gu, f32, bl.find(q + "up_proj.weight"), nullptr, width, D, &to_up);
+      if (!r) r = bl.gather(dn, f32, bl.find(q + "down_proj.weight"), nullptr, D, width);
+      return r;
+    };
+    const bool moe_layer = cfg->n_routed_experts > 0 && l >= cfg->first_k_dense_replace;
+    w.Fl = moe_layer ? cfg->n_shared_experts * cfg->moe_intermediate_size : F;
+    if (w.Fl) {
+      if ((rc = dev_alloc(m, &w.wgu, static_cast<size_t>(2 * w.Fl) * D * es))) return fail(rc);
+      if ((rc = dev_alloc(m, &w.wd, static_cast<size_t>(D) * w.Fl * es))) return fail(rc);
+      if ((rc = pack_mlp(moe_layer ? p + "mlp.shared_experts." : p + "mlp.", w.Fl, w.wgu, w.wd))) return fail(rc);
     }
-    if ((rc = dev_alloc(m, &w.wd, static_cast<size_t>(D) * F * es))) return fail(rc);
-    if ((rc = bl.gather(w.wd, f32, bl.find(p + "mlp.down_proj.weight"), nullptr, D, F))) return fail(rc);
+    if (moe_layer) {
+      // the stacked-experts formulation: expert e's gate/up rows at
+      // e * 2Fe, its down rows at e * D, of one tensor each
+      const int E = cfg->n_routed_experts, Fe = cfg->moe_intermediate_size;
+      w.moe = true;
+      void* rp = nullptr;
+      if ((rc = dev_alloc(m, &rp, static_cast<size_t>(E) * D * 4))) return fail(rc);
+      w.router = static_cast<float*>(rp);
+      if ((rc = bl.gather(w.router, true, bl.find(p + "mlp.gate.weight"), nullptr, E, D))) return fail(rc);
+      if ((rc = dev_alloc(m, &w.wgu_e, static_cast<size_t>(E) * 2 * Fe * D * es))) return fail(rc);
+      if ((rc = dev_alloc(m, &w.wd_e, static_cast<size_t>(E) * D * Fe * es))) return fail(rc);
+      for (int e = 0; e < E && !rc; ++e)
+        rc = pack_mlp(p + "mlp.experts." + std::to_string(e) + ".", Fe,
+                      static_cast<char*>(w.wgu_e) + static_cast<size_t>(e) * 2 * Fe * D * es,
+                      static_cast<char*>(w.wd_e) + static_cast<size_t>(e) * D * Fe * es);
+      if (rc) return fail(rc);
+    }
     void* g1 = nullptr;
     void* g2 = nullptr;
     if ((rc = dev_alloc(m, &g1, D * 4))) return fail(rc);
@@ -1139,14 +1316,17 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   m->ss = static_cast<float*>(p);
   if ((rc = dev_alloc(m, &m->q, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
   if ((rc = dev_alloc(m, &m->o, static_cast<size_t>(Mcap) * Hd * es))) return fail(rc);
-  if ((rc = dev_alloc(m, &m->u, static_cast<size_t>(Mcap) * F * es))) return fail(rc);
+  int Fmax = 0;  // widest dense MLP of any layer (shared experts included)
+  for (const LayerW& w : m->layers) Fmax = w.Fl > Fmax ? w.Fl : Fmax;
+  if (Fmax == 0) Fmax = 64;
+  if ((rc = dev_alloc(m, &m->u, static_cast<size_t>(Mcap) * Fmax * es))) return fail(rc);
   if (!f32) {
     const size_t rows = static_cast<size_t>(cfg->max_batch < 64 ? cfg->max_batch : 64);
     if ((rc = dev_alloc(m, &m->q_lo, rows * Hd * es))) return fail(rc);
   }
   if (m->f16) {
     if ((rc = dev_alloc(m, &m->o_lo, static_cast<size_t>(m->cfg.max_batch) * Hd * es))) return fail(rc);
-    if ((rc = dev_alloc(m, &m->u_lo, static_cast<size_t>(m->cfg.max_batch) * F * es))) return fail(rc);
+    if ((rc = dev_alloc(m, &m->u_lo, static_cast<size_t>(m->cfg.max_batch) * Fmax * es))) return fail(rc);
   }
   if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * 8))) return fail(rc);
   m->keys = static_cast<unsigned long long*>(p);
@@ -1157,6 +1337,44 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   if (cfg->qk_norm) {
     if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * (m->H + m->G) * m->d * 4))) return fail(rc);
     m->qk_raw = static_cast<float*>(p);
+  }
+  if (cfg->n_routed_experts > 0 && cfg->first_k_dense_replace < m->L) {
+    // sorted rows: every (token, expert) slot plus, per expert in use, up to
+    // 127 rows of padding to a whole 128-row block
+    m->moe = true;
+    m->E = cfg->n_routed_experts;
+    m->topk = cfg->num_experts_per_tok;
+    m->Fe = cfg->moe_intermediate_size;
+    const long long slots = static_cast<long long>(Mcap) * m->topk;
+    m->R_cap = (slots + std::min<long long>(m->E, slots) * 127 + 127) / 128 * 128;
+    const size_t R = static_cast<size_t>(m->R_cap);
+    if ((rc = dev_alloc(m, &p, slots * 4))) return fail(rc);
+    m->moe_topk_idx = static_cast<int*>(p);
+    if ((rc = dev_alloc(m, &p, slots * 4))) return fail(rc);
+    m->moe_topk_w = static_cast<float*>(p);
+    if ((rc = dev_alloc(m, &p, slots * 4))) return fail(rc);
+    m->moe_slot_row = static_cast<int*>(p);
+    if ((rc = dev_alloc(m, &p, R * 4))) return fail(rc);
+    m->moe_row_tok = static_cast<int*>(p);
+    if ((rc = dev_alloc(m, &p, R * 4))) return fail(rc);
+    m->moe_row_w = static_cast<float*>(p);
+    if ((rc = dev_alloc(m, &p, (R / 128) * 4 + 16))) return fail(rc);
+    m->moe_mb_expert = static_cast<int*>(p);
+    if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
+    m->moe_nmb = static_cast<int*>(p);
+    if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
+    m->moe_ones = static_cast<float*>(p);
+    const float one = 1.0f;
+    if (cudaMemcpy(m->moe_ones, &one, 4, cudaMemcpyHostToDevice) != cudaSuccess) return fail(AXON_ERR_CUDA);
+    if ((rc = dev_alloc(m, &m->moe_h, static_cast<size_t>(Mcap) * D * es))) return fail(rc);
+    if ((rc = dev_alloc(m, &m->moe_a_sorted, R * D * es))) return fail(rc);
+    if ((rc = dev_alloc(m, &m->moe_u_sorted, R * m->Fe * es))) return fail(rc);
+    if ((rc = dev_alloc(m, &p, R * D * 4))) return fail(rc);
+    m->moe_y_sorted = static_cast<float*>(p);
+    if (cudaMemsetAsync(m->moe_row_tok, 0xff, R * 4, st) != cudaSuccess ||
+        cudaMemsetAsync(m->moe_nmb, 0, 16, st) != cudaSuccess)
+      return fail(AXON_ERR_CUDA);
+    if (prepare_moe_kernels(D, m->E) != cudaSuccess) return fail(AXON_ERR_CUDA);
   }
   if ((rc = dev_alloc(m, &m->a_last, static_cast<size_t>(cfg->max_batch) * D * es))) return fail(rc);
   if (m->f16 && (rc = dev_alloc(m, &m->a_lo_last, static_cast<size_t>(cfg->max_batch) * D * es))) return fail(rc);
@@ -1197,13 +1415,15 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
       cudaMemsetAsync(m->x, 0, static_cast<size_t>(Mcap) * D * 4, st) != cudaSuccess ||
       cudaMemsetAsync(m->a, 0, static_cast<size_t>(Mcap) * D * es, st) != cudaSuccess ||
       cudaMemsetAsync(m->o, 0, static_cast<size_t>(Mcap) * Hd * es, st) != cudaSuccess ||
-      cudaMemsetAsync(m->u, 0, static_cast<size_t>(Mcap) * F * es, st) != cudaSuccess)
+      cudaMemsetAsync(m->u, 0, static_cast<size_t>(Mcap) * Fmax * es, st) != cudaSuccess)
     return fail(AXON_ERR_CUDA);
 
   // ---- TMA descriptors (bf16 tensor-core path)
   if (!f32) {
-    bool ok = make_tma_2d_16(&m->t_a, m->a, Mcap, D, 128, m->f16) && make_tma_2d_16(&m->t_o, m->o, Mcap, Hd, 128, m->f16) &&
-              make_tma_2d_16(&m->t_u, m->u, Mcap, F, 128, m->f16);
+    bool ok = make_tma_2d_16(&m->t_a, m->a, Mcap, D, 128, m->f16) && make_tma_2d_16(&m->t_o, m->o, Mcap, Hd, 128, m->f16);
+    if (ok && m->moe)
+      ok = make_tma_2d_16(&m->t_asorted, m->moe_a_sorted, m->R_cap, D, 128, m->f16) &&
+           make_tma_2d_16(&m->t_usorted, m->moe_u_sorted, m->R_cap, m->Fe, 128, m->f16);
     if (ok && m->a_lo) ok = make_tma_2d_16(&m->t_alo, m->a_lo, Mcap, D, 128, m->f16);
     for (int l = 0; l < m->L && ok; ++l) {
       LayerW& w = m->layers[l];
@@ -1215,18 +1435,36 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
       }
       w.m_o.a = m->t_o;
       ok = ok && make_tma_2d_16(&w.m_o.w, w.wo, D, Hd, 256, m->f16);
-      w.m_gu.a = m->t_a;
-      ok = ok && make_tma_2d_16(&w.m_gu.w, w.wgu, 2 * F, D, 256, m->f16);
-      w.m_d.a = m->t_u;
-      ok = ok && make_tma_2d_16(&w.m_d.w, w.wd, D, F, 256, m->f16);
+      if (w.Fl) {
+        w.m_gu.a = m->t_a;
+        ok = ok && make_tma_2d_16(&w.m_gu.w, w.wgu, 2 * w.Fl, D, 256, m->f16);
+        // the down projection reads u with this layer's row stride
+        ok = ok && make_tma_2d_16(&w.m_d.a, m->u, Mcap, w.Fl, 128, m->f16);
+        ok = ok && make_tma_2d_16(&w.m_d.w, w.wd, D, w.Fl, 256, m->f16);
+      }
+      if (w.moe) {
+        const int E = m->E, Fe = m->Fe;
+        w.m_gu_e.a = m->t_asorted;
+        ok = ok && make_tma_2d_16(&w.m_gu_e.w, w.wgu_e, static_cast<uint64_t>(E) * 2 * Fe, D, 256, m->f16);
+        w.m_d_e.a = m->t_usorted;
+        ok = ok && make_tma_2d_16(&w.m_d_e.w, w.wd_e, static_cast<uint64_t>(E) * D, Fe, 256, m->f16);
+        w.m_gu_e128 = w.m_gu_e;
+        ok = ok && make_tma_2d_16(&w.m_gu_e128.w, w.wgu_e, static_cast<uint64_t>(E) * 2 * Fe, D, 128, m->f16);
+        w.m_gu_e.n128 = &w.m_gu_e128;
+        w.m_d_e128 = w.m_d_e;
+        ok = ok && make_tma_2d_16(&w.m_d_e128.w, w.wd_e, static_cast<uint64_t>(E) * D, Fe, 128, m->f16);
+        w.m_d_e.n128 = &w.m_d_e128;
+      }
     }
     m->m_head.a = m->t_a;
     ok = ok && make_tma_2d_16(&m->m_head.w, m->head, V, D, 256, m->f16);
     // decode projections: weight boxes of 128 rows, activation boxes of 8..64 token rows
     for (int l = 0; l < m->L && ok; ++l) {
       LayerW& w = m->layers[l];
-      ok = make_tma_2d_16(&w.v_qkv, w.wqkv, m->Nqkv, D, 128, m->f16) && make_tma_2d_16(&w.v_o, w.wo, D, Hd, 128, m->f16) &&
-           make_tma_2d_16(&w.v_gu, w.wgu, 2 * F, D, 128, m->f16) && make_tma_2d_16(&w.v_d, w.wd, D, F, 128, m->f16);
+      ok = make_tma_2d_16(&w.v_qkv, w.wqkv, m->Nqkv, D, 128, m->f16) && make_tma_2d_16(&w.v_o, w.wo, D, Hd, 128, m->f16);
+      if (ok && w.Fl)
+        ok = make_tma_2d_16(&w.v_gu, w.wgu, 2 * w.Fl, D, 128, m->f16) &&
+             make_tma_2d_16(&w.v_d, w.wd, D, w.Fl, 128, m->f16);
     }
     ok = ok && make_tma_2d_16(&m->v_head, m->head, V, D, 128, m->f16);
     // 128-wide output tiles reuse the 128-row weight boxes of the decode maps
@@ -1252,7 +1490,7 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
   }
   // ---- persistent decode step: layer table and grid barrier state
   // default for B <= PERSIST_MAX_B; AXON_NO_PERSIST=1 keeps the launch chain
-  if (!f32 && !env_flag("AXON_NO_PERSIST") && (m->d == 64 || m->d == 128)) {
+  if (!f32 && !m->moe && !env_flag("AXON_NO_PERSIST") && (m->d == 64 || m->d == 128)) {
     const int per_sm = persist_ctas_per_sm(m->d, m->f16);
     if (per_sm >= 1) {
       std::vector<PersistLayer> pl(m->L);
@@ -1430,6 +1668,18 @@ int axon_profile_prefill(axon_model* m, const int32_t* d_ids, int32_t B, int32_t
   const int rc = enqueue_prefill(m, d_ids, B, S, d_block_table, AXON_LOGITS_LAST, nullptr, d_next, st, &pf);
   if (rc) return rc;
   return collect_profile(pf, out, max_out, n_out);
+}
+
+int axon_moe_routing_record(axon_model* m, int32_t* d_experts, int32_t rows) {
+  if (!m) return AXON_ERR_INVALID_ARG;
+  if (!m->moe) return AXON_ERR_UNSUPPORTED;
+  if (d_experts && rows < 1) return AXON_ERR_INVALID_ARG;
+  m->moe_record = d_experts;
+  m->moe_record_rows = d_experts ? rows : 0;
+  // recorded launches must not replay from graphs built without the record
+  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+  m->graphs.clear();
+  return AXON_OK;
 }
 
 int axon_reset(axon_model* m) {

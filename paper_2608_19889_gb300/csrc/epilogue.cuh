@@ -19,7 +19,7 @@
 
 #include "common.cuh"
 
-enum EpiKind : int { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LOGITS = 3 };
+enum EpiKind : int { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LOGITS = 3, EPI_ROWSCALE = 4 };
 // Gate activation of the gated MLP (axon_config.hidden_act).
 enum ActKind : int { ACT_SILU = 0, ACT_GELU_TANH = 1 };
 
@@ -81,6 +81,9 @@ struct EpiArgs {
   float* logits;  // [M][logits_stride] or null
   long long logits_stride;
   unsigned long long* keys;  // [M] argmax keys
+  // ROWSCALE (mixture-of-experts down projection): y_out[m][n] = v * row_w[m], fp32, row stride N
+  float* y_out;
+  const float* row_w;
   int* err;
 };
 
@@ -319,6 +322,15 @@ AXON_DEV void epi_swiglu16(const EpiArgs& e, int m, int n0, const float* v, floa
     for (int i = 0; i < 8; ++i) lo[i] = u[i] - to_f(from_f<T>(u[i]));
     store8<T>(reinterpret_cast<T*>(e.u_lo_out) + static_cast<long long>(m) * (e.N >> 1) + (n0 >> 1), lo);
   }
+}
+
+// Mixture-of-experts down projection: the 16 outputs of sorted row m times
+// the row's routing weight, stored fp32 for the combine kernel.
+AXON_DEV void epi_rowscale16(const EpiArgs& e, int m, int n0, const float* v) {
+  const float w = e.row_w[m];
+  float4* y = reinterpret_cast<float4*>(e.y_out + static_cast<long long>(m) * e.N + n0);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) y[i] = make_float4(v[4 * i] * w, v[4 * i + 1] * w, v[4 * i + 2] * w, v[4 * i + 3] * w);
 }
 
 // logits = r * v (columns >= N dropped); returns this chunk's argmax key.

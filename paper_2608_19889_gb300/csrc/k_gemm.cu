@@ -58,7 +58,7 @@ template <int KIND, typename T16, bool SPLIT, int BN_>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmAlo, int M, int N, int K, EpiArgs ep, int ks, float* ws,
-                   int* tickets) {
+                   int* tickets, GemmGroup grp) {
   using C = GCfg<SPLIT, BN_>;
   constexpr int BN = C::BN;
   constexpr int B_BYTES = C::B_BYTES;
@@ -105,7 +105,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem = *tmem_slot_ptr;
 
   grid_dep_wait();
-  const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN;
+  // grouped: the m-blocks the routing plan laid out (read after the wait,
+  // when the plan kernel's writes are visible)
+  const bool grouped = grp.mb_expert != nullptr;
+  const int num_m = grouped ? __ldcg(grp.n_mblocks) : (M + BM - 1) / BM, num_n = (N + BN - 1) / BN;
   const int tiles = num_m * num_n, KB = K / BK;
   // Work units: (tile, K split) pairs, the ks splits of a tile adjacent.
   // ks > 1 only with one M tile (M <= BM): each unit leaves its partial tile
@@ -120,6 +123,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int t = u / ks, sp = u - t * ks;
         int mb, nb;
         tile_coords(t, num_m, num_n, mb, nb);
+        if (grouped) {
+          mb = t / num_n;
+          nb = t - mb * num_n;
+        }
+        const int wrow = grouped ? __ldcg(grp.mb_expert + mb) * N + nb * BN : nb * BN;
         const int kb1 = (sp + 1) * KB / ks;
         for (int kb = sp * KB / ks; kb < kb1; ++kb, ++it) {
           const int s = it % STAGES;
@@ -131,7 +139,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           mbar_arrive_expect_tx(full_bar(s), STAGE_BYTES);
           tma_load_2d(sA + s * A_BYTES, &tmA, full_bar(s), kb * BK, mb * BM);
           if (SPLIT) tma_load_2d(sAlo + s * A_BYTES, &tmAlo, full_bar(s), kb * BK, mb * BM);
-          tma_load_2d(sB + s * B_BYTES, &tmB, full_bar(s), kb * BK, nb * BN);
+          tma_load_2d(sB + s * B_BYTES, &tmB, full_bar(s), kb * BK, wrow);
         }
       }
     }
@@ -185,6 +193,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int t = u / ks;
       int mb, nb;
       tile_coords(t, num_m, num_n, mb, nb);
+      if (grouped) {
+        mb = t / num_n;
+        nb = t - mb * num_n;
+      }
       const int buf = lt & 1;
       const uint32_t aph = (lt >> 1) & 1;
       const bool got = mbar_wait(accf_bar(buf), aph, ep.err);
@@ -263,9 +275,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         continue;
       }
       const int m = mb * BM + row;
-      const bool mval = m < M;
+      const bool mval = m < M && (!grp.row_valid || grp.row_valid[m] >= 0);
       float rinv = 1.f;
-      if (KIND != EPI_RESID && mval) rinv = row_rinv(ep, m);
+      if (KIND != EPI_RESID && KIND != EPI_ROWSCALE && mval) rinv = row_rinv(ep, m);
       float ssum = 0.f;
       unsigned long long best = 0ull;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(q4 * 32) << 16) + buf * BN;
@@ -312,6 +324,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             epi_qkv16<T16>(ep, m, n0, f, rinv);
           } else if (KIND == EPI_SWIGLU) {
             epi_swiglu16<T16>(ep, m, n0, f, rinv);
+          } else if (KIND == EPI_ROWSCALE) {
+            epi_rowscale16(ep, m, n0, f);
           } else {
             const unsigned long long k = epi_logits16(ep, m, n0, f, rinv);
             best = k > best ? k : best;
@@ -347,9 +361,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 template <int KIND, typename T16, bool SPLIT, int BN>
 cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
-                        const GemmSplitK& sk) {
+                        const GemmSplitK& sk, const GemmGroup& grp) {
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN) * sk.ks;
-  const int grid = tiles < lc.num_sms ? tiles : lc.num_sms;
+  // grouped: the tile count is known only on the device; one CTA per SM
+  const int grid = grp.mb_expert ? lc.num_sms : (tiles < lc.num_sms ? tiles : lc.num_sms);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(NUM_THREADS);
@@ -362,7 +377,7 @@ cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N,
   cfg.numAttrs = lc.pdl ? 1 : 0;
   const GemmMaps& g = BN == 256 ? maps : *maps.n128;
   return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN>, g.a, g.w, SPLIT ? g.a_lo : g.a, M, N, K, ep,
-                            sk.ks, sk.ws, sk.tickets);
+                            sk.ks, sk.ws, sk.tickets, grp);
 }
 
 }  // namespace
@@ -411,18 +426,20 @@ cudaError_t prepare_gemm_t() {
   if (e == cudaSuccess) e = set_smem<EPI_RESID, T16, false>();
   if (e == cudaSuccess) e = set_smem<EPI_SWIGLU, T16, false>();
   if (e == cudaSuccess) e = set_smem<EPI_LOGITS, T16, false>();
+  if (e == cudaSuccess) e = set_smem<EPI_ROWSCALE, T16, false>();
   return e;
 }
 template <typename T16, int BN>
 cudaError_t launch_t(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
-                     const GemmSplitK& sk) {
+                     const GemmSplitK& sk, const GemmGroup& grp) {
   switch (kind) {
     case EPI_QKV:
-      return maps.split ? launch_kind<EPI_QKV, T16, true, BN>(lc, maps, M, N, K, ep, sk)
-                        : launch_kind<EPI_QKV, T16, false, BN>(lc, maps, M, N, K, ep, sk);
-    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN>(lc, maps, M, N, K, ep, sk);
-    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN>(lc, maps, M, N, K, ep, sk);
-    default: return launch_kind<EPI_LOGITS, T16, false, BN>(lc, maps, M, N, K, ep, sk);
+      return maps.split ? launch_kind<EPI_QKV, T16, true, BN>(lc, maps, M, N, K, ep, sk, grp)
+                        : launch_kind<EPI_QKV, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_ROWSCALE: return launch_kind<EPI_ROWSCALE, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
+    default: return launch_kind<EPI_LOGITS, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
   }
 }
 }  // namespace
@@ -446,8 +463,11 @@ cudaError_t prepare_gemm_kernels() {
 }
 
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K,
-                           const EpiArgs& ep, int tile_n, const GemmSplitK* split) {
+                           const EpiArgs& ep, int tile_n, const GemmSplitK* split, const GemmGroup* group) {
   if (M < 1 || N < 1 || K < BK || (K % BK)) return cudaErrorInvalidValue;
+  const GemmGroup grp = group ? *group : GemmGroup{};
+  if (grp.mb_expert && (!grp.n_mblocks || (split && split->ks > 1) || (M % BM))) return cudaErrorInvalidValue;
+  if (kind == EPI_ROWSCALE && !grp.mb_expert) return cudaErrorInvalidValue;
   GemmSplitK sk;
   if (split && split->ks > 1) {
     // one M tile, 256-wide tiles, at most GEMM_MAX_UNITS units, at least one K block per unit
@@ -459,11 +479,11 @@ cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, 
   }
   if (tile_n == 128) {
     if (!maps.n128) return cudaErrorInvalidValue;
-    if (lc.f16) return launch_t<f16, 128>(lc, kind, maps, M, N, K, ep, sk);
-    return launch_t<bf16, 128>(lc, kind, maps, M, N, K, ep, sk);
+    if (lc.f16) return launch_t<f16, 128>(lc, kind, maps, M, N, K, ep, sk, grp);
+    return launch_t<bf16, 128>(lc, kind, maps, M, N, K, ep, sk, grp);
   }
-  if (lc.f16) return launch_t<f16, 256>(lc, kind, maps, M, N, K, ep, sk);
-  return launch_t<bf16, 256>(lc, kind, maps, M, N, K, ep, sk);
+  if (lc.f16) return launch_t<f16, 256>(lc, kind, maps, M, N, K, ep, sk, grp);
+  return launch_t<bf16, 256>(lc, kind, maps, M, N, K, ep, sk, grp);
 }
 
 int gemm_split_k(const LaunchCtx& lc, int M, int N, int K) {

@@ -77,6 +77,42 @@ cudaError_t launch_finalize_varlen(const LaunchCtx& lc, unsigned long long* keys
 // e is the QKV launch's epilogue argument block.
 cudaError_t launch_qk_norm_rope(const LaunchCtx& lc, bool fp32, const EpiArgs& e, int rows);
 
+// ---- mixture of experts (k_moe.cu): routing, the stable sort of
+// (token, expert) slots into 128-row expert segments, the sorted operand
+// rows and the combine into the residual; the expert products run on the
+// grouped tcgen05 GEMM (GemmGroup).
+constexpr int MOE_MAX_EXPERTS = 256;
+struct MoeArgs {
+  int D, E, k, norm_topk;
+  const void* act;     // normed operand a = x * g [T][act_stride] (16-bit)
+  const void* act_lo;  // its second term (fp16 mode), or null
+  long long act_stride;
+  const float* router;  // [E][D] fp32
+  void* h_hi;           // [T][D] normalised input, 16-bit
+  void* h_lo;           // its second term, or null
+  int* topk_idx;        // [T * k]
+  float* topk_w;        // [T * k]
+  int* slot_row;        // [T * k] sorted row of each (token, j) slot
+  int* row_tok;         // [rows] token of each sorted row, -1 for padding
+  float* row_w;         // [rows] routing weight of each sorted row
+  int* mb_expert;       // [rows / 128] expert of each 128-row block
+  int* n_mblocks;       // [1] blocks laid out
+  void* a_sorted;       // [rows][D] sorted operand rows
+  void* a_sorted_lo;    // second terms, or null
+  float* y_sorted;      // [rows][D] expert outputs times routing weight
+  int* record;          // optional [record_rows][k]: copy of the chosen experts (inspection)
+  int record_rows;
+  int* err;
+};
+// ns: the norm state of `act` (row_rinv); T tokens.
+cudaError_t prepare_moe_kernels(int D, int E);
+cudaError_t launch_moe_route(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ns);
+cudaError_t launch_moe_plan(const LaunchCtx& lc, const MoeArgs& a, int T);
+cudaError_t launch_moe_gather(const LaunchCtx& lc, const MoeArgs& a);
+// ep: residual x (ep.x, ep.N = D) and, when ep.a_out is set, the residual
+// epilogue's outputs (a_out, a_lo_out, gain, ss_out / ss_out_stride).
+cudaError_t launch_moe_combine(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ep);
+
 // ---- attention (k_attn.cu)
 struct AttnArgs {
   const void* q;  // [rows][H*d]
@@ -149,10 +185,22 @@ struct GemmSplitK {
   int* tickets = nullptr;    // [max_tiles]
   int max_tiles = 0;
 };
+// Grouped mode (mixture of experts, stacked experts): the activation rows
+// are sorted by expert, each expert's rows padded to whole 128-row blocks;
+// m-block b belongs to expert mb_expert[b], and *n_mblocks blocks exist
+// (both written on the device by the routing plan). The weight operand is
+// the experts' matrices stacked as one [E * N][K] tensor: block b's tiles
+// read rows mb_expert[b] * N + n. Rows whose row_valid entry is negative
+// are padding and get no epilogue. M bounds the sorted rows.
+struct GemmGroup {
+  const int* mb_expert = nullptr;  // null: ordinary GEMM
+  const int* n_mblocks = nullptr;
+  const int* row_valid = nullptr;
+};
 // tile_n: 256 or 128 (from gemm_tile_n); the residual epilogue writes one
 // norm partial per row and tile, i.e. ceil(N / tile_n) of them.
 cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
-                           int tile_n = 256, const GemmSplitK* split = nullptr);
+                           int tile_n = 256, const GemmSplitK* split = nullptr, const GemmGroup* group = nullptr);
 int gemm_tile_n(const LaunchCtx& lc, const GemmMaps& maps, int M, int N);
 // K split (1 = none) for a decode-sized M x N x K product whose 256-wide
 // tiles cannot fill half the GPU.

@@ -49,6 +49,8 @@ WORKLOADS = {
     "8b_paged_b64_ctx512-4096_n128": dict(model="8b", B=64, ctx=(512, 4096), n_new=128, layout="paged"),
     "32b_b1_s2048_n256": dict(model="32b", B=1, S=2048, n_new=256, layout="contiguous"),
     "32b_b16_s2048_n256": dict(model="32b", B=16, S=2048, n_new=256, layout="contiguous"),
+    # the paper's mixture-of-experts data point (DeepSeek-MoE 16B, Sec. Results)
+    "moe16b_b1_s512_n128": dict(model="moe16b", B=1, S=512, n_new=128, layout="contiguous"),
     # prompt twice the window: the window bounds prefill attention and every decode step's keys
     "7b_swa_b1_s8192_n256": dict(model="7b_swa", B=1, S=8192, n_new=256, layout="contiguous"),
 }
