@@ -83,11 +83,17 @@ def shape_from_hf_config(c: dict) -> dict:
         raise ValueError(f"model_type {mt!r} is not a Llama-family decoder this library implements")
     H = int(c["num_attention_heads"])
     D = int(c["hidden_size"])
+    # Transformers v5 keeps the rotary settings under rope_parameters; older
+    # configs keep rope_theta and rope_scaling at the top level
+    rp = c.get("rope_parameters") or {}
+    theta = rp.get("rope_theta", c.get("rope_theta"))
+    if theta is None:
+        raise ValueError("no rope_theta in the config (neither top level nor rope_parameters)")
     shape = dict(L=int(c["num_hidden_layers"]), D=D, H=H, G=int(c.get("num_key_value_heads", H)),
                  d=int(c.get("head_dim") or D // H), F=int(c["intermediate_size"]), V=int(c["vocab_size"]),
                  tie=bool(c.get("tie_word_embeddings", False)),
                  bias=bool(c.get("attention_bias", mt == "qwen2")),
-                 theta=float(c.get("rope_theta", 10000.0)), eps=float(c.get("rms_norm_eps", 1e-6)))
+                 theta=float(theta), eps=float(c.get("rms_norm_eps", 1e-6)))
     if c.get("mlp_bias"):
         raise ValueError("MLP biases are not implemented")
     act = c.get("hidden_act", "silu")
@@ -105,9 +111,11 @@ def shape_from_hf_config(c: dict) -> dict:
             raise ValueError("a sliding window on only some layers is not implemented")
         if first <= 0:
             shape["window"] = int(window)
-    rs = c.get("rope_scaling")
+    rs = c.get("rope_scaling") or (rp if rp.get("rope_type", "default") != "default" else None)
     if rs:
         kind = rs.get("rope_type", rs.get("type"))
+        if kind == "default":
+            return shape
         if kind != "llama3":
             raise ValueError(f"rope_scaling {kind!r} is not implemented")
         shape.update(rope_factor=float(rs["factor"]), rope_low=float(rs["low_freq_factor"]),

@@ -120,3 +120,21 @@ def test_head_dim_defaults_to_width_over_heads():
     c = {k: v for k, v in LLAMA31.items() if k != "rope_scaling"}
     assert ck.shape_from_hf_config(c)["d"] == 128
     assert ck.shape_from_hf_config(dict(c, head_dim=64))["d"] == 64
+
+
+def test_rope_parameters_of_newer_configs_and_default_rope_type():
+    """Transformers v5 configs keep the rotary settings under
+    rope_parameters; a 'default' rope type means no frequency scaling; a
+    config with no rotary base at all is refused rather than defaulted."""
+    top = {k: v for k, v in LLAMA31.items() if k not in ("rope_theta", "rope_scaling")}
+    v5 = dict(top, rope_parameters={"rope_type": "llama3", "rope_theta": 500000.0, "factor": 8.0,
+                                    "low_freq_factor": 1.0, "high_freq_factor": 4.0,
+                                    "original_max_position_embeddings": 8192})
+    s = ck.shape_from_hf_config(v5)
+    assert s["theta"] == 5e5 and (s["rope_factor"], s["rope_orig"]) == (8.0, 8192)
+    plain = ck.shape_from_hf_config(dict(top, rope_parameters={"rope_type": "default", "rope_theta": 1e6}))
+    assert plain["theta"] == 1e6 and "rope_factor" not in plain
+    old_default = ck.shape_from_hf_config(dict(LLAMA31, rope_scaling={"rope_type": "default"}))
+    assert "rope_factor" not in old_default
+    with pytest.raises(ValueError):
+        ck.shape_from_hf_config(top)

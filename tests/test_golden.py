@@ -1,8 +1,10 @@
-"""Regression pin of the oracle against tests/golden/tiny_decoder.json, which
+"""Change detector for the oracle: tests/golden/tiny_decoder.json holds what
 tests/golden/make_golden.py wrote from the oracle itself (the paper prints no
 worked numbers for this forward). It catches unintended changes to the
-oracle's arithmetic; the other oracle tests pin it to the paper and to
-mathematics."""
+oracle's arithmetic but pins the oracle only to itself; the other oracle
+tests pin it to the paper and to mathematics. The tolerance leaves room for
+the summation order of another BLAS build or thread count (float64 sums of
+a few hundred terms); the greedy tokens must match exactly."""
 import json
 import os
 
@@ -27,7 +29,7 @@ def test_oracle_reproduces_the_stored_generation(name):
     cache = o.new_contiguous_cache(DATA["batch"], DATA["prompt"] + DATA["decode_steps"])
     toks, logits = o.generate(ids, DATA["decode_steps"] + 1, cache)
     assert np.array_equal(toks, np.array(c["tokens"]))
-    assert np.allclose(logits, np.array(c["logits"]), rtol=1e-12, atol=1e-12)
+    assert np.allclose(logits, np.array(c["logits"]), rtol=1e-9, atol=1e-9)
 
 
 def test_cases_differ_from_each_other():
