@@ -36,11 +36,12 @@ struct LayerW {
   float* qn = nullptr;  // qk-norm gains [d] (null when off)
   float* kn = nullptr;
   int Fl = 0;  // width of the layer's dense SwiGLU MLP (the shared experts' in a MoE layer; 0: none)
-  // mixture of experts: fp32 router [E][D]; the experts stacked as one
+  // mixture of experts: router [E][D]; the experts stacked as one
   // [E * 2Fe][D] gate/up tensor (each expert's rows interleaved in 16-row
   // chunks like the dense one) and one [E * D][Fe] down tensor
   bool moe = false;
-  float* router = nullptr;
+  void* router = nullptr;  // [E][D] in the model's 16-bit type (the checkpoint's bf16 values)
+  GemmMaps m_router{}, m_router128{};
   void* wgu_e = nullptr;
   void* wd_e = nullptr;
   GemmMaps m_gu_e{}, m_d_e{}, m_gu_e128{}, m_d_e128{};
@@ -139,8 +140,9 @@ struct axon_model {
   float* moe_row_w = nullptr;
   int* moe_mb_expert = nullptr;
   int* moe_nmb = nullptr;
+  float* moe_logits = nullptr;  // [Mcap][E] router logits
+  unsigned long long* moe_keys = nullptr;  // [Mcap] argmax keys of the router projection (unused)
   float* moe_ones = nullptr;  // [1] = 1.0: the sorted operand is already normalised
-  void* moe_h = nullptr;      // [Mcap][D]
   void* moe_a_sorted = nullptr;
   void* moe_u_sorted = nullptr;
   float* moe_y_sorted = nullptr;
@@ -552,8 +554,7 @@ MoeArgs moe_args(const axon_model* m, const LayerW& w) {
   a.act = m->a;
   a.act_lo = m->a_lo;
   a.act_stride = m->D;
-  a.router = w.router;
-  a.h_hi = m->moe_h;
+  a.logits = m->moe_logits;
   a.topk_idx = m->moe_topk_idx;
   a.topk_w = m->moe_topk_w;
   a.slot_row = m->moe_slot_row;
@@ -586,6 +587,16 @@ int enqueue_mlp(axon_model* m, int l, Proj& pj, const LaunchCtx& lc, Prof* pf, c
     const int E = m->E, k = m->topk, Fe = m->Fe;
     const int R = static_cast<int>(m->R_cap);
     const double act = expected_active_experts(E, k, M);
+    // router logits [M][E] on the projection kernels (norm scale applied)
+    EpiArgs rl = row;
+    set_norm(m, ns, rl);
+    rl.logits = m->moe_logits;
+    rl.logits_stride = E;
+    rl.keys = m->moe_keys;
+    pbeg(pf, decode ? "decode_moe_router" : "prefill_moe_router");
+    pj.run(EPI_LOGITS, w.router, &w.m_router, E, D, m->a, D, M, rl);
+    CK(pj.rc);
+    pend(pf, static_cast<double>(E) * D * es + M * (D * es + E * 4.0), 2.0 * M * E * D);
     MoeArgs ma = moe_args(m, w);
     if (m->moe_record) {
       ma.record = m->moe_record + static_cast<size_t>(l) * m->moe_record_rows * k;
@@ -594,10 +605,9 @@ int enqueue_mlp(axon_model* m, int l, Proj& pj, const LaunchCtx& lc, Prof* pf, c
     EpiArgs nx = base_epi(m);
     set_norm(m, ns, nx);
     pbeg(pf, decode ? "decode_moe_route" : "prefill_moe_route");
-    CK(launch_moe_route(lc, ma, M, nx));
-    CK(launch_moe_plan(lc, ma, M));
-    CK(launch_moe_gather(lc, ma));
-    pend(pf, static_cast<double>(E) * D * 4 + M * D * (2 * es + es * k), 2.0 * M * E * D);
+    CK(launch_moe_route_plan(lc, ma, M));
+    CK(launch_moe_gather(lc, ma, M, nx));
+    pend(pf, M * (E * 4.0 + D * (2 * es + es * k)), 0);
     // tile width: 128 when the experts' blocks alone leave most SMs idle
     const int tn = (static_cast<long long>(M) * k * ((D + 255) / 256) < m->num_sms) ? 128 : 256;
     GemmGroup grp;
@@ -1219,10 +1229,8 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
       // e * 2Fe, its down rows at e * D, of one tensor each
       const int E = cfg->n_routed_experts, Fe = cfg->moe_intermediate_size;
       w.moe = true;
-      void* rp = nullptr;
-      if ((rc = dev_alloc(m, &rp, static_cast<size_t>(E) * D * 4))) return fail(rc);
-      w.router = static_cast<float*>(rp);
-      if ((rc = bl.gather(w.router, true, bl.find(p + "mlp.gate.weight"), nullptr, E, D))) return fail(rc);
+      if ((rc = dev_alloc(m, &w.router, static_cast<size_t>(E) * D * es))) return fail(rc);
+      if ((rc = bl.gather(w.router, f32, bl.find(p + "mlp.gate.weight"), nullptr, E, D))) return fail(rc);
       if ((rc = dev_alloc(m, &w.wgu_e, static_cast<size_t>(E) * 2 * Fe * D * es))) return fail(rc);
       if ((rc = dev_alloc(m, &w.wd_e, static_cast<size_t>(E) * D * Fe * es))) return fail(rc);
       for (int e = 0; e < E && !rc; ++e)
@@ -1362,11 +1370,14 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     m->moe_mb_expert = static_cast<int*>(p);
     if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
     m->moe_nmb = static_cast<int*>(p);
+    if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * m->E * 4))) return fail(rc);
+    m->moe_logits = static_cast<float*>(p);
+    if ((rc = dev_alloc(m, &p, static_cast<size_t>(Mcap) * 8))) return fail(rc);
+    m->moe_keys = static_cast<unsigned long long*>(p);
     if ((rc = dev_alloc(m, &p, 16))) return fail(rc);
     m->moe_ones = static_cast<float*>(p);
     const float one = 1.0f;
     if (cudaMemcpy(m->moe_ones, &one, 4, cudaMemcpyHostToDevice) != cudaSuccess) return fail(AXON_ERR_CUDA);
-    if ((rc = dev_alloc(m, &m->moe_h, static_cast<size_t>(Mcap) * D * es))) return fail(rc);
     if ((rc = dev_alloc(m, &m->moe_a_sorted, R * D * es))) return fail(rc);
     if ((rc = dev_alloc(m, &m->moe_u_sorted, R * m->Fe * es))) return fail(rc);
     if ((rc = dev_alloc(m, &p, R * D * 4))) return fail(rc);
@@ -1444,6 +1455,15 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
       }
       if (w.moe) {
         const int E = m->E, Fe = m->Fe;
+        w.m_router.a = m->t_a;
+        if (m->a_lo) {
+          w.m_router.a_lo = m->t_alo;
+          w.m_router.split = true;
+        }
+        ok = ok && make_tma_2d_16(&w.m_router.w, w.router, E, D, 256, m->f16);
+        w.m_router128 = w.m_router;
+        ok = ok && make_tma_2d_16(&w.m_router128.w, w.router, E, D, 128, m->f16);
+        w.m_router.n128 = &w.m_router128;
         w.m_gu_e.a = m->t_asorted;
         ok = ok && make_tma_2d_16(&w.m_gu_e.w, w.wgu_e, static_cast<uint64_t>(E) * 2 * Fe, D, 256, m->f16);
         w.m_d_e.a = m->t_usorted;

@@ -2,18 +2,20 @@
 // grouped experts; the stacked-experts formulation that the paper's graph
 // rewriting puts in place of a loop over experts):
 //
-//   moe_route_kernel    per token: h = (a [+ a_lo]) * r, the normalised
-//                       input (r from the producer's norm partials), router
-//                       logits h . Wr[e] in fp32, softmax, top-k (lowest
-//                       index on ties), weights (optionally renormalised);
-//                       h is also stored as 16-bit operand terms;
+//   [router logits: the decode GEMV or the tcgen05 GEMM with the LOGITS
+//    epilogue (norm scale applied), fp32 [T][E]]
+//   moe_route_kernel    per token: softmax of the router logits, top-k
+//                       (lowest index on ties), weights (optionally
+//                       renormalised); for few tokens the plan kernel's
+//                       CTA does this itself;
 //   moe_plan_kernel     one CTA: a stable counting sort of the T x k
 //                       (token, expert) slots by expert into segments padded
 //                       to 128-row blocks: the sorted row of every slot, the
 //                       token and weight of every sorted row (token -1 for
 //                       padding), the expert of every 128-row block and the
 //                       block count -- the grouped GEMM's tile list;
-//   moe_gather_kernel   the sorted operand rows (padding rows zero);
+//   moe_gather_kernel   the sorted operand rows: the normalised input
+//                       h = (a [+ a_lo]) * r, rounded once to 16 bits;
 //   [grouped tcgen05 GEMM gate/up + SwiGLU, grouped GEMM down scaled by the
 //    row's weight: k_gemm.cu]
 //   moe_combine_kernel  per token: x += the sum of its k expert outputs in
@@ -26,37 +28,16 @@ namespace {
 
 constexpr int ROUTE_THREADS = 256;
 constexpr int PLAN_THREADS = 1024;
+// Token counts up to which one CTA both routes and sorts (the decode path).
+constexpr int FUSED_ROUTE_MAX_T = 256;
 
-template <typename T16>
-__global__ void __launch_bounds__(ROUTE_THREADS) moe_route_kernel(MoeArgs a, EpiArgs ns) {
-  grid_dep_launch();
-  grid_dep_wait();
-  extern __shared__ float sh[];  // [D] normalised h, then [E] logits
-  const int t = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int D = a.D, E = a.E, k = a.k;
-  float* lg = sh + D;
-  const float r = row_rinv(ns, t);
-  const T16* ah = static_cast<const T16*>(a.act) + static_cast<long long>(t) * a.act_stride;
-  const T16* al = a.act_lo ? static_cast<const T16*>(a.act_lo) + static_cast<long long>(t) * a.act_stride : nullptr;
-  T16* hh = static_cast<T16*>(a.h_hi) + static_cast<long long>(t) * D;
-  T16* hl = a.h_lo ? static_cast<T16*>(a.h_lo) + static_cast<long long>(t) * D : nullptr;
-  for (int i = tid; i < D; i += ROUTE_THREADS) {
-    const float v = (to_f(ah[i]) + (al ? to_f(al[i]) : 0.f)) * r;
-    sh[i] = v;
-    const T16 h16 = from_f<T16>(v);
-    hh[i] = h16;
-    if (hl) hl[i] = from_f<T16>(v - to_f(h16));
-  }
-  __syncthreads();
-  for (int e = warp; e < E; e += ROUTE_THREADS / 32) {
-    const float* w = a.router + static_cast<long long>(e) * D;
-    float s = 0.f;
-    for (int i = lane; i < D; i += 32) s = fmaf(sh[i], w[i], s);
-    s = warp_sum(s);
-    if (lane == 0) lg[e] = s;
-  }
-  __syncthreads();
-  if (warp != 0) return;
+// Token t: softmax of its router logits, top-k by repeated arg-max over
+// (probability, lowest index), the weights (renormalised over the k chosen
+// when norm_topk). One warp; lg is the warp's [E] scratch.
+AXON_DEV void route_token(const MoeArgs& a, int t, float* lg, int lane) {
+  const int E = a.E, k = a.k;
+  __syncwarp();
+  for (int e = lane; e < E; e += 32) lg[e] = a.logits[static_cast<long long>(t) * E + e];
   float mx = -INFINITY;
   for (int e = lane; e < E; e += 32) mx = fmaxf(mx, lg[e]);
 #pragma unroll
@@ -69,7 +50,6 @@ __global__ void __launch_bounds__(ROUTE_THREADS) moe_route_kernel(MoeArgs a, Epi
   }
   den = warp_sum(den);
   __syncwarp();
-  // top-k by repeated arg-max over (probability, lowest index)
   float wsum = 0.f, wk[8];
   int ik[8];
   for (int j = 0; j < k; ++j) {
@@ -113,10 +93,23 @@ __global__ void __launch_bounds__(ROUTE_THREADS) moe_route_kernel(MoeArgs a, Epi
   }
 }
 
+// One warp per token (many tokens: prefill).
+__global__ void __launch_bounds__(ROUTE_THREADS) moe_route_kernel(MoeArgs a, int T) {
+  grid_dep_launch();
+  grid_dep_wait();
+  extern __shared__ float sh[];  // [warps][E]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * (ROUTE_THREADS / 32) + warp;
+  if (t < T) route_token(a, t, sh + warp * a.E, lane);
+}
+
 // Stable counting sort of the n = T * k slots by expert, in rounds of
 // PLAN_THREADS slots: within a warp, slots of one expert are ranked by
 // lane (match_any), warps are ranked in order by a per-expert prefix over
 // the round's warp counts, rounds in order by the running counts.
+// With ROUTE, the CTA's warps first route the T tokens themselves (the
+// per-warp scratch is the count table, unused until then).
+template <bool ROUTE>
 __global__ void __launch_bounds__(PLAN_THREADS) moe_plan_kernel(MoeArgs a, int T) {
   grid_dep_launch();
   grid_dep_wait();
@@ -125,6 +118,10 @@ __global__ void __launch_bounds__(PLAN_THREADS) moe_plan_kernel(MoeArgs a, int T
   __shared__ int wcnt[PLAN_THREADS / 32][MOE_MAX_EXPERTS];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int E = a.E, n = T * a.k;
+  if (ROUTE) {
+    for (int t = warp; t < T; t += PLAN_THREADS / 32) route_token(a, t, reinterpret_cast<float*>(wcnt[warp]), lane);
+    __syncthreads();
+  }
   for (int e = tid; e < E; e += PLAN_THREADS) cnt[e] = 0;
   for (int base = 0; base < n; base += PLAN_THREADS) {
     for (int c = tid; c < (PLAN_THREADS / 32) * E; c += PLAN_THREADS) wcnt[c / E][c % E] = 0;
@@ -183,26 +180,44 @@ __global__ void __launch_bounds__(PLAN_THREADS) moe_plan_kernel(MoeArgs a, int T
   }
 }
 
-// Sorted operand rows: row r is token row_tok[r]'s normalised h (both
-// terms), or zeros for padding. One warp per row, 16-byte copies.
+// Sorted operand rows: slot i = (token t, j) goes to row slot_row[i] as the
+// normalised input h = (a [+ a_lo]) * r of token t, rounded once to 16 bits.
+// Padding rows are left as they are: a row of the grouped GEMMs' operand
+// only reaches its own output row, which the epilogues skip. One warp per
+// slot, 8 elements per lane step.
 template <typename T16>
-__global__ void __launch_bounds__(256) moe_gather_kernel(MoeArgs a) {
+__global__ void __launch_bounds__(256) moe_gather_kernel(MoeArgs a, int T, EpiArgs ns) {
   grid_dep_launch();
   grid_dep_wait();
-  const int rows = __ldcg(a.n_mblocks) * 128;
-  const int per_row = a.D / 8;  // 16-byte pieces
+  const int n = T * a.k, per_row = a.D / 8;
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   const int nwarps = (gridDim.x * blockDim.x) >> 5;
-  for (int r = warp; r < rows; r += nwarps) {
-    const int tok = __ldcg(a.row_tok + r);
-    const uint4* sh = reinterpret_cast<const uint4*>(static_cast<const T16*>(a.h_hi) + static_cast<long long>(tok) * a.D);
-    uint4* dh = reinterpret_cast<uint4*>(static_cast<T16*>(a.a_sorted) + static_cast<long long>(r) * a.D);
-    const uint4* sl = a.h_lo ? reinterpret_cast<const uint4*>(static_cast<const T16*>(a.h_lo) + static_cast<long long>(tok) * a.D) : nullptr;
-    uint4* dl = a.a_sorted_lo ? reinterpret_cast<uint4*>(static_cast<T16*>(a.a_sorted_lo) + static_cast<long long>(r) * a.D) : nullptr;
-    const uint4 z = make_uint4(0, 0, 0, 0);
+  for (int i = warp; i < n; i += nwarps) {
+    const int row = a.slot_row[i];
+    if (row < 0) continue;
+    const int t = i / a.k;
+    const float r = row_rinv(ns, t);
+    const uint4* sh = reinterpret_cast<const uint4*>(static_cast<const T16*>(a.act) + t * a.act_stride);
+    const uint4* sl = a.act_lo ? reinterpret_cast<const uint4*>(static_cast<const T16*>(a.act_lo) + t * a.act_stride)
+                               : nullptr;
+    uint4* dh = reinterpret_cast<uint4*>(static_cast<T16*>(a.a_sorted) + static_cast<long long>(row) * a.D);
     for (int c = lane; c < per_row; c += 32) {
-      dh[c] = tok >= 0 ? __ldcg(sh + c) : z;
-      if (dl) dl[c] = (tok >= 0 && sl) ? __ldcg(sl + c) : z;
+      const uint4 hv = sh[c];
+      const T16* h8 = reinterpret_cast<const T16*>(&hv);
+      float v[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) v[q] = to_f(h8[q]);
+      if (sl) {
+        const uint4 lv = sl[c];
+        const T16* l8 = reinterpret_cast<const T16*>(&lv);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] += to_f(l8[q]);
+      }
+      uint4 o;
+      T16* o8 = reinterpret_cast<T16*>(&o);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) o8[q] = from_f<T16>(v[q] * r);
+      dh[c] = o;
     }
   }
 }
@@ -265,28 +280,27 @@ cudaError_t launch_k(const LaunchCtx& lc, K kernel, dim3 grid, dim3 block, size_
 }  // namespace
 
 cudaError_t prepare_moe_kernels(int D, int E) {
-  const int smem = (D + E) * 4;
-  cudaError_t e = cudaFuncSetAttribute(moe_route_kernel<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(moe_route_kernel<f16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  return e;
+  (void)D;
+  (void)E;
+  return cudaSuccess;
 }
 
-cudaError_t launch_moe_route(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ns) {
+cudaError_t launch_moe_route_plan(const LaunchCtx& lc, const MoeArgs& a, int T) {
   if (T < 1 || a.k < 1 || a.k > 8 || a.k > a.E || a.E > MOE_MAX_EXPERTS) return cudaErrorInvalidValue;
-  const size_t smem = static_cast<size_t>(a.D + a.E) * 4;
-  if (lc.f16) return launch_k(lc, moe_route_kernel<f16>, dim3(T), dim3(ROUTE_THREADS), smem, a, ns);
-  return launch_k(lc, moe_route_kernel<bf16>, dim3(T), dim3(ROUTE_THREADS), smem, a, ns);
+  if (T <= FUSED_ROUTE_MAX_T) return launch_k(lc, moe_plan_kernel<true>, dim3(1), dim3(PLAN_THREADS), 0, a, T);
+  const int warps = ROUTE_THREADS / 32;
+  const size_t smem = static_cast<size_t>(warps) * a.E * 4;
+  cudaError_t e = launch_k(lc, moe_route_kernel, dim3((T + warps - 1) / warps), dim3(ROUTE_THREADS), smem, a, T);
+  if (e != cudaSuccess) return e;
+  return launch_k(lc, moe_plan_kernel<false>, dim3(1), dim3(PLAN_THREADS), 0, a, T);
 }
 
-cudaError_t launch_moe_plan(const LaunchCtx& lc, const MoeArgs& a, int T) {
-  return launch_k(lc, moe_plan_kernel, dim3(1), dim3(PLAN_THREADS), 0, a, T);
-}
-
-cudaError_t launch_moe_gather(const LaunchCtx& lc, const MoeArgs& a) {
+cudaError_t launch_moe_gather(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ns) {
   if (a.D % 8) return cudaErrorInvalidValue;
-  if (lc.f16) return launch_k(lc, moe_gather_kernel<f16>, dim3(2 * lc.num_sms), dim3(256), 0, a);
-  return launch_k(lc, moe_gather_kernel<bf16>, dim3(2 * lc.num_sms), dim3(256), 0, a);
+  const long long warps = static_cast<long long>(T) * a.k;
+  const int grid = static_cast<int>(std::min<long long>((warps + 7) / 8, 4LL * lc.num_sms));
+  if (lc.f16) return launch_k(lc, moe_gather_kernel<f16>, dim3(grid), dim3(256), 0, a, T, ns);
+  return launch_k(lc, moe_gather_kernel<bf16>, dim3(grid), dim3(256), 0, a, T, ns);
 }
 
 cudaError_t launch_moe_combine(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ep) {

@@ -87,9 +87,7 @@ struct MoeArgs {
   const void* act;     // normed operand a = x * g [T][act_stride] (16-bit)
   const void* act_lo;  // its second term (fp16 mode), or null
   long long act_stride;
-  const float* router;  // [E][D] fp32
-  void* h_hi;           // [T][D] normalised input, 16-bit
-  void* h_lo;           // its second term, or null
+  const float* logits;  // [T][E] router logits (fp32, norm scale applied)
   int* topk_idx;        // [T * k]
   float* topk_w;        // [T * k]
   int* slot_row;        // [T * k] sorted row of each (token, j) slot
@@ -97,18 +95,17 @@ struct MoeArgs {
   float* row_w;         // [rows] routing weight of each sorted row
   int* mb_expert;       // [rows / 128] expert of each 128-row block
   int* n_mblocks;       // [1] blocks laid out
-  void* a_sorted;       // [rows][D] sorted operand rows
-  void* a_sorted_lo;    // second terms, or null
+  void* a_sorted;       // [rows][D] sorted operand rows (normalised, 16-bit)
   float* y_sorted;      // [rows][D] expert outputs times routing weight
   int* record;          // optional [record_rows][k]: copy of the chosen experts (inspection)
   int record_rows;
   int* err;
 };
-// ns: the norm state of `act` (row_rinv); T tokens.
 cudaError_t prepare_moe_kernels(int D, int E);
-cudaError_t launch_moe_route(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ns);
-cudaError_t launch_moe_plan(const LaunchCtx& lc, const MoeArgs& a, int T);
-cudaError_t launch_moe_gather(const LaunchCtx& lc, const MoeArgs& a);
+// Routing of T tokens from a.logits and the sorted layout (one or two launches).
+cudaError_t launch_moe_route_plan(const LaunchCtx& lc, const MoeArgs& a, int T);
+// ns: the norm state of `act` (row_rinv).
+cudaError_t launch_moe_gather(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ns);
 // ep: residual x (ep.x, ep.N = D) and, when ep.a_out is set, the residual
 // epilogue's outputs (a_out, a_lo_out, gain, ss_out / ss_out_stride).
 cudaError_t launch_moe_combine(const LaunchCtx& lc, const MoeArgs& a, int T, const EpiArgs& ep);
