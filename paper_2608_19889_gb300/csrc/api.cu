@@ -11,6 +11,7 @@
 // then final norm + LM head (+argmax) and the greedy-token finaliser.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -901,10 +902,11 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     // key blocks (8 per warp; measured at 40 blocks, head_dim 64: 0.743 ms
     // per step unsplit, 0.775-0.790 ms split). Beyond that the keys split
     // into items of persist_split_blocks blocks (80 blocks, head_dim 128:
-    // 3.170 ms per step in items of 16, 3.239 ms in items of 64).
-    int psplits = m->blocks_per_seq > 64
-                      ? (m->blocks_per_seq + m->persist_split_blocks - 1) / m->persist_split_blocks
-                      : 1;
+    // 3.170 ms per step in items of 16, 3.239 ms in items of 64). The small
+    // layout stages one block per warp: items of 8 blocks, one round.
+    const int kmax = std::max(std::max(m->D, m->H * m->d), m->F);
+    const int sblocks = persist_small(m->d, m->f16, B, kmax) ? 8 : m->persist_split_blocks;
+    int psplits = (m->blocks_per_seq > 64 || sblocks == 8) ? (m->blocks_per_seq + sblocks - 1) / sblocks : 1;
     if (psplits > cap) psplits = cap;
     PersistArgs pa = persist_args(m, tokens, B, ctx, bt, logits, next, psplits, attn_part ? attn_part : m->attn_part,
                                   attn_cnt ? attn_cnt : m->attn_cnt);

@@ -199,7 +199,7 @@ AXON_DEV void dec_sync() {
 // PAIR = 1: the caller guarantees a second term of q and at most 8 query
 // heads per kv head, so only the paired tile loop is compiled; PAIR = 0:
 // chosen at run time.
-template <int HD, typename T16, bool NAMED, int PAIR = 0>
+template <int HD, typename T16, bool NAMED, int PAIR = 0, int STAGES = 2>
 AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* sm, int tid) {
   constexpr int TILE = 16 * HD * 2;
   const int warp = tid >> 5, lane = tid & 31, r = lane >> 2, q = lane & 3;
@@ -221,7 +221,7 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
   if (s >= n_used) return;
   const int jb = jlo + s * per, je = min(jb + per, jlo + nblk);
 
-  const uint32_t wbase = smem_u32(sm) + warp * 4 * TILE;  // per warp: [stage][K | V]
+  const uint32_t wbase = smem_u32(sm) + warp * STAGES * 2 * TILE;  // per warp: [stage][K | V]
   const uint16_t* kp = static_cast<const uint16_t*>(p.k);
   const uint16_t* vp = static_cast<const uint16_t*>(p.v);
   auto issue = [&](int j, int stg) {
@@ -252,7 +252,7 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
     constexpr bool PAIRED = decltype(paired_tag)::value;
     for (; j < je; j += DEC_WARPS) {
       const int jn = j + DEC_WARPS;
-      if (jn < je) {
+      if (STAGES == 2 && jn < je) {
         issue(jn, stg ^ 1);
         cp_async_wait<1>();
       } else {
@@ -262,7 +262,10 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
       attn_tile16<HD, T16, PAIRED>(wbase + stg * 2 * TILE, wbase + stg * 2 * TILE + TILE, qa, st, j * 16, klo, T - 1,
                                    klo, T - 1, p.scale_log2, lane);
       __syncwarp();
-      stg ^= 1;
+      if (STAGES == 2)
+        stg ^= 1;
+      else if (jn < je)
+        issue(jn, 0);  // one stage: the next block loads once this one is consumed
     }
     if (PAIRED) fold_paired<HD>(st);
   };
@@ -334,54 +337,45 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
   if (n_used == 1) return;
 
   // Last CTA of this (sequence, kv head) merges the n_used partial states.
+  // The ticket is taken after the CTA barrier by one thread with an
+  // acquire-release atomic: its release covers the CTA's partial stores, its
+  // acquire (passed on by the second barrier) the other CTAs'.
   __shared__ int is_last;
-  __shared__ float cw[16][64];
-  __shared__ float cinv[16];
-  __threadfence();
   dec_sync<NAMED>();
-  if (tid == 0) is_last = (atomicAdd(p.counter + b * p.G + g, 1) == n_used - 1);
+  if (tid == 0) is_last = (atom_add_acq_rel_gpu(p.counter + b * p.G + g, 1) == n_used - 1);
   dec_sync<NAMED>();
   if (!is_last) return;
-  __threadfence();
-  float* cl = wo;  // reuse: [16][64] running sums
-  for (int idx = tid; idx < HPG * n_used; idx += DEC_WARPS * 32) {
-    const int i = idx / n_used, t = idx - i * n_used;
-    const float* pr = part + (static_cast<long long>(t) * 16 + i) * rowlen;
-    cw[i][t] = __ldcg(pr + HD);
-    cl[i * 64 + t] = __ldcg(pr + HD + 1);
-  }
-  dec_sync<NAMED>();
-  if (tid < HPG) {
-    const int i = tid;
-    float M = NEG_INF;
-    for (int t = 0; t < n_used; ++t) M = fmaxf(M, cw[i][t]);
-    float L = 0.f;
-    for (int t = 0; t < n_used; ++t) {
-      const float f = (cw[i][t] == NEG_INF) ? 0.f : exp2f(cw[i][t] - M);
-      cw[i][t] = f;
-      L += cl[i * 64 + t] * f;
-    }
-    cinv[i] = L > 0.f ? 1.f / L : 0.f;
-  }
-  dec_sync<NAMED>();
+  // Each thread folds the n_used (m, l, O) partial states of its outputs in
+  // split order with the online-softmax update; the loads of sixteen splits
+  // are issued together, so up to sixteen splits cost one L2 round trip.
   for (int idx = tid; idx < HPG * HD; idx += DEC_WARPS * 32) {
     const int i = idx / HD, dd = idx - i * HD;
-    const float* pc = part + static_cast<long long>(i) * rowlen + dd;
-    float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
-    int t = 0;
-    for (; t + 4 <= n_used; t += 4) {
-      const float v0 = __ldcg(pc + (t + 0) * 16 * rowlen), v1 = __ldcg(pc + (t + 1) * 16 * rowlen);
-      const float v2 = __ldcg(pc + (t + 2) * 16 * rowlen), v3 = __ldcg(pc + (t + 3) * 16 * rowlen);
-      O0 += cw[i][t] * v0;
-      O1 += cw[i][t + 1] * v1;
-      O2 += cw[i][t + 2] * v2;
-      O3 += cw[i][t + 3] * v3;
+    const float* pc = part + static_cast<long long>(i) * rowlen;
+    float M = NEG_INF, L = 0.f, O = 0.f;
+    for (int t0 = 0; t0 < n_used; t0 += 16) {
+      float mv[16], lv[16], ov[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const bool in = t0 + u < n_used;
+        const float* pr = pc + static_cast<long long>(in ? t0 + u : 0) * 16 * rowlen;
+        mv[u] = in ? __ldcg(pr + HD) : NEG_INF;
+        lv[u] = in ? __ldcg(pr + HD + 1) : 0.f;
+        ov[u] = in ? __ldcg(pr + dd) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        if (mv[u] == NEG_INF) continue;  // a split with no visible key
+        const float nm = fmaxf(M, mv[u]);
+        const float a = exp2f(M - nm), f = exp2f(mv[u] - nm);  // a = 0 while M = -inf
+        L = L * a + lv[u] * f;
+        O = O * a + ov[u] * f;
+        M = nm;
+      }
     }
-    for (; t < n_used; ++t) O0 += cw[i][t] * __ldcg(pc + t * 16 * rowlen);
     T16* og = static_cast<T16*>(p.o) + (static_cast<long long>(b) * p.H + g * HPG + i) * HD + dd;
-    const float ov = ((O0 + O1) + (O2 + O3)) * cinv[i];
-    *og = from_f<T16>(ov);
-    if (p.o_lo) static_cast<T16*>(p.o_lo)[og - static_cast<T16*>(p.o)] = from_f<T16>(ov - to_f(from_f<T16>(ov)));
+    const float res = L > 0.f ? O / L : 0.f;
+    *og = from_f<T16>(res);
+    if (p.o_lo) static_cast<T16*>(p.o_lo)[og - static_cast<T16*>(p.o)] = from_f<T16>(res - to_f(from_f<T16>(res)));
   }
   if (tid == 0) p.counter[b * p.G + g] = 0;
 }
@@ -389,5 +383,13 @@ AXON_DEV void attn_decode_item(const AttnArgs& p, int s, int g, int b, uint8_t* 
 
 template <int HD>
 constexpr size_t decode_smem() { return DEC_WARPS * 4 * 16 * HD * 2; }  // warps x 2 stages x (K, V)
+// One stage per warp (STAGES = 1), or the merge buffers of attn_decode_item
+// ([warps][16] maxima and sums, [warps][16][HD] outputs), whichever is larger.
+template <int HD>
+constexpr size_t decode_smem1() {
+  return DEC_WARPS * 2 * 16 * HD * 2 > (2 * DEC_WARPS * 16 + DEC_WARPS * 16 * HD) * 4
+             ? DEC_WARPS * 2 * 16 * HD * 2
+             : (2 * DEC_WARPS * 16 + DEC_WARPS * 16 * HD) * 4;
+}
 
 }  // namespace

@@ -35,6 +35,7 @@
 // (same barrier sequence, so named barriers stay matched) and the host sees
 // the error bit. Before it exits, the producer waits (bounded) for its copies
 // in flight.
+#include <algorithm>
 #include <type_traits>
 
 #include "attn_tile.cuh"
@@ -53,12 +54,19 @@ constexpr int SMEM_LIMIT = 232448;         // 227 KB opt-in per CTA
 
 static_assert(PCW == DEC_WARPS, "attention items run on the consumer warps");
 
-template <int HD>
+// How the 16-bit operand terms of the projections enter the MMAs (proj_phase).
+constexpr int TERMS_ONE = 0, TERMS_PAIRED = 1, TERMS_TWO = 2;
+
+// Shared-memory layout. SM ("small"): the attention items stage one key
+// block per warp (decode_smem1), so the weight ring gets the space a second
+// stage would take -- at head_dim 128, 8 ring stages instead of 5; taken
+// when the activations of the batch still stage next to the epilogue buffer.
+template <int HD, bool SM>
 struct PLayout {
-  static constexpr int ATTN = static_cast<int>(decode_smem<HD>());
+  static constexpr int ATTN = SM ? static_cast<int>(decode_smem1<HD>()) : static_cast<int>(decode_smem<HD>());
   static constexpr int RED = 2 * RED_FLOATS * 4;
   static constexpr int MISC = 256;  // rinv[8], abort flag
-  static constexpr int STATIC_EST = 8192;  // static shared of the attention merge, with margin
+  static constexpr int STATIC_EST = 1024;  // static shared (the merge flag), with margin
   static constexpr int NS = (SMEM_LIMIT - ATTN - RED - MISC - STATIC_EST - 1024) / (STAGE_BYTES + 16);
   static constexpr int BARS = 2 * NS * 8;
   static constexpr int RING_OFF = 0;
@@ -156,25 +164,28 @@ AXON_DEV int first_item(int rot) {
   return ((static_cast<int>(blockIdx.x) - rot) % n + n) % n;
 }
 
-template <int HD>
+template <int HD, bool SM>
 struct Ring {
   uint32_t base;  // shared address of stage 0
   uint32_t bars;  // full[NS] then empty[NS]
   AXON_DEV uint32_t full(int s) const { return bars + 8 * s; }
-  AXON_DEV uint32_t empty(int s) const { return bars + 8 * (PLayout<HD>::NS + s); }
+  AXON_DEV uint32_t empty(int s) const { return bars + 8 * (PLayout<HD, SM>::NS + s); }
 };
 
 // ----------------------------------------------------------------- producer
 // Streams this CTA's items of one matrix (in the item order the consumers
 // walk): per ring stage one or two TMA boxes of 16 rows x 256 columns, one
 // instruction each; rows >= N and columns >= K arrive as zeros.
-template <int HD>
-AXON_DEV void stream_matrix(const Ring<HD>& R, const CUtensorMap* map, int N, int K, int& rot, uint32_t& stage,
+template <int HD, bool SM>
+AXON_DEV void stream_matrix(const Ring<HD, SM>& R, const CUtensorMap* map, int N, int K, int& rot, uint32_t& stage,
                             bool& stop, PersistGrid* g, volatile int* s_abort, int* err, int lane) {
-  constexpr int NS = PLayout<HD>::NS;
+  constexpr int NS = PLayout<HD, SM>::NS;
   const int n = (N + 15) >> 4;
   const int i0 = first_item(rot);
   rot = (rot + n) % static_cast<int>(gridDim.x);
+  // Weights are read once per step: they should not evict the key/value
+  // cache or the activations from L2.
+  const uint64_t policy = createpolicy_evict_first();
   for (int i = i0; i < n && !stop; i += gridDim.x) {
     for (int k0 = 0; k0 < K && !stop; k0 += KC) {
       const int slot = static_cast<int>(stage % NS);
@@ -186,8 +197,8 @@ AXON_DEV void stream_matrix(const Ring<HD>& R, const CUtensorMap* map, int N, in
           const bool two = k0 + BOXC < K;
           mbar_arrive_expect_tx(R.full(slot), two ? STAGE_BYTES : BOX_BYTES);
           const uint32_t dst = R.base + slot * STAGE_BYTES;
-          tma_load_2d(dst, map, R.full(slot), k0, i * 16);
-          if (two) tma_load_2d(dst + BOX_BYTES, map, R.full(slot), k0 + BOXC, i * 16);
+          tma_load_2d_hint(dst, map, R.full(slot), k0, i * 16, policy);
+          if (two) tma_load_2d_hint(dst + BOX_BYTES, map, R.full(slot), k0 + BOXC, i * 16, policy);
         }
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -210,13 +221,13 @@ struct CState {
 // Stage t of a phase's stage sequence (spi stages per item): wait for the
 // ring slot, copy this warp's weight fragments (rows r, r+8 x 16 columns)
 // and the token-r activation fragments to registers, release the slot.
-template <int HD, typename T16, bool LO>
-AXON_DEV void load_stage(const Ring<HD>& R, CState& cs, const PersistArgs& A, PersistGrid* g, volatile int* s_abort,
+template <int HD, bool SM, typename T16, bool WANT_Y>
+AXON_DEV void load_stage(const Ring<HD, SM>& R, CState& cs, const PersistArgs& A, PersistGrid* g, volatile int* s_abort,
                          int t, int spi, int K, int warp, int lane, int r, int q, bool tok_ok, bool staged,
                          const uint8_t* act_sm, int pitch, const T16* xsrc, const T16* ysrc, int xrow_s, int yrow_s,
-                         bool want_y, uint4& w0, uint4& w1, uint4& w2, uint4& w3, uint4& x0, uint4& x1, uint4& y0,
+                         uint4& w0, uint4& w1, uint4& w2, uint4& w3, uint4& x0, uint4& x1, uint4& y0,
                          uint4& y1, bool& on) {
-  constexpr int NS = PLayout<HD>::NS;
+  constexpr int NS = PLayout<HD, SM>::NS;
   const int k0 = (t % spi) * KC;
   const int kc = min(KC, K - k0);
   const int sl = static_cast<int>(cs.stage % NS);
@@ -236,7 +247,7 @@ AXON_DEV void load_stage(const Ring<HD>& R, CState& cs, const PersistArgs& A, Pe
         const uint32_t sa = smem_u32(act_sm) + xrow_s * pitch + (k + 16 * q) * 2;
         x0 = lds16(sa);
         x1 = lds16(sa + 16);
-        if (LO && want_y) {
+        if (WANT_Y) {
           const uint32_t sb = smem_u32(act_sm) + yrow_s * pitch + (k + 16 * q) * 2;
           y0 = lds16(sb);
           y1 = lds16(sb + 16);
@@ -244,7 +255,7 @@ AXON_DEV void load_stage(const Ring<HD>& R, CState& cs, const PersistArgs& A, Pe
       } else {
         x0 = __ldcg(reinterpret_cast<const uint4*>(xsrc + k));
         x1 = __ldcg(reinterpret_cast<const uint4*>(xsrc + k + 8));
-        if (LO && want_y) {
+        if (WANT_Y) {
           y0 = __ldcg(reinterpret_cast<const uint4*>(ysrc + k));
           y1 = __ldcg(reinterpret_cast<const uint4*>(ysrc + k + 8));
         }
@@ -260,7 +271,16 @@ AXON_DEV void load_stage(const Ring<HD>& R, CState& cs, const PersistArgs& A, Pe
 
 // One projection phase: items of 16 rows x K, products on mma.sync with the
 // weight tile from the ring and the B <= 8 token rows of `act` (and of its
-// second term `act_lo` when LO); epilogue `KIND`.
+// second term `act_lo` in the two-term modes); epilogue `KIND`.
+//
+// MODE (compile time, so that each kernel carries only its own inner loop):
+//   TERMS_ONE    one 16-bit term per token (bf16 mode);
+//   TERMS_PAIRED two terms, B <= 4: token slot 2b of the MMA's N dimension
+//                holds token b's first term and slot 2b+1 its second, and
+//                the reduction adds the two accumulator columns (no extra
+//                MMA, no extra load);
+//   TERMS_TWO    two terms, B = 5..8: a second MMA set takes the second
+//                terms.
 //
 // Per item the consumer warps only run the products and the cross-warp sum;
 // the item's 16 x B sums go to a shared buffer and the epilogues run in
@@ -268,12 +288,14 @@ AXON_DEV void load_stage(const Ring<HD>& R, CState& cs, const PersistArgs& A, Pe
 // global reads (residual, rope table, bias, gains) overlap instead of
 // stalling the weight stream item after item. The LM head's argmax keeps a
 // per-CTA best key per token in shared memory and commits it once per phase.
-template <int HD, int KIND, typename T16, bool LO>
-AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, const T16* W, int N, int K,
+template <int HD, bool SM, int KIND, typename T16, int MODE>
+AXON_DEV void proj_phase(const Ring<HD, SM>& R, CState& cs, const PersistArgs& A, const T16* W, int N, int K,
                          const T16* act, const T16* act_lo, int act_stride, const EpiArgs& ep, float* red_base,
                          float* rinv_s, unsigned long long* best_s, uint8_t* act_sm, PersistGrid* g,
                          volatile int* s_abort, int tid) {
-  constexpr int ATTN = PLayout<HD>::ATTN;
+  constexpr int ATTN = PLayout<HD, SM>::ATTN;
+  constexpr bool LO = MODE != TERMS_ONE;
+  constexpr bool paired = MODE == TERMS_PAIRED;
   const int warp = tid >> 5, lane = tid & 31, r = lane >> 2, q = lane & 3;
   const int B = A.B;
   const int n = (N + 15) >> 4;
@@ -334,12 +356,8 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
   bool rinv_pending = KIND != EPI_RESID;
   if (KIND != EPI_RESID && warp < B)
     for (int j = lane; j < A.Pmax; j += 32) rp += __ldcg(A.ss + warp * A.Pmax + j);
-  // Token slot r of the MMA's N dimension normally holds token r (and, with
-  // the split operand, a second MMA set holds its second term). With B <= 4
-  // and the split operand the two terms share one MMA instead: slot 2b holds
-  // token b's first term and slot 2b+1 its second, and the reduction adds
-  // the two accumulator columns -- no extra MMA, no extra load.
-  const bool paired = LO && B <= 4;
+  // Token slot r of the MMA's N dimension holds token r, or (paired) the
+  // first or second term of token r / 2.
   const int tb = paired ? (r >> 1) : r;
   const bool term_lo = paired && (r & 1);
   const bool tok_ok = tb < B;
@@ -347,7 +365,7 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
   const T16* xsrc = (term_lo ? act_lo : act) + static_cast<long long>(tsafe) * act_stride + 16 * q;
   const T16* ysrc = LO ? act_lo + static_cast<long long>(tsafe) * act_stride + 16 * q : nullptr;
   const int xrow_s = term_lo ? B + tsafe : tsafe, yrow_s = B + tsafe;
-  const bool want_y = LO && !paired;
+  constexpr bool want_y = LO && !paired;
 
   // Epilogues of the buffered items slot 0 .. nslots-1 (items i0 + slot * grid).
   auto flush = [&](int i0, int nslots) {
@@ -389,8 +407,8 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
     for (int t = 0; t < spi; ++t) {
       uint4 w0, w1, w2, w3, x0, x1, y0, y1;
       bool on;
-      load_stage<HD, T16, LO>(R, cs, A, g, s_abort, t, spi, K, warp, lane, r, q, tok_ok, staged, act_sm, pitch, xsrc,
-                              ysrc, xrow_s, yrow_s, want_y, w0, w1, w2, w3, x0, x1, y0, y1, on);
+      load_stage<HD, SM, T16, want_y>(R, cs, A, g, s_abort, t, spi, K, warp, lane, r, q, tok_ok, staged, act_sm,
+                                      pitch, xsrc, ysrc, xrow_s, yrow_s, w0, w1, w2, w3, x0, x1, y0, y1, on);
       if (on) {
         const uint32_t A0[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
         const uint32_t A1[8] = {w2.x, w2.y, w2.z, w2.w, w3.x, w3.y, w3.z, w3.w};
@@ -403,7 +421,7 @@ AXON_DEV void proj_phase(const Ring<HD>& R, CState& cs, const PersistArgs& A, co
           const uint32_t bb[2] = {Bv[2 * j], Bv[2 * j + 1]};
           mma16816<T16>(acc[j & 1], a, bb);
         }
-        if (LO && want_y) {
+        if (want_y) {
           const uint32_t Bl[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
@@ -464,20 +482,20 @@ AXON_DEV EpiArgs base_ep(const PersistArgs& A) {
   return e;
 }
 
-template <int HD, typename T16>
+template <int HD, bool SM, typename T16, int MODE>
 __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs A) {
-  constexpr bool LO = std::is_same<T16, f16>::value;  // fp16 mode carries the split operand
-  constexpr int NS = PLayout<HD>::NS;
+  constexpr bool LO = MODE != TERMS_ONE;  // fp16 mode carries the split operand
+  constexpr int NS = PLayout<HD, SM>::NS;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  Ring<HD> R;
-  R.base = smem_u32(sm + PLayout<HD>::RING_OFF);
-  R.bars = smem_u32(sm + PLayout<HD>::BAR_OFF);
-  uint8_t* attn_sm = sm + PLayout<HD>::ATTN_OFF;
-  float* red_base = reinterpret_cast<float*>(sm + PLayout<HD>::RED_OFF);
-  float* rinv_s = reinterpret_cast<float*>(sm + PLayout<HD>::MISC_OFF);
-  volatile int* s_abort = reinterpret_cast<volatile int*>(sm + PLayout<HD>::MISC_OFF + 64);
-  unsigned long long* best_s = reinterpret_cast<unsigned long long*>(sm + PLayout<HD>::MISC_OFF + 128);
+  Ring<HD, SM> R;
+  R.base = smem_u32(sm + PLayout<HD, SM>::RING_OFF);
+  R.bars = smem_u32(sm + PLayout<HD, SM>::BAR_OFF);
+  uint8_t* attn_sm = sm + PLayout<HD, SM>::ATTN_OFF;
+  float* red_base = reinterpret_cast<float*>(sm + PLayout<HD, SM>::RED_OFF);
+  float* rinv_s = reinterpret_cast<float*>(sm + PLayout<HD, SM>::MISC_OFF);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(sm + PLayout<HD, SM>::MISC_OFF + 64);
+  unsigned long long* best_s = reinterpret_cast<unsigned long long*>(sm + PLayout<HD, SM>::MISC_OFF + 128);
   PersistGrid* g = A.grid;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -498,13 +516,13 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
     uint32_t stage = 0;
     bool stop = false;
     for (int l = 0; l < A.L && !stop; ++l) {
-      stream_matrix<HD>(R, A.wmaps + 4 * l + 0, A.Nqkv, A.D, rot, stage, stop, g, s_abort, A.err, lane);
-      stream_matrix<HD>(R, A.wmaps + 4 * l + 1, A.D, Hd, rot, stage, stop, g, s_abort, A.err, lane);
-      stream_matrix<HD>(R, A.wmaps + 4 * l + 2, 2 * A.F, A.D, rot, stage, stop, g, s_abort, A.err, lane);
-      stream_matrix<HD>(R, A.wmaps + 4 * l + 3, A.D, A.F, rot, stage, stop, g, s_abort, A.err, lane);
+      stream_matrix<HD, SM>(R, A.wmaps + 4 * l + 0, A.Nqkv, A.D, rot, stage, stop, g, s_abort, A.err, lane);
+      stream_matrix<HD, SM>(R, A.wmaps + 4 * l + 1, A.D, Hd, rot, stage, stop, g, s_abort, A.err, lane);
+      stream_matrix<HD, SM>(R, A.wmaps + 4 * l + 2, 2 * A.F, A.D, rot, stage, stop, g, s_abort, A.err, lane);
+      stream_matrix<HD, SM>(R, A.wmaps + 4 * l + 3, A.D, A.F, rot, stage, stop, g, s_abort, A.err, lane);
     }
     if (!stop)
-      stream_matrix<HD>(R, A.wmaps + 4 * A.L, A.V, A.D, rot, stage, stop, g, s_abort, A.err, lane);
+      stream_matrix<HD, SM>(R, A.wmaps + 4 * A.L, A.V, A.D, rot, stage, stop, g, s_abort, A.err, lane);
     // Copies still in flight must land before the CTA's shared memory goes
     // away: wait for the last use of every slot.
     if (lane == 0) {
@@ -585,7 +603,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       e.bt_stride = A.blocks_per_seq;
       e.blocks_per_seq = A.blocks_per_seq;
       e.num_blocks = A.num_blocks;
-      proj_phase<HD, EPI_QKV, T16, LO>(R, cs, A, static_cast<const T16*>(w.wqkv), A.Nqkv, A.D, a16, alo16, A.D, e,
+      proj_phase<HD, SM, EPI_QKV, T16, MODE>(R, cs, A, static_cast<const T16*>(w.wqkv), A.Nqkv, A.D, a16, alo16, A.D, e,
                                        red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
     }
     grid_sync(g, epoch, tid, s_abort, A.err);
@@ -617,7 +635,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       const int items = A.splits * A.G * B;
       for (int it = blockIdx.x; it < items; it += gridDim.x) {
         const int s = it % A.splits, gg = (it / A.splits) % A.G, b = it / (A.splits * A.G);
-        attn_decode_item<HD, T16, true, 1>(p, s, gg, b, attn_sm, tid);
+        attn_decode_item<HD, T16, true, 1, SM ? 1 : 2>(p, s, gg, b, attn_sm, tid);
       }
     }
     grid_sync(g, epoch, tid, s_abort, A.err);
@@ -629,7 +647,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       e.a_out = A.a;
       e.a_lo_out = A.a_lo;
       e.gain = w.g2;
-      proj_phase<HD, EPI_RESID, T16, LO>(R, cs, A, static_cast<const T16*>(w.wo), A.D, Hd,
+      proj_phase<HD, SM, EPI_RESID, T16, MODE>(R, cs, A, static_cast<const T16*>(w.wo), A.D, Hd,
                                          static_cast<const T16*>(A.o), static_cast<const T16*>(A.o_lo), Hd, e,
                                          red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
     }
@@ -640,7 +658,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       e.N = 2 * A.F;
       e.u_out = A.u;
       e.u_lo_out = A.u_lo;
-      proj_phase<HD, EPI_SWIGLU, T16, LO>(R, cs, A, static_cast<const T16*>(w.wgu), 2 * A.F, A.D, a16, alo16, A.D, e,
+      proj_phase<HD, SM, EPI_SWIGLU, T16, MODE>(R, cs, A, static_cast<const T16*>(w.wgu), 2 * A.F, A.D, a16, alo16, A.D, e,
                                           red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
     }
     grid_sync(g, epoch, tid, s_abort, A.err);
@@ -652,7 +670,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
       e.a_out = A.a;
       e.a_lo_out = A.a_lo;
       e.gain = w.gnext;
-      proj_phase<HD, EPI_RESID, T16, LO>(R, cs, A, static_cast<const T16*>(w.wd), A.D, A.F,
+      proj_phase<HD, SM, EPI_RESID, T16, MODE>(R, cs, A, static_cast<const T16*>(w.wd), A.D, A.F,
                                          static_cast<const T16*>(A.u), static_cast<const T16*>(A.u_lo), A.F, e,
                                          red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
     }
@@ -665,7 +683,7 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
     e.logits = A.logits;
     e.logits_stride = A.V;
     e.keys = A.keys;
-    proj_phase<HD, EPI_LOGITS, T16, LO>(R, cs, A, static_cast<const T16*>(A.head), A.V, A.D, a16, alo16, A.D, e,
+    proj_phase<HD, SM, EPI_LOGITS, T16, MODE>(R, cs, A, static_cast<const T16*>(A.head), A.V, A.D, a16, alo16, A.D, e,
                                         red_base, rinv_s, best_s, attn_sm, g, s_abort, tid);
   }
   grid_sync(g, epoch, tid, s_abort, A.err);
@@ -689,28 +707,75 @@ __global__ void __launch_bounds__(PTHREADS, 1) persist_decode_kernel(PersistArgs
   }
 }
 
-template <int HD, typename T16>
+template <int HD, bool SM, typename T16, int MODE>
 cudaError_t launch_t(const PersistArgs& a, int nctas, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(nctas);
   cfg.blockDim = dim3(PTHREADS);
-  cfg.dynamicSmemBytes = PLayout<HD>::BYTES;
+  cfg.dynamicSmemBytes = PLayout<HD, SM>::BYTES;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, persist_decode_kernel<HD, T16>, a);
+  return cudaLaunchKernelEx(&cfg, persist_decode_kernel<HD, SM, T16, MODE>, a);
+}
+
+template <int HD, bool SM, typename T16, int MODE>
+cudaError_t prepare_one(int* per_sm) {
+  cudaError_t e = cudaFuncSetAttribute(persist_decode_kernel<HD, SM, T16, MODE>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, PLayout<HD, SM>::BYTES);
+  if (e != cudaSuccess) return e;
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, persist_decode_kernel<HD, SM, T16, MODE>, PTHREADS,
+                                                       PLayout<HD, SM>::BYTES);
+}
+
+// Every kernel a (head_dim, type) may launch: bf16 one term, fp16 paired
+// (B <= 4) and two-set (B > 4); at head_dim 128 also the small layout of the
+// one-term and paired kernels. Resident CTAs per SM = the smallest.
+template <int HD, typename T16>
+cudaError_t prepare_t(int* per_sm) {
+  int n[4] = {0, 0, 0, 0};
+  cudaError_t e;
+  if constexpr (!std::is_same<T16, f16>::value) {
+    e = prepare_one<HD, false, T16, TERMS_ONE>(&n[0]);
+    n[1] = n[2] = n[3] = n[0];
+    if constexpr (HD == 128)
+      if (e == cudaSuccess) e = prepare_one<HD, true, T16, TERMS_ONE>(&n[1]);
+  } else {
+    e = prepare_one<HD, false, T16, TERMS_PAIRED>(&n[0]);
+    if (e == cudaSuccess) e = prepare_one<HD, false, T16, TERMS_TWO>(&n[1]);
+    n[2] = n[3] = n[0];
+    if constexpr (HD == 128)
+      if (e == cudaSuccess) e = prepare_one<HD, true, T16, TERMS_PAIRED>(&n[2]);
+  }
+  int m = n[0];
+  for (int i = 1; i < 4; ++i) m = n[i] < m ? n[i] : m;
+  *per_sm = m;
+  return e;
 }
 
 template <int HD, typename T16>
-cudaError_t prepare_t(int* per_sm) {
-  cudaError_t e = cudaFuncSetAttribute(persist_decode_kernel<HD, T16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       PLayout<HD>::BYTES);
-  if (e != cudaSuccess) return e;
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, persist_decode_kernel<HD, T16>, PTHREADS,
-                                                       PLayout<HD>::BYTES);
+cudaError_t launch_mode(const PersistArgs& a, bool small, int nctas, cudaStream_t st) {
+  if constexpr (!std::is_same<T16, f16>::value) {
+    if constexpr (HD == 128)
+      if (small) return launch_t<HD, true, T16, TERMS_ONE>(a, nctas, st);
+    return launch_t<HD, false, T16, TERMS_ONE>(a, nctas, st);
+  } else {
+    if (a.B > 4) return launch_t<HD, false, T16, TERMS_TWO>(a, nctas, st);
+    if constexpr (HD == 128)
+      if (small) return launch_t<HD, true, T16, TERMS_PAIRED>(a, nctas, st);
+    return launch_t<HD, false, T16, TERMS_PAIRED>(a, nctas, st);
+  }
+}
+
+// Whether the activations of B rows (both terms in fp16 mode, except when
+// paired) of width D stage in an attention region of `attn` bytes next to
+// the epilogue buffer.
+bool stages_in(int attn, bool use_f16, int B, int D) {
+  const int rows = use_f16 ? 2 * B : B;
+  return static_cast<long long>(rows) * (D * 2 + 16) <= attn - 8 * B * 16 * 4;
 }
 
 }  // namespace
@@ -734,17 +799,26 @@ int persist_ctas_per_sm(int head_dim, bool use_f16) {
 bool persist_fits(int head_dim, bool use_f16, int B, int D) {
   if (B < 1 || B > PERSIST_MAX_B) return false;
   // The normed operand of QKV, gate/up and the LM head (K = D; with its
-  // second term in fp16 mode, except when the two terms share one MMA) must
-  // stage in shared memory next to the epilogue buffer; streaming it from
-  // L2 stage by stage is slower than the launch chain.
-  const int attn = head_dim == 64 ? PLayout<64>::ATTN : PLayout<128>::ATTN;
-  const int rows = use_f16 ? 2 * B : B;
-  return rows * (D * 2 + 16) <= attn - 8 * B * 16 * 4;
+  // second term in fp16 mode) must stage in shared memory next to the
+  // epilogue buffer; streaming it from L2 stage by stage is slower than the
+  // launch chain.
+  const int attn = head_dim == 64 ? PLayout<64, false>::ATTN : PLayout<128, false>::ATTN;
+  return stages_in(attn, use_f16, B, D);
+}
+
+bool persist_small(int head_dim, bool use_f16, int B, int kmax) {
+  if (head_dim != 128 || B < 1 || B > (use_f16 ? 4 : PERSIST_MAX_B)) return false;
+  return stages_in(PLayout<128, true>::ATTN, use_f16, B, kmax);
 }
 
 cudaError_t launch_persist_decode(const PersistArgs& a, int head_dim, bool use_f16, int nctas, cudaStream_t st) {
   if (a.B < 1 || a.B > PERSIST_MAX_B || (a.D & 63) || (a.F & 63) || ((a.H * a.d) & 63)) return cudaErrorInvalidValue;
-  if (head_dim == 64) return use_f16 ? launch_t<64, f16>(a, nctas, st) : launch_t<64, bf16>(a, nctas, st);
-  if (head_dim == 128) return use_f16 ? launch_t<128, f16>(a, nctas, st) : launch_t<128, bf16>(a, nctas, st);
+  if (head_dim == 64)
+    return use_f16 ? launch_mode<64, f16>(a, false, nctas, st) : launch_mode<64, bf16>(a, false, nctas, st);
+  if (head_dim == 128) {
+    const int kmax = std::max(std::max(a.D, a.H * a.d), a.F);
+    const bool small = persist_small(128, use_f16, a.B, kmax);
+    return use_f16 ? launch_mode<128, f16>(a, small, nctas, st) : launch_mode<128, bf16>(a, small, nctas, st);
+  }
   return cudaErrorInvalidValue;
 }

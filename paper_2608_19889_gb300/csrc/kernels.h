@@ -270,4 +270,9 @@ int persist_ctas_per_sm(int head_dim, bool use_f16);
 // Whether B sequences of width D suit the kernel (their normed activations
 // stage in shared memory); else the decode step takes the launch chain.
 bool persist_fits(int head_dim, bool use_f16, int B, int D);
+// Whether the kernel takes its small layout for this batch (head_dim 128:
+// one staged key block per warp, a deeper weight ring): the activations of
+// every projection (widest K = kmax) must still stage next to the epilogue
+// buffer. Its attention items then hold 8 key blocks, one per warp.
+bool persist_small(int head_dim, bool use_f16, int B, int kmax);
 cudaError_t launch_persist_decode(const PersistArgs& a, int head_dim, bool use_f16, int nctas, cudaStream_t st);

@@ -122,7 +122,8 @@ def test_persistent_decode_paged_cache(prec):
 @pytest.mark.parametrize("shape", [TINY, TINY128])
 def test_persistent_decode_split_kv_long_context(shape):
     """A context of more than 64 key blocks: the persistent step splits each
-    sequence's keys into items of 16 blocks and merges them across CTAs."""
+    sequence's keys into items of 16 blocks (8 in the head_dim-128 small
+    layout, one staged block per warp) and merges them across CTAs."""
     ax = _ax()
     B, S, max_ctx = 2, 1100, 1152  # 72 key blocks of capacity: 5 splits
     w = gpu_weights(shape)
