@@ -124,6 +124,7 @@ struct axon_model {
   PersistGrid* pgrid = nullptr;
   int persist_ctas = 0;
   int decode_gemv_max = 32;  // decode projections with more tokens take the tcgen05 GEMM (AXON_DECODE_GEMV_MAX)
+  bool qkv_split = true;     // decode QKV of 9-16 tokens on the split-K GEMM (AXON_QKV_SPLITK=0: the GEMV)
   int persist_split_blocks = 16;  // persistent step: key blocks per split-KV item (AXON_PERSIST_SPLIT_BLOCKS)
   // decode attention grid budget in CTAs (AXON_ATTN_TARGET_CTAS; 0: the
   // split count with the smallest estimated makespan)
@@ -499,11 +500,14 @@ struct Proj {
     //    LM head);
     //  * the residual projections (O, down) on the split-K GEMM where the
     //    parts stay cheap to sum: a long K (>= 8192) or at most 16 tokens;
+    //    QKV too at most 16 tokens (qkv_split);
     //  * otherwise the GEMV up to gemv_max tokens, the plain GEMM above.
     const bool dec = gemv_max < 64 && maps != nullptr && !m->fp32 && M > 8;
     const bool wide = dec && static_cast<long long>((N + 127) / 128) * ((M + 127) / 128) >= m->num_sms;
-    const bool resid_split = dec && !wide && kind == EPI_RESID && (K >= 8192 || M <= 16) &&
-                             gemm_split_k(lc, M, N, K) > 1 && m->gemm_sk.ws != nullptr;
+    const bool split_kind =
+        (kind == EPI_RESID && (K >= 8192 || M <= 16)) || (kind == EPI_QKV && m->qkv_split && M <= 16);
+    const bool resid_split =
+        dec && !wide && split_kind && gemm_split_k(lc, M, N, K) > 1 && m->gemm_sk.ws != nullptr;
     const bool gemv = (M <= gemv_max && !wide && !resid_split) || (!m->fp32 && maps == nullptr);
     if (gemv && kind == EPI_RESID) {
       ep.rinv_out = m->rinv;
@@ -1091,6 +1095,7 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     const int t = atoi(v);
     if (t >= 0 && t <= 64) m->decode_gemv_max = t;
   }
+  if (const char* v = getenv("AXON_QKV_SPLITK")) m->qkv_split = atoi(v) != 0;
   g_trace = env_flag("AXON_TRACE");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   auto fail = [&](int code) {

@@ -222,14 +222,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         tc_fence_before();
         mbar_arrive(acce_bar(buf));
-        __threadfence();
+        // ticket after the epilogue warps' barrier: one acquire-release atomic
+        // publishes the four warps' partial stores and, for the last unit,
+        // orders its loads of the other units' partials after theirs
         asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (etid == 0) s_last = (atomicAdd(tickets + t, 1) == ks - 1);
+        if (etid == 0) s_last = (atom_add_acq_rel_gpu(tickets + t, 1) == ks - 1);
         asm volatile("bar.sync 1, 128;" ::: "memory");
         if (s_last) {
           // 2. last unit of the tile: sum the ks partials in split order
           // (deterministic) and run the epilogue, as (row, 16 columns) tasks
-          __threadfence();
           if (KIND != EPI_RESID && etid < M) s_rinv[etid] = row_rinv(ep, etid);
           asm volatile("bar.sync 1, 128;" ::: "memory");
           constexpr int CH = BN / 16;
@@ -240,15 +241,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             float f[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) f[i] = 0.f;
-            for (int sp = 0; sp < ks; ++sp) {
-              const float* pp = ws + ((static_cast<long long>(t) * ks + sp) * BM + m) * BN + c;
+            // four splits' loads in flight per round trip, added in split order
+            for (int sp0 = 0; sp0 < ks; sp0 += 4) {
+              float4 a4[4][4];
 #pragma unroll
-              for (int i = 0; i < 16; i += 4) {
-                const float4 a4 = __ldcg(reinterpret_cast<const float4*>(pp + i));
-                f[i] += a4.x;
-                f[i + 1] += a4.y;
-                f[i + 2] += a4.z;
-                f[i + 3] += a4.w;
+              for (int u = 0; u < 4; ++u) {
+                const bool in = sp0 + u < ks;
+                const float* pp = ws + ((static_cast<long long>(t) * ks + (in ? sp0 + u : 0)) * BM + m) * BN + c;
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                  a4[u][i] = in ? __ldcg(reinterpret_cast<const float4*>(pp + 4 * i)) : make_float4(0.f, 0.f, 0.f, 0.f);
+              }
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                if (sp0 + u >= ks) break;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  f[4 * i] += a4[u][i].x;
+                  f[4 * i + 1] += a4[u][i].y;
+                  f[4 * i + 2] += a4[u][i].z;
+                  f[4 * i + 3] += a4[u][i].w;
+                }
               }
             }
             if (KIND == EPI_QKV) {
