@@ -821,7 +821,7 @@ int enqueue_prefill(axon_model* m, const int32_t* ids, int B, int S, const int32
 // their routing kernels, so those models decode on the launch chain.
 bool persist_eligible(const axon_model* m, int B) {
   return m->persist_ctas > 0 && !m->fp32 && !m->cfg.qk_norm && !m->moe && m->H / m->G <= 8 &&
-         persist_fits(m->d, m->f16, B, m->D);
+         persist_fits(m->d, m->f16, B, m->D, std::max(std::max(m->D, m->H * m->d), m->F));
 }
 
 PersistArgs persist_args(const axon_model* m, const int32_t* tokens, int B, int32_t* ctx, const int32_t* bt,
@@ -906,10 +906,9 @@ int enqueue_decode(axon_model* m, const int32_t* tokens, int B, int32_t* ctx, co
     // key blocks (8 per warp; measured at 40 blocks, head_dim 64: 0.743 ms
     // per step unsplit, 0.775-0.790 ms split). Beyond that the keys split
     // into items of persist_split_blocks blocks (80 blocks, head_dim 128:
-    // 3.170 ms per step in items of 16, 3.239 ms in items of 64). The small
-    // layout stages one block per warp: items of 8 blocks, one round.
-    const int kmax = std::max(std::max(m->D, m->H * m->d), m->F);
-    const int sblocks = persist_small(m->d, m->f16, B, kmax) ? 8 : m->persist_split_blocks;
+    // 3.170 ms per step in items of 16, 3.239 ms in items of 64). Head_dim
+    // 128 stages one block per warp: items of 8 blocks, one round.
+    const int sblocks = m->d == 128 ? 8 : m->persist_split_blocks;
     int psplits = (m->blocks_per_seq > 64 || sblocks == 8) ? (m->blocks_per_seq + sblocks - 1) / sblocks : 1;
     if (psplits > cap) psplits = cap;
     PersistArgs pa = persist_args(m, tokens, B, ctx, bt, logits, next, psplits, attn_part ? attn_part : m->attn_part,

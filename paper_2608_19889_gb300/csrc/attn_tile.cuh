@@ -161,6 +161,90 @@ AXON_DEV void attn_tile16(uint32_t ks, uint32_t vs, const uint32_t (&qa)[HD / 16
   }
 }
 
+// Two consecutive 16-key blocks (keys tok0 .. tok0+31; block A's K and V at
+// ksa / vsa, block B's at ksb / vsb) as one tile: four independent score
+// accumulators in the QK^T loop instead of two, one online-softmax rescale
+// of the output for 32 keys instead of two. Rows as in attn_tile16 (not
+// paired).
+template <int HD, typename T16>
+AXON_DEV void attn_tile32(uint32_t ksa, uint32_t vsa, uint32_t ksb, uint32_t vsb, const uint32_t (&qa)[HD / 16][4],
+                          WarpState<HD>& st, int tok0, int lo0, int lim0, int lo1, int lim1, float sl2, int lane) {
+  const int q = lane & 3;
+  const int mi = lane >> 3, li = lane & 7;
+  float s[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
+#pragma unroll
+  for (int kk = 0; kk < HD / 16; ++kk) {
+    uint32_t ka[4], kb[4];
+    const int tok = (mi >> 1) * 8 + li, ch = 2 * kk + (mi & 1);
+    ldsm_x4(ka, swz<HD>(ksa, tok, ch));
+    ldsm_x4(kb, swz<HD>(ksb, tok, ch));
+    const uint32_t b0[2] = {ka[0], ka[1]}, b1[2] = {ka[2], ka[3]}, b2[2] = {kb[0], kb[1]}, b3[2] = {kb[2], kb[3]};
+    mma16816<T16>(s[0], qa[kk], b0);
+    mma16816<T16>(s[1], qa[kk], b1);
+    mma16816<T16>(s[2], qa[kk], b2);
+    mma16816<T16>(s[3], qa[kk], b3);
+  }
+  float mx0 = NEG_INF, mx1 = NEG_INF;
+#pragma unroll
+  for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int t = tok0 + nt * 8 + 2 * q + e;
+      s[nt][e] = (t <= lim0 && t >= lo0) ? s[nt][e] * sl2 : NEG_INF;
+      s[nt][2 + e] = (t <= lim1 && t >= lo1) ? s[nt][2 + e] * sl2 : NEG_INF;
+      mx0 = fmaxf(mx0, s[nt][e]);
+      mx1 = fmaxf(mx1, s[nt][2 + e]);
+    }
+  }
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+  const float nm0 = fmaxf(st.m0, mx0), nm1 = fmaxf(st.m1, mx1);
+  const float base0 = (nm0 == NEG_INF) ? 0.f : nm0, base1 = (nm1 == NEG_INF) ? 0.f : nm1;
+  const float a0 = exp2f(st.m0 - base0), a1 = exp2f(st.m1 - base1);
+  float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+  for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      s[nt][e] = exp2f(s[nt][e] - base0);
+      s[nt][2 + e] = exp2f(s[nt][2 + e] - base1);
+      ps0 += s[nt][e];
+      ps1 += s[nt][2 + e];
+    }
+  }
+  st.l0 = st.l0 * a0 + ps0;
+  st.l1 = st.l1 * a1 + ps1;
+  st.m0 = nm0;
+  st.m1 = nm1;
+#pragma unroll
+  for (int nd = 0; nd < HD / 8; ++nd) {
+    st.o[nd][0] *= a0;
+    st.o[nd][1] *= a0;
+    st.o[nd][2] *= a1;
+    st.o[nd][3] *= a1;
+  }
+  const uint32_t pa[4] = {pack2<T16>(s[0][0], s[0][1]), pack2<T16>(s[0][2], s[0][3]), pack2<T16>(s[1][0], s[1][1]),
+                          pack2<T16>(s[1][2], s[1][3])};
+  const uint32_t pb[4] = {pack2<T16>(s[2][0], s[2][1]), pack2<T16>(s[2][2], s[2][3]), pack2<T16>(s[3][0], s[3][1]),
+                          pack2<T16>(s[3][2], s[3][3])};
+#pragma unroll
+  for (int nd2 = 0; nd2 < HD / 16; ++nd2) {
+    uint32_t va[4], vb[4];
+    const int tok = (mi & 1) * 8 + li, ch = 2 * nd2 + (mi >> 1);
+    ldsm_x4_t(va, swz<HD>(vsa, tok, ch));
+    ldsm_x4_t(vb, swz<HD>(vsb, tok, ch));
+    const uint32_t a0v[2] = {va[0], va[1]}, a1v[2] = {va[2], va[3]}, b0v[2] = {vb[0], vb[1]}, b1v[2] = {vb[2], vb[3]};
+    mma16816<T16>(st.o[2 * nd2], pa, a0v);
+    mma16816<T16>(st.o[2 * nd2 + 1], pa, a1v);
+    mma16816<T16>(st.o[2 * nd2], pb, b0v);
+    mma16816<T16>(st.o[2 * nd2 + 1], pb, b1v);
+  }
+}
+
 // After the last PAIRED tile: add row r + 8's partial output into row r and
 // leave row r + 8 empty.
 template <int HD>

@@ -124,12 +124,23 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(AttnArgs p, int PW, A
     }
     __syncthreads();
     if (wfirst < S) {
-      for (int jj = 0; jj < 4; ++jj) {
+      // blocks in pairs where both are needed (32-key tiles), else singly
+      for (int jj = 0; jj < 4;) {
         const int j = jlo + sidx * 4 + jj;
         if (j >= jlo + nblk || j * 16 > wmax) break;
-        if (j * 16 + 15 < wlo) continue;  // slid out of every row of this warp
+        if (j * 16 + 15 < wlo) {  // slid out of every row of this warp
+          ++jj;
+          continue;
+        }
         const uint32_t t = base + buf * STAGE + jj * 2 * TILE;
-        attn_tile16<HD, T16>(t, t + TILE, qa, st, j * 16, lo0, pos0, lo1, pos1, p.scale_log2, lane);
+        if (jj + 1 < 4 && j + 1 < jlo + nblk && (j + 1) * 16 <= wmax) {
+          attn_tile32<HD, T16>(t, t + TILE, t + 2 * TILE, t + 3 * TILE, qa, st, j * 16, lo0, pos0, lo1, pos1,
+                               p.scale_log2, lane);
+          jj += 2;
+        } else {
+          attn_tile16<HD, T16>(t, t + TILE, qa, st, j * 16, lo0, pos0, lo1, pos1, p.scale_log2, lane);
+          ++jj;
+        }
       }
     }
     __syncthreads();

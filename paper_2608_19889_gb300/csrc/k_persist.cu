@@ -35,7 +35,6 @@
 // (same barrier sequence, so named barriers stay matched) and the host sees
 // the error bit. Before it exits, the producer waits (bounded) for its copies
 // in flight.
-#include <algorithm>
 #include <type_traits>
 
 #include "attn_tile.cuh"
@@ -57,10 +56,9 @@ static_assert(PCW == DEC_WARPS, "attention items run on the consumer warps");
 // How the 16-bit operand terms of the projections enter the MMAs (proj_phase).
 constexpr int TERMS_ONE = 0, TERMS_PAIRED = 1, TERMS_TWO = 2;
 
-// Shared-memory layout. SM ("small"): the attention items stage one key
-// block per warp (decode_smem1), so the weight ring gets the space a second
-// stage would take -- at head_dim 128, 8 ring stages instead of 5; taken
-// when the activations of the batch still stage next to the epilogue buffer.
+// Shared-memory layout. SM ("small", head_dim 128): the attention items stage
+// one key block per warp (decode_smem1), so the weight ring gets the space a
+// second stage would take: 9 ring stages instead of 5.
 template <int HD, bool SM>
 struct PLayout {
   static constexpr int ATTN = SM ? static_cast<int>(decode_smem1<HD>()) : static_cast<int>(decode_smem<HD>());
@@ -731,51 +729,42 @@ cudaError_t prepare_one(int* per_sm) {
                                                        PLayout<HD, SM>::BYTES);
 }
 
-// Every kernel a (head_dim, type) may launch: bf16 one term, fp16 paired
-// (B <= 4) and two-set (B > 4); at head_dim 128 also the small layout of the
-// one-term and paired kernels. Resident CTAs per SM = the smallest.
+// The kernels a (head_dim, type) launches: bf16 one term; fp16 paired
+// (B <= 4) and two sets (B > 4). Head_dim 64 takes the layout whose
+// attention region stages two key blocks per warp, head_dim 128 the small
+// one (measured at head_dim 128: the two-stage layout's 5-stage ring lost to
+// the launch chain at 8B width, B = 8, bf16, 4.19 against 3.59 ms per step,
+// and tied it at 32B width, B = 1, fp16). Resident CTAs per SM = the smaller
+// count.
 template <int HD, typename T16>
 cudaError_t prepare_t(int* per_sm) {
-  int n[4] = {0, 0, 0, 0};
-  cudaError_t e;
+  constexpr bool SMALL = HD == 128;
   if constexpr (!std::is_same<T16, f16>::value) {
-    e = prepare_one<HD, false, T16, TERMS_ONE>(&n[0]);
-    n[1] = n[2] = n[3] = n[0];
-    if constexpr (HD == 128)
-      if (e == cudaSuccess) e = prepare_one<HD, true, T16, TERMS_ONE>(&n[1]);
+    return prepare_one<HD, SMALL, T16, TERMS_ONE>(per_sm);
   } else {
-    e = prepare_one<HD, false, T16, TERMS_PAIRED>(&n[0]);
-    if (e == cudaSuccess) e = prepare_one<HD, false, T16, TERMS_TWO>(&n[1]);
-    n[2] = n[3] = n[0];
-    if constexpr (HD == 128)
-      if (e == cudaSuccess) e = prepare_one<HD, true, T16, TERMS_PAIRED>(&n[2]);
+    int a = 0, b = 0;
+    cudaError_t e = prepare_one<HD, SMALL, T16, TERMS_PAIRED>(&a);
+    if (e == cudaSuccess) e = prepare_one<HD, SMALL, T16, TERMS_TWO>(&b);
+    *per_sm = a < b ? a : b;
+    return e;
   }
-  int m = n[0];
-  for (int i = 1; i < 4; ++i) m = n[i] < m ? n[i] : m;
-  *per_sm = m;
-  return e;
 }
 
 template <int HD, typename T16>
-cudaError_t launch_mode(const PersistArgs& a, bool small, int nctas, cudaStream_t st) {
-  if constexpr (!std::is_same<T16, f16>::value) {
-    if constexpr (HD == 128)
-      if (small) return launch_t<HD, true, T16, TERMS_ONE>(a, nctas, st);
-    return launch_t<HD, false, T16, TERMS_ONE>(a, nctas, st);
-  } else {
-    if (a.B > 4) return launch_t<HD, false, T16, TERMS_TWO>(a, nctas, st);
-    if constexpr (HD == 128)
-      if (small) return launch_t<HD, true, T16, TERMS_PAIRED>(a, nctas, st);
-    return launch_t<HD, false, T16, TERMS_PAIRED>(a, nctas, st);
-  }
+cudaError_t launch_mode(const PersistArgs& a, int nctas, cudaStream_t st) {
+  constexpr bool SMALL = HD == 128;
+  if constexpr (!std::is_same<T16, f16>::value)
+    return launch_t<HD, SMALL, T16, TERMS_ONE>(a, nctas, st);
+  else
+    return a.B <= 4 ? launch_t<HD, SMALL, T16, TERMS_PAIRED>(a, nctas, st)
+                    : launch_t<HD, SMALL, T16, TERMS_TWO>(a, nctas, st);
 }
 
-// Whether the activations of B rows (both terms in fp16 mode, except when
-// paired) of width D stage in an attention region of `attn` bytes next to
-// the epilogue buffer.
-bool stages_in(int attn, bool use_f16, int B, int D) {
+// Whether B activation rows (two terms each in fp16 mode) of K columns stage
+// in an attention region of `attn` bytes next to the epilogue buffer.
+bool stages_in(int attn, bool use_f16, int B, int K) {
   const int rows = use_f16 ? 2 * B : B;
-  return static_cast<long long>(rows) * (D * 2 + 16) <= attn - 8 * B * 16 * 4;
+  return static_cast<long long>(rows) * (K * 2 + 16) <= attn - 8 * B * 16 * 4;
 }
 
 }  // namespace
@@ -796,29 +785,20 @@ int persist_ctas_per_sm(int head_dim, bool use_f16) {
   return n;
 }
 
-bool persist_fits(int head_dim, bool use_f16, int B, int D) {
+bool persist_fits(int head_dim, bool use_f16, int B, int D, int kmax) {
   if (B < 1 || B > PERSIST_MAX_B) return false;
-  // The normed operand of QKV, gate/up and the LM head (K = D; with its
-  // second term in fp16 mode) must stage in shared memory next to the
-  // epilogue buffer; streaming it from L2 stage by stage is slower than the
-  // launch chain.
-  const int attn = head_dim == 64 ? PLayout<64, false>::ATTN : PLayout<128, false>::ATTN;
-  return stages_in(attn, use_f16, B, D);
-}
-
-bool persist_small(int head_dim, bool use_f16, int B, int kmax) {
-  if (head_dim != 128 || B < 1 || B > (use_f16 ? 4 : PERSIST_MAX_B)) return false;
-  return stages_in(PLayout<128, true>::ATTN, use_f16, B, kmax);
+  // Head_dim 64: the normed operand of QKV, gate/up and the LM head (K = D)
+  // must stage in shared memory next to the epilogue buffer; streaming it
+  // from L2 stage by stage is slower than the launch chain. Head_dim 128
+  // (small layout): every projection's operand (K up to kmax) must.
+  if (head_dim == 64) return stages_in(PLayout<64, false>::ATTN, use_f16, B, D);
+  if (head_dim == 128) return stages_in(PLayout<128, true>::ATTN, use_f16, B, kmax);
+  return false;
 }
 
 cudaError_t launch_persist_decode(const PersistArgs& a, int head_dim, bool use_f16, int nctas, cudaStream_t st) {
   if (a.B < 1 || a.B > PERSIST_MAX_B || (a.D & 63) || (a.F & 63) || ((a.H * a.d) & 63)) return cudaErrorInvalidValue;
-  if (head_dim == 64)
-    return use_f16 ? launch_mode<64, f16>(a, false, nctas, st) : launch_mode<64, bf16>(a, false, nctas, st);
-  if (head_dim == 128) {
-    const int kmax = std::max(std::max(a.D, a.H * a.d), a.F);
-    const bool small = persist_small(128, use_f16, a.B, kmax);
-    return use_f16 ? launch_mode<128, f16>(a, small, nctas, st) : launch_mode<128, bf16>(a, small, nctas, st);
-  }
+  if (head_dim == 64) return use_f16 ? launch_mode<64, f16>(a, nctas, st) : launch_mode<64, bf16>(a, nctas, st);
+  if (head_dim == 128) return use_f16 ? launch_mode<128, f16>(a, nctas, st) : launch_mode<128, bf16>(a, nctas, st);
   return cudaErrorInvalidValue;
 }

@@ -267,12 +267,8 @@ struct PersistArgs {
 // Resident CTAs per SM of the kernel for this head_dim / type (0: not
 // available); also sets its shared-memory limit. Call before any launch.
 int persist_ctas_per_sm(int head_dim, bool use_f16);
-// Whether B sequences of width D suit the kernel (their normed activations
-// stage in shared memory); else the decode step takes the launch chain.
-bool persist_fits(int head_dim, bool use_f16, int B, int D);
-// Whether the kernel takes its small layout for this batch (head_dim 128:
-// one staged key block per warp, a deeper weight ring): the activations of
-// every projection (widest K = kmax) must still stage next to the epilogue
-// buffer. Its attention items then hold 8 key blocks, one per warp.
-bool persist_small(int head_dim, bool use_f16, int B, int kmax);
+// Whether B sequences of width D (widest projection input kmax) suit the
+// kernel (their activations stage in shared memory); else the decode step
+// takes the launch chain.
+bool persist_fits(int head_dim, bool use_f16, int B, int D, int kmax);
 cudaError_t launch_persist_decode(const PersistArgs& a, int head_dim, bool use_f16, int nctas, cudaStream_t st);
