@@ -44,6 +44,13 @@ struct GCfg {
   static constexpr int SMEM = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
 };
 
+// Residual epilogue staging: each epilogue warp's 32 rows x 32 accumulator
+// columns, rows padded to 36 floats (float4 stores of 8 consecutive rows
+// hit distinct banks).
+constexpr int EPI_TP = 36;
+template <int KIND>
+constexpr int epi_smem() { return KIND == EPI_RESID ? 4 * 32 * EPI_TP * 4 : 0; }
+
 AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
   const int per_group = GROUP_M * num_n;
   const int g = t / per_group;
@@ -72,6 +79,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t sA = base, sAlo = base + STAGES * A_BYTES, sB = base + STAGES * A_BYTES * C::A_TERMS;
   const uint32_t bars = base + STAGES * STAGE_BYTES;
   const uint32_t tmem_slot = bars + 8 * (2 * STAGES + 4);
+  float* const epi_tile = reinterpret_cast<float*>(smem_raw + (bars + C::BAR_BYTES - raw));  // epi_smem<KIND>()
   const uint32_t* tmem_slot_ptr =
       reinterpret_cast<const uint32_t*>(smem_raw + (tmem_slot - raw));
   auto full_bar = [&](int s) { return bars + 8 * s; };
@@ -291,36 +299,89 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const bool mval = m < M && (!grp.row_valid || grp.row_valid[m] >= 0);
       float rinv = 1.f;
       if (KIND != EPI_RESID && KIND != EPI_ROWSCALE && mval) rinv = row_rinv(ep, m);
-      float ssum = 0.f;
       unsigned long long best = 0ull;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(q4 * 32) << 16) + buf * BN;
       if (KIND == EPI_RESID) {
-        // 64 columns at a time: the 16 residual loads of a group are in
-        // flight together, and one TMEM wait covers 4 loads.
+        // Through shared memory, 32 columns at a time: the warp stages its 32
+        // rows x 32 accumulator columns, then every global access (residual
+        // read, x, a and a_lo writes) covers 4 rows x 128 bytes per
+        // instruction, lane (r, c) taking row 4i + r, columns 4c .. 4c+3.
+        float* tw = epi_tile + q4 * 32 * EPI_TP;
+        const int lr = lane >> 3, lc = (lane & 7) * 4;
+        const int mrow = mb * BM + q4 * 32 + lr;  // + 4i: the lane's rows
+        bool rv[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int mm = mrow + 4 * i;
+          rv[i] = mm < M && (!grp.row_valid || grp.row_valid[mm] >= 0);
+        }
+        // residual slices of group c0 (8 rows x 4 columns per lane), loaded
+        // one group ahead so that their round trip overlaps the previous
+        // group's stores
+        auto load_x = [&](int c0, float4 (&xr)[8]) {
+          const int n = nb * BN + c0 + lc;
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            xr[i] = (rv[i] && n < N) ? __ldcg(reinterpret_cast<const float4*>(
+                                           ep.x + static_cast<long long>(mrow + 4 * i) * ep.N + n))
+                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+        };
+        float rs[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) rs[i] = 0.f;
+        float4 xcur[8], xnext[8];
+        load_x(0, xcur);
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 64) {
-          float4 xin[4][4];
-          if (mval) {
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              if (nb * BN + c0 + j * 16 < N) load_resid16(ep, m, nb * BN + c0 + j * 16, xin[j]);
-          }
-          uint32_t v[4][16];
-#pragma unroll
-          for (int j = 0; j < 4; ++j) tmem_ld16(taddr + c0 + j * 16, v[j]);
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+          if (c0 + 32 < BN) load_x(c0 + 32, xnext);
+          uint32_t v[2][16];
+          tmem_ld16(taddr + c0, v[0]);
+          tmem_ld16(taddr + c0 + 16, v[1]);
           tmem_wait_ld();
-          if (mval) {
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const int n0 = nb * BN + c0 + j * 16;
-              if (n0 < N) {
-                float f[16];
+          for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(tw + lane * EPI_TP + 4 * j) =
+                make_float4(__uint_as_float(v[j >> 2][(j & 3) * 4]), __uint_as_float(v[j >> 2][(j & 3) * 4 + 1]),
+                            __uint_as_float(v[j >> 2][(j & 3) * 4 + 2]), __uint_as_float(v[j >> 2][(j & 3) * 4 + 3]));
+          __syncwarp();
+          const int n = nb * BN + c0 + lc;
+          const float4 g4 = n < N ? *reinterpret_cast<const float4*>(ep.gain + n) : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(v[j][i]);
-                ssum += epi_resid16x<T16>(ep, m, n0, f, xin[j]);
+          for (int i = 0; i < 8; ++i) {
+            const int rl = 4 * i + lr;
+            float part = 0.f;
+            if (rv[i] && n < N) {
+              const float4 acc = *reinterpret_cast<const float4*>(tw + rl * EPI_TP + lc);
+              const float4 xo = xcur[i];
+              const float xn[4] = {xo.x + acc.x, xo.y + acc.y, xo.z + acc.z, xo.w + acc.w};
+              const long long off = static_cast<long long>(mrow + 4 * i) * ep.N + n;
+              *reinterpret_cast<float4*>(ep.x + off) = make_float4(xn[0], xn[1], xn[2], xn[3]);
+              const float ag[4] = {xn[0] * g4.x, xn[1] * g4.y, xn[2] * g4.z, xn[3] * g4.w};
+              *reinterpret_cast<uint2*>(static_cast<T16*>(ep.a_out) + off) =
+                  make_uint2(pack2<T16>(ag[0], ag[1]), pack2<T16>(ag[2], ag[3]));
+              if (ep.a_lo_out) {
+                float lo[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) lo[k] = ag[k] - to_f(from_f<T16>(ag[k]));
+                *reinterpret_cast<uint2*>(static_cast<T16*>(ep.a_lo_out) + off) =
+                    make_uint2(pack2<T16>(lo[0], lo[1]), pack2<T16>(lo[2], lo[3]));
               }
+              part = ((xn[0] * xn[0] + xn[1] * xn[1]) + xn[2] * xn[2]) + xn[3] * xn[3];
             }
+            // the row's 32 columns: the 8 lanes of the row, fixed tree order
+            part += __shfl_xor_sync(0xffffffffu, part, 1);
+            part += __shfl_xor_sync(0xffffffffu, part, 2);
+            part += __shfl_xor_sync(0xffffffffu, part, 4);
+            rs[i] += part;
           }
+          __syncwarp();
+#pragma unroll
+          for (int i = 0; i < 8; ++i) xcur[i] = xnext[i];
+        }
+        if ((lane & 7) == 0) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (rv[i]) ep.ss_out[static_cast<long long>(mrow + 4 * i) * ep.ss_out_stride + nb] = rs[i];
         }
       }
 #pragma unroll 1
@@ -347,7 +408,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       tc_fence_before();
       mbar_arrive(acce_bar(buf));
-      if (KIND == EPI_RESID && mval) ep.ss_out[static_cast<long long>(m) * ep.ss_out_stride + nb] = ssum;
+
       if (KIND == EPI_LOGITS && mval) argmax_commit(ep.keys + m, best);
     }
   }
@@ -381,7 +442,7 @@ cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N,
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(NUM_THREADS);
-  cfg.dynamicSmemBytes = GCfg<SPLIT, BN>::SMEM;
+  cfg.dynamicSmemBytes = GCfg<SPLIT, BN>::SMEM + epi_smem<KIND>();
   cfg.stream = lc.stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -424,7 +485,7 @@ namespace {
 template <int KIND, typename T16, bool SPLIT, int BN>
 cudaError_t set_smem1() {
   return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              GCfg<SPLIT, BN>::SMEM);
+                              GCfg<SPLIT, BN>::SMEM + epi_smem<KIND>());
 }
 template <int KIND, typename T16, bool SPLIT>
 cudaError_t set_smem() {
