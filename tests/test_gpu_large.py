@@ -182,9 +182,9 @@ def test_32b_width_prefill_s2048():
 @pytest.mark.parametrize("name,B", [("8b", 12), ("32b", 16)])
 def test_wide_decode_batch_9_to_32(name, B):
     """Decode with 9-32 sequences at full width, one layer: the launch chain
-    with gate/up and the LM head on the tcgen05 GEMM, O and down on its split-K
-    mode and QKV on the 16-32-token GEMV (the plan the 32B batch-16 config
-    decodes with)."""
+    with gate/up and the LM head on the tcgen05 GEMM, QKV, O and down on its
+    split-K mode at up to 16 tokens (the plan the 32B batch-16 config decodes
+    with)."""
     import paper_2608_19889_gb300 as ax
     m = shape(name, L=1)
     S, n = 48, 4
