@@ -32,14 +32,25 @@ constexpr int NUM_THREADS = 192;
 // 16-bit terms (hi + lo) and every k-step issues two MMAs into the same
 // accumulator. The ring takes as many stages as fit in 200 KB, at most 6
 // (BN 256: 4, split 3; BN 128: 6, split 4).
-template <bool SPLIT, int BN_>
+//
+// SMALL (at most 16 activation rows, decode): each stage holds [A (16 rows)
+// | A_lo (16 rows, SPLIT) | B]; the MMA still reads 128 A rows from the
+// 16-row tile, rows 16..127 falling in the same stage's following bytes
+// (landed, so stable; their accumulator rows are never stored). Without the
+// 112 padding rows a stage is 2-3x smaller, so more of them -- more weight
+// bytes in flight per SM -- fit (up to 12).
+template <bool SPLIT, int BN_, bool SMALL = false>
 struct GCfg {
   static constexpr int BN = BN_;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
   static constexpr int A_TERMS = SPLIT ? 2 : 1;
-  static constexpr int STAGE_BYTES = A_TERMS * A_BYTES + B_BYTES;
-  static constexpr int STAGES = (200 * 1024) / STAGE_BYTES > 6 ? 6 : (200 * 1024) / STAGE_BYTES;
+  static constexpr int A_TILE = SMALL ? 16 * BK * 2 : A_BYTES;  // bytes of one A term in a stage
+  static constexpr int STAGE_BYTES = A_TERMS * A_TILE + B_BYTES;
+  static constexpr int MAX_STAGES = SMALL ? 12 : 6;
+  static constexpr int STAGES =
+      (200 * 1024) / STAGE_BYTES > MAX_STAGES ? MAX_STAGES : (200 * 1024) / STAGE_BYTES;
+  static_assert(!SMALL || STAGE_BYTES - (A_TERMS - 1) * A_TILE >= A_BYTES, "the MMA's 128-row read stays in its stage");
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
   static constexpr int SMEM = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
 };
@@ -61,12 +72,12 @@ AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
   mb = first_m + (local - nb * gm);
 }
 
-template <int KIND, typename T16, bool SPLIT, int BN_>
+template <int KIND, typename T16, bool SPLIT, int BN_, bool SMALL>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmAlo, int M, int N, int K, EpiArgs ep, int ks, float* ws,
                    int* tickets, GemmGroup grp) {
-  using C = GCfg<SPLIT, BN_>;
+  using C = GCfg<SPLIT, BN_, SMALL>;
   constexpr int BN = C::BN;
   constexpr int B_BYTES = C::B_BYTES;
   constexpr uint32_t TMEM_COLS = C::TMEM_COLS;
@@ -75,8 +86,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  // ring: [STAGES] A tiles, [STAGES] A_lo tiles (SPLIT), [STAGES] B tiles
+  // ring: [STAGES] A tiles, [STAGES] A_lo tiles (SPLIT), [STAGES] B tiles;
+  // SMALL: per stage [A | A_lo | B]
   const uint32_t sA = base, sAlo = base + STAGES * A_BYTES, sB = base + STAGES * A_BYTES * C::A_TERMS;
+  auto a_at = [&](int s) { return SMALL ? base + s * STAGE_BYTES : sA + s * A_BYTES; };
+  auto alo_at = [&](int s) { return SMALL ? base + s * STAGE_BYTES + C::A_TILE : sAlo + s * A_BYTES; };
+  auto b_at = [&](int s) { return SMALL ? base + s * STAGE_BYTES + C::A_TERMS * C::A_TILE : sB + s * B_BYTES; };
   const uint32_t bars = base + STAGES * STAGE_BYTES;
   const uint32_t tmem_slot = bars + 8 * (2 * STAGES + 4);
   float* const epi_tile = reinterpret_cast<float*>(smem_raw + (bars + C::BAR_BYTES - raw));  // epi_smem<KIND>()
@@ -145,9 +160,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             break;
           }
           mbar_arrive_expect_tx(full_bar(s), STAGE_BYTES);
-          tma_load_2d(sA + s * A_BYTES, &tmA, full_bar(s), kb * BK, mb * BM);
-          if (SPLIT) tma_load_2d(sAlo + s * A_BYTES, &tmAlo, full_bar(s), kb * BK, mb * BM);
-          tma_load_2d(sB + s * B_BYTES, &tmB, full_bar(s), kb * BK, wrow);
+          tma_load_2d(a_at(s), &tmA, full_bar(s), kb * BK, mb * BM);
+          if (SPLIT) tma_load_2d(alo_at(s), &tmAlo, full_bar(s), kb * BK, mb * BM);
+          tma_load_2d(b_at(s), &tmB, full_bar(s), kb * BK, wrow);
         }
       }
     }
@@ -173,13 +188,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc_sw128(sA + s * A_BYTES);
-          const uint64_t bd = smem_desc_sw128(sB + s * B_BYTES);
+          const uint64_t ad = smem_desc_sw128(a_at(s));
+          const uint64_t bd = smem_desc_sw128(b_at(s));
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K inside the swizzle atom
             tc_mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
           if (SPLIT) {
-            const uint64_t ald = smem_desc_sw128(sAlo + s * A_BYTES);
+            const uint64_t ald = smem_desc_sw128(alo_at(s));
 #pragma unroll
             for (int k = 0; k < BK / 16; ++k) tc_mma_f16(d, ald + 2 * k, bd + 2 * k, idesc, 1u);
           }
@@ -433,7 +448,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int KIND, typename T16, bool SPLIT, int BN>
+template <int KIND, typename T16, bool SPLIT, int BN, bool SMALL>
 cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
                         const GemmSplitK& sk, const GemmGroup& grp) {
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN) * sk.ks;
@@ -442,7 +457,7 @@ cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N,
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(NUM_THREADS);
-  cfg.dynamicSmemBytes = GCfg<SPLIT, BN>::SMEM + epi_smem<KIND>();
+  cfg.dynamicSmemBytes = GCfg<SPLIT, BN, SMALL>::SMEM + epi_smem<KIND>();
   cfg.stream = lc.stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -450,8 +465,10 @@ cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N,
   cfg.attrs = attr;
   cfg.numAttrs = lc.pdl ? 1 : 0;
   const GemmMaps& g = BN == 256 ? maps : *maps.n128;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN>, g.a, g.w, SPLIT ? g.a_lo : g.a, M, N, K, ep,
-                            sk.ks, sk.ws, sk.tickets, grp);
+  const CUtensorMap& ta = SMALL ? g.a16 : g.a;
+  const CUtensorMap& tlo = SPLIT ? (SMALL ? g.a_lo16 : g.a_lo) : ta;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN, SMALL>, ta, g.w, tlo, M, N, K, ep, sk.ks,
+                            sk.ws, sk.tickets, grp);
 }
 
 }  // namespace
@@ -482,15 +499,20 @@ bool make_tma_2d_plain(CUtensorMap* map, const void* base, uint64_t rows, uint64
 }
 
 namespace {
-template <int KIND, typename T16, bool SPLIT, int BN>
+template <int KIND, typename T16, bool SPLIT, int BN, bool SMALL>
 cudaError_t set_smem1() {
-  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              GCfg<SPLIT, BN>::SMEM + epi_smem<KIND>());
+  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT, BN, SMALL>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              GCfg<SPLIT, BN, SMALL>::SMEM + epi_smem<KIND>());
 }
 template <int KIND, typename T16, bool SPLIT>
 cudaError_t set_smem() {
-  cudaError_t e = set_smem1<KIND, T16, SPLIT, 256>();
-  if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128>();
+  cudaError_t e = set_smem1<KIND, T16, SPLIT, 256, false>();
+  if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128, false>();
+  if (KIND != EPI_ROWSCALE) {  // the small-M layout (decode kinds)
+    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 256, KIND != EPI_ROWSCALE>();
+    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128, KIND != EPI_ROWSCALE>();
+  }
   return e;
 }
 template <typename T16>
@@ -503,18 +525,27 @@ cudaError_t prepare_gemm_t() {
   if (e == cudaSuccess) e = set_smem<EPI_ROWSCALE, T16, false>();
   return e;
 }
-template <typename T16, int BN>
+template <typename T16, int BN, bool SMALL>
 cudaError_t launch_t(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
                      const GemmSplitK& sk, const GemmGroup& grp) {
   switch (kind) {
     case EPI_QKV:
-      return maps.split ? launch_kind<EPI_QKV, T16, true, BN>(lc, maps, M, N, K, ep, sk, grp)
-                        : launch_kind<EPI_QKV, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
-    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
-    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
-    case EPI_ROWSCALE: return launch_kind<EPI_ROWSCALE, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
-    default: return launch_kind<EPI_LOGITS, T16, false, BN>(lc, maps, M, N, K, ep, sk, grp);
+      return maps.split ? launch_kind<EPI_QKV, T16, true, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp)
+                        : launch_kind<EPI_QKV, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_ROWSCALE: return launch_kind<EPI_ROWSCALE, T16, false, BN, false>(lc, maps, M, N, K, ep, sk, grp);
+    default: return launch_kind<EPI_LOGITS, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
   }
+}
+template <int BN>
+cudaError_t launch_bn(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
+                      const GemmSplitK& sk, const GemmGroup& grp, bool small) {
+  if (small)
+    return lc.f16 ? launch_t<f16, BN, true>(lc, kind, maps, M, N, K, ep, sk, grp)
+                  : launch_t<bf16, BN, true>(lc, kind, maps, M, N, K, ep, sk, grp);
+  return lc.f16 ? launch_t<f16, BN, false>(lc, kind, maps, M, N, K, ep, sk, grp)
+                : launch_t<bf16, BN, false>(lc, kind, maps, M, N, K, ep, sk, grp);
 }
 }  // namespace
 
@@ -551,13 +582,13 @@ cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, 
       return cudaErrorInvalidValue;
     sk = *split;
   }
+  // at most 16 rows (one M block) and 16-row activation boxes: the small-M stage layout
+  const bool small = M <= 16 && maps.has16 && !grp.mb_expert && kind != EPI_ROWSCALE;
   if (tile_n == 128) {
     if (!maps.n128) return cudaErrorInvalidValue;
-    if (lc.f16) return launch_t<f16, 128>(lc, kind, maps, M, N, K, ep, sk, grp);
-    return launch_t<bf16, 128>(lc, kind, maps, M, N, K, ep, sk, grp);
+    return launch_bn<128>(lc, kind, maps, M, N, K, ep, sk, grp, small);
   }
-  if (lc.f16) return launch_t<f16, 256>(lc, kind, maps, M, N, K, ep, sk, grp);
-  return launch_t<bf16, 256>(lc, kind, maps, M, N, K, ep, sk, grp);
+  return launch_bn<256>(lc, kind, maps, M, N, K, ep, sk, grp, small);
 }
 
 int gemm_split_k(const LaunchCtx& lc, int M, int N, int K) {
