@@ -113,6 +113,7 @@ struct axon_model {
   int* err = nullptr;
   CUtensorMap t_a{}, t_o{}, t_alo{};
   CUtensorMap t_a16{}, t_o16{}, t_alo16{};  // the same in boxes of 16 rows (decode GEMMs)
+  CUtensorMap t_a64{}, t_o64{}, t_alo64{};  // and of 64 rows
   // decode graphs
   cudaStream_t cap_stream = nullptr;
   std::map<GraphKey, cudaGraphExec_t> graphs;
@@ -1444,12 +1445,19 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
            make_tma_2d_16(&m->t_usorted, m->moe_u_sorted, m->R_cap, m->Fe, 128, m->f16);
     if (ok && m->a_lo) ok = make_tma_2d_16(&m->t_alo, m->a_lo, Mcap, D, 128, m->f16);
     ok = ok && make_tma_2d_16(&m->t_a16, m->a, Mcap, D, 16, m->f16) &&
-         make_tma_2d_16(&m->t_o16, m->o, Mcap, Hd, 16, m->f16);
-    if (ok && m->a_lo) ok = make_tma_2d_16(&m->t_alo16, m->a_lo, Mcap, D, 16, m->f16);
-    auto small_a = [&](GemmMaps& g, const CUtensorMap& a16) {
+         make_tma_2d_16(&m->t_o16, m->o, Mcap, Hd, 16, m->f16) &&
+         make_tma_2d_16(&m->t_a64, m->a, Mcap, D, 64, m->f16) && make_tma_2d_16(&m->t_o64, m->o, Mcap, Hd, 64, m->f16);
+    if (ok && m->a_lo)
+      ok = make_tma_2d_16(&m->t_alo16, m->a_lo, Mcap, D, 16, m->f16) &&
+           make_tma_2d_16(&m->t_alo64, m->a_lo, Mcap, D, 64, m->f16);
+    auto small_a = [&](GemmMaps& g, const CUtensorMap& a16, const CUtensorMap& a64) {
       g.a16 = a16;
-      if (g.split) g.a_lo16 = m->t_alo16;
-      g.has16 = true;
+      g.a64 = a64;
+      if (g.split) {
+        g.a_lo16 = m->t_alo16;
+        g.a_lo64 = m->t_alo64;
+      }
+      g.has16 = g.has64 = true;
     };
     for (int l = 0; l < m->L && ok; ++l) {
       LayerW& w = m->layers[l];
@@ -1461,18 +1469,19 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
       }
       w.m_o.a = m->t_o;
       ok = ok && make_tma_2d_16(&w.m_o.w, w.wo, D, Hd, 256, m->f16);
-      small_a(w.m_qkv, m->t_a16);
-      small_a(w.m_o, m->t_o16);
+      small_a(w.m_qkv, m->t_a16, m->t_a64);
+      small_a(w.m_o, m->t_o16, m->t_o64);
       if (w.Fl) {
         w.m_gu.a = m->t_a;
         ok = ok && make_tma_2d_16(&w.m_gu.w, w.wgu, 2 * w.Fl, D, 256, m->f16);
         // the down projection reads u with this layer's row stride
         ok = ok && make_tma_2d_16(&w.m_d.a, m->u, Mcap, w.Fl, 128, m->f16);
         ok = ok && make_tma_2d_16(&w.m_d.w, w.wd, D, w.Fl, 256, m->f16);
-        small_a(w.m_gu, m->t_a16);
-        CUtensorMap u16;
-        ok = ok && make_tma_2d_16(&u16, m->u, Mcap, w.Fl, 16, m->f16);
-        small_a(w.m_d, u16);
+        small_a(w.m_gu, m->t_a16, m->t_a64);
+        CUtensorMap u16, u64;
+        ok = ok && make_tma_2d_16(&u16, m->u, Mcap, w.Fl, 16, m->f16) &&
+             make_tma_2d_16(&u64, m->u, Mcap, w.Fl, 64, m->f16);
+        small_a(w.m_d, u16, u64);
       }
       if (w.moe) {
         const int E = m->E, Fe = m->Fe;
@@ -1499,7 +1508,7 @@ int axon_model_create(const axon_config* cfg, const axon_tensor* weights, int32_
     }
     m->m_head.a = m->t_a;
     ok = ok && make_tma_2d_16(&m->m_head.w, m->head, V, D, 256, m->f16);
-    small_a(m->m_head, m->t_a16);
+    small_a(m->m_head, m->t_a16, m->t_a64);
     // decode projections: weight boxes of 128 rows, activation boxes of 8..64 token rows
     for (int l = 0; l < m->L && ok; ++l) {
       LayerW& w = m->layers[l];

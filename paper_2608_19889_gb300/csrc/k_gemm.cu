@@ -33,27 +33,35 @@ constexpr int NUM_THREADS = 192;
 // accumulator. The ring takes as many stages as fit in 200 KB, at most 6
 // (BN 256: 4, split 3; BN 128: 6, split 4).
 //
-// SMALL (at most 16 activation rows, decode): each stage holds [A (16 rows)
-// | A_lo (16 rows, SPLIT) | B]; the MMA still reads 128 A rows from the
-// 16-row tile, rows 16..127 falling in the same stage's following bytes
-// (landed, so stable; their accumulator rows are never stored). Without the
-// 112 padding rows a stage is 2-3x smaller, so more of them -- more weight
-// bytes in flight per SM -- fit (up to 12).
-template <bool SPLIT, int BN_, bool SMALL = false>
+// AROWS < 128 (at most AROWS activation rows, decode: 16 or 64): each stage
+// holds [A (AROWS rows) | A_lo (AROWS rows, SPLIT) | B]; the MMA still reads
+// 128 A rows from the tile, rows AROWS..127 falling in the same stage's
+// following bytes (landed, so stable; their accumulator rows are never
+// stored). Without the padding rows a stage is smaller, so more of them --
+// more weight bytes in flight per SM -- fit (up to 12).
+//
+// RING: the ring's byte budget. The residual kind at BN 256 keeps 8 KB of
+// static shared memory for its row sums, so its ring gets 196 KB.
+template <bool SPLIT, int BN_, int AROWS = 128, int RING = 200 * 1024>
 struct GCfg {
   static constexpr int BN = BN_;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
   static constexpr int A_TERMS = SPLIT ? 2 : 1;
-  static constexpr int A_TILE = SMALL ? 16 * BK * 2 : A_BYTES;  // bytes of one A term in a stage
+  static constexpr bool SMALL = AROWS < BM;
+  static constexpr int A_TILE = AROWS * BK * 2;  // bytes of one A term in a stage
   static constexpr int STAGE_BYTES = A_TERMS * A_TILE + B_BYTES;
   static constexpr int MAX_STAGES = SMALL ? 12 : 6;
-  static constexpr int STAGES =
-      (200 * 1024) / STAGE_BYTES > MAX_STAGES ? MAX_STAGES : (200 * 1024) / STAGE_BYTES;
+  static constexpr int STAGES = RING / STAGE_BYTES > MAX_STAGES ? MAX_STAGES : RING / STAGE_BYTES;
   static_assert(!SMALL || STAGE_BYTES - (A_TERMS - 1) * A_TILE >= A_BYTES, "the MMA's 128-row read stays in its stage");
   static constexpr int BAR_BYTES = 8 * (2 * STAGES + 4) + 16;
   static constexpr int SMEM = STAGES * STAGE_BYTES + BAR_BYTES + 1024;
 };
+
+template <int KIND, int BN>
+constexpr int ring_budget() { return KIND == EPI_RESID && BN == 256 ? 196 * 1024 : 200 * 1024; }
+template <int KIND, bool SPLIT, int BN, int AROWS>
+using GCfgK = GCfg<SPLIT, BN, AROWS, ring_budget<KIND, BN>()>;
 
 // Residual epilogue staging: each epilogue warp's 32 rows x 32 accumulator
 // columns, rows padded to 36 floats (float4 stores of 8 consecutive rows
@@ -72,12 +80,13 @@ AXON_DEV void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
   mb = first_m + (local - nb * gm);
 }
 
-template <int KIND, typename T16, bool SPLIT, int BN_, bool SMALL>
+template <int KIND, typename T16, bool SPLIT, int BN_, int AROWS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmAlo, int M, int N, int K, EpiArgs ep, int ks, float* ws,
                    int* tickets, GemmGroup grp) {
-  using C = GCfg<SPLIT, BN_, SMALL>;
+  using C = GCfgK<KIND, SPLIT, BN_, AROWS>;
+  constexpr bool SMALL = C::SMALL;
   constexpr int BN = C::BN;
   constexpr int B_BYTES = C::B_BYTES;
   constexpr uint32_t TMEM_COLS = C::TMEM_COLS;
@@ -87,7 +96,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   // ring: [STAGES] A tiles, [STAGES] A_lo tiles (SPLIT), [STAGES] B tiles;
-  // SMALL: per stage [A | A_lo | B]
+  // AROWS < 128: per stage [A | A_lo | B]
   const uint32_t sA = base, sAlo = base + STAGES * A_BYTES, sB = base + STAGES * A_BYTES * C::A_TERMS;
   auto a_at = [&](int s) { return SMALL ? base + s * STAGE_BYTES : sA + s * A_BYTES; };
   auto alo_at = [&](int s) { return SMALL ? base + s * STAGE_BYTES + C::A_TILE : sAlo + s * A_BYTES; };
@@ -448,7 +457,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int KIND, typename T16, bool SPLIT, int BN, bool SMALL>
+template <int KIND, typename T16, bool SPLIT, int BN, int AROWS>
 cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
                         const GemmSplitK& sk, const GemmGroup& grp) {
   const int tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN) * sk.ks;
@@ -457,7 +466,7 @@ cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N,
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(NUM_THREADS);
-  cfg.dynamicSmemBytes = GCfg<SPLIT, BN, SMALL>::SMEM + epi_smem<KIND>();
+  cfg.dynamicSmemBytes = GCfgK<KIND, SPLIT, BN, AROWS>::SMEM + epi_smem<KIND>();
   cfg.stream = lc.stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -465,9 +474,9 @@ cudaError_t launch_kind(const LaunchCtx& lc, const GemmMaps& maps, int M, int N,
   cfg.attrs = attr;
   cfg.numAttrs = lc.pdl ? 1 : 0;
   const GemmMaps& g = BN == 256 ? maps : *maps.n128;
-  const CUtensorMap& ta = SMALL ? g.a16 : g.a;
-  const CUtensorMap& tlo = SPLIT ? (SMALL ? g.a_lo16 : g.a_lo) : ta;
-  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN, SMALL>, ta, g.w, tlo, M, N, K, ep, sk.ks,
+  const CUtensorMap& ta = AROWS == 16 ? g.a16 : (AROWS == 64 ? g.a64 : g.a);
+  const CUtensorMap& tlo = SPLIT ? (AROWS == 16 ? g.a_lo16 : (AROWS == 64 ? g.a_lo64 : g.a_lo)) : ta;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, T16, SPLIT, BN, AROWS>, ta, g.w, tlo, M, N, K, ep, sk.ks,
                             sk.ws, sk.tickets, grp);
 }
 
@@ -499,19 +508,21 @@ bool make_tma_2d_plain(CUtensorMap* map, const void* base, uint64_t rows, uint64
 }
 
 namespace {
-template <int KIND, typename T16, bool SPLIT, int BN, bool SMALL>
+template <int KIND, typename T16, bool SPLIT, int BN, int AROWS>
 cudaError_t set_smem1() {
-  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT, BN, SMALL>,
+  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, T16, SPLIT, BN, AROWS>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              GCfg<SPLIT, BN, SMALL>::SMEM + epi_smem<KIND>());
+                              GCfgK<KIND, SPLIT, BN, AROWS>::SMEM + epi_smem<KIND>());
 }
 template <int KIND, typename T16, bool SPLIT>
 cudaError_t set_smem() {
-  cudaError_t e = set_smem1<KIND, T16, SPLIT, 256, false>();
-  if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128, false>();
-  if (KIND != EPI_ROWSCALE) {  // the small-M layout (decode kinds)
-    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 256, KIND != EPI_ROWSCALE>();
-    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128, KIND != EPI_ROWSCALE>();
+  cudaError_t e = set_smem1<KIND, T16, SPLIT, 256, 128>();
+  if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128, 128>();
+  if constexpr (KIND != EPI_ROWSCALE) {  // the small-M layouts (decode kinds)
+    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 256, 16>();
+    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128, 16>();
+    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 256, 64>();
+    if (e == cudaSuccess) e = set_smem1<KIND, T16, SPLIT, 128, 64>();
   }
   return e;
 }
@@ -525,27 +536,31 @@ cudaError_t prepare_gemm_t() {
   if (e == cudaSuccess) e = set_smem<EPI_ROWSCALE, T16, false>();
   return e;
 }
-template <typename T16, int BN, bool SMALL>
+template <typename T16, int BN, int AROWS>
 cudaError_t launch_t(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
                      const GemmSplitK& sk, const GemmGroup& grp) {
   switch (kind) {
     case EPI_QKV:
-      return maps.split ? launch_kind<EPI_QKV, T16, true, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp)
-                        : launch_kind<EPI_QKV, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
-    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
-    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
-    case EPI_ROWSCALE: return launch_kind<EPI_ROWSCALE, T16, false, BN, false>(lc, maps, M, N, K, ep, sk, grp);
-    default: return launch_kind<EPI_LOGITS, T16, false, BN, SMALL>(lc, maps, M, N, K, ep, sk, grp);
+      return maps.split ? launch_kind<EPI_QKV, T16, true, BN, AROWS>(lc, maps, M, N, K, ep, sk, grp)
+                        : launch_kind<EPI_QKV, T16, false, BN, AROWS>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_RESID: return launch_kind<EPI_RESID, T16, false, BN, AROWS>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, T16, false, BN, AROWS>(lc, maps, M, N, K, ep, sk, grp);
+    case EPI_ROWSCALE: return launch_kind<EPI_ROWSCALE, T16, false, BN, 128>(lc, maps, M, N, K, ep, sk, grp);
+    default: return launch_kind<EPI_LOGITS, T16, false, BN, AROWS>(lc, maps, M, N, K, ep, sk, grp);
   }
+}
+template <int BN, int AROWS>
+cudaError_t launch_ar(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
+                      const GemmSplitK& sk, const GemmGroup& grp) {
+  return lc.f16 ? launch_t<f16, BN, AROWS>(lc, kind, maps, M, N, K, ep, sk, grp)
+                : launch_t<bf16, BN, AROWS>(lc, kind, maps, M, N, K, ep, sk, grp);
 }
 template <int BN>
 cudaError_t launch_bn(const LaunchCtx& lc, int kind, const GemmMaps& maps, int M, int N, int K, const EpiArgs& ep,
-                      const GemmSplitK& sk, const GemmGroup& grp, bool small) {
-  if (small)
-    return lc.f16 ? launch_t<f16, BN, true>(lc, kind, maps, M, N, K, ep, sk, grp)
-                  : launch_t<bf16, BN, true>(lc, kind, maps, M, N, K, ep, sk, grp);
-  return lc.f16 ? launch_t<f16, BN, false>(lc, kind, maps, M, N, K, ep, sk, grp)
-                : launch_t<bf16, BN, false>(lc, kind, maps, M, N, K, ep, sk, grp);
+                      const GemmSplitK& sk, const GemmGroup& grp, int arows) {
+  if (arows == 16) return launch_ar<BN, 16>(lc, kind, maps, M, N, K, ep, sk, grp);
+  if (arows == 64) return launch_ar<BN, 64>(lc, kind, maps, M, N, K, ep, sk, grp);
+  return launch_ar<BN, 128>(lc, kind, maps, M, N, K, ep, sk, grp);
 }
 }  // namespace
 
@@ -582,13 +597,15 @@ cudaError_t launch_gemm_tc(const LaunchCtx& lc, int kind, const GemmMaps& maps, 
       return cudaErrorInvalidValue;
     sk = *split;
   }
-  // at most 16 rows (one M block) and 16-row activation boxes: the small-M stage layout
-  const bool small = M <= 16 && maps.has16 && !grp.mb_expert && kind != EPI_ROWSCALE;
+  // at most 16 (64) rows -- one M block -- and activation boxes of 16 (64)
+  // rows: the small-M stage layouts
+  const bool dec = !grp.mb_expert && kind != EPI_ROWSCALE;
+  const int arows = (dec && M <= 16 && maps.has16) ? 16 : ((dec && M <= 64 && maps.has64) ? 64 : 128);
   if (tile_n == 128) {
     if (!maps.n128) return cudaErrorInvalidValue;
-    return launch_bn<128>(lc, kind, maps, M, N, K, ep, sk, grp, small);
+    return launch_bn<128>(lc, kind, maps, M, N, K, ep, sk, grp, arows);
   }
-  return launch_bn<256>(lc, kind, maps, M, N, K, ep, sk, grp, small);
+  return launch_bn<256>(lc, kind, maps, M, N, K, ep, sk, grp, arows);
 }
 
 int gemm_split_k(const LaunchCtx& lc, int M, int N, int K) {

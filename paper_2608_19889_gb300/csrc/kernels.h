@@ -162,11 +162,14 @@ struct GemmMaps {
   CUtensorMap a;     // activations [rows][K], box 64 x 128
   CUtensorMap w;     // weights [N][K], box 64 x 256 (64 x 128 in the n128 set)
   CUtensorMap a_lo;  // second term of a split activation operand (used when split)
-  // the same activation operand (and second term) in boxes of 16 rows: at
-  // most 16 rows (decode), the ring stages hold only the rows that exist
+  // the same activation operand (and second term) in boxes of 16 and of 64
+  // rows: at most 16 (64) rows (decode), the ring stages hold only those
   CUtensorMap a16;
   CUtensorMap a_lo16;
+  CUtensorMap a64;
+  CUtensorMap a_lo64;
   bool has16 = false;
+  bool has64 = false;
   bool split = false;
   const GemmMaps* n128 = nullptr;  // the same operands with 128-row weight boxes (128-wide tiles), or null
 };
