@@ -6,11 +6,13 @@ CUDA library.
 
     mod = parse_module(text)                  # syntax.py
     g = build_graph(mod, config)              # graph.py: inlining, paths, loops
-    low = lower_decoder(g)                    # lower.py: shape + checkpoint names
+    stack_experts(g)                          # rewrite.py: loops over experts -> stacked experts
+    low = lower_decoder(g)                    # lower.py: shape + checkpoint names (runs the rewrite too)
     model = create_model(low, checkpoint, max_batch=..., max_context=...)
 """
 from .graph import AxonGraphError, Graph, Node, Ref, build_graph, dump
 from .lower import LoweredDecoder, LoweringError, lower_decoder
+from .rewrite import stack_experts
 from .syntax import AxonSyntaxError, parse_module
 
 
@@ -30,4 +32,5 @@ def create_model(lowered: LoweredDecoder, checkpoint: dict, max_batch: int, max_
 
 
 __all__ = ["AxonGraphError", "AxonSyntaxError", "Graph", "LoweredDecoder", "LoweringError", "Node", "Ref",
-           "build_graph", "compile_decoder", "create_model", "dump", "lower_decoder", "parse_module"]
+           "build_graph", "compile_decoder", "create_model", "dump", "lower_decoder", "parse_module",
+           "stack_experts"]

@@ -13,7 +13,18 @@ paper's language section and causal-LM listing:
 
 inside one ``for`` loop over the layers that carries the hidden state (and
 the cache), after an embedding and before a final rmsnorm and LM head
-(tied when the head reads the embedding's path). The matcher walks the
+(tied when the head reads the embedding's path).
+
+Mixture-of-experts layers replace m by
+
+    w, idx = softmax_topk_router(h2);  m = stacked_experts(h2, w, idx) [+ shared(h2)]
+
+where the stacked-experts node is what the Phase 2(b) rewrite (rewrite.py)
+makes of a loop over the experts, and ``shared`` is a gated MLP (the shared
+experts, one MLP whose width is a multiple of an expert's). Such a model is
+either one loop of MoE layers or a loop of leading dense layers followed by
+a loop of MoE layers that continues the first one's index range and carries
+its values (DeepSeek-MoE: the first layer dense). The matcher walks the
 loop body backwards from its hidden-state output and claims every node it
 recognises; any node left unclaimed, and any operation outside the
 supported set, is a LoweringError naming it -- there is no fallback.
@@ -29,6 +40,7 @@ from dataclasses import dataclass, field
 from typing import Dict, List, Optional
 
 from . import graph as gr
+from .rewrite import ACTIVATIONS as _ACTS, stack_experts
 
 # Operations allowed outside the layer loop and around the cache: they
 # carry positions, masks and cache bookkeeping, which the library keeps on
@@ -39,8 +51,8 @@ _PLUMBING = {
     "Positions.position_ids", "Masking.causal_mask_for_input", "Masking.mask_for_input",
     "Masking.mask_length_for_input", "input",
 }
-_ACTS = {"Act.silu": "silu", "Activations.silu": "silu", "Act.gelu_tanh": "gelu_tanh",
-         "Activations.gelu_new": "gelu_tanh", "Act.gelu_new": "gelu_tanh", "Activations.gelu_tanh": "gelu_tanh"}
+# limits of the mixture-of-experts kernels (the config's documented range)
+_MAX_EXPERTS, _MAX_TOPK = 256, 8
 
 
 class LoweringError(ValueError):
@@ -50,12 +62,15 @@ class LoweringError(ValueError):
 @dataclass
 class LoweredDecoder:
     """shape: the model shape for make_config (L, D, H, G, d, F, V, tie,
-    bias, theta, eps, window, act, qk_norm, rope scaling); names: library
-    checkpoint name -> module parameter path (per layer, already
-    instantiated)."""
+    bias, theta, eps, window, act, qk_norm, rope scaling; for MoE decoders
+    n_experts, top_k, moe_F, n_shared, first_dense, norm_topk); names:
+    library checkpoint name -> module parameter path (per layer and expert,
+    already instantiated)."""
     shape: dict
     names: Dict[str, str] = field(default_factory=dict)
-    paths: Dict[str, str] = field(default_factory=dict)  # role -> module path pattern ({i} per layer)
+    # role -> module path pattern ({var} per layer, {e} per expert); the roles
+    # of a second (mixture-of-experts) layer loop under "moe_layers."
+    paths: Dict[str, str] = field(default_factory=dict)
 
     def module_weights(self, library_named: dict) -> dict:
         """Re-key a library-named checkpoint under the module's own paths."""
@@ -105,54 +120,87 @@ def _bool(v):
     return bool(v) if v is not None else False
 
 
-def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
-    """Match the Graph IR of a causal-LM entry definition onto the fused
-    decoder kernels. `config`: the values the module read through Config
-    (for defaults of epsilon and rotary base); `g.config_reads` is used when
-    absent."""
-    cfg = dict(getattr(g, "config_reads", {}) or {})
-    cfg.update(config or {})
-    loops = [n for n in g.nodes if n.op == "loop"]
-    if len(loops) != 1:
-        raise LoweringError(f"expected one layer loop, found {len(loops)}")
-    loop = loops[0]
+@dataclass
+class _Layer:
+    """What the body of one layer loop lowered to."""
+    loop: gr.Node
+    params: dict  # H, G, d, bias, theta, act, qk_norm, rope scaling: equal across loops
+    eps: set
+    paths: dict  # role -> parameter path pattern with the loop's {var}
+    mlp: str  # "dense" or "moe"
+    F: int = 0  # dense MLP width
+    moe: dict = field(default_factory=dict)  # E, top_k, Fe, Fs, norm_topk
+
+
+def _gated_mlp(m: _Match, down_ref, what: str):
+    """down(act(gate(h)) * up(h)): (gate, up, down, activation, h)."""
+    down = m.node(down_ref, {"NN.linear"}, f"{what} output")
+    mul = m.node(down.inputs[0], {"mul"}, f"{what} product")
+    pa, pb = (m.byid.get(r.node) if isinstance(r, gr.Ref) else None for r in mul.inputs)
+    if pa is not None and pa.op in _ACTS:
+        act_n, up = m.node(mul.inputs[0]), m.node(mul.inputs[1], {"NN.linear"}, f"{what} up projection")
+    elif pb is not None and pb.op in _ACTS:
+        act_n, up = m.node(mul.inputs[1]), m.node(mul.inputs[0], {"NN.linear"}, f"{what} up projection")
+    else:
+        raise LoweringError(f"the {what} must multiply an activated gate projection with an up projection")
+    gate = m.node(act_n.inputs[0], {"NN.linear"}, f"{what} gate projection")
+    if gate.inputs[0] != up.inputs[0]:
+        raise LoweringError("gate and up projections must read the same normalised input")
+    return gate, up, down, _ACTS[act_n.op], gate.inputs[0]
+
+
+def _moe_mlp(m: _Match, mlp_ref):
+    """The MoE pattern at the MLP output, or None when the output is not a
+    stacked-experts sum: (stacked node, router node, shared MLP parts or
+    None, h)."""
+    n = m.byid.get(mlp_ref.node) if isinstance(mlp_ref, gr.Ref) else None
+    if n is None:
+        return None
+    stacked, shared_ref = None, None
+    if n.op == "MoE.stacked_experts":
+        stacked = n
+    elif n.op == "add":
+        for a, b in (tuple(n.inputs), tuple(n.inputs[::-1])):
+            s = m.byid.get(a.node) if isinstance(a, gr.Ref) else None
+            if s is not None and s.op == "MoE.stacked_experts":
+                stacked, shared_ref = s, b
+                break
+        if stacked is None:
+            return None
+        m.claimed.add(n.id)
+    else:
+        return None
+    m.claimed.add(stacked.id)
+    init, h, w, idx = stacked.inputs
+    init_n = m.byid.get(init.node) if isinstance(init, gr.Ref) else None
+    if init_n is not None and init_n.op == "Tensor.zeros_like":
+        m.claimed.add(init_n.id)
+    elif shared_ref is None:
+        shared_ref = init  # the experts' sum starts from the shared experts' output
+    else:
+        raise LoweringError("the experts' sum must start from zeros or from the shared experts' output")
+    if not (isinstance(w, gr.Ref) and isinstance(idx, gr.Ref) and w.node == idx.node
+            and (w.index, idx.index) == (0, 1)):
+        raise LoweringError("expert weights and indices must be the two outputs of one MoE.softmax_topk_router")
+    router = m.node(w, {"MoE.softmax_topk_router"}, "router")
+    if router.inputs[0] != h:
+        raise LoweringError("the router and the experts must read the same normalised input")
+    shared = None
+    if shared_ref is not None:
+        shared = _gated_mlp(m, shared_ref, "shared experts")
+        if shared[4] != h:
+            raise LoweringError("the shared experts must read the routed experts' input")
+    return stacked, router, shared, h
+
+
+def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
+    """Match one layer loop's body, backwards from its hidden-state output."""
     body = loop.body
-    L = loop.attrs["stop"] - loop.attrs["start"]
-    if loop.attrs["start"] != 0:
-        raise LoweringError("the layer loop must start at 0")
-
-    # ---- outside the loop: embedding -> loop -> final norm -> head
-    outer = {n.id: n for n in g.nodes}
-    emb = [n for n in g.nodes if n.op == "NN.embedding"]
-    if len(emb) != 1 or not emb[0].path:
-        raise LoweringError("expected one NN.embedding with a parameter path")
-    emb = emb[0]
-    if not loop.inputs or not isinstance(loop.inputs[0], gr.Ref) or loop.inputs[0].node != emb.id:
-        raise LoweringError("the layer loop must carry the embedding output as its first value")
-    heads_out = [n for n in g.nodes if n.op == "NN.linear"]
-    if len(heads_out) != 1:
-        raise LoweringError(f"expected one NN.linear (the LM head) outside the layer loop, found {len(heads_out)}")
-    head = heads_out[0]
-    fnorm = outer.get(head.inputs[0].node) if isinstance(head.inputs[0], gr.Ref) else None
-    if fnorm is None or fnorm.op != "NN.rmsnorm" or not fnorm.path:
-        raise LoweringError("the LM head must read an NN.rmsnorm of the final hidden state")
-    if not (isinstance(fnorm.inputs[0], gr.Ref) and fnorm.inputs[0].node == loop.id and fnorm.inputs[0].index == 0):
-        raise LoweringError("the final norm must read the layer loop's hidden state")
-    if not any(isinstance(o, gr.Ref) and o.node == head.id for o in g.outputs):
-        raise LoweringError("the entry definition must return the LM head's logits")
-    window = 0
-    for n in g.nodes:
-        if n.op in ("NN.embedding", "NN.linear", "NN.rmsnorm", "loop"):
-            continue
-        if n.op not in _PLUMBING:
-            raise LoweringError(f"operation {n.op} outside the layer loop has no GB300 kernel")
-        if n.op == "Masking.causal_mask_for_input":
-            window = int(n.attrs.get("window", 0) or 0)
-    tie = head.path == emb.path
-    if head.attrs.get("bias") or head.attrs.get("transpose"):
-        raise LoweringError("the LM head takes neither a bias nor a transposed matrix here")
-
-    # ---- the layer body, backwards from the hidden-state output
+    inner = [n for n in body.nodes if n.op == "loop"]
+    if inner:
+        raise LoweringError(f"a loop over {inner[0].attrs.get('scope') or inner[0].attrs.get('var')} inside the "
+                            "layer is not a router-weighted sum over experts (the stacked-experts rewrite does "
+                            "not apply), and the kernels run no other loop")
     m = _Match(body, g)
     x_in = body.inputs[0]
     out_x = body.outputs[0]
@@ -169,21 +217,16 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
         raise LoweringError("the attention residual must add the layer input (pre-norm block)")
     attn_out = add1.inputs[1] if add1.inputs[0] == x_in else add1.inputs[0]
 
-    # MLP: down(act(gate(h2)) * up(h2))
-    down = m.node(mlp_ref, {"NN.linear"}, "MLP output")
-    mul = m.node(down.inputs[0], {"mul"}, "MLP product")
-    pa, pb = (m.byid.get(r.node) if isinstance(r, gr.Ref) else None for r in mul.inputs)
-    if pa is not None and pa.op in _ACTS:
-        act_n, up = m.node(mul.inputs[0]), m.node(mul.inputs[1], {"NN.linear"}, "MLP up projection")
-    elif pb is not None and pb.op in _ACTS:
-        act_n, up = m.node(mul.inputs[1]), m.node(mul.inputs[0], {"NN.linear"}, "MLP up projection")
+    # MLP: down(act(gate(h2)) * up(h2)), or the mixture of experts
+    moe = _moe_mlp(m, mlp_ref)
+    if moe is None:
+        gate, up, down, act, h2 = _gated_mlp(m, mlp_ref, "MLP")
     else:
-        raise LoweringError("the MLP must multiply an activated gate projection with an up projection")
-    act = _ACTS[act_n.op]
-    gate = m.node(act_n.inputs[0], {"NN.linear"}, "MLP gate projection")
-    if gate.inputs[0] != up.inputs[0]:
-        raise LoweringError("gate and up projections must read the same normalised input")
-    norm2 = m.node(gate.inputs[0], {"NN.rmsnorm"}, "post-attention norm")
+        stacked, router, shared, h2 = moe
+        act = _ACTS.get(stacked.attrs.get("act"))
+        if shared is not None and shared[3] != act:
+            raise LoweringError("the shared and the routed experts must use one activation")
+    norm2 = m.node(h2, {"NN.rmsnorm"}, "post-attention norm")
     if norm2.inputs[0] != x1_ref:
         raise LoweringError("the post-attention norm must read x + attention")
 
@@ -243,61 +286,192 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
     biases = {_bool(n.attrs.get("bias")) for n in (q_lin, k_lin, v_lin)}
     if len(biases) != 1:
         raise LoweringError("q, k and v must all have biases or none")
-    for n in (o_proj, gate, up, down):
+    plain = [o_proj] + ([gate, up, down] if moe is None else [router] + (list(shared[:3]) if shared else []))
+    for n in plain:
         if _bool(n.attrs.get("bias")) or _bool(n.attrs.get("transpose")):
             raise LoweringError(f"{n.path}: the kernels take [out, in] matrices without bias here")
     for n in (q_lin, k_lin, v_lin):
         if _bool(n.attrs.get("transpose")):
             raise LoweringError(f"{n.path}: the kernels take [out, in] matrices here")
-    D = int(emb.attrs.get("dim", 0))
     qdim = int(q_lin.attrs.get("dim", 0))
     if not D or not qdim or not H or not G or qdim % H:
         raise LoweringError("hidden size, head counts and projection widths must be known")
     d = qdim // H
-    F = int(gate.attrs.get("dim", 0))
-    V = int(head.attrs.get("dim", 0)) or int(cfg.get("vocab_size", 0))
     if int(k_lin.attrs.get("dim", 0)) != G * d or int(v_lin.attrs.get("dim", 0)) != G * d:
         raise LoweringError("k and v widths must be kv_heads * head_dim")
-    if int(up.attrs.get("dim", 0)) != F or int(down.attrs.get("dim", 0)) != D or int(o_proj.attrs.get("dim", D)) != D:
+    if int(o_proj.attrs.get("dim", D)) != D:
         raise LoweringError("MLP and output projection widths disagree with the hidden size")
-    epss = {float(n.attrs.get("eps", cfg.get("rms_norm_eps", 1e-6))) for n in (norm1, norm2, fnorm)}
+    params = dict(H=H, G=G, d=d, bias=biases.pop(), theta=thetas.pop(), act=act, qk_norm=q_norm is not None,
+                  rope_scaling=tuple(sorted(rope_scaling.items())))
+    eps = {float(n.attrs.get("eps", cfg.get("rms_norm_eps", 1e-6))) for n in (norm1, norm2)}
+    paths = {"input_norm": norm1.path, "post_norm": norm2.path, "q": q_lin.path, "k": k_lin.path,
+             "v": v_lin.path, "o": o_proj.path}
+    if q_norm is not None:
+        paths.update(q_norm=q_norm.path, k_norm=k_norm.path)
+    layer = _Layer(loop, params, eps, paths, "dense" if moe is None else "moe")
+    if moe is None:
+        F = int(gate.attrs.get("dim", 0))
+        if int(up.attrs.get("dim", 0)) != F or int(down.attrs.get("dim", 0)) != D:
+            raise LoweringError("MLP and output projection widths disagree with the hidden size")
+        layer.F = F
+        paths.update(gate=gate.path, up=up.path, down=down.path)
+    else:
+        layer.moe = _moe_params(stacked, router, shared, D)
+        paths.update(router=router.path, expert_gate=stacked.attrs["gate"], expert_up=stacked.attrs["up"],
+                     expert_down=stacked.attrs["down"])
+        if shared is not None:
+            paths.update(shared_gate=shared[0].path, shared_up=shared[1].path, shared_down=shared[2].path)
+    var = "{" + loop.attrs["var"] + "}"
+    for role, p in paths.items():
+        if not p:
+            raise LoweringError(f"{role}: parameterised operation without a path")
+        if var not in p:
+            raise LoweringError(f"{role}: the layer's parameter path {p!r} does not vary with the layer")
+    return layer
+
+
+def _moe_params(stacked: gr.Node, router: gr.Node, shared, D: int) -> dict:
+    """Sizes of a matched MoE MLP, within the kernels' limits."""
+    a = stacked.attrs
+    if a.get("bias"):
+        raise LoweringError("expert projections: the kernels take [out, in] matrices without bias here")
+    E, Fe = int(a.get("experts", 0)), int(a.get("dim") or 0)
+    if not 1 <= E <= _MAX_EXPERTS:
+        raise LoweringError(f"{E} experts: the kernels take 1 to {_MAX_EXPERTS}")
+    if Fe <= 0 or int(a.get("up_dim") or 0) != Fe or int(a.get("down_dim") or 0) != D:
+        raise LoweringError("expert widths must be known and the down projection must return the hidden size")
+    if "{" + str(a.get("var")) + "}" not in str(a.get("gate")):
+        raise LoweringError("expert parameters must vary with the expert")
+    top_k = router.attrs.get("top_k")
+    if not isinstance(top_k, int) or not 1 <= top_k <= min(_MAX_TOPK, E):
+        raise LoweringError(f"router top_k {top_k!r}: the kernels take 1 to min({_MAX_TOPK}, experts)")
+    if router.attrs.get("dim") not in (None, E):
+        raise LoweringError("the router's width must be the number of experts")
+    Fs = 0
+    if shared is not None:
+        Fs = int(shared[0].attrs.get("dim", 0))
+        if int(shared[1].attrs.get("dim", 0)) != Fs or int(shared[2].attrs.get("dim", 0)) != D:
+            raise LoweringError("shared experts' widths disagree with each other or with the hidden size")
+        if Fs <= 0 or Fs % Fe:
+            raise LoweringError("the shared experts' width must be a multiple of one expert's width")
+    return dict(E=E, top_k=top_k, Fe=Fe, Fs=Fs, norm_topk=_bool(router.attrs.get("normalize")),
+                evar="{" + str(a["var"]) + "}")
+
+
+def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
+    """Match the Graph IR of a causal-LM entry definition onto the fused
+    decoder kernels, after the stacked-experts rewrite. `config`: the values
+    the module read through Config (for defaults of epsilon and rotary
+    base); `g.config_reads` is used when absent."""
+    cfg = dict(getattr(g, "config_reads", {}) or {})
+    cfg.update(config or {})
+    stack_experts(g)
+    loops = [n for n in g.nodes if n.op == "loop"]
+    if not 1 <= len(loops) <= 2:
+        raise LoweringError(f"expected one layer loop (or a dense one, then a mixture-of-experts one), "
+                            f"found {len(loops)}")
+    if loops[0].attrs["start"] != 0:
+        raise LoweringError("the layer loop must start at 0")
+    if len(loops) == 2:
+        a, b = loops
+        if b.attrs["start"] != a.attrs["stop"]:
+            raise LoweringError("the second layer loop must continue the first one's index range")
+        if len(b.inputs) != a.n_out or any(not (isinstance(r, gr.Ref) and r.node == a.id and r.index == i)
+                                           for i, r in enumerate(b.inputs)):
+            raise LoweringError("the second layer loop must carry the values the first one yields")
+    last = loops[-1]
+    L = last.attrs["stop"]
+
+    # ---- outside the loops: embedding -> loop(s) -> final norm -> head
+    outer = {n.id: n for n in g.nodes}
+    emb = [n for n in g.nodes if n.op == "NN.embedding"]
+    if len(emb) != 1 or not emb[0].path:
+        raise LoweringError("expected one NN.embedding with a parameter path")
+    emb = emb[0]
+    first = loops[0]
+    if not first.inputs or not isinstance(first.inputs[0], gr.Ref) or first.inputs[0].node != emb.id:
+        raise LoweringError("the layer loop must carry the embedding output as its first value")
+    heads_out = [n for n in g.nodes if n.op == "NN.linear"]
+    if len(heads_out) != 1:
+        raise LoweringError(f"expected one NN.linear (the LM head) outside the layer loop, found {len(heads_out)}")
+    head = heads_out[0]
+    fnorm = outer.get(head.inputs[0].node) if isinstance(head.inputs[0], gr.Ref) else None
+    if fnorm is None or fnorm.op != "NN.rmsnorm" or not fnorm.path:
+        raise LoweringError("the LM head must read an NN.rmsnorm of the final hidden state")
+    if not (isinstance(fnorm.inputs[0], gr.Ref) and fnorm.inputs[0].node == last.id and fnorm.inputs[0].index == 0):
+        raise LoweringError("the final norm must read the layer loop's hidden state")
+    if not any(isinstance(o, gr.Ref) and o.node == head.id for o in g.outputs):
+        raise LoweringError("the entry definition must return the LM head's logits")
+    window = 0
+    for n in g.nodes:
+        if n.op in ("NN.embedding", "NN.linear", "NN.rmsnorm", "loop"):
+            continue
+        if n.op not in _PLUMBING:
+            raise LoweringError(f"operation {n.op} outside the layer loop has no GB300 kernel")
+        if n.op == "Masking.causal_mask_for_input":
+            window = int(n.attrs.get("window", 0) or 0)
+    tie = head.path == emb.path
+    if head.attrs.get("bias") or head.attrs.get("transpose"):
+        raise LoweringError("the LM head takes neither a bias nor a transposed matrix here")
+
+    # ---- the layer bodies
+    D = int(emb.attrs.get("dim", 0))
+    layers = [_match_layer(lp, g, cfg, D) for lp in loops]
+    if len(layers) == 2 and [ly.mlp for ly in layers] != ["dense", "moe"]:
+        raise LoweringError("two layer loops must be the leading dense layers, then the mixture-of-experts ones")
+    p0 = layers[0].params
+    for ly in layers[1:]:
+        for key, v in ly.params.items():
+            if p0[key] != v:
+                raise LoweringError(f"the dense and the mixture-of-experts layers disagree on {key}")
+    epss = set().union(*(ly.eps for ly in layers))
+    epss.add(float(fnorm.attrs.get("eps", cfg.get("rms_norm_eps", 1e-6))))
     if len(epss) != 1:
         raise LoweringError("every RMSNorm must use one epsilon")
-    shape = dict(L=L, D=D, H=H, G=G, d=d, F=F, V=V, tie=tie, bias=biases.pop(), theta=thetas.pop(),
-                 eps=epss.pop(), window=window, act=act, qk_norm=q_norm is not None)
+    V = int(head.attrs.get("dim", 0)) or int(cfg.get("vocab_size", 0))
+    moe = layers[-1].moe if layers[-1].mlp == "moe" else None
+    F = layers[0].F if layers[0].mlp == "dense" else (moe["Fs"] or moe["Fe"])
+    shape = dict(L=L, D=D, H=p0["H"], G=p0["G"], d=p0["d"], F=F, V=V, tie=tie, bias=p0["bias"],
+                 theta=p0["theta"], eps=epss.pop(), window=window, act=p0["act"], qk_norm=p0["qk_norm"])
+    rope_scaling = dict(p0["rope_scaling"])
     if rope_scaling:
         shape.update(rope_factor=float(rope_scaling.get("factor", 0.0)),
                      rope_low=float(rope_scaling.get("low_freq_factor", 1.0)),
                      rope_high=float(rope_scaling.get("high_freq_factor", 4.0)),
                      rope_orig=int(rope_scaling.get("original_max_position", 8192)))
+    if moe is not None:
+        shape.update(n_experts=moe["E"], top_k=moe["top_k"], moe_F=moe["Fe"], n_shared=moe["Fs"] // moe["Fe"],
+                     first_dense=first.attrs["stop"] if len(layers) == 2 else 0, norm_topk=moe["norm_topk"])
 
-    paths = {"embed": emb.path, "final_norm": fnorm.path, "head": head.path, "input_norm": norm1.path,
-             "post_norm": norm2.path, "q": q_lin.path, "k": k_lin.path, "v": v_lin.path, "o": o_proj.path,
-             "gate": gate.path, "up": up.path, "down": down.path}
-    if q_norm is not None:
-        paths.update(q_norm=q_norm.path, k_norm=k_norm.path)
-    for role, p in paths.items():
-        if not p:
-            raise LoweringError(f"{role}: parameterised operation without a path")
-    var = "{" + loop.attrs["var"] + "}"
+    # ---- library checkpoint name -> module parameter path
     names = {"model.embed_tokens.weight": emb.path + ".weight", "model.norm.weight": fnorm.path + ".weight"}
     if not tie:
         names["lm_head.weight"] = head.path + ".weight"
-    per_layer = [("input_layernorm.weight", "input_norm", "weight"),
-                 ("post_attention_layernorm.weight", "post_norm", "weight"),
-                 ("self_attn.q_proj.weight", "q", "weight"), ("self_attn.k_proj.weight", "k", "weight"),
-                 ("self_attn.v_proj.weight", "v", "weight"), ("self_attn.o_proj.weight", "o", "weight"),
-                 ("mlp.gate_proj.weight", "gate", "weight"), ("mlp.up_proj.weight", "up", "weight"),
-                 ("mlp.down_proj.weight", "down", "weight")]
+    attn = [("input_layernorm.weight", "input_norm"), ("post_attention_layernorm.weight", "post_norm"),
+            ("self_attn.q_proj.weight", "q"), ("self_attn.k_proj.weight", "k"),
+            ("self_attn.v_proj.weight", "v"), ("self_attn.o_proj.weight", "o")]
     if shape["bias"]:
-        per_layer += [("self_attn.q_proj.bias", "q", "bias"), ("self_attn.k_proj.bias", "k", "bias"),
-                      ("self_attn.v_proj.bias", "v", "bias")]
+        attn += [("self_attn.q_proj.bias", "q"), ("self_attn.k_proj.bias", "k"), ("self_attn.v_proj.bias", "v")]
     if shape["qk_norm"]:
-        per_layer += [("self_attn.q_norm.weight", "q_norm", "weight"), ("self_attn.k_norm.weight", "k_norm", "weight")]
-    for role in ("input_norm", "post_norm", "q", "k", "v", "o", "gate", "up", "down"):
-        if var not in paths[role]:
-            raise LoweringError(f"{role}: the layer's parameter path {paths[role]!r} does not vary with the layer")
-    for l in range(L):
-        for lib, role, leaf in per_layer:
-            names[f"model.layers.{l}.{lib}"] = paths[role].replace(var, str(l)) + "." + leaf
+        attn += [("self_attn.q_norm.weight", "q_norm"), ("self_attn.k_norm.weight", "k_norm")]
+    dense = [("mlp.gate_proj.weight", "gate"), ("mlp.up_proj.weight", "up"), ("mlp.down_proj.weight", "down")]
+    shared = [("mlp.shared_experts.gate_proj.weight", "shared_gate"), ("mlp.shared_experts.up_proj.weight", "shared_up"),
+              ("mlp.shared_experts.down_proj.weight", "shared_down")]
+    expert = [("gate_proj.weight", "expert_gate"), ("up_proj.weight", "expert_up"), ("down_proj.weight", "expert_down")]
+    paths = {"embed": emb.path, "final_norm": fnorm.path, "head": head.path}
+    for k, ly in enumerate(layers):
+        var = "{" + ly.loop.attrs["var"] + "}"
+        per_layer = attn + (dense if ly.mlp == "dense" else [("mlp.gate.weight", "router")] +
+                            (shared if ly.moe["Fs"] else []))
+        paths.update({(role if k == 0 else f"moe_layers.{role}"): p for role, p in ly.paths.items()})
+        for l in range(ly.loop.attrs["start"], ly.loop.attrs["stop"]):
+            for lib, role in per_layer:
+                leaf = lib.rsplit(".", 1)[1]
+                names[f"model.layers.{l}.{lib}"] = ly.paths[role].replace(var, str(l)) + "." + leaf
+            if ly.mlp == "moe":
+                evar = ly.moe["evar"]
+                for e in range(ly.moe["E"]):
+                    for lib, role in expert:
+                        names[f"model.layers.{l}.mlp.experts.{e}.{lib}"] = (
+                            ly.paths[role].replace(var, str(l)).replace(evar, str(e)) + ".weight")
     return LoweredDecoder(shape, names, paths)

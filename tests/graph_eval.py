@@ -1,0 +1,188 @@
+"""Direct evaluation of a front-end Graph IR on the CPU (float64 numpy).
+
+Test infrastructure for the Axon-subset front end: it runs a module's Graph
+IR node by node on its own parameter paths, so a test can check that what a
+module states (before or after the stacked-experts rewrite) is the function
+the lowered model computes -- the oracle run on the checkpoint re-keyed
+through the lowering's name map. It covers a prompt pass from an empty
+cache (the cache operations pass the new keys and values through) and the
+operations the decoder modules use; each follows the library operation's
+meaning in the paper's built-ins (Sec. Built-In Libraries):
+
+  NN.embedding / NN.rmsnorm / NN.linear   rows of E; x / sqrt(mean x^2 + eps) * g;
+                                          x W^T (+ b), W stored [out, in]
+  Attention.reshape_heads / merge_heads   [.., n*d] <-> [.., n, d]
+  Positions.position_ids / rope           past + i; rotate-half pairs (j, j + d/2),
+                                          angle p * theta^(-2j/d)
+  Attention.attention                     softmax(q k^T / sqrt(d)) v over keys at
+                                          positions <= the query's (and > p - window),
+                                          query head h on kv head floor(h / (H/G))
+  Act.silu / Act.gelu_tanh                z / (1 + e^-z); tanh form of gelu
+  MoE.softmax_topk_router                 p = softmax(x Wr^T); the top_k experts by p
+                                          (lower index first on ties) and their p,
+                                          divided by their sum with normalize=true
+  MoE.expert_weight w idx e               the weight expert e received (0 if none)
+  MoE.stacked_experts                     init + sum_e expert_weight(e) * ffn_e(h)
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+from paper_2608_19889_gb300.frontend import graph as gr
+
+
+class GraphEval:
+    """weights: module parameter path + ".weight" / ".bias" -> array."""
+
+    def __init__(self, weights: dict):
+        self.W = {k: np.asarray(v, dtype=np.float64) for k, v in weights.items()}
+
+    def run(self, g: gr.Graph, ids) -> list:
+        ids = np.asarray(ids, dtype=np.int64)
+        env: dict = {}
+        return self._graph(g, [ids, None], env, {})
+
+    # ------------------------------------------------------------ plumbing
+    def _graph(self, g, args, env, loopvars):
+        for n in g.nodes:
+            if n.op == "input":
+                idx = n.attrs["index"]
+                env[n.id] = (args[idx] if idx < len(args) else None,)
+            else:
+                out = self._node(n, env, loopvars)
+                env[n.id] = out if n.n_out > 1 else (out,)
+        return [self._val(o, env, loopvars) for o in g.outputs]
+
+    def _val(self, x, env, loopvars):
+        if isinstance(x, gr.Ref):
+            return env[x.node][x.index]
+        if isinstance(x, gr.LoopVar):
+            return loopvars[x.name]
+        return x
+
+    @staticmethod
+    def _path(p, loopvars):
+        for k, v in loopvars.items():
+            p = p.replace("{" + k + "}", str(v))
+        return p
+
+    def _w(self, path, loopvars, leaf="weight"):
+        return self.W[self._path(path, loopvars) + "." + leaf]
+
+    # ---------------------------------------------------------- operations
+    def _node(self, n, env, lv):
+        ins = [self._val(x, env, lv) for x in n.inputs]
+        at = {k: self._val(v, env, lv) for k, v in n.attrs.items()}
+        op = n.op
+        if op == "loop":
+            vals = ins
+            for i in range(at["start"], at["stop"]):
+                inner = dict(lv)
+                inner[at["var"]] = i
+                vals = self._graph(n.body, vals, env, inner)
+            return tuple(vals) if n.n_out > 1 else vals[0]
+        if op in ("add", "sub", "mul", "div"):
+            a, b = ins
+            return {"add": np.add, "sub": np.subtract, "mul": np.multiply, "div": np.divide}[op](a, b)
+        if op == "NN.embedding":
+            return self._w(n.path, lv)[ins[0]]
+        if op == "NN.rmsnorm":
+            x = ins[0]
+            return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + float(at["eps"])) * self._w(n.path, lv)
+        if op == "NN.linear":
+            y = ins[0] @ self._w(n.path, lv).T
+            return y + self._w(n.path, lv, "bias") if at.get("bias") else y
+        if op == "Attention.reshape_heads":
+            x = ins[0]
+            return x.reshape(x.shape[:-1] + (int(at["heads"]), -1))
+        if op == "Attention.merge_heads":
+            x = ins[0]
+            return x.reshape(x.shape[:-2] + (-1,))
+        if op == "Cache.past_length":
+            return 0
+        if op == "Positions.position_ids":
+            ids = ins[0]
+            return np.broadcast_to(np.arange(ids.shape[-1]) + int(at.get("past_length") or 0), ids.shape)
+        if op == "Masking.causal_mask_for_input":
+            return {"window": int(at.get("window", 0) or 0)}
+        if op in ("Cache.prepare", "Cache.index", "Cache.append"):
+            return None
+        if op == "Cache.update":
+            return ins[1], ins[2], None
+        if op == "Positions.rope":
+            return self._rope(ins[0], ins[1], float(at["theta"]), at)
+        if op == "Attention.attention":
+            return self._attention(ins[0], ins[1], ins[2], ins[3] or {})
+        if op == "Act.silu":
+            z = ins[0]
+            return z / (1.0 + np.exp(-z))
+        if op in ("Act.gelu_tanh", "Act.gelu_new", "Activations.gelu_new"):
+            z = ins[0]
+            return 0.5 * z * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (z + 0.044715 * z ** 3)))
+        if op == "Tensor.zeros_like":
+            return np.zeros_like(ins[0])
+        if op == "MoE.softmax_topk_router":
+            return self._route(ins[0], self._w(n.path, lv), int(at["top_k"]), bool(at.get("normalize", False)))
+        if op == "MoE.expert_weight":
+            w, idx, e = ins
+            return np.sum(np.where(idx == e, w, 0.0), axis=-1, keepdims=True)
+        if op == "MoE.stacked_experts":
+            return self._stacked(ins, at, lv)
+        raise NotImplementedError(op)
+
+    @staticmethod
+    def _rope(x, pos, theta, at):
+        if any(k in at for k in ("factor", "low_freq_factor", "high_freq_factor")):
+            raise NotImplementedError("rope frequency scaling")
+        d = x.shape[-1]
+        inv = theta ** (-2.0 * np.arange(d // 2) / d)
+        ang = np.asarray(pos, dtype=np.float64)[..., None, None] * inv  # [B, S, 1, d/2]
+        c, s = np.cos(ang), np.sin(ang)
+        a, b = x[..., : d // 2], x[..., d // 2:]
+        return np.concatenate([a * c - b * s, b * c + a * s], axis=-1)
+
+    @staticmethod
+    def _attention(q, k, v, mask):
+        B, S, H, d = q.shape
+        G = k.shape[2]
+        t = np.arange(S)
+        keep = t[None, :] <= t[:, None]
+        W = mask.get("window", 0)
+        if W > 0:
+            keep &= t[None, :] > t[:, None] - W
+        out = np.empty_like(q)
+        for b in range(B):
+            for h in range(H):
+                g = h // (H // G)
+                s = q[b, :, h, :] @ k[b, :, g, :].T / math.sqrt(d)
+                s = np.where(keep, s, -np.inf)
+                s = np.exp(s - s.max(axis=-1, keepdims=True))
+                out[b, :, h, :] = (s / s.sum(axis=-1, keepdims=True)) @ v[b, :, g, :]
+        return out
+
+    @staticmethod
+    def _route(x, Wr, top_k, normalize):
+        s = x @ Wr.T
+        p = np.exp(s - s.max(axis=-1, keepdims=True))
+        p /= p.sum(axis=-1, keepdims=True)
+        idx = np.argsort(-p, axis=-1, kind="stable")[..., :top_k]
+        w = np.take_along_axis(p, idx, axis=-1)
+        if normalize:
+            w = w / w.sum(axis=-1, keepdims=True)
+        return w, idx
+
+    def _stacked(self, ins, at, lv):
+        init, h, w, idx = ins
+        act = {"Act.silu": lambda z: z / (1.0 + np.exp(-z))}.get(at["act"])
+        if act is None:
+            raise NotImplementedError(at["act"])
+        y = np.array(init, dtype=np.float64)
+        for e in range(int(at["experts"])):
+            inner = dict(lv)
+            inner[at["var"]] = e
+            ffn = (act(h @ self._w(at["gate"], inner).T) * (h @ self._w(at["up"], inner).T)) @ self._w(at["down"],
+                                                                                                      inner).T
+            y = y + np.sum(np.where(idx == e, w, 0.0), axis=-1, keepdims=True) * ffn
+        return y

@@ -1,20 +1,34 @@
 """CPU tests of the Axon-subset front end: lexing and parsing, Graph IR
 building (definition inlining, scoped parameter paths, loops, configuration
-reads), and the lowering of a decoder module onto the library's kernels
-(shape and checkpoint-name map), including the variants it accepts and the
-modules it must refuse."""
+reads), the stacked-experts rewrite, and the lowering of decoder modules
+onto the library's kernels (shape and checkpoint-name map), including the
+variants it accepts and the modules it must refuse. The lowering is also
+checked for meaning: a module's Graph IR, evaluated directly on its own
+parameter paths (graph_eval.py), gives the oracle's logits for the lowered
+shape on the checkpoint re-keyed through the name map."""
 import os
 import re
 
+import numpy as np
 import pytest
 
+import synth_inputs as si
+from graph_eval import GraphEval
+from helpers import oracle_for
 from paper_2608_19889_gb300 import frontend as fe
+from paper_2608_19889_gb300.frontend import rewrite as rw
 from paper_2608_19889_gb300.frontend import syntax as sx
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 LLAMA = open(os.path.join(HERE, "data", "llama_decoder.axon")).read()
+MOE = open(os.path.join(HERE, "data", "moe_decoder.axon")).read()
 CFG = dict(hidden_size=128, num_hidden_layers=2, num_attention_heads=4, num_key_value_heads=2, head_dim=32,
            intermediate_size=192, vocab_size=1000, rope_theta=10000.0, rms_norm_eps=1e-5)
+# DeepSeek-MoE-like at toy width: layer 0 dense, layers 1-2 with 6 experts
+# (2 per token) of width 16 and a shared MLP of 2 experts' width
+MOE_CFG = dict(hidden_size=32, num_hidden_layers=3, first_k_dense_replace=1, num_attention_heads=4,
+               num_key_value_heads=2, head_dim=8, intermediate_size=48, n_routed_experts=6, num_experts_per_tok=2,
+               moe_intermediate_size=16, n_shared_experts=2, vocab_size=64, rope_theta=10000.0, rms_norm_eps=1e-5)
 
 
 # ------------------------------------------------------------------ syntax
@@ -186,3 +200,119 @@ def test_checkpoint_renaming_both_ways_and_missing_tensors():
     mod.pop("layers.1.feed_forward.w3.weight")
     with pytest.raises(fe.LoweringError, match="w3"):
         low.library_weights(mod)
+
+
+# ------------------------------------------------------ mixture of experts
+def _moe_body(g):
+    """The body graph of the mixture-of-experts layer loop."""
+    return [n for n in g.nodes if n.op == "loop"][-1].body
+
+
+def test_stacked_experts_rewrite_replaces_the_loop_over_experts():
+    g = fe.build_graph(sx.parse_module(MOE), MOE_CFG)
+    inner = [n for n in _moe_body(g).nodes if n.op == "loop"]
+    assert len(inner) == 1 and inner[0].attrs["var"] == "e" and inner[0].attrs["stop"] == 6
+    loop_id = inner[0].id
+    assert rw.stack_experts(g) == 1
+    assert rw.stack_experts(g) == 0  # nothing left to rewrite
+    body = _moe_body(g)
+    assert not [n for n in body.nodes if n.op == "loop"]
+    st = [n for n in body.nodes if n.op == "MoE.stacked_experts"]
+    assert len(st) == 1 and st[0].id == loop_id  # uses of the loop's value now read the stacked node
+    a = st[0].attrs
+    assert (a["experts"], a["dim"], a["act"], a["var"]) == (6, 16, "Act.silu", "e")
+    assert (a["gate"], a["up"], a["down"]) == tuple(f"blocks.{{i}}.ffn.experts.{{e}}.{w}"
+                                                     for w in ("w_gate", "w_up", "w_down"))
+    router = [n for n in body.nodes if n.op == "MoE.softmax_topk_router"][0]
+    init, h, w, idx = st[0].inputs
+    assert (w, idx) == (fe.Ref(router.id, 0), fe.Ref(router.id, 1)) and router.inputs[0] == h
+
+
+def test_dense_loops_are_not_rewritten():
+    g = fe.build_graph(sx.parse_module(LLAMA), CFG)
+    before = fe.dump(g)
+    assert rw.stack_experts(g) == 0 and fe.dump(g) == before
+
+
+def test_moe_module_lowers_to_the_kernels_shape_and_names():
+    low = fe.compile_decoder(MOE, MOE_CFG)
+    assert low.shape == dict(L=3, D=32, H=4, G=2, d=8, F=48, V=64, tie=False, bias=False, theta=10000.0, eps=1e-5,
+                             window=0, act="silu", qk_norm=False, n_experts=6, top_k=2, moe_F=16, n_shared=2,
+                             first_dense=1, norm_topk=False)
+    # exactly the tensors the library reads for that shape, each from its module path
+    assert set(low.names) == set(si.weight_shapes(low.shape))
+    assert low.names["model.layers.0.mlp.down_proj.weight"] == "blocks.0.ffn.w_down.weight"
+    assert low.names["model.layers.2.mlp.gate.weight"] == "blocks.2.ffn.router.weight"
+    assert low.names["model.layers.1.mlp.experts.5.up_proj.weight"] == "blocks.1.ffn.experts.5.w_up.weight"
+    assert low.names["model.layers.2.mlp.shared_experts.down_proj.weight"] == "blocks.2.ffn.shared.w_down.weight"
+    assert low.paths["moe_layers.expert_gate"] == "blocks.{i}.ffn.experts.{e}.w_gate"
+
+
+def test_llama_module_names_are_the_librarys_tensors():
+    low = fe.compile_decoder(LLAMA, CFG)
+    assert set(low.names) == set(si.weight_shapes(low.shape))
+
+
+def test_moe_config_variants():
+    low = fe.compile_decoder(MOE, dict(MOE_CFG, norm_topk_prob=True, first_k_dense_replace=0, n_shared_experts=1))
+    s = low.shape
+    assert s["norm_topk"] and s["first_dense"] == 0 and s["n_shared"] == 1
+    assert set(low.names) == set(si.weight_shapes(s))
+    assert not any(".mlp.gate_proj." in k for k in low.names)  # no dense layer left
+
+
+def _moe_variant(old, new):
+    assert MOE.count(old) >= 1, old
+    return MOE.replace(old, new)
+
+
+@pytest.mark.parametrize("src,cfg,msg", [
+    (None, dict(num_experts_per_tok=9), "top_k"),
+    (None, dict(n_routed_experts=300, num_experts_per_tok=2), "experts"),
+    (("s <- gated@shared h (SHARED * EXPERT_FFN)", "s <- gated@shared h (SHARED * EXPERT_FFN + 8)"), {}, "multiple"),
+    # no router weight on the expert term: not a mixture, every expert on every token
+    (("y <- y + MoE.expert_weight w idx e * gated h EXPERT_FFN", "y <- y + gated h EXPERT_FFN"), {},
+     "sum over experts"),
+    # a loop that skips expert 0
+    (("[0..EXPERTS) carry (y)", "[1..EXPERTS) carry (y)"), {}, "sum over experts"),
+    # the same parameters for every expert
+    (("y <- y + MoE.expert_weight w idx e * gated h EXPERT_FFN",
+      "y <- y + MoE.expert_weight w idx e * gated@@blocks.one h EXPERT_FFN"), {}, "sum over experts"),
+    (("  x, new_i <- dense_layer x pos mask past_i", "  x, new_i <- moe_layer x pos mask past_i"), {},
+     "leading dense"),
+    (("w, idx <- MoE.softmax_topk_router@router h top_k=TOPK",
+      "w, idx <- MoE.softmax_topk_router@router (h * 2.0) top_k=TOPK"), {}, "router"),
+    (("mixture h = do", "mixture h = do\n  h <- Tensor.dropout h"), {}, "post-attention norm"),
+])
+def test_moe_modules_outside_the_kernels_are_refused(src, cfg, msg):
+    text = MOE if src is None else _moe_variant(*src)
+    with pytest.raises(fe.LoweringError, match=msg):
+        fe.compile_decoder(text, dict(MOE_CFG, **cfg))
+
+
+@pytest.mark.parametrize("case", ["llama", "moe", "moe_normalised_all_moe"])
+def test_lowered_modules_compute_what_the_oracle_computes(case):
+    """The module's own Graph IR on its own parameter paths against the
+    oracle on the lowered shape and the re-keyed checkpoint (float64 both):
+    the lowering keeps the module's meaning. For MoE modules both the literal
+    loop over experts and its stacked-experts rewrite are evaluated."""
+    src, cfg = {"llama": (LLAMA, dict(CFG, num_hidden_layers=2)), "moe": (MOE, MOE_CFG),
+                "moe_normalised_all_moe": (MOE, dict(MOE_CFG, norm_topk_prob=True, first_k_dense_replace=0))}[case]
+    low = fe.compile_decoder(src, cfg)
+    w = si.make_weights(low.shape, seed=11)
+    lib = si.weights_as_f32_numpy(w)
+    mod = low.module_weights(lib)
+    ids = si.make_ids(2, 7, low.shape["V"], seed=12)
+    o = oracle_for(low.shape, w)
+    ref = o.prefill(ids, o.new_contiguous_cache(2, 8))
+    g = fe.build_graph(sx.parse_module(src), cfg)
+    graphs = [g]
+    if "moe" in case:
+        g2 = fe.build_graph(sx.parse_module(src), cfg)
+        assert rw.stack_experts(g2) == 1
+        graphs.append(g2)
+    for gg in graphs:
+        got = GraphEval(mod).run(gg, ids)[0]
+        assert got.shape == ref.shape
+        err = float(np.max(np.abs(got - ref)))
+        assert err < 1e-10 * max(1.0, float(np.max(np.abs(ref)))), err
