@@ -290,15 +290,31 @@ def test_moe_modules_outside_the_kernels_are_refused(src, cfg, msg):
         fe.compile_decoder(text, dict(MOE_CFG, **cfg))
 
 
-@pytest.mark.parametrize("case", ["llama", "moe", "moe_normalised_all_moe"])
+def _llama_variants():
+    """q/k/v biases, qk-norm, the tanh gelu gate and a tied head."""
+    src = LLAMA
+    for proj in ("wq", "wk", "wv"):
+        src = re.sub(rf"(NN\.linear@{proj} h dim=\([A-Z_]+ \* HEAD_DIM\))", r"\1 bias=true", src)
+    src = src.replace("  q <- rope q pos theta=THETA", "  q <- NN.rmsnorm@q_norm q eps=EPS\n  q <- rope q pos theta=THETA")
+    src = src.replace("  k <- rope k pos theta=THETA", "  k <- NN.rmsnorm@k_norm k eps=EPS\n  k <- rope k pos theta=THETA")
+    return src.replace("Act.silu g", "Act.gelu_tanh g").replace("NN.linear@output dim=VOCAB",
+                                                              "NN.linear@tok_embeddings dim=VOCAB")
+
+
+@pytest.mark.parametrize("case", ["llama", "llama_variants_window", "moe", "moe_normalised_all_moe"])
 def test_lowered_modules_compute_what_the_oracle_computes(case):
     """The module's own Graph IR on its own parameter paths against the
     oracle on the lowered shape and the re-keyed checkpoint (float64 both):
     the lowering keeps the module's meaning. For MoE modules both the literal
     loop over experts and its stacked-experts rewrite are evaluated."""
-    src, cfg = {"llama": (LLAMA, dict(CFG, num_hidden_layers=2)), "moe": (MOE, MOE_CFG),
+    src, cfg = {"llama": (LLAMA, dict(CFG, num_hidden_layers=2)),
+                "llama_variants_window": (_llama_variants(), dict(CFG, sliding_window=3)),
+                "moe": (MOE, MOE_CFG),
                 "moe_normalised_all_moe": (MOE, dict(MOE_CFG, norm_topk_prob=True, first_k_dense_replace=0))}[case]
     low = fe.compile_decoder(src, cfg)
+    if case == "llama_variants_window":
+        s = low.shape
+        assert s["bias"] and s["qk_norm"] and s["act"] == "gelu_tanh" and s["tie"] and s["window"] == 3
     w = si.make_weights(low.shape, seed=11)
     lib = si.weights_as_f32_numpy(w)
     mod = low.module_weights(lib)
