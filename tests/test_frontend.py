@@ -332,3 +332,16 @@ def test_lowered_modules_compute_what_the_oracle_computes(case):
         assert got.shape == ref.shape
         err = float(np.max(np.abs(got - ref)))
         assert err < 1e-10 * max(1.0, float(np.max(np.abs(ref)))), err
+
+
+def test_lowered_moe_shape_fills_the_config_the_library_reads():
+    """The lowered MoE shape through make_config (host-side ctypes struct,
+    no library call): the config.json keys the module read land in the
+    C config's mixture-of-experts fields."""
+    import paper_2608_19889_gb300 as ax
+    low = fe.compile_decoder(MOE, dict(MOE_CFG, norm_topk_prob=True))
+    c = ax.make_config(low.shape, max_batch=4, max_context=64)
+    assert (c.num_hidden_layers, c.hidden_size, c.intermediate_size, c.vocab_size) == (3, 32, 48, 64)
+    assert (c.n_routed_experts, c.num_experts_per_tok, c.moe_intermediate_size, c.n_shared_experts,
+            c.first_k_dense_replace, c.norm_topk_prob) == (6, 2, 16, 2, 1, 1)
+    assert (c.num_attention_heads, c.num_key_value_heads, c.head_dim, c.hidden_act) == (4, 2, 8, ax.AXON_ACT_SILU)
