@@ -301,7 +301,15 @@ def _llama_variants():
                                                               "NN.linear@tok_embeddings dim=VOCAB")
 
 
-@pytest.mark.parametrize("case", ["llama", "llama_variants_window", "moe", "moe_normalised_all_moe"])
+def _moe_shared_first():
+    """The experts' sum accumulated onto the shared MLP's output instead of
+    zeros, the router weights renormalised."""
+    src = MOE.replace("  y <- Tensor.zeros_like h\n", "  y <- gated@shared h (SHARED * EXPERT_FFN)\n")
+    return src.replace("  s <- gated@shared h (SHARED * EXPERT_FFN)\n  return y + s", "  return y")
+
+
+@pytest.mark.parametrize("case", ["llama", "llama_variants_window", "moe", "moe_normalised_all_moe",
+                                  "moe_shared_first"])
 def test_lowered_modules_compute_what_the_oracle_computes(case):
     """The module's own Graph IR on its own parameter paths against the
     oracle on the lowered shape and the re-keyed checkpoint (float64 both):
@@ -310,8 +318,11 @@ def test_lowered_modules_compute_what_the_oracle_computes(case):
     src, cfg = {"llama": (LLAMA, dict(CFG, num_hidden_layers=2)),
                 "llama_variants_window": (_llama_variants(), dict(CFG, sliding_window=3)),
                 "moe": (MOE, MOE_CFG),
-                "moe_normalised_all_moe": (MOE, dict(MOE_CFG, norm_topk_prob=True, first_k_dense_replace=0))}[case]
+                "moe_normalised_all_moe": (MOE, dict(MOE_CFG, norm_topk_prob=True, first_k_dense_replace=0)),
+                "moe_shared_first": (_moe_shared_first(), dict(MOE_CFG, norm_topk_prob=True))}[case]
     low = fe.compile_decoder(src, cfg)
+    if case == "moe_shared_first":
+        assert "zeros_like" not in src and low.shape["n_shared"] == 2 and low.shape["norm_topk"]
     if case == "llama_variants_window":
         s = low.shape
         assert s["bias"] and s["qk_norm"] and s["act"] == "gelu_tanh" and s["tie"] and s["window"] == 3
