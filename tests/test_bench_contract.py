@@ -1,7 +1,10 @@
 """CPU checks of bench.py's accounting and of its reference-arm JSON line:
-the algorithmic byte and FLOP counts on shapes small enough to count by hand,
-the DRAM-traffic record lookup (valid only for the CUDA sources it was taken
-on), and `--impl reference` on the 135M workload."""
+the algorithmic byte and FLOP counts on shapes small enough to count by hand
+(dense and mixture-of-experts, against the checkpoint's own matrix shapes
+and, for the expected number of routed experts, exact enumeration), the
+DRAM-traffic record lookup (valid only for the CUDA sources it was taken
+on), the peak and clock bookkeeping, and `--impl reference` on the 135M
+workload."""
 import json
 import os
 import subprocess
@@ -115,3 +118,84 @@ def test_sliding_window_counts_only_the_visible_keys():
     assert bench.prefill_flops(W, 1, 7) == 2 * 7 * lin + 2 * 4 * 4 * 16 * 18 + 2 * head
     assert bench.varlen_prefill_flops(W, [[(4, 3)]]) == 2 * 3 * lin + 2 * 4 * 4 * 16 * 9 + 2 * head
     assert bench.keys_seen_by_run(4, 3, 0) == 5 + 6 + 7
+
+
+# mixture of experts: the decode step's weight bytes and the prefill FLOPs
+MOE_SHAPE = dict(L=3, D=32, H=4, G=2, d=8, F=48, V=64, tie=False, bias=False, n_experts=6, top_k=2, moe_F=16,
+                 n_shared=2, first_dense=1)
+
+
+def _matrices(shape):
+    """Weight elements of every per-layer matrix, by its HF name."""
+    import numpy as np
+    import synth_inputs as si
+    return {k: int(np.prod(v)) for k, v in si.weight_shapes(shape).items() if ".layers." in k and len(v) == 2}
+
+
+@pytest.mark.parametrize("shape", [dict(SHAPE, tie=False), MOE_SHAPE])
+def test_model_bytes_match_the_checkpoints_matrices(shape):
+    """All experts counted (active None): the per-layer matrices of the
+    checkpoint the library reads, counted from their shapes."""
+    lin, head = bench.model_bytes(shape)
+    assert lin == sum(_matrices(shape).values())
+    assert head == shape["V"] * shape["D"]
+
+
+def test_moe_model_bytes_with_some_experts_active():
+    m = _matrices(MOE_SHAPE)
+    one_expert = sum(v for k, v in m.items() if ".layers.1.mlp.experts.0." in k)
+    lin_all, _ = bench.model_bytes(MOE_SHAPE)
+    lin_3, _ = bench.model_bytes(MOE_SHAPE, active_experts=3)
+    assert lin_all - lin_3 == 2 * (6 - 3) * one_expert  # two MoE layers, three experts fewer each
+
+
+def test_expected_active_experts_against_enumeration():
+    """E (1 - (1 - k/E)^T) against the exact mean over every assignment of
+    T tokens to k-subsets of E experts (uniform, independent)."""
+    import itertools
+    E, k = 6, 2
+    subsets = list(itertools.combinations(range(E), k))
+    for T in (1, 2, 3):
+        total = sum(len(set().union(*pick)) for pick in itertools.product(subsets, repeat=T))
+        exact = total / len(subsets) ** T
+        assert abs(bench.expected_active_experts(dict(n_experts=E, top_k=k), T) - exact) < 1e-12
+
+
+def test_moe_linear_flops_per_token_by_hand():
+    """Per token: every attention matrix, the dense layer's MLP, and in each
+    MoE layer the router, the shared MLP and top_k experts, 2 FLOPs per
+    weight element."""
+    m = _matrices(MOE_SHAPE)
+    per = sum(v for k, v in m.items() if ".experts." not in k)
+    per += 2 * MOE_SHAPE["top_k"] * sum(v for k, v in m.items() if ".layers.1.mlp.experts.0." in k)
+    assert bench.linear_flops_per_token(MOE_SHAPE) == 2 * per
+
+
+def test_tensor_peak_takes_the_sustained_figure_for_long_phases():
+    assert bench.tensor_peak(1900.0, 1700.0, 99.9) == (1900.0, "burst")
+    assert bench.tensor_peak(1900.0, 1700.0, 100.0) == (1700.0, "sustained")
+    assert bench.tensor_peak(1900.0, None, 5000.0) == (1900.0, "burst")
+
+
+def test_clock_sampler_reads_median_clock_and_active_reasons():
+    class FakeProc:
+        def terminate(self):
+            pass
+
+        def communicate(self, timeout=None):
+            rows = ["0, 2070, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active",
+                    "0, 1980, 2070, 1390.5, 0x4, Not Active, Not Active, Not Active, Active",
+                    "0, 2070, 2070, 1200.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+                    "garbled line"]
+            return "\n".join(rows) + "\n", ""
+
+    s = bench.ClockSampler.__new__(bench.ClockSampler)
+    s.p = FakeProc()
+    c = s.stop()
+    assert c == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+
+
+def test_default_precision_by_width():
+    assert bench.default_precision("32b_b16_s2048_n256") == "fp16"
+    assert bench.default_precision("8b_paged_b64_ctx512-4096_n128") == "fp16"
+    assert bench.default_precision("0.5b_b1_s512_n128") == "bf16"
