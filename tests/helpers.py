@@ -26,7 +26,10 @@ def tiny_tol(prec: str) -> float:
 def parity(gpu: np.ndarray, ref: np.ndarray):
     """(max |delta|, top-1 agreement, hard mismatches). A hard mismatch is a
     top-1 disagreement where the oracle's top-2 gap exceeds twice the
-    observed max |delta| (i.e. not explainable as a near tie)."""
+    observed max |delta|. It cannot occur: a flip needs a delta of at least
+    half the gap (tests/test_parity_stats.py), so the count is a diagnostic
+    and the binding checks are max |delta| against the tolerance and the
+    raw top-1 floors."""
     gpu = np.asarray(gpu, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
     maxd = float(np.max(np.abs(gpu - ref)))

@@ -74,11 +74,12 @@ def decode_steps(m, first_tokens, ctx0, n_steps, V, block_table=None):
 
 
 def check(gpu, ref, tol=LOGIT_TOL, what="", top1=False):
-    """max |delta logit| <= tol and no top-1 mismatch outside a near tie;
-    with top1=True also >= 99% top-1 agreement among the positions whose
-    oracle top-2 gap is outside the bf16 noise band (2 max |delta|): random
-    init leaves many positions with gaps inside it, where either token is a
-    correct greedy choice at this precision."""
+    """max |delta logit| <= tol, the binding check. The top-1 statistics are
+    printed; the no-hard-mismatch assertion and the top1=True agreement on
+    positions whose oracle top-2 gap exceeds 2 max |delta| hold by
+    construction (a flip needs a delta of at least half the gap), so they
+    guard only against a broken statistic. Raw top-1 floors are asserted by
+    the callers that state them."""
     maxd, agree, hard = parity(gpu, ref)
     srt = np.sort(np.asarray(ref), axis=-1)
     near = float(np.mean((srt[..., -1] - srt[..., -2]) <= 2 * maxd))
