@@ -48,9 +48,11 @@ from .rewrite import ACTIVATIONS as _ACTS, stack_experts
 # attention kernels, the paged or contiguous cache).
 _PLUMBING = {
     "Cache.past_length", "Cache.prepare", "Cache.read", "Cache.index", "Cache.append", "Cache.finish",
-    "Positions.position_ids", "Masking.causal_mask_for_input", "Masking.mask_for_input",
+    "Positions.position_ids", "Masking.causal_mask_for_input", "Masking.causal_mask", "Masking.mask_for_input",
     "Masking.mask_length_for_input", "input",
 }
+# masks the attention kernels implement: causal, optionally windowed
+_CAUSAL_MASKS = ("Masking.causal_mask_for_input", "Masking.causal_mask")
 # limits of the mixture-of-experts kernels (the config's documented range)
 _MAX_EXPERTS, _MAX_TOPK = 256, 8
 
@@ -124,7 +126,7 @@ def _bool(v):
 class _Layer:
     """What the body of one layer loop lowered to."""
     loop: gr.Node
-    params: dict  # H, G, d, bias, theta, act, qk_norm, rope scaling: equal across loops
+    params: dict  # H, G, d, bias, theta, act, qk_norm, rope scaling, window: equal across loops
     eps: set
     paths: dict  # role -> parameter path pattern with the loop's {var}
     mlp: str  # "dense" or "moe"
@@ -240,6 +242,19 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
         n = m.byid.get(r.node) if isinstance(r, gr.Ref) else None
         if n is not None and n.op == "Cache.update":
             m.claimed.add(n.id)
+    # the mask: built before the loop from the ids, or in the layer from q
+    # and k; the kernels attend causally, so nothing else is accepted
+    mask_ref = att.inputs[3] if len(att.inputs) > 3 else None
+    mask = None
+    if isinstance(mask_ref, gr.Ref):
+        mask = m.byid.get(mask_ref.node) or m.outer_byid.get(mask_ref.node)
+    if mask is None or mask.op not in _CAUSAL_MASKS:
+        raise LoweringError("attention must take a causal mask (Masking.causal_mask_for_input or "
+                            "Masking.causal_mask): the kernels attend causally"
+                            + (f", found {mask.op}" if mask is not None else ", found none"))
+    if mask.attrs.get("padding_mask") is not None:
+        raise LoweringError("padding masks: the kernels take per-sequence lengths instead")
+    window = int(mask.attrs.get("window", 0) or 0)
     rope_scaling = {}
 
     def qk_chain(ref, what):
@@ -302,7 +317,7 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
     if int(o_proj.attrs.get("dim", D)) != D:
         raise LoweringError("MLP and output projection widths disagree with the hidden size")
     params = dict(H=H, G=G, d=d, bias=biases.pop(), theta=thetas.pop(), act=act, qk_norm=q_norm is not None,
-                  rope_scaling=tuple(sorted(rope_scaling.items())))
+                  rope_scaling=tuple(sorted(rope_scaling.items())), window=window)
     eps = {float(n.attrs.get("eps", cfg.get("rms_norm_eps", 1e-6))) for n in (norm1, norm2)}
     paths = {"input_norm": norm1.path, "post_norm": norm2.path, "q": q_lin.path, "k": k_lin.path,
              "v": v_lin.path, "o": o_proj.path}
@@ -402,14 +417,11 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
         raise LoweringError("the final norm must read the layer loop's hidden state")
     if not any(isinstance(o, gr.Ref) and o.node == head.id for o in g.outputs):
         raise LoweringError("the entry definition must return the LM head's logits")
-    window = 0
     for n in g.nodes:
         if n.op in ("NN.embedding", "NN.linear", "NN.rmsnorm", "loop"):
             continue
         if n.op not in _PLUMBING:
             raise LoweringError(f"operation {n.op} outside the layer loop has no GB300 kernel")
-        if n.op == "Masking.causal_mask_for_input":
-            window = int(n.attrs.get("window", 0) or 0)
     tie = head.path == emb.path
     if head.attrs.get("bias") or head.attrs.get("transpose"):
         raise LoweringError("the LM head takes neither a bias nor a transposed matrix here")
@@ -432,7 +444,7 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
     moe = layers[-1].moe if layers[-1].mlp == "moe" else None
     F = layers[0].F if layers[0].mlp == "dense" else (moe["Fs"] or moe["Fe"])
     shape = dict(L=L, D=D, H=p0["H"], G=p0["G"], d=p0["d"], F=F, V=V, tie=tie, bias=p0["bias"],
-                 theta=p0["theta"], eps=epss.pop(), window=window, act=p0["act"], qk_norm=p0["qk_norm"])
+                 theta=p0["theta"], eps=epss.pop(), window=p0["window"], act=p0["act"], qk_norm=p0["qk_norm"])
     rope_scaling = dict(p0["rope_scaling"])
     if rope_scaling:
         shape.update(rope_factor=float(rope_scaling.get("factor", 0.0)),

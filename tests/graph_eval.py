@@ -105,7 +105,9 @@ class GraphEval:
         if op == "Positions.position_ids":
             ids = ins[0]
             return np.broadcast_to(np.arange(ids.shape[-1]) + int(at.get("past_length") or 0), ids.shape)
-        if op == "Masking.causal_mask_for_input":
+        if op in ("Masking.causal_mask_for_input", "Masking.causal_mask"):
+            if at.get("padding_mask") is not None:
+                raise NotImplementedError("padding masks")
             return {"window": int(at.get("window", 0) or 0)}
         if op in ("Cache.prepare", "Cache.index", "Cache.append"):
             return None
@@ -114,7 +116,9 @@ class GraphEval:
         if op == "Positions.rope":
             return self._rope(ins[0], ins[1], float(at["theta"]), at)
         if op == "Attention.attention":
-            return self._attention(ins[0], ins[1], ins[2], ins[3] or {})
+            if len(ins) < 4 or ins[3] is None:
+                raise NotImplementedError("attention without a causal mask")
+            return self._attention(ins[0], ins[1], ins[2], ins[3])
         if op == "Act.silu":
             z = ins[0]
             return z / (1.0 + np.exp(-z))

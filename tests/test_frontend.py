@@ -185,6 +185,11 @@ def test_variants_bias_qk_norm_gelu_tied_window_and_rope_scaling():
      "  m <- NN.rmsnorm@ffn_norm x eps=EPS |> ffn@feed_forward\n  x <- x + a", "post-attention norm"),
     ("  past_len <- Cache.past_length past", "  past_len <- Cache.past_length past\n  z <- Tensor.noise ids",
      "outside the layer loop"),
+    # no mask (bidirectional attention) or a non-causal one: the kernels attend causally
+    ("attention q k v mask |>", "attention q k v |>", "causal mask"),
+    ("  mask <- causal_mask_for_input ids past_len window=WINDOW",
+     "  mask <- Masking.mask_for_input ids past_len", "causal mask"),
+    ("attention q k v mask |>", "attention q k v (Masking.causal_mask q k padding_mask=pos) |>", "padding"),
 ])
 def test_modules_outside_the_kernels_are_refused(old, new, msg):
     with pytest.raises(fe.LoweringError, match=msg):
@@ -308,8 +313,20 @@ def _moe_shared_first():
     return src.replace("  s <- gated@shared h (SHARED * EXPERT_FFN)\n  return y + s", "  return y")
 
 
-@pytest.mark.parametrize("case", ["llama", "llama_variants_window", "moe", "moe_normalised_all_moe",
-                                  "moe_shared_first"])
+def _llama_layer_mask():
+    """The mask built inside the layer from q and k (the attention built-ins'
+    self-attention pattern), windowed."""
+    return LLAMA.replace("  y <- attention q k v mask |>",
+                         "  keep <- Masking.causal_mask q k window=5\n  y <- attention q k v keep |>")
+
+
+def test_mask_built_in_the_layer_is_plumbing_with_its_window():
+    low = fe.compile_decoder(_llama_layer_mask(), CFG)
+    assert low.shape["window"] == 5 and low.names == fe.compile_decoder(LLAMA, CFG).names
+
+
+@pytest.mark.parametrize("case", ["llama", "llama_variants_window", "llama_layer_mask", "moe",
+                                  "moe_normalised_all_moe", "moe_shared_first"])
 def test_lowered_modules_compute_what_the_oracle_computes(case):
     """The module's own Graph IR on its own parameter paths against the
     oracle on the lowered shape and the re-keyed checkpoint (float64 both):
@@ -317,6 +334,7 @@ def test_lowered_modules_compute_what_the_oracle_computes(case):
     loop over experts and its stacked-experts rewrite are evaluated."""
     src, cfg = {"llama": (LLAMA, dict(CFG, num_hidden_layers=2)),
                 "llama_variants_window": (_llama_variants(), dict(CFG, sliding_window=3)),
+                "llama_layer_mask": (_llama_layer_mask(), CFG),
                 "moe": (MOE, MOE_CFG),
                 "moe_normalised_all_moe": (MOE, dict(MOE_CFG, norm_topk_prob=True, first_k_dense_replace=0)),
                 "moe_shared_first": (_moe_shared_first(), dict(MOE_CFG, norm_topk_prob=True))}[case]
