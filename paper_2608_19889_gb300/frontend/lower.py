@@ -53,6 +53,36 @@ _PLUMBING = {
 }
 # masks the attention kernels implement: causal, optionally windowed
 _CAUSAL_MASKS = ("Masking.causal_mask_for_input", "Masking.causal_mask")
+_ROPE_SCALING = ("factor", "low_freq_factor", "high_freq_factor", "original_max_position")
+# keyword arguments the kernels implement, per operation; any other keyword
+# would change the function and is refused rather than dropped
+_KWARGS = {
+    "NN.embedding": {"dim"}, "NN.linear": {"dim", "bias", "transpose"}, "NN.rmsnorm": {"eps"},
+    "Attention.reshape_heads": {"heads"}, "Attention.merge_heads": set(), "Attention.attention": set(),
+    "Positions.rope": {"theta", *_ROPE_SCALING}, "Positions.position_ids": {"past_length"},
+    "Masking.causal_mask_for_input": {"window", "padding_mask"}, "Masking.causal_mask": {"window", "padding_mask"},
+    "MoE.softmax_topk_router": {"top_k", "normalize", "dim"}, "MoE.expert_weight": set(),
+    "Tensor.zeros_like": set(), "add": set(), "mul": set(),
+    **{a: set() for a in _ACTS},
+}
+
+
+def _check_kwargs(nodes):
+    for n in nodes:
+        if n.op == "MoE.stacked_experts":  # the keywords of the operations the rewrite replaced
+            for op, keys in n.attrs.get("kwargs", {}).items():
+                extra = sorted(set(keys) - _KWARGS.get(op, set()))
+                if extra:
+                    raise LoweringError(f"{op} in the experts: keyword argument(s) {extra} are not implemented "
+                                        "by the kernels")
+            continue
+        allowed = _KWARGS.get(n.op)
+        if allowed is None:
+            continue
+        extra = sorted(set(n.attrs) - allowed)
+        if extra:
+            raise LoweringError(f"{n.op}{' @@' + n.path if n.path else ''}: keyword argument(s) {extra} "
+                                "are not implemented by the kernels")
 # limits of the mixture-of-experts kernels (the config's documented range)
 _MAX_EXPERTS, _MAX_TOPK = 256, 8
 
@@ -281,13 +311,23 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
         raise LoweringError("the input norm must read the layer input")
     if (q_norm is None) != (k_norm is None):
         raise LoweringError("qk-norm must apply to both q and k")
-    for r in (q_rope, k_rope):
-        for key in ("factor", "low_freq_factor", "high_freq_factor", "original_max_position"):
-            if key in r.attrs:
-                rope_scaling[key] = r.attrs[key]
+    scalings = [tuple((key, r.attrs[key]) for key in _ROPE_SCALING if key in r.attrs) for r in (q_rope, k_rope)]
+    if scalings[0] != scalings[1]:
+        raise LoweringError("q and k must use one rotary frequency scaling")
+    rope_scaling.update(scalings[0])
     thetas = {float(r.attrs.get("theta", cfg.get("rope_theta", 10000.0))) for r in (q_rope, k_rope)}
     if len(thetas) != 1:
         raise LoweringError("q and k must use one rotary base")
+    # rotary positions: the new tokens' positions after the cached ones
+    for r in (q_rope, k_rope):
+        pos = r.inputs[1] if len(r.inputs) > 1 else None
+        pn = (m.byid.get(pos.node) or m.outer_byid.get(pos.node)) if isinstance(pos, gr.Ref) else None
+        past = pn.attrs.get("past_length") if pn is not None and pn.op == "Positions.position_ids" else None
+        pl = (m.byid.get(past.node) or m.outer_byid.get(past.node)) if isinstance(past, gr.Ref) else None
+        if pl is None or pl.op != "Cache.past_length":
+            raise LoweringError("rotary positions must be Positions.position_ids offset by the cache's past "
+                                "length (past_length=Cache.past_length ...): the kernels place token i of a "
+                                "sequence at its cached length + i")
 
     # claimed plumbing inside the body (cache index/append, inputs)
     for n in body.nodes:
@@ -297,6 +337,7 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
     if left:
         raise LoweringError("layer operations with no GB300 kernel: " +
                             ", ".join(f"{n.op}{' @@' + n.path if n.path else ''}" for n in left))
+    _check_kwargs(body.nodes)
 
     biases = {_bool(n.attrs.get("bias")) for n in (q_lin, k_lin, v_lin)}
     if len(biases) != 1:
@@ -422,6 +463,7 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
             continue
         if n.op not in _PLUMBING:
             raise LoweringError(f"operation {n.op} outside the layer loop has no GB300 kernel")
+    _check_kwargs(g.nodes)
     tie = head.path == emb.path
     if head.attrs.get("bias") or head.attrs.get("transpose"):
         raise LoweringError("the LM head takes neither a bias nor a transposed matrix here")

@@ -18,7 +18,8 @@ feeds only the expert-weight selection and the parameter paths, the
 accumulator is only added to -- and replaces the loop node by
 
     MoE.stacked_experts(init, h, w, idx)   attrs: experts E, dim (expert
-        width), act, var, gate / up / down path patterns with {var}
+        width), act, var, gate / up / down path patterns with {var}, and
+        the replaced operations' keyword names (kwargs)
 
 whose value is init + sum_e expert_weight(w, idx, e) * ffn_e(h): the
 experts' matrices stacked along a leading expert axis, each token computed
@@ -111,7 +112,10 @@ def _expert_loop(loop: gr.Node) -> Optional[gr.Node]:
     attrs = {"experts": loop.attrs["stop"], "var": var, "dim": gate.attrs.get("dim"), "act": act.op,
              "gate": gate.path, "up": up.path, "down": down.path, "down_dim": down.attrs.get("dim"),
              "up_dim": up.attrs.get("dim"),
-             "bias": any(bool(n.attrs.get("bias")) or bool(n.attrs.get("transpose")) for n in (gate, up, down))}
+             "bias": any(bool(n.attrs.get("bias")) or bool(n.attrs.get("transpose")) for n in (gate, up, down)),
+             # the replaced operations' own keyword arguments, for the backend to vet
+             "kwargs": {"NN.linear": sorted(set(gate.attrs) | set(up.attrs) | set(down.attrs)),
+                        act.op: sorted(act.attrs), "MoE.expert_weight": sorted(sel.attrs)}}
     return gr.Node(loop.id, "MoE.stacked_experts", [loop.inputs[0], h, w, idx], attrs, None, 1, None)
 
 

@@ -190,6 +190,12 @@ def test_variants_bias_qk_norm_gelu_tied_window_and_rope_scaling():
     ("  mask <- causal_mask_for_input ids past_len window=WINDOW",
      "  mask <- Masking.mask_for_input ids past_len", "causal mask"),
     ("attention q k v mask |>", "attention q k v (Masking.causal_mask q k padding_mask=pos) |>", "padding"),
+    # positions that restart at 0 on every decode step
+    ("  pos <- position_ids ids past_length=past_len", "  pos <- position_ids ids", "rotary positions"),
+    ("  k <- rope k pos theta=THETA", "  k <- rope k pos theta=THETA factor=8.0", "frequency scaling"),
+    # keywords that would change the function
+    ("NN.rmsnorm@attention_norm x eps=EPS", "NN.rmsnorm@attention_norm x eps=EPS offset=1.0", "offset"),
+    ("attention q k v mask |>", "attention q k v mask scale=0.5 |>", "scale"),
 ])
 def test_modules_outside_the_kernels_are_refused(old, new, msg):
     with pytest.raises(fe.LoweringError, match=msg):
@@ -288,6 +294,7 @@ def _moe_variant(old, new):
     (("w, idx <- MoE.softmax_topk_router@router h top_k=TOPK",
       "w, idx <- MoE.softmax_topk_router@router (h * 2.0) top_k=TOPK"), {}, "router"),
     (("mixture h = do", "mixture h = do\n  h <- Tensor.dropout h"), {}, "post-attention norm"),
+    (("  g <- NN.linear@w_gate x dim=width", "  g <- NN.linear@w_gate x dim=width scale=2.0"), {}, "scale"),
 ])
 def test_moe_modules_outside_the_kernels_are_refused(src, cfg, msg):
     text = MOE if src is None else _moe_variant(*src)
