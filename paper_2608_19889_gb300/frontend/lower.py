@@ -359,7 +359,8 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
         raise LoweringError("MLP and output projection widths disagree with the hidden size")
     params = dict(H=H, G=G, d=d, bias=biases.pop(), theta=thetas.pop(), act=act, qk_norm=q_norm is not None,
                   rope_scaling=tuple(sorted(rope_scaling.items())), window=window)
-    eps = {float(n.attrs.get("eps", cfg.get("rms_norm_eps", 1e-6))) for n in (norm1, norm2)}
+    norms = (norm1, norm2) + ((q_norm, k_norm) if q_norm is not None else ())
+    eps = {float(n.attrs.get("eps", cfg.get("rms_norm_eps", 1e-6))) for n in norms}
     paths = {"input_norm": norm1.path, "post_norm": norm2.path, "q": q_lin.path, "k": k_lin.path,
              "v": v_lin.path, "o": o_proj.path}
     if q_norm is not None:

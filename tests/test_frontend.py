@@ -196,6 +196,9 @@ def test_variants_bias_qk_norm_gelu_tied_window_and_rope_scaling():
     # keywords that would change the function
     ("NN.rmsnorm@attention_norm x eps=EPS", "NN.rmsnorm@attention_norm x eps=EPS offset=1.0", "offset"),
     ("attention q k v mask |>", "attention q k v mask scale=0.5 |>", "scale"),
+    # qk-norm with its own epsilon: the kernels use one rms_norm_eps
+    ("  q <- rope q pos theta=THETA", "  q <- NN.rmsnorm@q_norm q eps=0.5\n  q <- rope q pos theta=THETA\n"
+     "  k <- NN.rmsnorm@k_norm k eps=0.5", "epsilon"),
 ])
 def test_modules_outside_the_kernels_are_refused(old, new, msg):
     with pytest.raises(fe.LoweringError, match=msg):
