@@ -13,6 +13,12 @@ checkpoint directory holds for that:
 Only what `axon_model_create` accepts is returned: bf16 and fp32 tensors pass
 through; fp16 tensors are widened to fp32 (exact). Host memory only; the
 create call copies and repacks on the device.
+
+Mixture-of-experts checkpoints: DeepSeek-MoE configs map onto the library's
+expert fields and use its tensor names as they are; Mixtral configs map with
+norm_topk (Mixtral's router takes the softmax of the top-k logits, which is
+the top-k softmax probabilities divided by their sum) and their
+`block_sparse_moe.*` tensors are renamed (`hf_to_library_names`).
 """
 from __future__ import annotations
 
@@ -74,12 +80,31 @@ def read_checkpoint(directory: str) -> dict:
     return read_safetensors(single)
 
 
+def _moe_fields(c: dict, mt: str) -> dict:
+    """Mixture-of-experts fields of the shape dict (empty for dense models)."""
+    if mt == "deepseek":
+        if int(c.get("moe_layer_freq", 1)) != 1:
+            raise ValueError("MoE layers at a stride (moe_layer_freq > 1) are not implemented")
+        if c.get("scoring_func", "softmax") != "softmax" or c.get("topk_method", "greedy") != "greedy":
+            raise ValueError("only softmax scoring with greedy top-k routing is implemented")
+        if not c.get("n_routed_experts"):
+            return {}
+        return dict(n_experts=int(c["n_routed_experts"]), top_k=int(c["num_experts_per_tok"]),
+                    moe_F=int(c["moe_intermediate_size"]), n_shared=int(c.get("n_shared_experts") or 0),
+                    first_dense=int(c.get("first_k_dense_replace", 0)), norm_topk=bool(c.get("norm_topk_prob", False)))
+    if mt == "mixtral":
+        return dict(n_experts=int(c["num_local_experts"]), top_k=int(c["num_experts_per_tok"]),
+                    moe_F=int(c["intermediate_size"]), n_shared=0, first_dense=0, norm_topk=True)
+    return {}
+
+
 def shape_from_hf_config(c: dict) -> dict:
     """The shape dict of `make_config` from an HF config.json of a
-    Llama-family decoder (Llama, Mistral, Qwen2, SmolLM, ...). Raises on a
-    model this library does not implement."""
+    Llama-family decoder (Llama, Mistral, Qwen2, Qwen3, SmolLM, ...) or of a
+    DeepSeek-MoE or Mixtral mixture of experts. Raises on a model this
+    library does not implement."""
     mt = c.get("model_type", "llama")
-    if mt not in ("llama", "mistral", "qwen2"):
+    if mt not in ("llama", "mistral", "qwen2", "qwen3", "deepseek", "mixtral"):
         raise ValueError(f"model_type {mt!r} is not a Llama-family decoder this library implements")
     H = int(c["num_attention_heads"])
     D = int(c["hidden_size"])
@@ -96,6 +121,9 @@ def shape_from_hf_config(c: dict) -> dict:
                  theta=float(theta), eps=float(c.get("rms_norm_eps", 1e-6)))
     if c.get("mlp_bias"):
         raise ValueError("MLP biases are not implemented")
+    if mt == "qwen3":
+        shape["qk_norm"] = True  # per-head RMSNorm of q and k (q_norm / k_norm gains)
+    shape.update(_moe_fields(c, mt))
     act = c.get("hidden_act", "silu")
     if act in ("gelu_pytorch_tanh", "gelu_new"):
         shape["act"] = "gelu_tanh"
@@ -130,9 +158,33 @@ def load_model(directory: str, max_batch: int, max_context: int, **config_kw):
     them to the device. config_kw go to make_config (layout, precision, ...)."""
     from . import axon_model_create, make_config
     with open(os.path.join(directory, "config.json")) as f:
-        shape = shape_from_hf_config(json.load(f))
-    weights = read_checkpoint(directory)
+        hf = json.load(f)
+    shape = shape_from_hf_config(hf)
+    weights = hf_to_library_names(shape, hf.get("model_type", "llama"), read_checkpoint(directory))
     if shape["tie"]:
         weights.pop("lm_head.weight", None)
     cfg = make_config(shape, max_batch=max_batch, max_context=max_context, **config_kw)
     return axon_model_create(cfg, weights), shape
+
+
+def hf_to_library_names(shape: dict, model_type: str, weights: dict) -> dict:
+    """Rename a checkpoint's tensors to the names axon_model_create reads:
+    Mixtral's router and experts (block_sparse_moe.gate -> mlp.gate,
+    experts.{e}.w1 / w3 / w2 -> mlp.experts.{e}.gate_proj / up_proj /
+    down_proj); every other family already uses them."""
+    if model_type != "mixtral":
+        return weights
+    leaf = {"w1": "gate_proj", "w3": "up_proj", "w2": "down_proj"}
+    out = {}
+    for name, t in weights.items():
+        parts = name.split(".")
+        if ".block_sparse_moe." in name:
+            i = parts.index("block_sparse_moe")
+            rest = parts[i + 1:]
+            if len(rest) == 4 and rest[0] == "experts" and rest[2] in leaf:
+                rest = ["experts", rest[1], leaf[rest[2]], rest[3]]
+            elif rest != ["gate", "weight"]:  # the router keeps its leaf name
+                raise ValueError(f"unexpected mixture-of-experts tensor {name}")
+            name = ".".join(parts[:i] + ["mlp"] + rest)
+        out[name] = t
+    return out

@@ -1,6 +1,8 @@
 """Checkpoint loading on the host: the hand-written safetensors reader (single
 file and sharded index, bf16 / fp16 / fp32) against tensors written here, and
-the HF config.json mapping of the Llama-family variants the kernels implement."""
+the HF config.json mapping of the Llama-family variants and the
+mixture-of-experts families (DeepSeek-MoE, Mixtral with its tensor renaming)
+the kernels implement."""
 import json
 import struct
 
@@ -138,3 +140,80 @@ def test_rope_parameters_of_newer_configs_and_default_rope_type():
     assert "rope_factor" not in old_default
     with pytest.raises(ValueError):
         ck.shape_from_hf_config(top)
+
+
+# ------------------------------------------------------ mixture of experts
+DEEPSEEK_MOE_16B = {  # the config.json keys of a DeepSeek-MoE-16B-shaped model
+    "model_type": "deepseek", "num_hidden_layers": 28, "hidden_size": 2048, "num_attention_heads": 16,
+    "num_key_value_heads": 16, "intermediate_size": 10944, "vocab_size": 102400, "rope_theta": 10000.0,
+    "rms_norm_eps": 1e-6, "tie_word_embeddings": False, "attention_bias": False, "hidden_act": "silu",
+    "n_routed_experts": 64, "num_experts_per_tok": 6, "moe_intermediate_size": 1408, "n_shared_experts": 2,
+    "first_k_dense_replace": 1, "moe_layer_freq": 1, "norm_topk_prob": False, "scoring_func": "softmax",
+    "topk_method": "greedy"}
+MIXTRAL = {
+    "model_type": "mixtral", "num_hidden_layers": 2, "hidden_size": 64, "num_attention_heads": 4,
+    "num_key_value_heads": 2, "intermediate_size": 96, "vocab_size": 50, "rope_theta": 1e6, "rms_norm_eps": 1e-5,
+    "num_local_experts": 4, "num_experts_per_tok": 2, "sliding_window": None, "tie_word_embeddings": False}
+
+
+def test_deepseek_moe_config_is_the_moe_workloads_shape():
+    s = ck.shape_from_hf_config(DEEPSEEK_MOE_16B)
+    want = dict(si.MODEL_SHAPES["moe16b"])
+    assert {k: s[k] for k in want} == want
+
+
+@pytest.mark.parametrize("key,value", [("moe_layer_freq", 2), ("scoring_func", "sigmoid"),
+                                       ("topk_method", "group_limited_greedy")])
+def test_deepseek_routing_the_kernels_do_not_implement_is_refused(key, value):
+    with pytest.raises(ValueError):
+        ck.shape_from_hf_config(dict(DEEPSEEK_MOE_16B, **{key: value}))
+
+
+def test_qwen3_has_qk_norm_and_moe_families_without_kernels_are_refused():
+    q3 = {"model_type": "qwen3", "num_hidden_layers": 2, "hidden_size": 64, "num_attention_heads": 4,
+          "num_key_value_heads": 2, "head_dim": 32, "intermediate_size": 96, "vocab_size": 50, "rope_theta": 1e6,
+          "attention_bias": False}
+    s = ck.shape_from_hf_config(q3)
+    assert s["qk_norm"] and not s["bias"] and s["d"] == 32
+    for mt in ("qwen2_moe", "deepseek_v2"):
+        with pytest.raises(ValueError):
+            ck.shape_from_hf_config(dict(q3, model_type=mt))
+
+
+def test_mixtral_config_and_tensor_names():
+    s = ck.shape_from_hf_config(MIXTRAL)
+    assert (s["n_experts"], s["top_k"], s["moe_F"], s["n_shared"], s["first_dense"], s["norm_topk"]) == \
+        (4, 2, 96, 0, 0, True)
+    lib = si.make_weights(s)
+    inv = {"gate_proj": "w1", "up_proj": "w3", "down_proj": "w2"}
+    mixtral = {}
+    for name, t in lib.items():  # the library's names written the way a Mixtral checkpoint stores them
+        p = name.split(".")
+        if ".mlp.gate." in name:
+            name = ".".join(p[:3] + ["block_sparse_moe", "gate", "weight"])
+        elif ".mlp.experts." in name:
+            name = ".".join(p[:3] + ["block_sparse_moe", "experts", p[5], inv[p[6]], "weight"])
+        mixtral[name] = t
+    assert not any(".mlp." in k for k in mixtral)
+    back = ck.hf_to_library_names(s, "mixtral", mixtral)
+    assert set(back) == set(lib) == set(si.weight_shapes(s))
+    assert all(torch.equal(back[k], lib[k]) for k in lib)
+    with pytest.raises(ValueError):
+        ck.hf_to_library_names(s, "mixtral", {"model.layers.0.block_sparse_moe.experts.0.w9.weight": lib[
+            "model.embed_tokens.weight"]})
+
+
+def test_softmax_of_the_top_k_logits_is_the_renormalised_top_k():
+    """Mixtral routes by the softmax of its top-k router logits; the library
+    (and the oracle) take the softmax over all experts, keep the top k and,
+    with norm_topk, divide by their sum. The two are the same weights."""
+    from oracle import decoder as od
+    rng = np.random.Generator(np.random.PCG64(3))
+    h, Wr = rng.normal(size=(9, 16)), rng.normal(size=(8, 16))
+    idx, w, _ = od.moe_route(h, Wr, 2, norm_topk=True)
+    logits = h @ Wr.T
+    top = np.take_along_axis(logits, idx, axis=-1)
+    direct = np.exp(top - top.max(-1, keepdims=True))
+    direct /= direct.sum(-1, keepdims=True)
+    assert np.allclose(w, direct, rtol=1e-13, atol=1e-15)
+    assert np.all(idx == np.argsort(-logits, axis=-1, kind="stable")[:, :2])  # the same experts too
