@@ -130,7 +130,7 @@ def shape_from_hf_config(c: dict) -> dict:
     elif act != "silu":
         raise ValueError(f"hidden_act {act!r} is not implemented")
     window = c.get("sliding_window")
-    if window and mt == "mistral":
+    if window and mt in ("mistral", "mixtral"):
         shape["window"] = int(window)
     elif window and c.get("use_sliding_window", False):
         # Qwen2 windows the layers from max_window_layers on

@@ -184,6 +184,7 @@ def test_mixtral_config_and_tensor_names():
     s = ck.shape_from_hf_config(MIXTRAL)
     assert (s["n_experts"], s["top_k"], s["moe_F"], s["n_shared"], s["first_dense"], s["norm_topk"]) == \
         (4, 2, 96, 0, 0, True)
+    assert "window" not in s and ck.shape_from_hf_config(dict(MIXTRAL, sliding_window=4096))["window"] == 4096
     lib = si.make_weights(s)
     inv = {"gate_proj": "w1", "up_proj": "w3", "down_proj": "w2"}
     mixtral = {}
