@@ -18,7 +18,10 @@ Mixture-of-experts checkpoints: DeepSeek-MoE configs map onto the library's
 expert fields and use its tensor names as they are; Mixtral configs map with
 norm_topk (Mixtral's router takes the softmax of the top-k logits, which is
 the top-k softmax probabilities divided by their sum) and their
-`block_sparse_moe.*` tensors are renamed (`hf_to_library_names`).
+`block_sparse_moe.*` tensors are renamed (`hf_to_library_names`). Phi-3
+checkpoints store q/k/v as one `qkv_proj` and gate/up as one `gate_up_proj`
+matrix; they are split by rows into the library's separate tensors (the
+kernels fuse them again in their own layout at create).
 """
 from __future__ import annotations
 
@@ -104,7 +107,7 @@ def shape_from_hf_config(c: dict) -> dict:
     DeepSeek-MoE or Mixtral mixture of experts. Raises on a model this
     library does not implement."""
     mt = c.get("model_type", "llama")
-    if mt not in ("llama", "mistral", "qwen2", "qwen3", "deepseek", "mixtral"):
+    if mt not in ("llama", "mistral", "qwen2", "qwen3", "deepseek", "mixtral", "phi3"):
         raise ValueError(f"model_type {mt!r} is not a Llama-family decoder this library implements")
     H = int(c["num_attention_heads"])
     D = int(c["hidden_size"])
@@ -123,6 +126,8 @@ def shape_from_hf_config(c: dict) -> dict:
         raise ValueError("MLP biases are not implemented")
     if mt == "qwen3":
         shape["qk_norm"] = True  # per-head RMSNorm of q and k (q_norm / k_norm gains)
+    if mt == "phi3" and float(c.get("partial_rotary_factor", 1.0)) != 1.0:
+        raise ValueError("partial rotary embeddings are not implemented")
     shape.update(_moe_fields(c, mt))
     act = c.get("hidden_act", "silu")
     if act in ("gelu_pytorch_tanh", "gelu_new"):
@@ -130,7 +135,7 @@ def shape_from_hf_config(c: dict) -> dict:
     elif act != "silu":
         raise ValueError(f"hidden_act {act!r} is not implemented")
     window = c.get("sliding_window")
-    if window and mt in ("mistral", "mixtral"):
+    if window and mt in ("mistral", "mixtral", "phi3"):
         shape["window"] = int(window)
     elif window and c.get("use_sliding_window", False):
         # Qwen2 windows the layers from max_window_layers on
@@ -172,6 +177,8 @@ def hf_to_library_names(shape: dict, model_type: str, weights: dict) -> dict:
     Mixtral's router and experts (block_sparse_moe.gate -> mlp.gate,
     experts.{e}.w1 / w3 / w2 -> mlp.experts.{e}.gate_proj / up_proj /
     down_proj); every other family already uses them."""
+    if model_type == "phi3":
+        return _split_phi3(shape, weights)
     if model_type != "mixtral":
         return weights
     leaf = {"w1": "gate_proj", "w3": "up_proj", "w2": "down_proj"}
@@ -187,4 +194,29 @@ def hf_to_library_names(shape: dict, model_type: str, weights: dict) -> dict:
                 raise ValueError(f"unexpected mixture-of-experts tensor {name}")
             name = ".".join(parts[:i] + ["mlp"] + rest)
         out[name] = t
+    return out
+
+
+def _split_phi3(shape: dict, weights: dict) -> dict:
+    """Phi-3's fused matrices split by rows: qkv_proj [(H + 2G) d, D] into
+    q_proj, k_proj, v_proj (in that order); gate_up_proj [2F, D] into
+    gate_proj (first F rows) and up_proj."""
+    H, G, d, F = shape["H"], shape["G"], shape["d"], shape["F"]
+    out = {}
+    for name, t in weights.items():
+        if name.endswith(".self_attn.qkv_proj.weight"):
+            if tuple(t.shape)[0] != (H + 2 * G) * d:
+                raise ValueError(f"{name}: {tuple(t.shape)} rows, expected {(H + 2 * G) * d}")
+            p = name[: -len("qkv_proj.weight")]
+            out[p + "q_proj.weight"] = t[: H * d].contiguous()
+            out[p + "k_proj.weight"] = t[H * d:(H + G) * d].contiguous()
+            out[p + "v_proj.weight"] = t[(H + G) * d:].contiguous()
+        elif name.endswith(".mlp.gate_up_proj.weight"):
+            if tuple(t.shape)[0] != 2 * F:
+                raise ValueError(f"{name}: {tuple(t.shape)} rows, expected {2 * F}")
+            p = name[: -len("gate_up_proj.weight")]
+            out[p + "gate_proj.weight"] = t[:F].contiguous()
+            out[p + "up_proj.weight"] = t[F:].contiguous()
+        else:
+            out[name] = t
     return out

@@ -218,3 +218,35 @@ def test_softmax_of_the_top_k_logits_is_the_renormalised_top_k():
     direct /= direct.sum(-1, keepdims=True)
     assert np.allclose(w, direct, rtol=1e-13, atol=1e-15)
     assert np.all(idx == np.argsort(-logits, axis=-1, kind="stable")[:, :2])  # the same experts too
+
+
+PHI3 = {"model_type": "phi3", "num_hidden_layers": 2, "hidden_size": 64, "num_attention_heads": 4,
+        "num_key_value_heads": 2, "intermediate_size": 96, "vocab_size": 50, "rope_theta": 10000.0,
+        "rms_norm_eps": 1e-5, "sliding_window": 2047, "tie_word_embeddings": False, "hidden_act": "silu"}
+
+
+def test_phi3_fused_matrices_split_into_the_librarys_tensors():
+    s = ck.shape_from_hf_config(PHI3)
+    assert (s["d"], s["window"], s["bias"]) == (16, 2047, False)
+    lib = si.make_weights(s)
+    fused = {}
+    for name, t in lib.items():  # the library's tensors fused the way a Phi-3 checkpoint stores them
+        if ".self_attn.q_proj." in name:
+            p = name.replace("q_proj", "{}")
+            fused[p.format("qkv_proj")] = torch.cat([lib[p.format(x)] for x in ("q_proj", "k_proj", "v_proj")])
+        elif ".mlp.gate_proj." in name:
+            p = name.replace("gate_proj", "{}")
+            fused[p.format("gate_up_proj")] = torch.cat([lib[p.format("gate_proj")], lib[p.format("up_proj")]])
+        elif not any(x in name for x in (".k_proj.", ".v_proj.", ".up_proj.")):
+            fused[name] = t
+    back = ck.hf_to_library_names(s, "phi3", fused)
+    assert set(back) == set(lib) == set(si.weight_shapes(s))
+    assert all(torch.equal(back[k], lib[k]) for k in lib)
+    bad = dict(fused)
+    bad["model.layers.0.mlp.gate_up_proj.weight"] = bad["model.layers.0.mlp.gate_up_proj.weight"][:-1]
+    with pytest.raises(ValueError):
+        ck.hf_to_library_names(s, "phi3", bad)
+    with pytest.raises(ValueError):
+        ck.shape_from_hf_config(dict(PHI3, rope_scaling={"type": "longrope", "short_factor": [1.0], "long_factor": [1.0]}))
+    with pytest.raises(ValueError):
+        ck.shape_from_hf_config(dict(PHI3, partial_rotary_factor=0.5))
