@@ -40,7 +40,7 @@ from dataclasses import dataclass, field
 from typing import Dict, List, Optional
 
 from . import graph as gr
-from .rewrite import ACTIVATIONS as _ACTS, stack_experts
+from .rewrite import ACTIVATIONS as _ACTS, SWIGLU as _SWIGLU, stack_experts
 
 # Operations allowed outside the layer loop and around the cache: they
 # carry positions, masks and cache bookkeeping, which the library keeps on
@@ -62,8 +62,8 @@ _KWARGS = {
     "Positions.rope": {"theta", *_ROPE_SCALING}, "Positions.position_ids": {"past_length"},
     "Masking.causal_mask_for_input": {"window", "padding_mask"}, "Masking.causal_mask": {"window", "padding_mask"},
     "MoE.softmax_topk_router": {"top_k", "normalize", "dim"}, "MoE.expert_weight": set(),
-    "Tensor.zeros_like": set(), "add": set(), "mul": set(),
-    **{a: set() for a in _ACTS},
+    "Tensor.zeros_like": set(), "add": set(), "mul": set(), "Attention.split_qkv": {"heads", "kv_heads"},
+    **{a: set() for a in _ACTS}, **{a: set() for a in _SWIGLU},
 }
 
 
@@ -103,20 +103,49 @@ class LoweredDecoder:
     # role -> module path pattern ({var} per layer, {e} per expert); the roles
     # of a second (mixture-of-experts) layer loop under "moe_layers."
     paths: Dict[str, str] = field(default_factory=dict)
+    # library name -> (first row, end row) of the module tensor it is cut
+    # from: q/k/v of a fused projection split by Attention.split_qkv, gate
+    # and up of a fused projection under swiglu
+    rows: Dict[str, tuple] = field(default_factory=dict)
 
     def module_weights(self, library_named: dict) -> dict:
-        """Re-key a library-named checkpoint under the module's own paths."""
-        return {self.names[k]: v for k, v in library_named.items()}
+        """Re-key a library-named checkpoint under the module's own paths
+        (row slices of one module tensor concatenated in row order)."""
+        out, parts = {}, {}
+        for k, v in library_named.items():
+            if k in self.rows:
+                parts.setdefault(self.names[k], []).append((self.rows[k][0], v))
+            else:
+                out[self.names[k]] = v
+        for mod, ps in parts.items():
+            ts = [t for _, t in sorted(ps, key=lambda x: x[0])]
+            out[mod] = _concat_rows(ts)
+        return out
 
     def library_weights(self, module_named: dict) -> dict:
         """Re-key a checkpoint stored under the module's paths to the names
-        axon_model_create expects; every expected tensor must be present."""
+        axon_model_create expects (cutting fused tensors by rows); every
+        expected tensor must be present."""
         out = {}
         for lib, mod in self.names.items():
             if mod not in module_named:
                 raise LoweringError(f"checkpoint has no tensor {mod!r} (needed as {lib})")
-            out[lib] = module_named[mod]
+            t = module_named[mod]
+            if lib in self.rows:
+                a, b = self.rows[lib]
+                if t.shape[0] < b:
+                    raise LoweringError(f"{mod}: {t.shape[0]} rows, {lib} needs rows {a}..{b}")
+                t = t[a:b]
+            out[lib] = t
         return out
+
+
+def _concat_rows(ts):
+    if hasattr(ts[0], "detach"):  # torch tensors
+        import torch
+        return torch.cat(ts, 0)
+    import numpy as np
+    return np.concatenate(ts, 0)
 
 
 class _Match:
@@ -162,11 +191,19 @@ class _Layer:
     mlp: str  # "dense" or "moe"
     F: int = 0  # dense MLP width
     moe: dict = field(default_factory=dict)  # E, top_k, Fe, Fs, norm_topk
+    rows: dict = field(default_factory=dict)  # role -> row range of a fused projection
 
 
 def _gated_mlp(m: _Match, down_ref, what: str):
-    """down(act(gate(h)) * up(h)): (gate, up, down, activation, h)."""
+    """down(act(gate(h)) * up(h)), or down(swiglu(gate_up(h))) with gate and
+    up the two halves of one projection: (gate, up, down, activation, h,
+    fused)."""
     down = m.node(down_ref, {"NN.linear"}, f"{what} output")
+    src = m.byid.get(down.inputs[0].node) if isinstance(down.inputs[0], gr.Ref) else None
+    if src is not None and src.op in _SWIGLU:
+        sw = m.node(down.inputs[0])
+        fused = m.node(sw.inputs[0], {"NN.linear"}, f"{what} fused gate/up projection")
+        return fused, fused, down, "silu", fused.inputs[0], True
     mul = m.node(down.inputs[0], {"mul"}, f"{what} product")
     pa, pb = (m.byid.get(r.node) if isinstance(r, gr.Ref) else None for r in mul.inputs)
     if pa is not None and pa.op in _ACTS:
@@ -178,7 +215,19 @@ def _gated_mlp(m: _Match, down_ref, what: str):
     gate = m.node(act_n.inputs[0], {"NN.linear"}, f"{what} gate projection")
     if gate.inputs[0] != up.inputs[0]:
         raise LoweringError("gate and up projections must read the same normalised input")
-    return gate, up, down, _ACTS[act_n.op], gate.inputs[0]
+    return gate, up, down, _ACTS[act_n.op], gate.inputs[0], False
+
+
+def _mlp_width(gate, up, fused, what):
+    """Width F of a gated MLP (half the fused projection's width)."""
+    F = int(gate.attrs.get("dim", 0) or 0)
+    if fused:
+        if F <= 0 or F % 2:
+            raise LoweringError(f"{what}: the fused gate/up projection's width must be even (two halves)")
+        return F // 2
+    if int(up.attrs.get("dim", 0) or 0) != F:
+        raise LoweringError(f"{what}: gate and up projection widths differ")
+    return F
 
 
 def _moe_mlp(m: _Match, mlp_ref):
@@ -252,10 +301,12 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
     # MLP: down(act(gate(h2)) * up(h2)), or the mixture of experts
     moe = _moe_mlp(m, mlp_ref)
     if moe is None:
-        gate, up, down, act, h2 = _gated_mlp(m, mlp_ref, "MLP")
+        gate, up, down, act, h2, mlp_fused = _gated_mlp(m, mlp_ref, "MLP")
     else:
         stacked, router, shared, h2 = moe
-        act = _ACTS.get(stacked.attrs.get("act"))
+        act = "silu" if stacked.attrs.get("fused") else _ACTS.get(stacked.attrs.get("act"))
+        if act is None:
+            raise LoweringError(f"expert activation {stacked.attrs.get('act')} has no kernel")
         if shared is not None and shared[3] != act:
             raise LoweringError("the shared and the routed experts must use one activation")
     norm2 = m.node(h2, {"NN.rmsnorm"}, "post-attention norm")
@@ -287,23 +338,41 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
     window = int(mask.attrs.get("window", 0) or 0)
     rope_scaling = {}
 
-    def qk_chain(ref, what):
-        """rope([rmsnorm](reshape_heads(linear(h1)))): (linear, heads, norm or None, rope node)."""
-        rope = m.node(ref, {"Positions.rope"}, f"{what} rotary positions")
-        inner = m.node(rope.inputs[0], {"Attention.reshape_heads", "NN.rmsnorm"}, f"{what} heads")
-        qn = None
-        if inner.op == "NN.rmsnorm":
-            qn = inner
-            inner = m.node(inner.inputs[0], {"Attention.reshape_heads"}, f"{what} heads")
-        lin = m.node(inner.inputs[0], {"NN.linear"}, f"{what} projection")
-        return lin, int(inner.attrs.get("heads", 0)), qn, rope
+    heads_ops = {"Attention.reshape_heads", "Attention.split_qkv"}
+    splits = []  # (split node, output index) of a fused q/k/v projection
 
-    q_lin, H, q_norm, q_rope = qk_chain(q_ref, "query")
-    k_lin, G, k_norm, k_rope = qk_chain(k_ref, "key")
-    v_heads = m.node(v_ref, {"Attention.reshape_heads"}, "value heads")
-    v_lin = m.node(v_heads.inputs[0], {"NN.linear"}, "value projection")
-    if int(v_heads.attrs.get("heads", 0)) != G:
+    def heads_of(ref, what, index):
+        """The projection behind reshape_heads, or behind output `index` of
+        split_qkv (q 0, k 1, v 2): (linear, heads)."""
+        inner = m.node(ref, heads_ops, f"{what} heads")
+        if inner.op == "Attention.split_qkv":
+            if ref.index != index:
+                raise LoweringError(f"{what}: Attention.split_qkv gives q, k, v in that order")
+            splits.append(inner)
+            n = int(inner.attrs.get("heads" if index == 0 else "kv_heads", 0) or 0)
+        else:
+            n = int(inner.attrs.get("heads", 0) or 0)
+        return m.node(inner.inputs[0], {"NN.linear"}, f"{what} projection"), n
+
+    def qk_chain(ref, what, index):
+        """rope([rmsnorm](heads(linear(h1)))): (linear, heads, norm or None, rope node)."""
+        rope = m.node(ref, {"Positions.rope"}, f"{what} rotary positions")
+        qn = None
+        src = m.byid.get(rope.inputs[0].node) if isinstance(rope.inputs[0], gr.Ref) else None
+        inner_ref = rope.inputs[0]
+        if src is not None and src.op == "NN.rmsnorm":
+            qn = m.node(inner_ref)
+            inner_ref = qn.inputs[0]
+        lin, n = heads_of(inner_ref, what, index)
+        return lin, n, qn, rope
+
+    q_lin, H, q_norm, q_rope = qk_chain(q_ref, "query", 0)
+    k_lin, G, k_norm, k_rope = qk_chain(k_ref, "key", 1)
+    v_lin, Gv = heads_of(v_ref, "value", 2)
+    if Gv != G:
         raise LoweringError("keys and values must have the same number of heads")
+    if splits and (len(splits) != 3 or len({n.id for n in splits}) != 1):
+        raise LoweringError("q, k and v must all come from one Attention.split_qkv, or none")
     if not (q_lin.inputs[0] == k_lin.inputs[0] == v_lin.inputs[0]):
         raise LoweringError("q, k and v must project the same normalised input")
     norm1 = m.node(q_lin.inputs[0], {"NN.rmsnorm"}, "input norm")
@@ -349,12 +418,20 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
     for n in (q_lin, k_lin, v_lin):
         if _bool(n.attrs.get("transpose")):
             raise LoweringError(f"{n.path}: the kernels take [out, in] matrices here")
-    qdim = int(q_lin.attrs.get("dim", 0))
-    if not D or not qdim or not H or not G or qdim % H:
-        raise LoweringError("hidden size, head counts and projection widths must be known")
-    d = qdim // H
-    if int(k_lin.attrs.get("dim", 0)) != G * d or int(v_lin.attrs.get("dim", 0)) != G * d:
-        raise LoweringError("k and v widths must be kv_heads * head_dim")
+    rows = {}
+    if splits:  # one fused projection [(H + 2G) d, D]: q, k, v rows in that order
+        qkv = int(q_lin.attrs.get("dim", 0) or 0)
+        if not D or not H or not G or not qkv or qkv % (H + 2 * G):
+            raise LoweringError("the fused q/k/v projection's width must be (heads + 2 kv_heads) * head_dim")
+        d = qkv // (H + 2 * G)
+        rows.update(q=(0, H * d), k=(H * d, (H + G) * d), v=((H + G) * d, (H + 2 * G) * d))
+    else:
+        qdim = int(q_lin.attrs.get("dim", 0))
+        if not D or not qdim or not H or not G or qdim % H:
+            raise LoweringError("hidden size, head counts and projection widths must be known")
+        d = qdim // H
+        if int(k_lin.attrs.get("dim", 0)) != G * d or int(v_lin.attrs.get("dim", 0)) != G * d:
+            raise LoweringError("k and v widths must be kv_heads * head_dim")
     if int(o_proj.attrs.get("dim", D)) != D:
         raise LoweringError("MLP and output projection widths disagree with the hidden size")
     params = dict(H=H, G=G, d=d, bias=biases.pop(), theta=thetas.pop(), act=act, qk_norm=q_norm is not None,
@@ -366,18 +443,26 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
     if q_norm is not None:
         paths.update(q_norm=q_norm.path, k_norm=k_norm.path)
     layer = _Layer(loop, params, eps, paths, "dense" if moe is None else "moe")
+    layer.rows = rows
     if moe is None:
-        F = int(gate.attrs.get("dim", 0))
-        if int(up.attrs.get("dim", 0)) != F or int(down.attrs.get("dim", 0)) != D:
+        F = _mlp_width(gate, up, mlp_fused, "MLP")
+        if int(down.attrs.get("dim", 0)) != D:
             raise LoweringError("MLP and output projection widths disagree with the hidden size")
         layer.F = F
         paths.update(gate=gate.path, up=up.path, down=down.path)
+        if mlp_fused:
+            rows.update(gate=(0, F), up=(F, 2 * F))
     else:
         layer.moe = _moe_params(stacked, router, shared, D)
         paths.update(router=router.path, expert_gate=stacked.attrs["gate"], expert_up=stacked.attrs["up"],
                      expert_down=stacked.attrs["down"])
+        Fe, Fs = layer.moe["Fe"], layer.moe["Fs"]
+        if stacked.attrs.get("fused"):
+            rows.update(expert_gate=(0, Fe), expert_up=(Fe, 2 * Fe))
         if shared is not None:
             paths.update(shared_gate=shared[0].path, shared_up=shared[1].path, shared_down=shared[2].path)
+            if shared[5]:
+                rows.update(shared_gate=(0, Fs), shared_up=(Fs, 2 * Fs))
     var = "{" + loop.attrs["var"] + "}"
     for role, p in paths.items():
         if not p:
@@ -406,8 +491,8 @@ def _moe_params(stacked: gr.Node, router: gr.Node, shared, D: int) -> dict:
         raise LoweringError("the router's width must be the number of experts")
     Fs = 0
     if shared is not None:
-        Fs = int(shared[0].attrs.get("dim", 0))
-        if int(shared[1].attrs.get("dim", 0)) != Fs or int(shared[2].attrs.get("dim", 0)) != D:
+        Fs = _mlp_width(shared[0], shared[1], shared[5], "shared experts")
+        if int(shared[2].attrs.get("dim", 0)) != D:
             raise LoweringError("shared experts' widths disagree with each other or with the hidden size")
         if Fs <= 0 or Fs % Fe:
             raise LoweringError("the shared experts' width must be a multiple of one expert's width")
@@ -514,6 +599,7 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
               ("mlp.shared_experts.down_proj.weight", "shared_down")]
     expert = [("gate_proj.weight", "expert_gate"), ("up_proj.weight", "expert_up"), ("down_proj.weight", "expert_down")]
     paths = {"embed": emb.path, "final_norm": fnorm.path, "head": head.path}
+    rows = {}
     for k, ly in enumerate(layers):
         var = "{" + ly.loop.attrs["var"] + "}"
         per_layer = attn + (dense if ly.mlp == "dense" else [("mlp.gate.weight", "router")] +
@@ -522,11 +608,16 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
         for l in range(ly.loop.attrs["start"], ly.loop.attrs["stop"]):
             for lib, role in per_layer:
                 leaf = lib.rsplit(".", 1)[1]
-                names[f"model.layers.{l}.{lib}"] = ly.paths[role].replace(var, str(l)) + "." + leaf
+                name = f"model.layers.{l}.{lib}"
+                names[name] = ly.paths[role].replace(var, str(l)) + "." + leaf
+                if role in ly.rows:
+                    rows[name] = ly.rows[role]
             if ly.mlp == "moe":
                 evar = ly.moe["evar"]
                 for e in range(ly.moe["E"]):
                     for lib, role in expert:
-                        names[f"model.layers.{l}.mlp.experts.{e}.{lib}"] = (
-                            ly.paths[role].replace(var, str(l)).replace(evar, str(e)) + ".weight")
-    return LoweredDecoder(shape, names, paths)
+                        name = f"model.layers.{l}.mlp.experts.{e}.{lib}"
+                        names[name] = ly.paths[role].replace(var, str(l)).replace(evar, str(e)) + ".weight"
+                        if role in ly.rows:
+                            rows[name] = ly.rows[role]
+    return LoweredDecoder(shape, names, paths, rows)

@@ -18,7 +18,8 @@ feeds only the expert-weight selection and the parameter paths, the
 accumulator is only added to -- and replaces the loop node by
 
     MoE.stacked_experts(init, h, w, idx)   attrs: experts E, dim (expert
-        width), act, var, gate / up / down path patterns with {var}, and
+        width), act, var, gate / up / down path patterns with {var}, fused
+        (gate and up as the two halves of one projection under swiglu), and
         the replaced operations' keyword names (kwargs)
 
 whose value is init + sum_e expert_weight(w, idx, e) * ffn_e(h): the
@@ -36,6 +37,9 @@ from . import graph as gr
 # gate activations of the gated MLP the kernels implement (op -> kernel name)
 ACTIVATIONS = {"Act.silu": "silu", "Activations.silu": "silu", "Act.gelu_tanh": "gelu_tanh",
                "Activations.gelu_new": "gelu_tanh", "Act.gelu_new": "gelu_tanh", "Activations.gelu_tanh": "gelu_tanh"}
+# swiglu of one fused projection z of width 2F: silu(z[:F]) * z[F:] (gate
+# half first), the MLP idiom `linear@up |> swiglu |> linear@down`
+SWIGLU = {"Act.swiglu", "Activations.swiglu"}
 
 
 def _other(pair, ref):
@@ -89,17 +93,24 @@ def _expert_loop(loop: gr.Node) -> Optional[gr.Node]:
     down = inner(ffn_ref, {"NN.linear"})
     if down is None:
         return None
-    prod = inner(down.inputs[0], {"mul"})
-    if prod is None:
-        return None
-    a, b = (inner(r, set(ACTIVATIONS)) for r in prod.inputs)
-    act, up_ref = (a, prod.inputs[1]) if a is not None else (b, prod.inputs[0])
-    if act is None:
-        return None
-    gate = inner(act.inputs[0], {"NN.linear"})
-    up = inner(up_ref, {"NN.linear"})
-    if gate is None or up is None or gate.inputs[0] != up.inputs[0]:
-        return None
+    sw = inner(down.inputs[0], SWIGLU)
+    if sw is not None:  # one fused gate/up projection
+        act = prod = sw
+        gate = up = inner(sw.inputs[0], {"NN.linear"})
+        if gate is None:
+            return None
+    else:
+        prod = inner(down.inputs[0], {"mul"})
+        if prod is None:
+            return None
+        a, b = (inner(r, set(ACTIVATIONS)) for r in prod.inputs)
+        act, up_ref = (a, prod.inputs[1]) if a is not None else (b, prod.inputs[0])
+        if act is None:
+            return None
+        gate = inner(act.inputs[0], {"NN.linear"})
+        up = inner(up_ref, {"NN.linear"})
+        if gate is None or up is None or gate.inputs[0] != up.inputs[0]:
+            return None
     h = gate.inputs[0]
     if not isinstance(h, gr.Ref) or h.node in byid:
         return None  # the experts read a value computed before the loop
@@ -109,9 +120,13 @@ def _expert_loop(loop: gr.Node) -> Optional[gr.Node]:
     used = {y_in.node, acc.id, term.id, sel.id, down.id, prod.id, act.id, gate.id, up.id}
     if set(byid) != used:
         return None  # anything else in the body: not a plain sum over experts
-    attrs = {"experts": loop.attrs["stop"], "var": var, "dim": gate.attrs.get("dim"), "act": act.op,
+    fused = sw is not None
+    dim = gate.attrs.get("dim")
+    if fused:
+        dim = dim // 2 if isinstance(dim, int) and dim % 2 == 0 else None
+    attrs = {"experts": loop.attrs["stop"], "var": var, "dim": dim, "act": act.op, "fused": fused,
              "gate": gate.path, "up": up.path, "down": down.path, "down_dim": down.attrs.get("dim"),
-             "up_dim": up.attrs.get("dim"),
+             "up_dim": dim if fused else up.attrs.get("dim"),
              "bias": any(bool(n.attrs.get("bias")) or bool(n.attrs.get("transpose")) for n in (gate, up, down)),
              # the replaced operations' own keyword arguments, for the backend to vet
              "kwargs": {"NN.linear": sorted(set(gate.attrs) | set(up.attrs) | set(down.attrs)),

@@ -18,6 +18,9 @@ meaning in the paper's built-ins (Sec. Built-In Libraries):
                                           positions <= the query's (and > p - window),
                                           query head h on kv head floor(h / (H/G))
   Act.silu / Act.gelu_tanh                z / (1 + e^-z); tanh form of gelu
+  Act.swiglu z                            silu(z[.., :F]) * z[.., F:], F = width / 2
+  Attention.split_qkv t heads kv_heads    rows of t cut into q (heads * d), k and v
+                                          (kv_heads * d each), each split into heads
   MoE.softmax_topk_router                 p = softmax(x Wr^T); the top_k experts by p
                                           (lower index first on ties) and their p,
                                           divided by their sum with normalize=true
@@ -125,6 +128,14 @@ class GraphEval:
         if op in ("Act.gelu_tanh", "Act.gelu_new", "Activations.gelu_new"):
             z = ins[0]
             return 0.5 * z * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (z + 0.044715 * z ** 3)))
+        if op in ("Act.swiglu", "Activations.swiglu"):
+            return self._swiglu(ins[0])
+        if op == "Attention.split_qkv":
+            t, H, G = ins[0], int(at["heads"]), int(at["kv_heads"])
+            d = t.shape[-1] // (H + 2 * G)
+            q, k, v = t[..., : H * d], t[..., H * d:(H + G) * d], t[..., (H + G) * d:]
+            return (q.reshape(q.shape[:-1] + (H, d)), k.reshape(k.shape[:-1] + (G, d)),
+                    v.reshape(v.shape[:-1] + (G, d)))
         if op == "Tensor.zeros_like":
             return np.zeros_like(ins[0])
         if op == "MoE.softmax_topk_router":
@@ -177,16 +188,25 @@ class GraphEval:
             w = w / w.sum(axis=-1, keepdims=True)
         return w, idx
 
+    @staticmethod
+    def _swiglu(z):
+        F = z.shape[-1] // 2
+        g = z[..., :F]
+        return g / (1.0 + np.exp(-g)) * z[..., F:]
+
     def _stacked(self, ins, at, lv):
         init, h, w, idx = ins
-        act = {"Act.silu": lambda z: z / (1.0 + np.exp(-z))}.get(at["act"])
-        if act is None:
-            raise NotImplementedError(at["act"])
         y = np.array(init, dtype=np.float64)
         for e in range(int(at["experts"])):
             inner = dict(lv)
             inner[at["var"]] = e
-            ffn = (act(h @ self._w(at["gate"], inner).T) * (h @ self._w(at["up"], inner).T)) @ self._w(at["down"],
-                                                                                                      inner).T
+            if at.get("fused"):
+                u = self._swiglu(h @ self._w(at["gate"], inner).T)
+            elif at["act"] == "Act.silu":
+                g = h @ self._w(at["gate"], inner).T
+                u = g / (1.0 + np.exp(-g)) * (h @ self._w(at["up"], inner).T)
+            else:
+                raise NotImplementedError(at["act"])
+            ffn = u @ self._w(at["down"], inner).T
             y = y + np.sum(np.where(idx == e, w, 0.0), axis=-1, keepdims=True) * ffn
         return y

@@ -335,8 +335,71 @@ def test_mask_built_in_the_layer_is_plumbing_with_its_window():
     assert low.shape["window"] == 5 and low.names == fe.compile_decoder(LLAMA, CFG).names
 
 
-@pytest.mark.parametrize("case", ["llama", "llama_variants_window", "llama_layer_mask", "moe",
-                                  "moe_normalised_all_moe", "moe_shared_first"])
+def _llama_fused(bias=True):
+    """The attention's q, k, v as one projection cut by Attention.split_qkv,
+    and the MLP in the composition idiom linear@up |> swiglu |> linear@down."""
+    src = LLAMA.replace(
+        "  q <- NN.linear@wq h dim=(HEADS * HEAD_DIM) |> reshape_heads heads=HEADS\n"
+        "  k <- NN.linear@wk h dim=(KV_HEADS * HEAD_DIM) |> reshape_heads heads=KV_HEADS\n"
+        "  v <- NN.linear@wv h dim=(KV_HEADS * HEAD_DIM) |> reshape_heads heads=KV_HEADS\n",
+        f"  qkv <- NN.linear@wqkv h dim=((HEADS + 2 * KV_HEADS) * HEAD_DIM){' bias=true' if bias else ''}\n"
+        "  q, k, v <- Attention.split_qkv qkv heads=HEADS kv_heads=KV_HEADS\n")
+    src = src.replace("  g <- NN.linear@w1 x dim=FFN\n  u <- NN.linear@w3 x dim=FFN\n"
+                      "  return Act.silu g * u |> NN.linear@w2 dim=HIDDEN",
+                      "  return NN.linear@w13 x dim=(2 * FFN) |> Act.swiglu |> NN.linear@w2 dim=HIDDEN")
+    assert "split_qkv" in src and "swiglu" in src
+    return src
+
+
+def _moe_fused():
+    """Experts and shared MLP in the swiglu idiom (one gate/up projection each)."""
+    src = MOE.replace("gated x width = do\n  g <- NN.linear@w_gate x dim=width\n  u <- NN.linear@w_up x dim=width\n"
+                      "  return Act.silu g * u |> NN.linear@w_down dim=HIDDEN",
+                      "gated x width = NN.linear@w_gate_up x dim=(2 * width) |> Act.swiglu |> NN.linear@w_down dim=HIDDEN")
+    assert "w_gate_up" in src
+    return src
+
+
+def test_fused_projections_map_to_row_ranges():
+    low = fe.compile_decoder(_llama_fused(), CFG)
+    assert low.shape["bias"] and (low.shape["H"], low.shape["G"], low.shape["d"], low.shape["F"]) == (4, 2, 32, 192)
+    assert set(low.names) == set(si.weight_shapes(low.shape))
+    p = "model.layers.1."
+    assert low.names[p + "self_attn.k_proj.weight"] == "layers.1.attention.wqkv.weight"
+    assert low.rows[p + "self_attn.q_proj.weight"] == (0, 128)
+    assert low.rows[p + "self_attn.k_proj.bias"] == (128, 192)
+    assert low.rows[p + "self_attn.v_proj.weight"] == (192, 256)
+    assert (low.rows[p + "mlp.gate_proj.weight"], low.rows[p + "mlp.up_proj.weight"]) == ((0, 192), (192, 384))
+    lib = {k: np.full(tuple(v), float(i)) for i, (k, v) in enumerate(si.weight_shapes(low.shape).items())}
+    mod = low.module_weights(lib)
+    assert mod["layers.1.attention.wqkv.weight"].shape == (256, 128)
+    back = low.library_weights(mod)
+    assert set(back) == set(lib) and all(np.array_equal(back[k], lib[k]) for k in lib)
+    lowm = fe.compile_decoder(_moe_fused(), MOE_CFG)
+    assert set(lowm.names) == set(si.weight_shapes(lowm.shape)) and lowm.shape["moe_F"] == 16
+    assert lowm.rows["model.layers.2.mlp.experts.4.up_proj.weight"] == (16, 32)
+    assert lowm.rows["model.layers.1.mlp.shared_experts.up_proj.weight"] == (32, 64)
+    assert lowm.rows["model.layers.0.mlp.up_proj.weight"] == (48, 96)
+
+
+@pytest.mark.parametrize("old,new,msg", [
+    ("dim=((HEADS + 2 * KV_HEADS) * HEAD_DIM)", "dim=((HEADS + 2 * KV_HEADS) * HEAD_DIM + 1)", "fused q/k/v"),
+    ("dim=(2 * FFN)", "dim=(2 * FFN + 1)", "even"),
+    ("  q, k, v <- Attention.split_qkv qkv heads=HEADS kv_heads=KV_HEADS\n",
+     "  q, k, v0 <- Attention.split_qkv qkv heads=HEADS kv_heads=KV_HEADS\n"
+     "  v <- NN.linear@wv h dim=(KV_HEADS * HEAD_DIM) bias=true |> reshape_heads heads=KV_HEADS\n", "split_qkv"),
+    ("  q, k, v <- Attention.split_qkv qkv heads=HEADS kv_heads=KV_HEADS\n",
+     "  k, q, v <- Attention.split_qkv qkv heads=HEADS kv_heads=KV_HEADS\n", "order"),
+])
+def test_fused_projections_that_do_not_fit_are_refused(old, new, msg):
+    src = _llama_fused()
+    assert old in src
+    with pytest.raises(fe.LoweringError, match=msg):
+        fe.compile_decoder(src.replace(old, new), CFG)
+
+
+@pytest.mark.parametrize("case", ["llama", "llama_variants_window", "llama_layer_mask", "llama_fused", "moe",
+                                  "moe_normalised_all_moe", "moe_shared_first", "moe_fused"])
 def test_lowered_modules_compute_what_the_oracle_computes(case):
     """The module's own Graph IR on its own parameter paths against the
     oracle on the lowered shape and the re-keyed checkpoint (float64 both):
@@ -345,6 +408,8 @@ def test_lowered_modules_compute_what_the_oracle_computes(case):
     src, cfg = {"llama": (LLAMA, dict(CFG, num_hidden_layers=2)),
                 "llama_variants_window": (_llama_variants(), dict(CFG, sliding_window=3)),
                 "llama_layer_mask": (_llama_layer_mask(), CFG),
+                "llama_fused": (_llama_fused(), CFG),
+                "moe_fused": (_moe_fused(), dict(MOE_CFG, norm_topk_prob=True)),
                 "moe": (MOE, MOE_CFG),
                 "moe_normalised_all_moe": (MOE, dict(MOE_CFG, norm_topk_prob=True, first_k_dense_replace=0)),
                 "moe_shared_first": (_moe_shared_first(), dict(MOE_CFG, norm_topk_prob=True))}[case]
