@@ -4,10 +4,17 @@ Test infrastructure for the Axon-subset front end: it runs a module's Graph
 IR node by node on its own parameter paths, so a test can check that what a
 module states (before or after the stacked-experts rewrite) is the function
 the lowered model computes -- the oracle run on the checkpoint re-keyed
-through the lowering's name map. It covers a prompt pass from an empty
-cache (the cache operations pass the new keys and values through) and the
+through the lowering's name map. It runs a pass over new tokens after the
+ones a cache already holds (a prompt from an empty cache, then decode
+steps), with the cache the module threads through its layer loop, and the
 operations the decoder modules use; each follows the library operation's
 meaning in the paper's built-ins (Sec. Built-In Libraries):
+
+  Cache.past_length / prepare / index     tokens cached; the work cache; layer i's
+  Cache.update / append                   (K, V) so far; keys and values appended
+                                          along the sequence; the layer's new entry
+  Masking.causal_mask_for_input / causal_mask
+                                          causal (and windowed) over cached + new keys
 
   NN.embedding / NN.rmsnorm / NN.linear   rows of E; x / sqrt(mean x^2 + eps) * g;
                                           x W^T (+ b), W stored [out, in]
@@ -42,10 +49,17 @@ class GraphEval:
     def __init__(self, weights: dict):
         self.W = {k: np.asarray(v, dtype=np.float64) for k, v in weights.items()}
 
-    def run(self, g: gr.Graph, ids) -> list:
+    def run(self, g: gr.Graph, ids, past=None) -> list:
+        """The entry's outputs for new tokens ids [B, S] after `past` (None:
+        empty; else the cache of the previous run, see next_past)."""
         ids = np.asarray(ids, dtype=np.int64)
         env: dict = {}
-        return self._graph(g, [ids, None], env, {})
+        return self._graph(g, [ids, past], env, {})
+
+    @staticmethod
+    def next_past(work, ids):
+        """The cache after a run that returned `work` for new tokens ids."""
+        return {"layers": dict(enumerate(work["out"])), "len": work["len"] + np.asarray(ids).shape[-1]}
 
     # ------------------------------------------------------------ plumbing
     def _graph(self, g, args, env, loopvars):
@@ -104,18 +118,30 @@ class GraphEval:
             x = ins[0]
             return x.reshape(x.shape[:-2] + (-1,))
         if op == "Cache.past_length":
-            return 0
+            return 0 if ins[0] is None else ins[0]["len"]
         if op == "Positions.position_ids":
             ids = ins[0]
             return np.broadcast_to(np.arange(ids.shape[-1]) + int(at.get("past_length") or 0), ids.shape)
         if op in ("Masking.causal_mask_for_input", "Masking.causal_mask"):
             if at.get("padding_mask") is not None:
                 raise NotImplementedError("padding masks")
-            return {"window": int(at.get("window", 0) or 0)}
-        if op in ("Cache.prepare", "Cache.index", "Cache.append"):
-            return None
+            if op == "Masking.causal_mask":  # from q and k: the keys beyond the queries are cached ones
+                return {"window": int(at.get("window", 0) or 0), "past": ins[1].shape[1] - ins[0].shape[1]}
+            return {"window": int(at.get("window", 0) or 0), "past": int(ins[1] or 0)}
+        if op == "Cache.prepare":
+            past = ins[0]
+            return {"in": dict(past["layers"]) if past else {}, "out": [], "len": past["len"] if past else 0}
+        if op == "Cache.index":
+            return ins[0]["in"].get(int(ins[1]))
+        if op == "Cache.append":
+            work = ins[0]
+            return dict(work, out=work["out"] + [ins[1]])
         if op == "Cache.update":
-            return ins[1], ins[2], None
+            kv, k, v = ins
+            if kv is not None:
+                k = np.concatenate([kv[0], k], axis=1)
+                v = np.concatenate([kv[1], v], axis=1)
+            return k, v, (k, v)
         if op == "Positions.rope":
             return self._rope(ins[0], ins[1], float(at["theta"]), at)
         if op == "Attention.attention":
@@ -162,11 +188,12 @@ class GraphEval:
     def _attention(q, k, v, mask):
         B, S, H, d = q.shape
         G = k.shape[2]
-        t = np.arange(S)
-        keep = t[None, :] <= t[:, None]
+        tq = mask.get("past", 0) + np.arange(S)  # query positions after the cached keys
+        tk = np.arange(k.shape[1])
+        keep = tk[None, :] <= tq[:, None]
         W = mask.get("window", 0)
         if W > 0:
-            keep &= t[None, :] > t[:, None] - W
+            keep &= tk[None, :] > tq[:, None] - W
         out = np.empty_like(q)
         for b in range(B):
             for h in range(H):

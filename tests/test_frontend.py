@@ -402,9 +402,11 @@ def test_fused_projections_that_do_not_fit_are_refused(old, new, msg):
                                   "moe_normalised_all_moe", "moe_shared_first", "moe_fused"])
 def test_lowered_modules_compute_what_the_oracle_computes(case):
     """The module's own Graph IR on its own parameter paths against the
-    oracle on the lowered shape and the re-keyed checkpoint (float64 both):
-    the lowering keeps the module's meaning. For MoE modules both the literal
-    loop over experts and its stacked-experts rewrite are evaluated."""
+    oracle on the lowered shape and the re-keyed checkpoint (float64 both),
+    for a prompt and then three KV-cached decode steps through the cache the
+    module threads: the lowering keeps the module's meaning. For MoE modules
+    both the literal loop over experts and its stacked-experts rewrite are
+    evaluated."""
     src, cfg = {"llama": (LLAMA, dict(CFG, num_hidden_layers=2)),
                 "llama_variants_window": (_llama_variants(), dict(CFG, sliding_window=3)),
                 "llama_layer_mask": (_llama_layer_mask(), CFG),
@@ -423,19 +425,31 @@ def test_lowered_modules_compute_what_the_oracle_computes(case):
     lib = si.weights_as_f32_numpy(w)
     mod = low.module_weights(lib)
     ids = si.make_ids(2, 7, low.shape["V"], seed=12)
+    fed = si.make_ids(2, 3, low.shape["V"], seed=13)  # the decode steps' input tokens
     o = oracle_for(low.shape, w)
-    ref = o.prefill(ids, o.new_contiguous_cache(2, 8))
     g = fe.build_graph(sx.parse_module(src), cfg)
     graphs = [g]
     if "moe" in case:
         g2 = fe.build_graph(sx.parse_module(src), cfg)
         assert rw.stack_experts(g2) == 1
         graphs.append(g2)
-    for gg in graphs:
-        got = GraphEval(mod).run(gg, ids)[0]
+
+    def close(got, ref):
         assert got.shape == ref.shape
         err = float(np.max(np.abs(got - ref)))
         assert err < 1e-10 * max(1.0, float(np.max(np.abs(ref)))), err
+
+    for gg in graphs:
+        cache = o.new_contiguous_cache(2, 16)
+        ev = GraphEval(mod)
+        got, work = ev.run(gg, ids)
+        close(got, o.prefill(ids, cache))
+        past, lens = ev.next_past(work, ids), np.full(2, 7)
+        for t in range(fed.shape[1]):
+            step = fed[:, t:t + 1]
+            got, work = ev.run(gg, step, past)
+            close(got[:, 0], o.decode_step(fed[:, t], cache, lens))
+            past, lens = ev.next_past(work, step), lens + 1
 
 
 def test_lowered_moe_shape_fills_the_config_the_library_reads():
