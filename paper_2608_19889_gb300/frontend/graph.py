@@ -252,6 +252,13 @@ class Builder:
                     raise AxonGraphError(f"line {st.line}: yield outside a loop body")
                 vals = [self.eval(x, env, prefix) for x in st.exprs]
                 return ("__yield__", vals)
+            if isinstance(st, sx.IfS):
+                # only the taken branch is built; its return (or yield) ends this suite
+                c = self.eval(st.cond, env, prefix)
+                if not _is_const(c):
+                    raise AxonGraphError(f"line {st.line}: a branch condition must be known when the graph "
+                                         "is built")
+                return self.run_suite(st.then if c else st.other, dict(env), prefix, yield_ok)
             if isinstance(st, sx.BindS):
                 self.want = len(st.targets)
                 v = self.eval(st.expr, env, prefix)

@@ -9,7 +9,8 @@ values, symbolic-dimension types, Haskell-style syntax; appendix
     definitions ``name[@scope] p1 p2 = expr`` or ``= do`` + an indented suite;
   * statements: ``targets <- expr``, ``return e1, e2``, ``yield e1, e2``,
     ``targets <- for[@scope] i <- [a..b) [carry (x, y)] do`` + suite,
-    ``targets <- scope@path do`` + suite;
+    ``targets <- scope@path do`` + suite, and the statement-level
+    conditional ``if c then do`` + suite ``else do`` + suite;
   * expressions, lowest precedence first: ``::`` ascription (inside
     parentheses), ``>>=`` with a lambda, ``|>`` pipes, ``if/then/else`` and
     ``c ? a : b``, ``or``, ``and``, comparisons, ``+ -``, ``* /``, bare-call
@@ -116,6 +117,16 @@ class BindS:
 @dataclass
 class ReturnS:
     exprs: list
+    line: int = 0
+
+
+@dataclass
+class IfS:
+    """Statement-level conditional between two do suites; the taken suite's
+    return (or yield) ends the enclosing suite."""
+    cond: object
+    then: list
+    other: list
     line: int = 0
 
 
@@ -372,7 +383,7 @@ class Parser:
 
     # suites
     def suite(self) -> list:
-        """After `do`: an indented block, or one inline statement."""
+        """After `do`: an indented block, or inline statements separated by `;`."""
         if self.at("NEWLINE"):
             self.eat("NEWLINE")
             self.eat("INDENT")
@@ -386,7 +397,10 @@ class Parser:
                 self.skip_newlines()
             self.eat("DEDENT")
             return stmts
-        return [self.statement()]
+        stmts = [self.statement()]  # inline: `do s1; s2; return e`
+        while self.opt("OP", ";"):
+            stmts.append(self.statement())
+        return stmts
 
     def statement(self):
         tok = self.peek()
@@ -396,6 +410,18 @@ class Parser:
         if tok.kind == "NAME" and tok.text == "yield":
             self.i += 1
             return YieldS(self.expr_list(), tok.line)
+        if tok.kind == "NAME" and tok.text == "if":
+            self.i += 1
+            cond = self.expr()
+            self.eat("NAME", "then")
+            self.eat("NAME", "do")
+            then = self.suite()
+            self.skip_newlines()
+            if not self.at("NAME", "else"):
+                raise AxonSyntaxError("a statement-level if needs an else branch", self.peek().line)
+            self.eat("NAME", "else")
+            self.eat("NAME", "do")
+            return IfS(cond, then, self.suite(), tok.line)
         # targets <- ...
         targets = [self.eat("NAME").text]
         while self.opt("OP", ","):

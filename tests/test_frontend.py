@@ -463,3 +463,55 @@ def test_lowered_moe_shape_fills_the_config_the_library_reads():
     assert (c.n_routed_experts, c.num_experts_per_tok, c.moe_intermediate_size, c.n_shared_experts,
             c.first_k_dense_replace, c.norm_topk_prob) == (6, 2, 16, 2, 1, 1)
     assert (c.num_attention_heads, c.num_key_value_heads, c.head_dim, c.hidden_act) == (4, 2, 8, ax.AXON_ACT_SILU)
+
+
+# ------------------------------------------------------------ conditionals
+COND = """import NN
+USE <- Config.value @@use_norm default=true
+expr_if x = if USE then NN.rmsnorm@a x eps=0.1 else x
+ternary x = USE ? NN.rmsnorm@b x eps=0.1 : null
+stmt_if x = do
+  if USE then do
+    return x
+  else do
+    y <- NN.rmsnorm@c x eps=0.1
+    return y
+inline x = do h <- NN.rmsnorm@d x eps=0.1; return h
+"""
+
+
+@pytest.mark.parametrize("use", [True, False])
+def test_conditional_forms_build_only_the_taken_branch(use):
+    mod = sx.parse_module(COND)
+    ops = {e: [n.op + ("@" + n.path if n.path else "") for n in fe.build_graph(mod, {"use_norm": use}, entry=e).nodes]
+           for e in ("expr_if", "ternary", "stmt_if", "inline")}
+    norm = ["input", "NN.rmsnorm@{}"]
+    assert ops["expr_if"] == ([norm[0], norm[1].format("a")] if use else ["input"])
+    assert ops["ternary"] == ([norm[0], norm[1].format("b")] if use else ["input"])
+    assert ops["stmt_if"] == (["input"] if use else [norm[0], norm[1].format("c")])
+    assert ops["inline"] == [norm[0], norm[1].format("d")]
+
+
+def test_statement_if_needs_an_else():
+    with pytest.raises(fe.AxonSyntaxError, match="else"):
+        sx.parse_module("f x = do\n  if true then do\n    return x\n  y <- x\n  return y\n")
+
+
+@pytest.mark.parametrize("qk", [True, False])
+def test_a_config_switch_in_the_module_selects_the_variant(qk):
+    """qk-norm behind a configuration flag, written with the statement-level
+    conditional: the lowering sees only the taken branch."""
+    src = LLAMA.replace("WINDOW <- Config.value @@sliding_window default=0",
+                        "WINDOW <- Config.value @@sliding_window default=0\nQK_NORM <- Config.value @@qk_norm default=false")
+    src = src.replace("  q <- rope q pos theta=THETA\n  k <- rope k pos theta=THETA\n",
+                      "  q, k <- qk_norm_rope q k pos\n")
+    src = src.replace("ffn :: ", "qk_norm_rope q k pos = do\n"
+                      "  if QK_NORM then do\n"
+                      "    return rope (NN.rmsnorm@q_norm q eps=EPS) pos theta=THETA, "
+                      "rope (NN.rmsnorm@k_norm k eps=EPS) pos theta=THETA\n"
+                      "  else do\n"
+                      "    return rope q pos theta=THETA, rope k pos theta=THETA\n\n"
+                      "ffn :: ")
+    low = fe.compile_decoder(src, dict(CFG, qk_norm=qk))
+    assert low.shape["qk_norm"] == qk
+    assert ("model.layers.0.self_attn.q_norm.weight" in low.names) == qk
