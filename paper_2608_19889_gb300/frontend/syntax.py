@@ -5,8 +5,11 @@ values, symbolic-dimension types, Haskell-style syntax; appendix
 "Operations" paragraphs and the grammar figure):
 
   * module items: pragmas ``{-# KEY value #-}``, ``import M`` / ``import M (a, b)``,
-    constants ``NAME <- expr``, signatures ``name :: type`` (kept as text),
-    definitions ``name[@scope] p1 p2 = expr`` or ``= do`` + an indented suite;
+    ``export a b``, type aliases ``type T[x] = type`` and signatures
+    ``name[@scope] :: type`` (both kept as text: types are not checked),
+    constants ``NAME <- expr``, definitions ``name[@scope] p1 p2 = expr`` or
+    ``= do`` + an indented suite (a scope on the signature applies to the
+    definition);
   * statements: ``targets <- expr``, ``return e1, e2``, ``yield e1, e2``,
     ``targets <- for[@scope] i <- [a..b) [carry (x, y)] do`` + suite,
     ``targets <- scope@path do`` + suite, and the statement-level
@@ -174,6 +177,8 @@ class Module:
     pragmas: dict = field(default_factory=dict)
     imports: list = field(default_factory=list)
     constants: list = field(default_factory=list)  # [(name, expr)] in order
+    exports: list = field(default_factory=list)  # exported names
+    types: dict = field(default_factory=dict)  # alias -> type text
     definitions: dict = field(default_factory=dict)  # name -> Definition
     order: list = field(default_factory=list)  # definition names in source order
 
@@ -337,6 +342,20 @@ class Parser:
                         self.opt("OP", ",")
                     self.eat("OP", ")")
                 mod.imports.append((name, names))
+            elif tok.kind == "NAME" and tok.text == "export" and self.at("NAME", None, 1):
+                self.i += 1
+                while self.at("NAME"):
+                    mod.exports.append(self.eat("NAME").text)
+            elif tok.kind == "NAME" and tok.text == "type" and self.at("NAME", None, 1):
+                self.i += 1
+                name = self.eat("NAME").text
+                parts = []
+                while not self.at("NEWLINE") and not self.at("EOF"):
+                    parts.append(self.peek().text)
+                    self.i += 1
+                if not parts or parts[0] not in ("=", "[") or "=" not in parts:
+                    raise AxonSyntaxError(f"type alias {name}: expected [params] = type", tok.line)
+                mod.types[name] = " ".join(parts)
             elif tok.kind == "NAME" and self.at("OP", "<-", 1):
                 name = self.eat("NAME").text
                 self.eat("OP", "<-")
@@ -377,6 +396,8 @@ class Parser:
         if d is not None and d.body is not None:
             raise AxonSyntaxError(f"definition {start.text} given twice", start.line)
         sig = d.signature if d else None
+        if scope is None and d is not None:
+            scope = d.scope  # `name@scope :: type` then `name x = ...`
         mod.definitions[start.text] = Definition(start.text, scope, params, body, sig, start.line)
         if start.text not in mod.order:
             mod.order.append(start.text)

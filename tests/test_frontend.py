@@ -515,3 +515,17 @@ def test_a_config_switch_in_the_module_selects_the_variant(qk):
     low = fe.compile_decoder(src, dict(CFG, qk_norm=qk))
     assert low.shape["qk_norm"] == qk
     assert ("model.layers.0.self_attn.q_norm.weight" in low.names) == qk
+
+
+def test_exports_type_aliases_and_a_scope_on_the_signature():
+    src = ("import NN\nexport layer Twin\n\ntype Twin[T] = (T, T)\n\nwidth <- 64\n\n"
+           "layer@blk :: Tensor[B,S,D] -> ?Tensor[B,K] -> Tensor[B,S,D]\n"
+           "layer x m = do\n  h <- NN.rmsnorm@norm x eps=0.5\n  return x + h\n")
+    mod = sx.parse_module(src)
+    assert mod.exports == ["layer", "Twin"] and "Twin" in mod.types
+    assert mod.definitions["layer"].scope == "blk"
+    g = fe.build_graph(mod, {}, entry="layer")
+    assert [n.path for n in g.nodes if n.path] == ["blk.norm"]
+    assert [n.op for n in g.nodes if n.op == "input"] == ["input", "input"]  # the optional argument too
+    with pytest.raises(fe.AxonSyntaxError, match="type alias"):
+        sx.parse_module("type Twin T\n")
