@@ -37,7 +37,7 @@ loads through ``axon_model_create``.
 from __future__ import annotations
 
 from dataclasses import dataclass, field
-from typing import Dict, List, Optional
+from typing import Dict, Optional
 
 from . import graph as gr
 from .rewrite import ACTIVATIONS as _ACTS, SWIGLU as _SWIGLU, stack_experts
