@@ -39,28 +39,34 @@ POINTS = ("a", "q", "k", "v", "P", "o", "u")
 
 
 def rounder(kind):
-    """float64 array -> the same values rounded to bf16 or fp16."""
+    """float64 array -> the same values rounded to bf16 or fp16; kind
+    "bf16x2" / "fp16x2": two terms, hi = round(x) plus round(x - hi)."""
     import torch
-    dt = {"bf16": torch.bfloat16, "fp16": torch.float16}[kind]
+    dt = {"bf16": torch.bfloat16, "fp16": torch.float16}[kind.replace("x2", "")]
 
-    def r(x):
+    def r1(x):
         return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float64)).to(dt).to(torch.float64).numpy()
-    return r
+
+    if kind.endswith("x2"):
+        return lambda x: r1(x) + r1(np.asarray(x, dtype=np.float64) - r1(x))
+    return r1
 
 
 def forward(cfg: od.DecoderConfig, W: dict, ids, rounded=(), kind="fp16"):
     """Prompt pass of B sequences from an empty cache with 16-bit rounding at
-    the points named in `rounded`. Returns logits [B, S, V]."""
-    rnd = rounder(kind)
+    the points named in `rounded`, all of one kind, or with `kind` a dict
+    {point: kind}. Returns logits [B, S, V]."""
+    kinds = kind if isinstance(kind, dict) else {pt: kind for pt in POINTS}
+    rnds = {pt: rounder(k) for pt, k in kinds.items()}
 
     def at(point, x):
-        return rnd(x) if point in rounded else x
+        return rnds[point](x) if point in rounded else x
 
     def norm(x, g):
         if "a" not in rounded:
             return od.rmsnorm(x, g, cfg.eps)
         r = 1.0 / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + cfg.eps)
-        return rnd(x * g) * r
+        return rnds["a"](x * g) * r
 
     ids = np.asarray(ids, dtype=np.int64)
     B, S = ids.shape
@@ -131,11 +137,21 @@ def main():
     shape = dict(si.MODEL_SHAPES[args.width], L=args.layers)
     W = {k: np.asarray(v, dtype=np.float64) for k, v in si.weights_as_f32_numpy(si.make_weights(shape)).items()}
     ids = si.make_ids(1, args.seq, shape["V"])
-    res = table(od.DecoderConfig.from_dict(shape), W, ids)
+    cfg = od.DecoderConfig.from_dict(shape)
+    res = table(cfg, W, ids)
     print("| rounded to | " + " | ".join(POINTS) + " | all but a |")
     print("|---" * (len(POINTS) + 2) + "|")
     for kind, row in res.items():
         print(f"| {kind} | " + " | ".join(f"{row[p][0]:.1e} / {row[p][1]:.1e}" for p in POINTS + ("all",)) + " |")
+    # whole modes: every point rounded as the mode stores it
+    ref = forward(cfg, W, ids)
+    modes = {"bf16 (one term everywhere)": "bf16",
+             "bf16, two terms everywhere but the KV cache": {**{pt: "bf16x2" for pt in POINTS}, "k": "bf16",
+                                                             "v": "bf16"},
+             "fp16, two-term a (the fp16 prefill)": {**{pt: "fp16" for pt in POINTS}, "a": "fp16x2"}}
+    for name, kind in modes.items():
+        e = forward(cfg, W, ids, POINTS, kind) - ref
+        print(f"{name}: rms {np.sqrt(np.mean(e * e)):.1e}, max {np.max(np.abs(e)):.1e}")
 
 
 if __name__ == "__main__":

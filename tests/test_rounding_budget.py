@@ -34,3 +34,14 @@ def test_fp16_rounding_costs_less_than_bf16_at_every_point():
     for pt in POINTS + ("all",):
         f_rms, b_rms = t["fp16"][pt][0], t["bf16"][pt][0]
         assert 0 < f_rms < b_rms, (pt, f_rms, b_rms)
+
+
+def test_two_term_rounding_keeps_about_twice_the_bits():
+    from rounding_budget import rounder
+    # magnitudes in [0.25, 4): the second fp16 term stays out of fp16's subnormal range
+    rng = np.random.Generator(np.random.PCG64(8))
+    x = rng.choice([-1.0, 1.0], size=10000) * 2.0 ** rng.uniform(-2, 2, size=10000)
+    for kind, one, two in (("bf16", 2.0 ** -8, 2.0 ** -16), ("fp16", 2.0 ** -11, 2.0 ** -21)):
+        e1 = np.max(np.abs(rounder(kind)(x) - x) / np.abs(x))
+        e2 = np.max(np.abs(rounder(kind + "x2")(x) - x) / np.abs(x))
+        assert e1 <= one and 0 < e2 <= two, (kind, e1, e2)
