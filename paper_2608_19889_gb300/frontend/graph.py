@@ -282,6 +282,9 @@ class Builder:
             raise AxonGraphError("loop bounds must be known when the graph is built")
         lo = start if e.lo_closed else start + 1
         hi = stop + 1 if e.hi_closed else stop
+        step = 1 if e.step is None else self.eval(e.step, env, prefix)
+        if not isinstance(step, int) or step < 1:
+            raise AxonGraphError("a loop step must be a positive integer known when the graph is built")
         init = [env[c] for c in e.carry]
         body = Graph()
         self.graphs.append(body)
@@ -299,7 +302,7 @@ class Builder:
         body.outputs = out[1]
         if len(body.outputs) != len(e.carry):
             raise AxonGraphError("yield must give one value per carried name")
-        refs = self.emit("loop", init, {"var": e.var, "start": lo, "stop": hi,
+        refs = self.emit("loop", init, {"var": e.var, "start": lo, "stop": hi, "step": step,
                                          "scope": e.scope or ""}, n_out=len(e.carry), body=body)
         return refs
 

@@ -514,6 +514,8 @@ def lower_decoder(g: gr.Graph, config: Optional[dict] = None) -> LoweredDecoder:
                             f"found {len(loops)}")
     if loops[0].attrs["start"] != 0:
         raise LoweringError("the layer loop must start at 0")
+    if any(lp.attrs.get("step", 1) != 1 for lp in loops):
+        raise LoweringError("a layer loop must advance one layer per iteration (step=1)")
     if len(loops) == 2:
         a, b = loops
         if b.attrs["start"] != a.attrs["stop"]:

@@ -58,8 +58,8 @@ def _expert_loop(loop: gr.Node) -> Optional[gr.Node]:
     body = loop.body
     if body is None or loop.n_out != 1 or len(body.inputs) != 1 or len(body.outputs) != 1:
         return None
-    if loop.attrs.get("start") != 0 or loop.attrs.get("stop", 0) <= 0:
-        return None
+    if loop.attrs.get("start") != 0 or loop.attrs.get("stop", 0) <= 0 or loop.attrs.get("step", 1) != 1:
+        return None  # not every expert once
     var = loop.attrs.get("var")
     byid = {n.id: n for n in body.nodes}
 

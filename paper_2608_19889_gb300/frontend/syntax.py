@@ -11,7 +11,7 @@ values, symbolic-dimension types, Haskell-style syntax; appendix
     ``= do`` + an indented suite (a scope on the signature applies to the
     definition);
   * statements: ``targets <- expr``, ``return e1, e2``, ``yield e1, e2``,
-    ``targets <- for[@scope] i <- [a..b) [carry (x, y)] do`` + suite,
+    ``targets <- for[@scope] i <- [a..b) [step=n] [carry (x, y)] do`` + suite,
     ``targets <- scope@path do`` + suite, and the statement-level
     conditional ``if c then do`` + suite ``else do`` + suite;
   * expressions, lowest precedence first: ``::`` ascription (inside
@@ -149,6 +149,7 @@ class ForE:
     hi_closed: bool
     carry: List[str]
     body: list
+    step: object = None  # `step=n` (an expression), None: 1
 
 
 @dataclass
@@ -471,12 +472,11 @@ class Parser:
         if hi not in ")]":
             raise AxonSyntaxError("range must end with ) or ]", self.peek().line)
         carry = []
+        step = None
         if self.at("NAME", "step"):
             self.i += 1
             self.eat("OP", "=")
             step = self.atom()
-            if not (isinstance(step, Num) and step.value == 1):
-                raise AxonSyntaxError("only step=1 loops are in this subset", self.peek().line)
         if self.opt("NAME", "carry"):
             self.eat("OP", "(")
             while not self.at("OP", ")"):
@@ -484,7 +484,7 @@ class Parser:
                 self.opt("OP", ",")
             self.eat("OP", ")")
         self.eat("NAME", "do")
-        return ForE(scope, var, start, stop, lo == "[", hi == "]", carry, self.suite())
+        return ForE(scope, var, start, stop, lo == "[", hi == "]", carry, self.suite(), step)
 
     def scope_expr(self) -> ScopeE:
         self.eat("NAME", "scope")

@@ -95,7 +95,7 @@ class GraphEval:
         op = n.op
         if op == "loop":
             vals = ins
-            for i in range(at["start"], at["stop"]):
+            for i in range(at["start"], at["stop"], at.get("step", 1)):
                 inner = dict(lv)
                 inner[at["var"]] = i
                 vals = self._graph(n.body, vals, env, inner)

@@ -529,3 +529,16 @@ def test_exports_type_aliases_and_a_scope_on_the_signature():
     assert [n.op for n in g.nodes if n.op == "input"] == ["input", "input"]  # the optional argument too
     with pytest.raises(fe.AxonSyntaxError, match="type alias"):
         sx.parse_module("type Twin T\n")
+
+
+def test_loops_with_a_step():
+    src = ("import NN\nf x = do\n  y <- for i <- [0..7) step=2 carry (x) do\n    x <- x + 1.0\n    yield x\n"
+           "  return y\n")
+    g = fe.build_graph(sx.parse_module(src), {}, entry="f")
+    loop = [n for n in g.nodes if n.op == "loop"][0]
+    assert (loop.attrs["start"], loop.attrs["stop"], loop.attrs["step"]) == (0, 7, 2)
+    assert GraphEval({}).run(g, np.zeros((1, 1)))[0] == 4.0  # i = 0, 2, 4, 6
+    with pytest.raises(fe.AxonGraphError, match="step"):
+        fe.build_graph(sx.parse_module(src.replace("step=2", "step=0")), {}, entry="f")
+    with pytest.raises(fe.LoweringError, match="one layer per iteration"):
+        fe.compile_decoder(LLAMA.replace("[0..LAYERS) carry", "[0..LAYERS) step=2 carry"), CFG)
