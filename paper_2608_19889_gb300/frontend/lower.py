@@ -339,7 +339,7 @@ def _match_layer(loop: gr.Node, g: gr.Graph, cfg: dict, D: int) -> _Layer:
     rope_scaling = {}
 
     heads_ops = {"Attention.reshape_heads", "Attention.split_qkv"}
-    splits = []  # (split node, output index) of a fused q/k/v projection
+    splits = []  # the split_qkv node behind q, k and v (fused projection)
 
     def heads_of(ref, what, index):
         """The projection behind reshape_heads, or behind output `index` of
